@@ -1,0 +1,198 @@
+/*
+ * gleam.h -- C ABI of libgleam.so, the GB300 (sm_103a) chunk-dedup library.
+ *
+ * The operation (paper Sec. 4.1.2, "Hash-based Weight Chunk Retrieval"): before
+ * a host-to-device cudaMemcpy payload crosses the network, the payload is
+ * identified by hash against the set of chunks already resident on the
+ * server; a resident chunk is replaced by (hash, size) metadata and only the
+ * others travel in full, after which they are resident too.  App. B.1 ("Hash
+ * Cost and Collision") describes the paper's own identifier (MD5 of a 128-byte
+ * prefix, no byte check).  This library generalises it: every fixed C-byte
+ * chunk is identified by XXH64 (seed 0) over its whole length, looked up in a
+ * device-resident open-addressing index, and every key match is confirmed
+ * byte for byte against the cached copy, so a hash collision can never make
+ * two different chunks alias.
+ *
+ * Conventions shared by every call:
+ *  - Plain C types only.  A "device pointer" is memory the calling process
+ *    allocated on the cache's GPU (cudaMalloc, cudaMallocAsync or managed
+ *    memory); host pointers are rejected with GLEAM_ERR_NOT_DEVICE_PTR.
+ *  - The caller owns every buffer it passes.  The library owns the cache's
+ *    arena, index and per-call workspace, allocated on the GPU that was
+ *    current when the cache was created.
+ *  - Errors are negative return values (enum gleam_status).  A call that
+ *    returns an error other than GLEAM_ERR_CUDA leaves the cache unchanged.
+ *  - Chunk i of an n-byte payload covers bytes [i*C, min(n, (i+1)*C)); the last
+ *    chunk keeps its true length, and length is part of chunk equality.
+ */
+#ifndef GLEAM_H
+#define GLEAM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A CUDA stream handle (ABI-identical to cudaStream_t).  NULL means the legacy
+ * default stream, which orders against every blocking stream like cudaMemcpy. */
+typedef struct CUstream_st* gleam_stream_t;
+
+/* Opaque weight cache: device arena of fixed C-byte slots, device index, stats. */
+typedef struct gleam_cache gleam_cache_t;
+
+/* Opaque device-side copy of a cache's index and counters (test/bench helper). */
+typedef struct gleam_snapshot gleam_snapshot_t;
+
+enum gleam_status {
+  GLEAM_OK = 0,
+  GLEAM_ERR_INVALID_ARG = -1,   /* NULL handle/pointer, bad sizes, bad flags   */
+  GLEAM_ERR_NOT_DEVICE_PTR = -2,/* a buffer is not device memory of this GPU  */
+  GLEAM_ERR_CUDA = -3,          /* a CUDA runtime call failed                 */
+  GLEAM_ERR_CAPACITY = -4,      /* misses do not fit the free slots           */
+  GLEAM_ERR_TIMEOUT = -5,       /* a bounded device-side wait ran out         */
+  GLEAM_ERR_NOMEM = -6,         /* device allocation failed                   */
+  GLEAM_ERR_INTERNAL = -7       /* a device-side consistency check failed     */
+};
+
+/* Flags for gleam_cache_create_ex. */
+#define GLEAM_KEY16 0x1u        /* test mode: index key = low 16 bits of XXH64,
+                                   so unrelated chunks collide and every hit
+                                   must be separated from them by the verify */
+#define GLEAM_DEBUG_CHECKS 0x2u /* extra device-side index/arena checks      */
+
+/* Cumulative counters of one cache (successful calls only). */
+typedef struct gleam_stats {
+  uint64_t calls;          /* gleam_dedup_copy* calls with n > 0             */
+  uint64_t chunks;         /* chunks examined                                */
+  uint64_t hits_cache;     /* chunks found byte-equal in the cache as it was
+                              when their call started                        */
+  uint64_t hits_intra;     /* chunks equal to an earlier miss of their call  */
+  uint64_t misses;         /* chunks returned as misses (and inserted)       */
+  uint64_t inserts;        /* entries added (misses + debug inserts)         */
+  uint64_t verify_rejects; /* misses that had a key+length candidate whose
+                              bytes differed (collisions caught by verify)   */
+  uint64_t slots_used;     /* arena slots in use                             */
+  uint64_t bytes_used;     /* sum of the stored chunks' true lengths         */
+  uint64_t capacity_bytes; /* as passed to create                            */
+  uint64_t nslots;         /* capacity_bytes / chunk_bytes                   */
+  uint64_t chunk_bytes;    /* C                                              */
+} gleam_stats_t;
+
+/* Written by the device when an asynchronous dedup call completes. */
+typedef struct gleam_result {
+  int64_t status;          /* GLEAM_OK or a negative gleam_status            */
+  uint64_t n_miss;         /* misses = entries of miss_idx written           */
+  uint64_t n_hit_cache;
+  uint64_t n_hit_intra;
+  uint64_t verify_rejects;
+  uint64_t miss_bytes;     /* bytes written to the packed miss buffer        */
+} gleam_result_t;
+
+/* ---- cache lifetime ---------------------------------------------------- */
+
+/* Creates a cache on the current GPU with floor(capacity_bytes/chunk_bytes)
+ * slots of chunk_bytes each and an empty index (paper Sec. 4.1.3: the
+ * server-side shareable pool; Sec. 4.1.2: the set of resident identifiers).
+ * chunk_bytes: multiple of 32, 32..16 MiB.  The slot count must be 1..2^32-2.
+ * flags: 0 or a combination of GLEAM_KEY16 and GLEAM_DEBUG_CHECKS.
+ * On success *out owns about capacity_bytes + 32 B * slots of device memory.
+ * Returns GLEAM_OK, GLEAM_ERR_INVALID_ARG, GLEAM_ERR_NOMEM or GLEAM_ERR_CUDA. */
+int gleam_cache_create(size_t capacity_bytes, size_t chunk_bytes, gleam_cache_t** out);
+int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t flags,
+                          gleam_cache_t** out);
+
+/* Frees the arena, index and workspace after the cache's work has finished.
+ * NULL is accepted.  The handle is invalid afterwards. */
+void gleam_cache_destroy(gleam_cache_t* cache);
+
+/* Pre-sizes the per-call workspace for payloads of up to max_chunks chunks,
+ * so that later calls of that size allocate nothing.  Synchronous. */
+int gleam_cache_reserve(gleam_cache_t* cache, uint64_t max_chunks);
+
+/* ---- the hot path ------------------------------------------------------ */
+
+/* Fingerprints (paper Sec. 4.1.2's per-payload hash; App. B.1):
+ * d_out[i] = XXH64(seed 0) of chunk i of the n-byte device buffer d_buf, for
+ * i < ceil(n/chunk_bytes).  chunk_bytes == 0 hashes the whole buffer into
+ * d_out[0] (also for n == 0).  d_out: device array of u64, caller-owned.
+ * Asynchronous on `stream`; any alignment of d_buf is accepted. */
+int gleam_fingerprint(const void* d_buf, size_t n, size_t chunk_bytes, uint64_t* d_out,
+                      gleam_stream_t stream);
+
+/* Dedups one host-to-device payload already copied to the device (paper
+ * Sec. 4.1.2).  Chunks are decided in ascending order, as if one at a time:
+ * chunk i is a hit iff its bytes equal a cached chunk of the same length, or
+ * an earlier miss of this same call; otherwise it is a miss, is appended to
+ * the outputs and is inserted into the cache.
+ * Outputs (device memory, caller-owned, sized for the worst case):
+ *   d_hit_mask   u32[ceil(N/32)]: bit i%32 of word i/32 = chunk i is a hit,
+ *                bits past N are 0;
+ *   d_miss_idx   u32[N]: ascending indices of the misses;
+ *   d_miss_bytes u8[n]: the r-th miss's bytes at offset r*C (true length for
+ *                the last chunk) -- the bytes that must cross the network.
+ * Synchronous like cudaMemcpy (runs on the legacy default stream).
+ * Returns the number of misses (>= 0) or a negative gleam_status; on
+ * GLEAM_ERR_CAPACITY and GLEAM_ERR_TIMEOUT the cache is unchanged and the
+ * outputs are unspecified.  n == 0 returns 0 and touches nothing. */
+int64_t gleam_dedup_copy(gleam_cache_t* cache, const void* d_buf, size_t n,
+                         uint32_t* d_hit_mask, uint32_t* d_miss_idx, void* d_miss_bytes);
+
+/* Same as gleam_dedup_copy, enqueued on `stream` without a host sync.  The
+ * outcome is written to the device struct *d_result (may be NULL) when the
+ * call's work completes.  Calls on one cache must be ordered (one stream, or
+ * explicit events): they share the cache's workspace.  Returns GLEAM_OK once
+ * enqueued, or an argument/launch error.  The first call that needs a larger
+ * workspace than any before it synchronises the stream to grow it (see
+ * gleam_cache_reserve). */
+int gleam_dedup_copy_async(gleam_cache_t* cache, const void* d_buf, size_t n,
+                           uint32_t* d_hit_mask, uint32_t* d_miss_idx, void* d_miss_bytes,
+                           gleam_result_t* d_result, gleam_stream_t stream);
+
+/* Copies the cache's counters to *out (host struct).  Waits for the cache's
+ * outstanding work on the device. */
+int gleam_cache_stats(const gleam_cache_t* cache, gleam_stats_t* out);
+
+/* ---- inspection and test helpers (not on the hot path) ------------------ */
+
+/* Index contents ordered by slot: h_keys[s], h_lens[s] for s < min(max,
+ * slots_used) (host arrays).  *count receives the number of index entries. */
+int gleam_cache_export(const gleam_cache_t* cache, uint64_t* h_keys, uint32_t* h_lens,
+                       uint64_t max, uint64_t* count);
+
+/* Copies the stored bytes of `slot` to host memory h_out (at most max bytes);
+ * *len receives the stored length. */
+int gleam_cache_read_slot(const gleam_cache_t* cache, uint64_t slot, void* h_out,
+                          uint64_t max, uint64_t* len);
+
+/* Stores len bytes from device memory d_bytes under an arbitrary key (masked
+ * to 16 bits in GLEAM_KEY16 mode) in the next free slot.  Used to plant
+ * colliding entries that the verify must reject.  Synchronous. */
+int gleam_cache_debug_insert(gleam_cache_t* cache, uint64_t key, const void* d_bytes,
+                             size_t len);
+
+/* Test hooks.  what = GLEAM_DEBUG_WAIT_LIMIT_NS: limit of every device-side
+ * wait in nanoseconds (default 4e9); what = GLEAM_DEBUG_SKIP_ARRIVE: the block
+ * with this index (-1 = none) leaves the next call's first grid barrier
+ * without arriving, so the other blocks' bounded waits run out and the call
+ * returns GLEAM_ERR_TIMEOUT with the cache unchanged. */
+#define GLEAM_DEBUG_WAIT_LIMIT_NS 1
+#define GLEAM_DEBUG_SKIP_ARRIVE 2
+int gleam_cache_debug_set(gleam_cache_t* cache, int what, int64_t value);
+
+/* Device-side copy of the index, slot count and counters, for restoring the
+ * cache between timed repetitions.  Arena bytes past the saved slot count are
+ * never read, so they are not copied. */
+int gleam_cache_snapshot(gleam_cache_t* cache, gleam_snapshot_t** out);
+int gleam_cache_restore(gleam_cache_t* cache, const gleam_snapshot_t* snap);
+void gleam_snapshot_destroy(gleam_snapshot_t* snap);
+
+/* Short English name of a gleam_status value. */
+const char* gleam_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GLEAM_H */

@@ -1,0 +1,163 @@
+"""Gleam chunk-dedup oracle -- TEST INFRASTRUCTURE ONLY.
+
+A ctypes wrapper over ``gleam_oracle.cpp``: the plain, single-threaded CPU
+statement of the dedup hot path (paper Sec. 4.1.2, "Hash-based Weight Chunk
+Retrieval", and App. B.1, "Hash Cost and Collision"; XXH64 from the public
+xxHash specification).  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` may import it.  The CUDA library never does,
+and the two share no code.
+
+Every function here is pinned by ``tests/test_oracle_*.py`` against values the
+oracle does not produce itself: published XXH64 vectors, the installed
+libxxhash, zstd frame checksums, a pure-Python brute-force dedup on tiny
+inputs, and closed forms of the synthetic workloads.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "gleam_oracle.cpp")
+_LIB = os.path.join(_HERE, "liboracle.so")
+
+OK = 0
+ERR_INVALID_ARG = -1
+ERR_CAPACITY = -4
+KEY16 = 1
+
+STAT_FIELDS = (
+    "calls", "chunks", "hits_cache", "hits_intra", "misses", "inserts",
+    "verify_rejects", "slots_used", "bytes_used", "capacity_bytes", "nslots",
+    "chunk_bytes",
+)
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with the host C++ compiler (portable C++17)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + ".tmp%d" % os.getpid()
+        subprocess.check_call(
+            ["g++", "-O2", "-std=c++17", "-shared", "-fPIC", "-o", tmp, _SRC])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        l = ctypes.CDLL(build())
+        u64, sz, vp = ctypes.c_uint64, ctypes.c_size_t, ctypes.c_void_p
+        l.oracle_xxh64.restype = u64
+        l.oracle_xxh64.argtypes = [vp, sz, u64]
+        l.oracle_fingerprint.restype = ctypes.c_int
+        l.oracle_fingerprint.argtypes = [vp, sz, sz, vp]
+        l.oracle_cache_create.restype = vp
+        l.oracle_cache_create.argtypes = [sz, sz, ctypes.c_uint32, ctypes.POINTER(ctypes.c_int)]
+        l.oracle_cache_destroy.restype = None
+        l.oracle_cache_destroy.argtypes = [vp]
+        l.oracle_dedup.restype = ctypes.c_int64
+        l.oracle_dedup.argtypes = [vp, vp, sz, vp, vp, vp]
+        l.oracle_debug_insert.restype = ctypes.c_int
+        l.oracle_debug_insert.argtypes = [vp, u64, vp, sz]
+        l.oracle_cache_stats.restype = None
+        l.oracle_cache_stats.argtypes = [vp, vp]
+        l.oracle_cache_entries.restype = u64
+        l.oracle_cache_entries.argtypes = [vp, vp, vp, u64]
+        l.oracle_slot_bytes.restype = ctypes.c_int64
+        l.oracle_slot_bytes.argtypes = [vp, u64, vp, u64]
+        _lib = l
+    return _lib
+
+
+def _u8(buf) -> np.ndarray:
+    a = np.frombuffer(buf, dtype=np.uint8) if isinstance(buf, (bytes, bytearray, memoryview)) \
+        else np.ascontiguousarray(buf).view(np.uint8).reshape(-1)
+    return a
+
+
+def xxh64(data, seed: int = 0) -> int:
+    a = _u8(data)
+    return int(lib().oracle_xxh64(a.ctypes.data, a.size, seed))
+
+
+def fingerprint(data, chunk_bytes: int) -> np.ndarray:
+    """XXH64 (seed 0) of every chunk_bytes-byte chunk; chunk_bytes == 0: of the whole buffer."""
+    a = _u8(data)
+    n = a.size
+    count = 1 if chunk_bytes == 0 else (n + chunk_bytes - 1) // chunk_bytes
+    out = np.zeros(count, dtype=np.uint64)
+    rc = lib().oracle_fingerprint(a.ctypes.data, n, chunk_bytes, out.ctypes.data)
+    assert rc == OK
+    return out
+
+
+class OracleCache:
+    """The sequential weight cache: index + stored chunk bytes + statistics."""
+
+    def __init__(self, capacity_bytes: int, chunk_bytes: int, flags: int = 0):
+        err = ctypes.c_int(0)
+        self._h = lib().oracle_cache_create(capacity_bytes, chunk_bytes, flags, ctypes.byref(err))
+        if not self._h:
+            raise ValueError("oracle_cache_create rejected its arguments (%d)" % err.value)
+        self.chunk_bytes = chunk_bytes
+        self.flags = flags
+
+    def close(self):
+        if self._h:
+            lib().oracle_cache_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        self.close()
+
+    def dedup(self, data):
+        """Returns (rc, hit_mask u32[], miss_idx u32[n_miss], packed u8[packed_bytes])."""
+        a = _u8(data)
+        n = a.size
+        C = self.chunk_bytes
+        nch = (n + C - 1) // C
+        mask = np.zeros(max(1, (nch + 31) // 32), dtype=np.uint32)
+        miss = np.zeros(max(1, nch), dtype=np.uint32)
+        packed = np.zeros(max(1, n), dtype=np.uint8)
+        rc = int(lib().oracle_dedup(self._h, a.ctypes.data, n, mask.ctypes.data,
+                                    miss.ctypes.data, packed.ctypes.data))
+        if rc < 0:
+            return rc, None, None, None
+        miss = miss[:rc].copy()
+        nbytes = 0
+        if rc:
+            last = int(miss[-1])
+            tail = n - last * C if last == nch - 1 else C
+            nbytes = (rc - 1) * C + min(C, tail)
+        return rc, mask[: (nch + 31) // 32].copy(), miss, packed[:nbytes].copy()
+
+    def debug_insert(self, key: int, data) -> int:
+        a = _u8(data)
+        return int(lib().oracle_debug_insert(self._h, key, a.ctypes.data, a.size))
+
+    def stats(self) -> dict:
+        out = np.zeros(len(STAT_FIELDS), dtype=np.uint64)
+        lib().oracle_cache_stats(self._h, out.ctypes.data)
+        return {k: int(v) for k, v in zip(STAT_FIELDS, out)}
+
+    def entries(self):
+        """(keys u64[slots_used], lens u32[slots_used]) ordered by slot."""
+        used = self.stats()["slots_used"]
+        keys = np.zeros(max(1, used), dtype=np.uint64)
+        lens = np.zeros(max(1, used), dtype=np.uint32)
+        lib().oracle_cache_entries(self._h, keys.ctypes.data, lens.ctypes.data, used)
+        return keys[:used], lens[:used]
+
+    def slot_bytes(self, slot: int) -> bytes:
+        out = np.zeros(self.chunk_bytes, dtype=np.uint8)
+        ln = int(lib().oracle_slot_bytes(self._h, slot, out.ctypes.data, out.size))
+        if ln < 0:
+            raise IndexError(slot)
+        return out[:ln].tobytes()

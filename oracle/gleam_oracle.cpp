@@ -1,0 +1,331 @@
+// Gleam chunk-dedup ORACLE -- test infrastructure only.
+//
+// A plain, slow, single-threaded CPU statement of what the dedup hot path
+// computes.  Only the test suite, the package's smoke check and the CPU
+// baseline leg of the benchmark load this file's library; the product path
+// never does.  It shares no code, header or table with the CUDA library.
+//
+// What it follows:
+//  * Paper Sec. 4.1.2 ("Hash-based Weight Chunk Retrieval"): before a
+//    host-to-device payload is forwarded, a hash of the source bytes is looked
+//    up in the server's set of resident chunk identifiers; on a hit only
+//    (hash, size) metadata crosses the network, otherwise the full chunk does
+//    and it becomes reusable later.
+//  * Paper App. B.1 ("Hash Cost and Collision"): the paper hashes a prefix with
+//    MD5 and relies on never having seen a collision.  Here the identifier is
+//    XXH64 (seed 0) of each fixed C-byte chunk, and every key match is
+//    confirmed byte for byte so a collision can never alias two chunks.
+//  * XXH64 itself is written from the public xxHash specification (the
+//    "xxhash_spec" document): four accumulators over 32-byte stripes,
+//    convergence, merge rounds, length, 8/4/1-byte tails, avalanche.
+//
+// Readings taken where the paper is silent (each also listed in the design doc):
+//  R1 identifier = XXH64(seed 0) of the whole chunk, as a native u64.
+//  R2 chunks are fixed C bytes; chunk_bytes == 0 in oracle_fingerprint means
+//     one hash over the whole payload (the paper's per-payload identifier).
+//  R3 the last chunk keeps its true length; length is part of equality.
+//  R5 duplicates inside one call: chunks are decided strictly in ascending
+//     order, so a later copy of an earlier miss is a hit on that fresh insert.
+//  R6 verify_rejects counts chunks that had a key+length candidate and no
+//     byte-equal candidate.
+//  R7 running out of slots returns CAPACITY and leaves the cache unchanged.
+//  R8 miss indices ascending, packed bytes in the same order at rank*C,
+//     hit-mask bit i is bit (i % 32) of 32-bit word i / 32, trailing bits 0.
+//  R10 KEY16 mode keys the index by the low 16 bits of the fingerprint.
+#include <cstddef>
+#include <cstdint>
+#include <cstring>
+#include <unordered_map>
+#include <vector>
+
+namespace {
+
+// ---- XXH64, public xxHash specification ---------------------------------
+const uint64_t kP1 = 0x9E3779B185EBCA87ULL;
+const uint64_t kP2 = 0xC2B2AE3D27D4EB4FULL;
+const uint64_t kP3 = 0x165667B19E3779F9ULL;
+const uint64_t kP4 = 0x85EBCA77C2B2AE63ULL;
+const uint64_t kP5 = 0x27D4EB2F165667C5ULL;
+
+uint64_t rotl64(uint64_t x, int r) { return (x << r) | (x >> (64 - r)); }
+
+// Inputs are read as little-endian words regardless of the host's byte order.
+uint64_t read_le64(const uint8_t* p) {
+  uint64_t v = 0;
+  for (int k = 0; k < 8; ++k) v |= static_cast<uint64_t>(p[k]) << (8 * k);
+  return v;
+}
+
+uint32_t read_le32(const uint8_t* p) {
+  uint32_t v = 0;
+  for (int k = 0; k < 4; ++k) v |= static_cast<uint32_t>(p[k]) << (8 * k);
+  return v;
+}
+
+// One accumulator step: acc + input*P2, rotate left 31, times P1.
+uint64_t xxh_round(uint64_t acc, uint64_t input) {
+  acc += input * kP2;
+  acc = rotl64(acc, 31);
+  acc *= kP1;
+  return acc;
+}
+
+// Folding one accumulator into the converged hash.
+uint64_t xxh_merge(uint64_t h, uint64_t acc) {
+  h ^= xxh_round(0, acc);
+  h = h * kP1 + kP4;
+  return h;
+}
+
+uint64_t xxh64(const uint8_t* p, size_t len, uint64_t seed) {
+  size_t off = 0;
+  uint64_t h;
+  if (len >= 32) {
+    // Step 1: accumulator initialisation.
+    uint64_t v[4] = {seed + kP1 + kP2, seed + kP2, seed, seed - kP1};
+    // Step 2: every full 32-byte stripe; lane l takes the word at 8*l.
+    while (len - off >= 32) {
+      for (int l = 0; l < 4; ++l) v[l] = xxh_round(v[l], read_le64(p + off + 8 * l));
+      off += 32;
+    }
+    // Step 3: convergence.
+    h = rotl64(v[0], 1) + rotl64(v[1], 7) + rotl64(v[2], 12) + rotl64(v[3], 18);
+    // Step 4: merge every accumulator, in lane order.
+    for (int l = 0; l < 4; ++l) h = xxh_merge(h, v[l]);
+  } else {
+    h = seed + kP5;  // short-input start value
+  }
+  // Step 5: total length.
+  h += static_cast<uint64_t>(len);
+  // Step 6: remaining input, 8 bytes, then 4, then single bytes.
+  while (len - off >= 8) {
+    h ^= xxh_round(0, read_le64(p + off));
+    h = rotl64(h, 27) * kP1 + kP4;
+    off += 8;
+  }
+  if (len - off >= 4) {
+    h ^= static_cast<uint64_t>(read_le32(p + off)) * kP1;
+    h = rotl64(h, 23) * kP2 + kP3;
+    off += 4;
+  }
+  while (off < len) {
+    h ^= static_cast<uint64_t>(p[off]) * kP5;
+    h = rotl64(h, 11) * kP1;
+    ++off;
+  }
+  // Step 7: avalanche.
+  h ^= h >> 33;
+  h *= kP2;
+  h ^= h >> 29;
+  h *= kP3;
+  h ^= h >> 32;
+  return h;
+}
+
+// ---- the weight cache -----------------------------------------------------
+const int kOk = 0;
+const int kErrInvalidArg = -1;
+const int kErrCapacity = -4;
+const uint32_t kFlagKey16 = 1u;
+
+struct Entry {
+  uint64_t key;
+  uint32_t len;
+  uint32_t slot;
+};
+
+struct Cache {
+  size_t capacity_bytes = 0;
+  size_t chunk = 0;
+  uint64_t nslots = 0;
+  uint32_t flags = 0;
+  std::unordered_multimap<uint64_t, Entry> index;  // key -> entries
+  std::vector<std::vector<uint8_t>> slot_bytes;    // slot -> stored bytes
+  // statistics, same meaning as the CUDA library's
+  uint64_t calls = 0, chunks = 0, hits_cache = 0, hits_intra = 0, misses = 0,
+           inserts = 0, verify_rejects = 0, bytes_used = 0;
+};
+
+uint64_t key_of(const Cache& c, uint64_t fp) {
+  return (c.flags & kFlagKey16) ? (fp & 0xFFFFull) : fp;
+}
+
+bool bytes_equal(const std::vector<uint8_t>& stored, const uint8_t* p, size_t len) {
+  return stored.size() == len && (len == 0 || std::memcmp(stored.data(), p, len) == 0);
+}
+
+}  // namespace
+
+extern "C" {
+
+uint64_t oracle_xxh64(const void* p, size_t n, uint64_t seed) {
+  return xxh64(static_cast<const uint8_t*>(p), n, seed);
+}
+
+// out[i] = XXH64 of chunk i; chunk_bytes == 0 -> out[0] = XXH64 of all n bytes.
+int oracle_fingerprint(const void* buf, size_t n, size_t chunk_bytes, uint64_t* out) {
+  const uint8_t* p = static_cast<const uint8_t*>(buf);
+  if (chunk_bytes == 0) {
+    out[0] = xxh64(p, n, 0);
+    return kOk;
+  }
+  size_t nchunks = (n + chunk_bytes - 1) / chunk_bytes;
+  for (size_t i = 0; i < nchunks; ++i) {
+    size_t begin = i * chunk_bytes;
+    size_t len = (n - begin < chunk_bytes) ? (n - begin) : chunk_bytes;
+    out[i] = xxh64(p + begin, len, 0);
+  }
+  return kOk;
+}
+
+void* oracle_cache_create(size_t capacity_bytes, size_t chunk_bytes, uint32_t flags, int* err) {
+  if (chunk_bytes < 32 || chunk_bytes % 32 != 0 || chunk_bytes > (16u << 20) ||
+      (flags & ~kFlagKey16) != 0 || capacity_bytes / (chunk_bytes ? chunk_bytes : 1) == 0 ||
+      capacity_bytes / chunk_bytes > 0xFFFFFFFEull) {
+    if (err) *err = kErrInvalidArg;
+    return nullptr;
+  }
+  Cache* c = new Cache();
+  c->capacity_bytes = capacity_bytes;
+  c->chunk = chunk_bytes;
+  c->nslots = capacity_bytes / chunk_bytes;
+  c->flags = flags;
+  if (err) *err = kOk;
+  return c;
+}
+
+void oracle_cache_destroy(void* cache) { delete static_cast<Cache*>(cache); }
+
+// The sequential dedup of one payload (paper Sec. 4.1.2 with readings R1-R8).
+// Returns the number of misses, or a negative error code.  The cache is only
+// changed when the whole call succeeds.
+int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
+                     uint32_t* miss_idx, uint8_t* packed) {
+  Cache* c = static_cast<Cache*>(cache);
+  const uint8_t* p = static_cast<const uint8_t*>(buf);
+  if (c == nullptr || (n > 0 && buf == nullptr)) return kErrInvalidArg;
+  if (n == 0) return 0;
+  const size_t C = c->chunk;
+  const uint64_t nchunks = (n + C - 1) / C;
+  if (nchunks >= (1ull << 32)) return kErrInvalidArg;
+
+  // Entries inserted by this call, kept aside until the call commits.
+  std::unordered_multimap<uint64_t, Entry> fresh_index;
+  std::vector<std::vector<uint8_t>> fresh_bytes;
+  const uint64_t slots0 = c->slot_bytes.size();
+  uint64_t rank = 0, hits_cache = 0, hits_intra = 0, rejects = 0;
+
+  for (uint64_t w = 0; w < (nchunks + 31) / 32; ++w) hit_mask[w] = 0;
+
+  for (uint64_t i = 0; i < nchunks; ++i) {
+    const uint8_t* chunk = p + i * C;
+    const size_t len = (n - i * C < C) ? (n - i * C) : C;
+    const uint64_t key = key_of(*c, xxh64(chunk, len, 0));
+
+    bool candidate = false, hit = false, hit_is_fresh = false;
+    auto look = [&](const std::unordered_multimap<uint64_t, Entry>& idx,
+                    const std::vector<std::vector<uint8_t>>& store, uint64_t slot_base,
+                    bool fresh) {
+      auto range = idx.equal_range(key);
+      for (auto it = range.first; it != range.second; ++it) {
+        if (it->second.len != len) continue;
+        candidate = true;
+        if (bytes_equal(store[it->second.slot - slot_base], chunk, len)) {
+          hit = true;
+          hit_is_fresh = fresh;
+        }
+      }
+    };
+    look(c->index, c->slot_bytes, 0, false);
+    look(fresh_index, fresh_bytes, slots0, true);
+
+    if (hit) {
+      hit_mask[i / 32] |= 1u << (i % 32);
+      if (hit_is_fresh) ++hits_intra; else ++hits_cache;
+      continue;
+    }
+    if (candidate) ++rejects;
+    if (slots0 + rank >= c->nslots) return kErrCapacity;  // nothing committed
+    miss_idx[rank] = static_cast<uint32_t>(i);
+    std::memcpy(packed + rank * C, chunk, len);
+    Entry e{key, static_cast<uint32_t>(len), static_cast<uint32_t>(slots0 + rank)};
+    fresh_index.emplace(key, e);
+    fresh_bytes.emplace_back(chunk, chunk + len);
+    ++rank;
+  }
+
+  // Commit.
+  for (auto& kv : fresh_index) c->index.emplace(kv.first, kv.second);
+  for (auto& b : fresh_bytes) {
+    c->bytes_used += b.size();
+    c->slot_bytes.emplace_back(std::move(b));
+  }
+  c->calls += 1;
+  c->chunks += nchunks;
+  c->hits_cache += hits_cache;
+  c->hits_intra += hits_intra;
+  c->misses += rank;
+  c->inserts += rank;
+  c->verify_rejects += rejects;
+  return static_cast<int64_t>(rank);
+}
+
+// Test hook: store `bytes` under an arbitrary key (crafted collisions).
+int oracle_debug_insert(void* cache, uint64_t key, const void* bytes, size_t len) {
+  Cache* c = static_cast<Cache*>(cache);
+  if (c == nullptr || len == 0 || len > c->chunk || bytes == nullptr) return kErrInvalidArg;
+  if (c->slot_bytes.size() >= c->nslots) return kErrCapacity;
+  const uint8_t* b = static_cast<const uint8_t*>(bytes);
+  Entry e{key_of(*c, key), static_cast<uint32_t>(len), static_cast<uint32_t>(c->slot_bytes.size())};
+  c->index.emplace(e.key, e);
+  c->slot_bytes.emplace_back(b, b + len);
+  c->bytes_used += len;
+  c->inserts += 1;
+  return kOk;
+}
+
+// Stats in the CUDA library's field order:
+// calls, chunks, hits_cache, hits_intra, misses, inserts, verify_rejects,
+// slots_used, bytes_used, capacity_bytes, nslots, chunk_bytes.
+void oracle_cache_stats(const void* cache, uint64_t* out) {
+  const Cache* c = static_cast<const Cache*>(cache);
+  out[0] = c->calls;
+  out[1] = c->chunks;
+  out[2] = c->hits_cache;
+  out[3] = c->hits_intra;
+  out[4] = c->misses;
+  out[5] = c->inserts;
+  out[6] = c->verify_rejects;
+  out[7] = c->slot_bytes.size();
+  out[8] = c->bytes_used;
+  out[9] = c->capacity_bytes;
+  out[10] = c->nslots;
+  out[11] = c->chunk;
+}
+
+// Index contents, ordered by slot: keys[s], lens[s] for s < slots_used.
+uint64_t oracle_cache_entries(const void* cache, uint64_t* keys, uint32_t* lens, uint64_t max) {
+  const Cache* c = static_cast<const Cache*>(cache);
+  uint64_t count = 0;
+  for (const auto& kv : c->index) {
+    const Entry& e = kv.second;
+    if (e.slot < max) {
+      keys[e.slot] = e.key;
+      lens[e.slot] = e.len;
+    }
+    ++count;
+  }
+  return count;
+}
+
+// Stored bytes of one slot; returns its length, or -1 for a bad slot.
+int64_t oracle_slot_bytes(const void* cache, uint64_t slot, uint8_t* out, uint64_t max) {
+  const Cache* c = static_cast<const Cache*>(cache);
+  if (slot >= c->slot_bytes.size()) return -1;
+  const auto& b = c->slot_bytes[slot];
+  uint64_t m = b.size() < max ? b.size() : max;
+  if (m) std::memcpy(out, b.data(), m);
+  return static_cast<int64_t>(b.size());
+}
+
+}  // extern "C"
