@@ -188,6 +188,16 @@ int gleam_cache_snapshot(gleam_cache_t* cache, gleam_snapshot_t** out);
 int gleam_cache_restore(gleam_cache_t* cache, const gleam_snapshot_t* snap);
 void gleam_snapshot_destroy(gleam_snapshot_t* snap);
 
+/* Kernel timing for benchmarks.  While enabled, every dedup call records CUDA
+ * events on its own stream around its two kernels: kernel 0 fingerprints,
+ * probes and verifies; kernel 1 resolves duplicates, compacts, packs and
+ * inserts.  gleam_cache_profile_read waits for the recorded calls, writes the
+ * summed device time (ms) and launch count of kernel k to h_ms[k] and
+ * h_launches[k] for k < nkernels (host arrays), and starts a new tally. */
+int gleam_cache_profile(gleam_cache_t* cache, int enable);
+int gleam_cache_profile_read(gleam_cache_t* cache, double* h_ms, uint64_t* h_launches,
+                             int nkernels);
+
 /* Short English name of a gleam_status value. */
 const char* gleam_status_string(int status);
 

@@ -1,0 +1,192 @@
+// Internal types and device helpers of libgleam (not part of the C ABI).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "gleam.h"
+
+namespace gleam {
+
+// ---------------------------------------------------------------------------
+// Device data layout
+// ---------------------------------------------------------------------------
+
+constexpr uint32_t kEmptySlot = 0xFFFFFFFFu;
+
+// One entry of the cache index: open addressing, linear probing, load <= 1/2.
+// An entry is free iff slot == kEmptySlot; key/len are valid once the insert
+// kernel that claimed it has finished.
+struct __align__(16) IndexEntry {
+  unsigned long long key;  // XXH64 of the stored chunk (low 16 bits in KEY16 mode)
+  uint32_t slot;           // arena slot holding the bytes
+  uint32_t len;            // true length of the stored chunk
+};
+
+// One entry of the per-call group table used to find the first occurrence of
+// each distinct chunk inside a call.  owner = 1 + index of the chunk that
+// claimed the entry (0 = free); minv = ~(smallest unresolved chunk index of
+// the group) so that a zero-filled table means "no minimum yet".
+struct __align__(8) CallEntry {
+  uint32_t owner;
+  uint32_t minv;
+};
+
+// Per-chunk outcome of the probe/verify kernel.
+enum : uint8_t { kMissNoCand = 0, kMissCand = 1, kHit0 = 2 };
+
+// Per-chunk resolution word of the dedup kernel.
+constexpr uint32_t kResUnresolved = 0;
+constexpr uint32_t kResHit0 = 0x20000000u;     // byte-equal to a cached chunk
+constexpr uint32_t kResDup = 0x40000000u;      // byte-equal to an earlier miss
+constexpr uint32_t kResLeader = 0x80000000u;   // | round in which it was resolved
+constexpr uint32_t kResRoundMask = 0x1FFFFFFFu;
+
+// Device counters of one cache, in gleam_stats_t order (first nine fields).
+enum StatIdx {
+  ST_CALLS = 0, ST_CHUNKS, ST_HITS_CACHE, ST_HITS_INTRA, ST_MISSES, ST_INSERTS,
+  ST_REJECTS, ST_SLOTS_USED, ST_BYTES_USED, ST_COUNT
+};
+
+// Per-call control block, zeroed before every call.
+struct DevCtl {
+  unsigned int bar_count;
+  unsigned int bar_gen;
+  int err;
+  unsigned int done;
+  unsigned int unres[3];
+  unsigned int pad0;
+  unsigned long long acc_hits_cache;
+  unsigned long long acc_hits_intra;
+  unsigned long long acc_rejects;
+  unsigned long long acc_misses;
+  unsigned long long acc_miss_bytes;
+};
+
+// Position of a key in a power-of-two table: the 64-bit finaliser of
+// MurmurHash3 (Appleby), so that 16-bit test keys spread as well as full ones.
+__host__ __device__ __forceinline__ unsigned long long mix64(unsigned long long k) {
+  k ^= k >> 33;
+  k *= 0xff51afd7ed558ccdULL;
+  k ^= k >> 33;
+  k *= 0xc4ceb9fe1a85ec53ULL;
+  k ^= k >> 33;
+  return k;
+}
+
+// ---------------------------------------------------------------------------
+// Kernel argument blocks and launchers (defined in the kernel TUs)
+// ---------------------------------------------------------------------------
+
+struct HashArgs {
+  const uint8_t* buf;
+  uint64_t n;
+  uint64_t C;                  // chunk length (bytes)
+  uint32_t N;                  // number of chunks
+  unsigned long long* fp_out;  // optional: XXH64 per chunk
+  // probe + verify (index == nullptr: fingerprint only)
+  const IndexEntry* index;
+  uint64_t index_mask;
+  const uint8_t* arena;
+  const unsigned long long* dstats;
+  uint32_t key16;
+  uint8_t* status;
+  unsigned long long* key_out;
+  DevCtl* ctl;
+};
+
+struct DedupArgs {
+  const uint8_t* buf;
+  uint64_t n;
+  uint64_t C;
+  uint32_t N;
+  uint32_t* mask;
+  uint32_t* miss_idx;
+  uint8_t* packed;
+  uint8_t* arena;
+  IndexEntry* index;
+  uint64_t index_mask;
+  uint64_t nslots;
+  uint32_t* slot_len;
+  unsigned long long* dstats;
+  const uint8_t* status;
+  const unsigned long long* key;
+  uint32_t* res;
+  uint32_t* ent;
+  CallEntry* tbl;
+  uint64_t tbl_mask;
+  uint32_t* bcount;
+  DevCtl* ctl;
+  gleam_result_t* result;
+  unsigned long long wait_ns;
+  int skip_block;
+};
+
+cudaError_t launch_hash(const HashArgs& a, cudaStream_t s);
+cudaError_t launch_dedup(const DedupArgs& a, int grid, cudaStream_t s);
+cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
+                                unsigned long long* dstats, unsigned long long key,
+                                uint32_t slot, uint32_t len, DevCtl* ctl, cudaStream_t s);
+int dedup_threads();
+int dedup_blocks_per_sm();
+
+// ---------------------------------------------------------------------------
+// Device helpers
+// ---------------------------------------------------------------------------
+
+#ifdef __CUDACC__
+
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ unsigned int ld_acquire_u32(const unsigned int* p) {
+  unsigned int v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ int ld_volatile_s32(const int* p) {
+  return *reinterpret_cast<const volatile int*>(p);
+}
+
+// Grid-wide barrier for a cooperative launch.  Every wait is bounded by
+// `wait_ns`: a block that gives up records GLEAM_ERR_TIMEOUT and every block
+// then leaves through its epilogue.  `skip` makes the calling block leave
+// without arriving (test hook for the bounded wait).  Returns true if the
+// whole grid arrived and no error is recorded.
+__device__ __forceinline__ bool grid_barrier(DevCtl* ctl, unsigned int nblocks,
+                                             unsigned long long wait_ns, bool skip) {
+  __shared__ int s_ok;  // the block's verdict, so that every thread agrees
+  __syncthreads();
+  if (threadIdx.x == 0 && !skip) {
+    const unsigned int gen = ld_acquire_u32(&ctl->bar_gen);
+    __threadfence();
+    const unsigned int arrived = atomicAdd(&ctl->bar_count, 1u);
+    if (arrived == nblocks - 1) {
+      atomicExch(&ctl->bar_count, 0u);
+      __threadfence();
+      atomicAdd(&ctl->bar_gen, 1u);
+    } else {
+      const unsigned long long t0 = globaltimer_ns();
+      while (ld_acquire_u32(&ctl->bar_gen) == gen) {
+        if (ld_volatile_s32(&ctl->err) != 0) break;
+        if (globaltimer_ns() - t0 > wait_ns) {
+          atomicCAS(&ctl->err, 0, (int)GLEAM_ERR_TIMEOUT);
+          break;
+        }
+        __nanosleep(100);
+      }
+    }
+    __threadfence();
+  }
+  if (threadIdx.x == 0) s_ok = (!skip && ld_volatile_s32(&ctl->err) == 0) ? 1 : 0;
+  __syncthreads();
+  return s_ok != 0;
+}
+
+#endif  // __CUDACC__
+
+}  // namespace gleam

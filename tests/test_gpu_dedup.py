@@ -1,0 +1,218 @@
+"""gleam_dedup_copy vs the oracle, bit for bit, on seeded workloads shaped like
+the five benchmark configurations (scaled so the oracle takes seconds) and on
+the edge cases of the method."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_23115_gb300 import binding as B
+from paper_2607_23115_gb300 import workloads as W
+from paper_2607_23115_gb300.cache import Cache, DedupOutputs, result_dict
+from tests._parity import DEV, compare_cache, dedup_both
+
+pytestmark = pytest.mark.gpu
+KiB, MiB = 1024, 1 << 20
+
+
+def _pair(capacity, C, flags=0):
+    return Cache(capacity, C, flags), oracle.OracleCache(capacity, C, flags)
+
+
+@pytest.mark.parametrize("tail", [0, 1000])
+def test_fp16_payload_half_prefilled(tail):
+    C = 4 * KiB
+    host = W.fp16_payload(8 * MiB, seed=0)
+    N = host.numel() // C
+    sel = W.select_chunks(N, 0.5)
+    gc, oc = _pair(16 * MiB, C)
+    with gc:
+        assert dedup_both(gc, oc, W.gather_chunks(host, C, sel)) == N // 2
+        payload = torch.cat([host, host[:tail]]) if tail else host
+        rc = dedup_both(gc, oc, payload)
+        assert rc == N - N // 2 + (1 if tail else 0)
+        compare_cache(gc, oc)
+
+
+def test_gpt2_shaped_upload_two_passes():
+    C = 4 * KiB
+    up = W.weight_upload(W.scaled_shapes(W.gpt2_small_shapes(), 4), torch.float32)
+    gc, oc = _pair(256 * MiB, C)
+    with gc:
+        for _ in range(2):
+            for k in range(len(up.sizes)):
+                dedup_both(gc, oc, up.payload(k))
+        compare_cache(gc, oc)
+        st = gc.stats()
+        assert st["misses"] == len(up.chunks(C)) == st["hits_cache"]
+
+
+def test_llama_shaped_upload_bit_flips():
+    C = 64 * KiB
+    up = W.weight_upload(W.scaled_shapes(W.llama3_8b_shapes(), 8)[:60], torch.bfloat16)
+    gc, oc = _pair(512 * MiB, C)
+    with gc:
+        for k in range(len(up.sizes)):
+            dedup_both(gc, oc, up.payload(k))
+        chunks = up.chunks(C)
+        ids = W.select_chunks(len(chunks), 0.10)
+        W.flip_one_bit_per_chunk(up.buf, chunks, ids)
+        before = gc.stats()["misses"]
+        for k in range(len(up.sizes)):
+            dedup_both(gc, oc, up.payload(k))
+        assert gc.stats()["misses"] - before == len(ids)
+        compare_cache(gc, oc)
+
+
+def test_small_call_stream():
+    C = 4 * KiB
+    up = W.small_call_upload(300, lo=4 * KiB, hi=256 * KiB)
+    gc, oc = _pair(256 * MiB, C)
+    with gc:
+        dedup_both(gc, oc, W.random_bytes(2 * MiB, seed=W.SEED_PREFILL))
+        for k in range(len(up.sizes)):
+            dedup_both(gc, oc, up.payload(k))
+        compare_cache(gc, oc)
+
+
+@pytest.mark.parametrize("C", [1 * KiB, 4 * KiB, 16 * KiB, 64 * KiB])
+@pytest.mark.parametrize("key16", [False, True])
+def test_adversarial_payload(C, key16):
+    adv = W.adversarial_payload(16 * MiB, C)
+    flags = B.GLEAM_KEY16 if key16 else 0
+    gc, oc = _pair(64 * MiB, C, flags)
+    with gc:
+        if key16:
+            pick, rows = W.crafted_collisions(adv, C, count=64)
+            host_rows = adv.buf.view(-1, C)[pick].numpy()
+            for i, r in enumerate(rows):
+                key = oracle.xxh64(host_rows[i])
+                assert oc.debug_insert(key, r.numpy()) == 0
+                gc.debug_insert(key, r.to(DEV))
+        rc = dedup_both(gc, oc, adv.buf)
+        rnd = int((adv.kind == 2).sum())
+        npat = len(set(adv.pattern_id[adv.kind == 1].tolist()))
+        assert rc == 1 + npat + rnd
+        if key16:
+            assert gc.stats()["verify_rejects"] >= 64
+        compare_cache(gc, oc)
+
+
+@pytest.mark.parametrize("key16", [False, True])
+@pytest.mark.parametrize("C", [32, 64, 1024])
+def test_random_alphabet_sequences(C, key16):
+    rng = np.random.default_rng(C + key16)
+    flags = B.GLEAM_KEY16 if key16 else 0
+    gc, oc = _pair(20000 * C, C, flags)
+    alphabet = [W.random_bytes(C, seed=1000 + k) for k in range(200)] + [torch.zeros(C, dtype=torch.uint8)]
+    with gc:
+        for call in range(12):
+            nch = int(rng.integers(1, 3000))
+            parts = [alphabet[int(rng.integers(len(alphabet)))] for _ in range(nch)]
+            if rng.random() < 0.5:
+                parts.append(W.random_bytes(int(rng.integers(1, C)), seed=call))
+            payload = torch.cat(parts)
+            dedup_both(gc, oc, payload, offset=int(rng.choice([0, 0, 16, 4, 1])),
+                       packed_offset=int(rng.choice([0, 0, 3])))
+        compare_cache(gc, oc)
+
+
+def test_many_blocks_and_intra_call_duplicates():
+    C = 1 * KiB
+    base = W.random_bytes(6000 * C, seed=5).view(-1, C)
+    idx = torch.from_numpy(np.random.default_rng(3).integers(0, 6000, 40000))
+    payload = base[idx].reshape(-1).contiguous()
+    gc, oc = _pair(64 * MiB, C)
+    with gc:
+        dedup_both(gc, oc, payload)
+        compare_cache(gc, oc)
+        st = gc.stats()
+        assert st["hits_intra"] + st["misses"] == 40000
+
+
+def test_edge_sizes():
+    C = 4 * KiB
+    gc, oc = _pair(64 * C, C)
+    with gc:
+        assert dedup_both(gc, oc, torch.zeros(0, dtype=torch.uint8)) == 0
+        assert gc.stats()["calls"] == 0
+        dedup_both(gc, oc, W.random_bytes(1, seed=1))            # one 1-byte chunk
+        dedup_both(gc, oc, W.random_bytes(C - 1, seed=2))        # one short chunk
+        dedup_both(gc, oc, W.random_bytes(C, seed=3))            # exactly one chunk
+        dedup_both(gc, oc, W.random_bytes(C, seed=3))            # ... again: a hit
+        dedup_both(gc, oc, W.random_bytes(C + 1, seed=3))        # chunk + 1-byte tail
+        compare_cache(gc, oc)
+
+
+def test_largest_chunk_size():
+    C = 16 * MiB
+    gc, oc = _pair(4 * C, C)
+    with gc:
+        host = W.random_bytes(2 * C + 12345, seed=9)
+        dedup_both(gc, oc, host)
+        dedup_both(gc, oc, host[: C])
+        compare_cache(gc, oc)
+
+
+def test_capacity_error_leaves_cache_unchanged_then_recovers():
+    C = 1 * KiB
+    gc, oc = _pair(100 * C, C)
+    with gc:
+        dedup_both(gc, oc, W.random_bytes(60 * C, seed=1))
+        before = gc.stats()
+        assert dedup_both(gc, oc, W.random_bytes(50 * C, seed=2)) == B.GLEAM_ERR_CAPACITY
+        assert gc.stats() == before
+        assert dedup_both(gc, oc, W.random_bytes(40 * C, seed=2)) == 40
+        compare_cache(gc, oc)
+
+
+def test_async_calls_match_sync_and_report_results():
+    C = 4 * KiB
+    up = W.weight_upload(W.scaled_shapes(W.gpt2_small_shapes(), 8), torch.float32)
+    ga = Cache(64 * MiB, C)
+    oc = oracle.OracleCache(64 * MiB, C)
+    s = torch.cuda.Stream()
+    outs, results = [], []
+    dbuf = up.buf.to(DEV)
+    with ga:
+        for rep in range(2):
+            for k in range(len(up.sizes)):
+                n = up.sizes[k]
+                out = DedupOutputs.alloc(n, C, DEV)
+                res = torch.zeros(B.RESULT_WORDS, dtype=torch.int64, device=DEV)
+                with torch.cuda.stream(s):
+                    ga.dedup_async(dbuf[up.offsets[k]: up.offsets[k] + n], out, res, stream=s)
+                outs.append(out)
+                results.append(res)
+        s.synchronize()
+        i = 0
+        for rep in range(2):
+            for k in range(len(up.sizes)):
+                rc, mask_o, miss_o, packed_o = oc.dedup(up.payload(k).numpy())
+                r = result_dict(results[i])
+                assert r["status"] == 0 and r["n_miss"] == rc
+                assert r["miss_bytes"] == len(packed_o)
+                o = outs[i]
+                assert np.array_equal(o.hit_mask.cpu().numpy().view(np.uint32)[: len(mask_o)], mask_o)
+                assert np.array_equal(o.miss_idx.cpu().numpy().view(np.uint32)[:rc], miss_o)
+                assert np.array_equal(o.miss_bytes.cpu().numpy()[: len(packed_o)], packed_o)
+                i += 1
+        compare_cache(ga, oc)
+
+
+def test_snapshot_restore_repeats_identically():
+    C = 4 * KiB
+    host = W.fp16_payload(4 * MiB, seed=0)
+    with Cache(16 * MiB, C) as gc:
+        gc.dedup(host[: 2 * MiB].to(DEV))
+        snap = gc.snapshot()
+        st0 = gc.stats()
+        d = host.to(DEV)
+        n1, o1 = gc.dedup(d)
+        st1 = gc.stats()
+        gc.restore(snap)
+        assert gc.stats() == st0
+        n2, o2 = gc.dedup(d)
+        assert n1 == n2 and gc.stats() == st1
+        assert torch.equal(o1.hit_mask, o2.hit_mask) and torch.equal(o1.miss_idx[:n1], o2.miss_idx[:n2])
+        snap.close()
