@@ -1,0 +1,565 @@
+#!/usr/bin/env python
+"""Benchmark of the chunk-dedup hot path (paper Sec. 4.1.2) on GB300.
+
+One step = one pass of the whole path (fingerprint, probe, verify, in-call
+dedup, compaction, packing, insertion) over one upload: every tensor of the
+workload is one gleam_dedup_copy_async call, as one cudaMemcpy per tensor
+would be.  The cache is restored from a device snapshot at the start of each
+step (16 MiB index copy, inside the timed region), so every step does the
+same work.  Inputs (16 GB for the default workload) are resident in HBM and
+far larger than L2, so no L2 flush is needed between steps.
+
+Default workload: a Llama-3-8B-shaped bf16 weight upload (291 tensors,
+~16.06 GB, values ~N(0, 0.02)), chunk C = 64 KiB, a 24 GiB cache pre-filled
+with the base weights, and 10% of the chunks carrying one flipped bit (a
+fine-tuned variant), so ~90% of chunks hit and ~10% miss and are inserted.
+
+Printed line: payload GB/s (value), the pipeline's minimal-traffic roofline
+fraction (payload read + cached bytes read for hits + miss bytes written =
+2 x payload), the dominant kernel's roofline, the oracle's CPU rate on a
+bounded sample, the end-to-end rate with host buffers, clocks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "dedup payload GB/s on 1 GB300 and fraction of HBM roofline; vs CPU oracle"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+KiB, MiB, GiB = 1 << 10, 1 << 20, 1 << 30
+
+
+def parse_args():
+    p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=100)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["gleam", "reference"], default="gleam")
+    p.add_argument("--workload", choices=["llama3-8b", "llama3-8b-layer", "gpt2-small"], default="llama3-8b")
+    p.add_argument("--cpu-sample-bytes", type=int, default=3 * GiB,
+                   help="payload bytes of the oracle's bounded CPU sample")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--e2e-steps", type=int, default=5)
+    p.add_argument("--profile-launches", action="store_true",
+                   help="few steps, no baselines: for an ncu launch list")
+    return p.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# workloads
+# ---------------------------------------------------------------------------
+
+def workload_spec(name):
+    import torch
+    from paper_2607_23115_gb300 import workloads as W
+    if name == "llama3-8b":
+        return dict(name="llama3-8b-bf16-per-tensor", shapes=W.llama3_8b_shapes(),
+                    dtype=torch.bfloat16, C=64 * KiB, capacity=24 * GiB, flip_frac=0.10,
+                    desc="Llama-3-8B-shaped bf16 upload, 291 tensors, ~N(0,0.02); cache "
+                         "prefilled with the base weights; 10% of 64 KiB chunks bit-flipped")
+    if name == "llama3-8b-layer":
+        return dict(name="llama3-8b-bf16-one-layer", shapes=W.llama3_8b_shapes()[1:10],
+                    dtype=torch.bfloat16, C=64 * KiB, capacity=512 * MiB, flip_frac=0.10,
+                    desc="one Llama-3-8B layer (9 bf16 tensors, 436 MB): the small case of "
+                         "the llama3-8b workload for ncu captures")
+    if name == "gpt2-small":
+        return dict(name="gpt2-small-fp32-per-tensor-second-pass", shapes=W.gpt2_small_shapes(),
+                    dtype=torch.float32, C=4 * KiB, capacity=1 * GiB, flip_frac=0.0,
+                    desc="GPT-2-small-shaped fp32 upload, 148 tensors, ~N(0,0.02); second "
+                         "identical pass (all hits) after a first pass filled the cache")
+    raise ValueError(name)
+
+
+def make_upload(spec, device):
+    from paper_2607_23115_gb300 import workloads as W
+    return W.weight_upload(spec["shapes"], spec["dtype"], device=device)
+
+
+def perturb(spec, up):
+    from paper_2607_23115_gb300 import workloads as W
+    if spec["flip_frac"] <= 0:
+        return 0
+    chunks = up.chunks(spec["C"])
+    ids = W.select_chunks(len(chunks), spec["flip_frac"])
+    W.flip_one_bit_per_chunk(up.buf, chunks, ids)
+    return len(ids)
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "50", "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.6)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        sm = []
+        smax = None
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                smax = float(r[2])
+            except ValueError:
+                continue
+            for k, name in enumerate(names):
+                if r[5 + k].lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# the oracle on the host cores (bounded sample)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(spec, up_base_host, up_pert_host, sample_bytes, offset_tensor=0):
+    """Oracle dedup of a bounded sample of tensors: prefill with the base
+    tensors (untimed), then time the pass over the perturbed tensors."""
+    import oracle
+    ks, tot, k = [], 0, offset_tensor
+    n_t = len(up_base_host)
+    while tot < sample_bytes and len(ks) < n_t:
+        ks.append(k % n_t)
+        tot += up_base_host[k % n_t].size
+        k += 1
+    oc = oracle.OracleCache(spec["capacity"], spec["C"])
+    for kk in ks:
+        oc.dedup(up_base_host[kk])
+    src = up_pert_host if up_pert_host is not None else up_base_host
+    t0 = time.perf_counter()
+    for kk in ks:
+        oc.dedup(src[kk])
+    dt = time.perf_counter() - t0
+    oc.close()
+    return tot, dt, len(ks)
+
+
+def host_tensors(up, limit_bytes):
+    """numpy copies of the first tensors of an upload, up to limit_bytes."""
+    out, tot = [], 0
+    for k in range(len(up.sizes)):
+        if tot >= limit_bytes:
+            break
+        out.append(up.payload(k).cpu().numpy().copy())
+        tot += up.sizes[k]
+    return out
+
+
+# ---------------------------------------------------------------------------
+# roofline helpers
+# ---------------------------------------------------------------------------
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            j = json.load(f)
+        return float(j["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_digest():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2607_23115_gb300", "csrc")
+    for f in ("hash_probe.cu", "xxh64_device.cuh", "gleam_internal.cuh"):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(workload_name):
+    """ncu DRAM bytes per launch of the dominant kernel from the committed
+    profile summary, or None if absent or taken on a different kernel source."""
+    path = os.path.join(ROOT, "profiles", "k_hash_probe.%s.md" % workload_name)
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)\s+source_digest:\s*([0-9a-f]+)", text)
+    if not m or m.group(2) != kernel_source_digest():
+        return None
+    return float(m.group(1))
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+
+def run_gleam(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2607_23115_gb300 import binding as B
+    from paper_2607_23115_gb300.cache import Cache, DedupOutputs
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    spec = workload_spec(args.workload)
+    C = spec["C"]
+
+    up = make_upload(spec, dev)
+    nt = len(up.sizes)
+    total = up.total_bytes
+    do_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_launches
+    base_host = host_tensors(up, args.cpu_sample_bytes) if do_cpu else None
+
+    cache = Cache(spec["capacity"], C)
+    cache.reserve(max((s + C - 1) // C for s in up.sizes))
+    outs = [DedupOutputs.alloc(s, C, dev) for s in up.sizes]
+    results = torch.zeros(nt, B.RESULT_WORDS, dtype=torch.int64, device=dev)
+
+    bufs = [up.payload(k) for k in range(nt)]
+    items = cache.batch_items(bufs, outs, [results[k] for k in range(nt)])
+    total_res = torch.zeros(B.RESULT_WORDS, dtype=torch.int64, device=dev)
+
+    def one_pass():
+        cache.dedup_batch(None, items=items, total=total_res, stream=None)
+
+    def one_pass_calls():
+        for k in range(nt):
+            cache.dedup_async(bufs[k], outs[k], results[k], stream=None)
+
+    # prefill with the base upload (untimed), then perturb
+    one_pass()
+    n_flipped = perturb(spec, up)
+    torch.cuda.synchronize()
+    snap = cache.snapshot()
+    pert_host = None
+    if do_cpu and spec["flip_frac"] > 0:
+        pert_host = [up.payload(k).cpu().numpy().copy() for k in range(len(base_host))]
+
+    def step():
+        cache.restore(snap)
+        one_pass()
+
+    def step_calls():
+        cache.restore(snap)
+        one_pass_calls()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    r = results.cpu().numpy()
+    assert (r[:, 0] == 0).all(), "a dedup call failed: %s" % r[r[:, 0] != 0][:3]
+    miss_bytes = int(r[:, 5].sum())
+    n_miss = int(r[:, 1].sum())
+    hit_intra = int(r[:, 3].sum())
+    if spec["flip_frac"] > 0:
+        assert n_miss == n_flipped, (n_miss, n_flipped)
+    # algorithmic bytes: the fused fingerprint/probe/verify kernel reads the
+    # payload once and the cached copy of every cache hit
+    hit_cache_bytes = total - miss_bytes - hit_intra * C
+    kernel0_bytes = total + hit_cache_bytes
+    pipeline_bytes = 2 * total  # payload read + hit bytes read + miss bytes written
+
+    clocks = ClockSampler(local_rank)
+    if not args.profile_launches:
+        clocks.start()
+    B.gleam_cache_profile(cache.handle, True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_start.record()
+    for _ in range(args.steps):
+        step()
+    t_end.record()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    ms = t_start.elapsed_time(t_end)
+    clk = clocks.stop() if not args.profile_launches else None
+    rc, kms, klaunch = B.gleam_cache_profile_read(cache.handle, 2)
+    B.gleam_cache_profile(cache.handle, False)
+
+    # the same pass as one call per tensor (secondary figure)
+    calls_ms = None
+    if not args.profile_launches:
+        calls_steps = max(1, min(args.steps, 5))
+        step_calls()
+        torch.cuda.synchronize()
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        c0.record()
+        for _ in range(calls_steps):
+            step_calls()
+        c1.record()
+        torch.cuda.synchronize()
+        calls_ms = c0.elapsed_time(c1) / calls_steps
+        rcall = results.cpu().numpy()
+        assert (rcall[:, 0] == 0).all() and int(rcall[:, 1].sum()) == n_miss
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_per_step = ms / args.steps
+    value = world * total / (ms_per_step * 1e-3) / 1e9
+
+    hbm, hbm_src = measured_peaks()
+    k0_ms = kms[0] / max(1, klaunch[0])
+    k0_bytes = kernel0_bytes  # one launch covers the whole upload
+    k0_gbs = k0_bytes / (k0_ms * 1e-3) / 1e9
+    traffic = committed_traffic(spec["name"])
+    roofline = {"bound": "hbm", "kernel": "k_hash_probe (fingerprint + probe + verify)",
+                "achieved": round(k0_gbs, 1), "peak": hbm, "peak_source": hbm_src,
+                "unit": "GB/s", "frac": round(k0_gbs / hbm, 4),
+                "traffic": traffic, "algorithmic_bytes_per_launch": round(k0_bytes),
+                "avg_launch_ms": round(k0_ms, 5),
+                "kernel_share_of_step": round((kms[0]) / ms if ms else 0, 4),
+                "k_dedup_avg_launch_ms": round(kms[1] / max(1, klaunch[1]), 5)}
+    pipe_gbs = pipeline_bytes / (ms_per_step * 1e-3) / 1e9
+    pipeline = {"min_bytes_per_step": pipeline_bytes,
+                "achieved_gbs": round(pipe_gbs, 1),
+                "frac_of_measured_hbm": round(pipe_gbs / hbm, 4),
+                "frac_of_nominal_8tbs": round(pipe_gbs / NOMINAL_HBM_GBS, 4),
+                "with_arena_write_bytes": pipeline_bytes + miss_bytes,
+                "with_arena_write_frac_of_measured": round(
+                    (pipeline_bytes + miss_bytes) / (ms_per_step * 1e-3) / 1e9 / hbm, 4)}
+
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+        "data": "synthetic",
+        "config": {"workload": spec["name"], "description": spec["desc"],
+                   "payload_bytes_per_step": total, "payloads_per_step": nt, "calls_per_step": 1,
+                   "api": "gleam_dedup_copy_batch (one call = %d per-tensor payloads)" % nt, "chunk_bytes": C,
+                   "chunks_per_step": sum((s + C - 1) // C for s in up.sizes),
+                   "misses_per_step": n_miss, "cache_capacity_bytes": spec["capacity"],
+                   "l2": "inputs (%.1f GB per step) far larger than the 129 MB L2; no flush"
+                         % (total / 1e9),
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "pipeline_roofline": pipeline,
+        "roofline": roofline,
+        "per_call_async": None if calls_ms is None else {
+            "ms_per_step": round(calls_ms, 3),
+            "value": round(total / (calls_ms * 1e-3) / 1e9, 2),
+            "how": "same step as %d gleam_dedup_copy_async calls (one per tensor) instead "
+                   "of one gleam_dedup_copy_batch call" % nt},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clk,
+    }
+
+    if do_cpu:
+        nbytes, dt, ntens = oracle_sample(spec, base_host, pert_host, args.cpu_sample_bytes)
+        line["cpu_baseline"] = {
+            "value": round(nbytes / dt / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": "first %d tensors (%.2f GB) of the same upload: oracle prefilled with "
+                      "their base bytes (untimed), then timed over their perturbed bytes"
+                      % (ntens, nbytes / 1e9), "host_cpus": os.cpu_count()}
+
+    if not args.no_e2e and not args.profile_launches:
+        line["e2e"] = run_e2e(args, spec, up, cache, snap, outs, results, miss_bytes)
+
+    cache.close()
+    return line
+
+
+def run_e2e(args, spec, up, cache, snap, outs, results, miss_bytes):
+    """The same metric through the C ABI with HOST buffers: per step, every
+    tensor is copied host->device from pinned memory and deduped, and every
+    call's result, hit mask, miss indices and packed miss bytes are read back.
+    Tensors go in groups of >= 1 GiB, one gleam_dedup_copy_batch call per
+    group, so that the copy of group g+1 overlaps the dedup of group g."""
+    import torch
+    nt = len(up.sizes)
+    host = torch.empty(up.buf.numel(), dtype=torch.uint8, pin_memory=True)
+    host.copy_(up.buf)
+    groups, cur, acc = [], [], 0
+    for k in range(nt):
+        cur.append(k)
+        acc += up.sizes[k]
+        if acc >= GiB:
+            groups.append(cur)
+            cur, acc = [], 0
+    if cur:
+        groups.append(cur)
+    items = [cache.batch_items([up.payload(k) for k in g], [outs[k] for k in g],
+                               [results[k] for k in g]) for g in groups]
+    s_copy, s_comp, s_back = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    ev_in = [torch.cuda.Event() for _ in groups]
+    ev_out = [torch.cuda.Event() for _ in groups]
+    nmask = [o.hit_mask.numel() for o in outs]
+    res_host = torch.empty_like(results, device="cpu").pin_memory()
+    mask_host = [torch.empty(m, dtype=torch.int32, pin_memory=True) for m in nmask]
+    idx_host = [torch.empty(o.miss_idx.numel(), dtype=torch.int32, pin_memory=True) for o in outs]
+    packed_host = torch.empty(max(1, miss_bytes), dtype=torch.uint8, pin_memory=True)
+
+    def e2e_step():
+        cache.restore(snap)
+        torch.cuda.current_stream().synchronize()
+        d2h = 0
+        for gi, g in enumerate(groups):
+            with torch.cuda.stream(s_copy):
+                for k in g:
+                    o, sz = up.offsets[k], up.sizes[k]
+                    up.buf[o:o + sz].copy_(host[o:o + sz], non_blocking=True)
+                ev_in[gi].record(s_copy)
+            s_comp.wait_event(ev_in[gi])
+            cache.dedup_batch(None, items=items[gi], stream=s_comp)
+            ev_out[gi].record(s_comp)
+            s_back.wait_event(ev_out[gi])
+            with torch.cuda.stream(s_back):
+                for k in g:
+                    mask_host[k].copy_(outs[k].hit_mask, non_blocking=True)
+                    res_host[k].copy_(results[k], non_blocking=True)
+                    d2h += nmask[k] * 4 + 48
+        s_back.synchronize()
+        r = res_host.numpy()
+        pos = 0
+        with torch.cuda.stream(s_back):
+            for k in range(nt):
+                nm, mb = int(r[k, 1]), int(r[k, 5])
+                if nm:
+                    idx_host[k][:nm].copy_(outs[k].miss_idx[:nm], non_blocking=True)
+                    packed_host[pos:pos + mb].copy_(outs[k].miss_bytes[:mb], non_blocking=True)
+                pos += mb
+                d2h += nm * 4 + mb
+        s_back.synchronize()
+        return d2h
+
+    e2e_step()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    d2h = 0
+    for _ in range(args.e2e_steps):
+        d2h = e2e_step()
+    torch.cuda.synchronize()
+    dt = (time.perf_counter() - t0) / args.e2e_steps
+    return {"value": round(up.total_bytes / dt / 1e9, 2), "unit": "GB/s",
+            "h2d_bytes_per_step": up.total_bytes, "d2h_bytes_per_step": d2h,
+            "ms_per_step": round(dt * 1e3, 3), "steps": args.e2e_steps,
+            "how": "pinned host upload; per group of tensors (>= 1 GiB): H2D copies, one "
+                   "batch dedup call, D2H of results and hit masks, overlapped on three "
+                   "streams; then D2H of miss indices and packed miss bytes; wall clock"}
+
+
+# ---------------------------------------------------------------------------
+# the reference arm: the oracle on the host cores
+# ---------------------------------------------------------------------------
+
+def run_reference(args, rank, world):
+    import torch
+    spec = workload_spec(args.workload)
+    C = spec["C"]
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    # per step a bounded sample: a ~96 MiB slice of tensors, cycling through
+    # the first tensors of the upload, on a freshly prefilled oracle cache
+    slice_bytes = 96 * MiB
+    from paper_2607_23115_gb300 import workloads as W
+    shapes = spec["shapes"]
+    pool_shapes, acc = [], 0
+    for s in shapes[1:]:
+        pool_shapes.append(s)
+        acc += 1
+        if acc >= 40:
+            break
+    up = W.weight_upload(pool_shapes, spec["dtype"], device=dev)
+    base = [up.payload(k).cpu().numpy().copy() for k in range(len(up.sizes))]
+    perturb(spec, up)
+    pert = [up.payload(k).cpu().numpy().copy() for k in range(len(up.sizes))] \
+        if spec["flip_frac"] > 0 else None
+    times, nbytes = [], 0
+    for i in range(args.warmup + args.steps):
+        nb, dt, nk = oracle_sample(spec, base, pert, slice_bytes, offset_tensor=3 * i)
+        if i >= args.warmup:
+            times.append(dt)
+            nbytes += nb
+    t = sum(times)
+    value = nbytes / t / 1e9
+    line = {
+        "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(t / args.steps * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u8", "data": "synthetic",
+        "impl": "reference",
+        "config": {"workload": spec["name"], "description": spec["desc"], "chunk_bytes": C},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": "per step ~96 MiB of whole tensors (layer tensors of the "
+                                   "same upload), oracle cache prefilled with their base bytes "
+                                   "(untimed)", "host_cpus": os.cpu_count()},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    return line
+
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.profile_launches:
+        args.no_e2e = True
+        args.no_cpu_baseline = True
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        print(json.dumps(run_reference(args, rank, world)))
+        return 0
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    line = run_gleam(args, rank, world, local_rank)
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -90,6 +90,17 @@ typedef struct gleam_result {
   uint64_t miss_bytes;     /* bytes written to the packed miss buffer        */
 } gleam_result_t;
 
+/* One payload of gleam_dedup_copy_batch: the arguments of one
+ * gleam_dedup_copy_async call.  d_result may be NULL. */
+typedef struct gleam_payload {
+  const void* d_buf;
+  size_t n;
+  uint32_t* d_hit_mask;
+  uint32_t* d_miss_idx;
+  void* d_miss_bytes;
+  gleam_result_t* d_result;
+} gleam_payload_t;
+
 /* ---- cache lifetime ---------------------------------------------------- */
 
 /* Creates a cache on the current GPU with floor(capacity_bytes/chunk_bytes)
@@ -149,6 +160,21 @@ int64_t gleam_dedup_copy(gleam_cache_t* cache, const void* d_buf, size_t n,
 int gleam_dedup_copy_async(gleam_cache_t* cache, const void* d_buf, size_t n,
                            uint32_t* d_hit_mask, uint32_t* d_miss_idx, void* d_miss_bytes,
                            gleam_result_t* d_result, gleam_stream_t stream);
+
+/* Dedups `count` payloads in one call: the outputs, per-payload results and
+ * final cache state are exactly those of `count` gleam_dedup_copy_async calls
+ * made in array order (paper Sec. 4.1.2 applied to each intercepted
+ * host-to-device copy in turn; a chunk equal to an earlier payload's miss is
+ * a hit on the cache, as that payload's call would have inserted it).  All
+ * chunks of all payloads are processed together, so per-call latency is paid
+ * once.  Exception: if the misses of the whole batch do not fit the free
+ * slots, the batch returns GLEAM_ERR_CAPACITY as a unit and the cache is
+ * unchanged.  payloads: host array, read before the call returns (each
+ * entry's buffers as for gleam_dedup_copy).  d_total (device, may be NULL)
+ * receives the sums over the batch.  Asynchronous on `stream`; ordered after
+ * the cache's previous call whatever its stream. */
+int gleam_dedup_copy_batch(gleam_cache_t* cache, const gleam_payload_t* payloads, size_t count,
+                           gleam_result_t* d_total, gleam_stream_t stream);
 
 /* Copies the cache's counters to *out (host struct).  Waits for the cache's
  * outstanding work on the device. */

@@ -31,7 +31,7 @@ GLEAM_DEBUG_SKIP_ARRIVE = 2
 EXPORTS = (
     "gleam_cache_create", "gleam_cache_create_ex", "gleam_cache_destroy",
     "gleam_cache_reserve", "gleam_fingerprint", "gleam_dedup_copy",
-    "gleam_dedup_copy_async", "gleam_cache_stats", "gleam_cache_export",
+    "gleam_dedup_copy_async", "gleam_dedup_copy_batch", "gleam_cache_stats", "gleam_cache_export",
     "gleam_cache_read_slot", "gleam_cache_debug_insert", "gleam_cache_debug_set",
     "gleam_cache_snapshot", "gleam_cache_restore", "gleam_snapshot_destroy",
     "gleam_cache_profile", "gleam_cache_profile_read", "gleam_status_string",
@@ -43,6 +43,12 @@ class gleam_stats_t(ctypes.Structure):
         "calls", "chunks", "hits_cache", "hits_intra", "misses", "inserts",
         "verify_rejects", "slots_used", "bytes_used", "capacity_bytes", "nslots",
         "chunk_bytes")]
+
+
+class gleam_payload_t(ctypes.Structure):
+    _fields_ = [("d_buf", ctypes.c_void_p), ("n", ctypes.c_size_t),
+                ("d_hit_mask", ctypes.c_void_p), ("d_miss_idx", ctypes.c_void_p),
+                ("d_miss_bytes", ctypes.c_void_p), ("d_result", ctypes.c_void_p)]
 
 
 RESULT_FIELDS = ("status", "n_miss", "n_hit_cache", "n_hit_intra", "verify_rejects",
@@ -78,6 +84,7 @@ def lib() -> ctypes.CDLL:
         "gleam_fingerprint": (i32, [vp, sz, sz, vp, vp]),
         "gleam_dedup_copy": (ctypes.c_int64, [vp, vp, sz, vp, vp, vp]),
         "gleam_dedup_copy_async": (i32, [vp, vp, sz, vp, vp, vp, vp, vp]),
+        "gleam_dedup_copy_batch": (i32, [vp, ctypes.POINTER(gleam_payload_t), sz, vp, vp]),
         "gleam_cache_stats": (i32, [vp, ctypes.POINTER(gleam_stats_t)]),
         "gleam_cache_export": (i32, [vp, vp, vp, u64, ctypes.POINTER(u64)]),
         "gleam_cache_read_slot": (i32, [vp, u64, vp, u64, ctypes.POINTER(u64)]),
@@ -158,6 +165,22 @@ def gleam_dedup_copy_async(cache, d_buf, n: int, d_hit_mask, d_miss_idx, d_miss_
     return lib().gleam_dedup_copy_async(cache, _ptr(d_buf), n, _ptr(d_hit_mask),
                                         _ptr(d_miss_idx), _ptr(d_miss_bytes), _ptr(d_result),
                                         _stream(stream))
+
+
+def payload_array(payloads):
+    """ctypes gleam_payload_t[] from (d_buf, n, d_hit_mask, d_miss_idx,
+    d_miss_bytes, d_result) tuples; reusable across calls."""
+    arr = (gleam_payload_t * max(1, len(payloads)))()
+    for k, (buf, n, mask, idx, packed, res) in enumerate(payloads):
+        arr[k] = gleam_payload_t(_ptr(buf), n, _ptr(mask), _ptr(idx), _ptr(packed), _ptr(res))
+    arr.count = len(payloads)
+    return arr
+
+
+def gleam_dedup_copy_batch(cache, payloads, d_total=None, stream=None) -> int:
+    """payloads: a payload_array(), or a sequence of tuples for it."""
+    arr = payloads if hasattr(payloads, "count") else payload_array(payloads)
+    return lib().gleam_dedup_copy_batch(cache, arr, arr.count, _ptr(d_total), _stream(stream))
 
 
 def gleam_cache_stats(cache):

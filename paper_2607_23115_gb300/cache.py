@@ -89,6 +89,25 @@ class Cache:
                                         out.miss_bytes, result, stream),
                "gleam_dedup_copy_async")
 
+    @staticmethod
+    def batch_items(bufs, outs, results=None):
+        """Payload array for dedup_batch (build once, reuse for repeated calls)."""
+        items = []
+        for k, (b, o) in enumerate(zip(bufs, outs)):
+            n = b.numel() * b.element_size()
+            r = results[k] if results is not None else None
+            items.append((b, n, o.hit_mask, o.miss_idx, o.miss_bytes, r))
+        return B.payload_array(items)
+
+    def dedup_batch(self, bufs, outs=None, results=None, total: Optional[torch.Tensor] = None,
+                    stream=None, items=None):
+        """One call over several payloads, equivalent to dedup_async on each in
+        order.  results: per-payload int64[6] tensors (or None)."""
+        if items is None:
+            items = self.batch_items(bufs, outs, results)
+        _check(B.gleam_dedup_copy_batch(self.handle, items, total, stream),
+               "gleam_dedup_copy_batch")
+
     def stats(self) -> dict:
         rc, st = B.gleam_cache_stats(self.handle)
         _check(rc, "gleam_cache_stats")

@@ -1,29 +1,33 @@
 // First-occurrence resolution, stream compaction, packing and insertion for
-// one dedup call (paper Sec. 4.1.2: a chunk that is not resident "is
-// transmitted in full" and becomes reusable).
+// one dedup call over one or more payloads (paper Sec. 4.1.2: a chunk that is
+// not resident travels in full and becomes reusable).
 //
-// The result must equal deciding the chunks one at a time in ascending
-// order.  Given the probe/verify outcome against the cache as it was at the
-// start of the call (kHit0 or not), that sequential rule reduces to:
-//   * a non-resident chunk is a hit iff an earlier chunk of the call has the
-//     same bytes, and its leader is the first such chunk;
+// The result must equal deciding the chunks one at a time, payload after
+// payload, in ascending order.  Given the probe/verify outcome against the
+// cache as it was when the call started (kHit0 or not), that rule reduces to:
+//   * any other chunk is a hit iff an earlier chunk of the call has the same
+//     length and bytes; its leader is the first such chunk;
 //   * the misses are the leaders, inserted in ascending order at
 //     slot = slots_used + rank;
+//   * a hit on a leader from an earlier payload is, for its own payload, a hit
+//     on the cache (that payload's call would have found the insert);
 //   * a leader counts as a verify reject iff the cache had a key+length
 //     candidate for it, or an earlier leader of the call has its key+length.
 //
 // One cooperative launch does it all, separated by bounded grid barriers:
-//   A  every non-resident full chunk claims its key's entry in a per-call
-//      table and posts its index as the group minimum;
+//   A  outputs are cleared; every non-resident chunk claims the entry of its
+//      (key, length) in a per-call table and posts its number as the group
+//      minimum;
 //   B  each unresolved chunk compares itself (whole warp, 16-byte loads) with
-//      its group's minimum: equal -> duplicate, index == minimum -> leader
-//      of this round, else it stays for the next round (only different bytes
-//      under one key: a true 64-bit collision, or KEY16 test mode);
+//      its group's minimum: equal -> duplicate, number == minimum -> leader
+//      of this round, else it stays for the next round (different bytes under
+//      one key: a true 64-bit collision, or KEY16 test mode);
 //   C  group minima of the remaining chunks are reset and re-posted (A);
-//   D  leaders are counted per contiguous block range, ranks come from the
-//      block totals plus warp ballots, and the hit mask, miss indices,
-//      packed bytes, arena copies and index entries are written.
-// The last block to finish publishes the counters and the call result.
+//   D  leaders are counted per contiguous block range; the exclusive rank of
+//      every chunk follows from the block totals plus warp ballots; then hit
+//      masks, miss indices, packed bytes, arena copies and index entries are
+//      written.
+// The last block to finish publishes the counters and the results.
 #include "gleam_internal.cuh"
 
 namespace gleam {
@@ -33,11 +37,6 @@ constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 
 __device__ __forceinline__ uint32_t ldcg_u32(const uint32_t* p) { return __ldcg(p); }
-
-__device__ __forceinline__ uint32_t chunk_len(const DedupArgs& a, uint32_t i) {
-  const uint64_t start = (uint64_t)i * a.C;
-  return (uint32_t)min(a.C, a.n - start);
-}
 
 // Whole-warp byte equality of two full chunks of the payload.
 __device__ bool warp_equal(const uint8_t* x, const uint8_t* y, uint32_t len, bool vec) {
@@ -122,19 +121,24 @@ __device__ bool index_insert(IndexEntry* index, uint64_t mask, unsigned long lon
   return false;
 }
 
-// Finds or claims the per-call table entry of a full chunk's key.
-__device__ uint32_t group_entry(const DedupArgs& a, uint32_t i, unsigned long long k) {
-  uint64_t pos = mix64(k) & a.tbl_mask;
+// Finds or claims the per-call group entry of (key, len) for chunk g.
+__device__ uint32_t group_entry(const DedupArgs& a, uint32_t g, unsigned long long k,
+                                uint32_t len) {
+  uint64_t pos = mix64(k ^ ((unsigned long long)len << 40)) & a.tbl_mask;
   for (uint64_t probe = 0; probe <= a.tbl_mask; ++probe) {
     uint32_t o = ldcg_u32(&a.tbl[pos].owner);
     if (o == 0) {
-      o = atomicCAS(&a.tbl[pos].owner, 0u, i + 1);
+      o = atomicCAS(&a.tbl[pos].owner, 0u, g + 1);
       if (o == 0) return (uint32_t)pos;
     }
-    if (a.key[o - 1] == k) return (uint32_t)pos;
+    if (a.ch.key[o - 1] == k && a.ch.len[o - 1] == len) return (uint32_t)pos;
     pos = (pos + 1) & a.tbl_mask;
   }
-  return 0xFFFFFFFFu;  // cannot happen: the table has >= 2N entries
+  return 0xFFFFFFFFu;  // cannot happen: the table has >= 2 Ntot entries
+}
+
+__device__ __forceinline__ const PayloadDesc& desc(const DedupArgs& a, uint32_t p) {
+  return a.count > 1 ? a.table[p] : a.one;
 }
 
 template <typename T>
@@ -151,11 +155,19 @@ __device__ __forceinline__ T block_sum(T v, T* red) {
   return t;
 }
 
+// Adds v to *dst once per group of lanes that share `key` (warp-aggregated).
+__device__ __forceinline__ void add_by_key(unsigned long long* dst, uint32_t key, uint32_t v,
+                                           bool active) {
+  const unsigned peers = __match_any_sync(0xffffffffu, active ? key : 0xFFFFFFFFu);
+  const uint32_t sum = __reduce_add_sync(peers, active ? v : 0u);
+  if (active && (threadIdx.x & 31) == (uint32_t)(__ffs(peers) - 1) && sum) atomicAdd(dst, sum);
+}
+
 __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ uint32_t warp_cnt[kWarps];
   __shared__ uint32_t warp_off[kWarps];
-  __shared__ uint32_t list_i[kThreads];
+  __shared__ uint32_t list_g[kThreads];
   __shared__ uint32_t list_r[kThreads];
   __shared__ unsigned long long s_slots0;
 
@@ -163,35 +175,43 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const uint32_t tid = blockIdx.x * kThreads + threadIdx.x;
   const uint32_t nth = G * kThreads;
-  const uint32_t N = a.N;
+  const uint32_t N = (uint32_t)a.Ntot;
   const bool skip = (int)blockIdx.x == a.skip_block;
-  const bool vec_buf = ((uintptr_t)a.buf % 16) == 0;
+  const ChunkArrays& ch = a.ch;
 
   if (threadIdx.x == 0) s_slots0 = *(volatile const unsigned long long*)&a.dstats[ST_SLOTS_USED];
   __syncthreads();
   const unsigned long long slots0 = s_slots0;
 
-  // ---- A: round-1 claims -------------------------------------------------
+  // ---- A: clear outputs, round-1 claims -------------------------------------
   if (!skip) {
-    for (uint32_t i = tid; i < N; i += nth) {
-      if (a.status[i] == kHit0) {
-        a.res[i] = kResHit0;
+    for (uint32_t p = tid; p < a.count; p += nth) {
+      gleam_result_t* r = desc(a, p).result;
+      if (r) {
+        r->n_miss = 0;
+        r->n_hit_cache = 0;
+        r->n_hit_intra = 0;
+        r->verify_rejects = 0;
+        r->miss_bytes = 0;
+      }
+    }
+    for (uint32_t g = tid; g < N; g += nth) {
+      const PayloadDesc& P = desc(a, ch.pidx[g]);
+      const unsigned long long i = g - P.chunk_base;
+      if ((i & 31) == 0) P.mask[i >> 5] = 0;
+      if (ch.status[g] == kHit0) {
+        ch.res[g] = kResHit0;
         continue;
       }
-      if (chunk_len(a, i) != a.C) {  // the short last chunk: unique length
-        a.res[i] = kResLeader | 1u;
-        a.ent[i] = 0xFFFFFFFFu;
-        continue;
-      }
-      const uint32_t e = group_entry(a, i, a.key[i]);
+      const uint32_t e = group_entry(a, g, ch.key[g], ch.len[g]);
       if (e == 0xFFFFFFFFu) {
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-        a.res[i] = kResLeader | 1u;
+        ch.res[g] = kResLeader | 1u;
         continue;
       }
-      a.ent[i] = e;
-      a.res[i] = kResUnresolved;
-      atomicMax(&a.tbl[e].minv, ~i);
+      ch.ent[g] = e;
+      ch.res[g] = kResUnresolved;
+      atomicMax(&a.tbl[e].minv, ~g);
     }
   }
   bool ok = grid_barrier(a.ctl, G, a.wait_ns, skip);
@@ -202,16 +222,16 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     if (tid == 0) atomicExch(&a.ctl->unres[(round + 1) % 3], 0u);
     const uint32_t nwarps = nth / 32;
     for (uint32_t base = (tid / 32) * 32; base < N; base += nwarps * 32) {
-      const uint32_t i = base + lane;
+      const uint32_t g = base + lane;
       bool need = false;
       uint32_t m = 0;
-      if (i < N && ldcg_u32(&a.res[i]) == kResUnresolved) {
-        m = ~ldcg_u32(&a.tbl[a.ent[i]].minv);
-        if (m == i) {
-          a.res[i] = kResLeader | round;
-        } else if (m > i) {  // the group minimum can only be below i: table damaged
+      if (g < N && ldcg_u32(&ch.res[g]) == kResUnresolved) {
+        m = ~ldcg_u32(&a.tbl[ch.ent[g]].minv);
+        if (m == g) {
+          ch.res[g] = kResLeader | round;
+        } else if (m > g) {  // the group minimum can only be below g: table damaged
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-          a.res[i] = kResLeader | round;
+          ch.res[g] = kResLeader | round;
         } else {
           need = true;
         }
@@ -220,43 +240,51 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       while (todo) {
         const int j = __ffs(todo) - 1;
         todo &= todo - 1;
-        const uint32_t ii = base + j;
+        const uint32_t gg = base + j;
         const uint32_t mm = __shfl_sync(0xffffffffu, m, j);
-        const bool eq = warp_equal(a.buf + (uint64_t)ii * a.C, a.buf + (uint64_t)mm * a.C,
-                                   (uint32_t)a.C, vec_buf);
+        const uint8_t* x = reinterpret_cast<const uint8_t*>(ch.src[gg]);
+        const uint8_t* y = reinterpret_cast<const uint8_t*>(ch.src[mm]);
+        const uint32_t len = ch.len[gg];
+        const bool vec = (((uintptr_t)x | (uintptr_t)y) & 15) == 0;
+        const bool eq = warp_equal(x, y, len, vec);
         if (lane == (uint32_t)j) {
-          if (eq) a.res[ii] = kResDup;
-          else atomicAdd(&a.ctl->unres[round % 3], 1u);
+          if (eq) {
+            ch.ent[gg] = mm;  // the leader, for the hit's classification
+            ch.res[gg] = kResDup;
+          } else {
+            atomicAdd(&a.ctl->unres[round % 3], 1u);
+          }
         }
       }
     }
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
     if (!ok) break;
     if (ldcg_u32(&a.ctl->unres[round % 3]) == 0) break;
-    for (uint32_t i = tid; i < N; i += nth)
-      if (ldcg_u32(&a.res[i]) == kResUnresolved) a.tbl[a.ent[i]].minv = 0;
+    for (uint32_t g = tid; g < N; g += nth)
+      if (ldcg_u32(&ch.res[g]) == kResUnresolved) a.tbl[ch.ent[g]].minv = 0;
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
     if (!ok) break;
-    for (uint32_t i = tid; i < N; i += nth)
-      if (ldcg_u32(&a.res[i]) == kResUnresolved) atomicMax(&a.tbl[a.ent[i]].minv, ~i);
+    for (uint32_t g = tid; g < N; g += nth)
+      if (ldcg_u32(&ch.res[g]) == kResUnresolved) atomicMax(&a.tbl[ch.ent[g]].minv, ~g);
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
     ++round;
   }
 
-  // ---- D: count, rank, write ------------------------------------------------
+  // ---- D1: misses per contiguous block range --------------------------------
   const uint64_t per = (((uint64_t)N + G - 1) / G + 31) & ~31ull;
   const uint32_t lo = (uint32_t)min((uint64_t)N, blockIdx.x * per);
   const uint32_t hi = (uint32_t)min((uint64_t)N, lo + per);
+  unsigned long long before = 0, total = 0;
   if (ok) {
     uint32_t cnt = 0;
-    for (uint32_t i = lo + threadIdx.x; i < hi; i += kThreads)
-      cnt += (ldcg_u32(&a.res[i]) & kResLeader) ? 1u : 0u;
+    for (uint32_t g = lo + threadIdx.x; g < hi; g += kThreads)
+      cnt += (ldcg_u32(&ch.res[g]) & kResLeader) ? 1u : 0u;
     const unsigned long long c = block_sum<unsigned long long>(cnt, red64);
     if (threadIdx.x == 0) a.bcount[blockIdx.x] = (uint32_t)c;
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   }
+  // ---- D2: exclusive miss rank of every chunk; per-payload start ranks ------
   if (ok) {
-    unsigned long long before = 0, total = 0;
     for (uint32_t j = threadIdx.x; j < G; j += kThreads) {
       const uint32_t v = ldcg_u32(&a.bcount[j]);
       total += v;
@@ -267,110 +295,174 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     if (slots0 + total > a.nslots) {
       if (threadIdx.x == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_CAPACITY);
       ok = false;
-    } else {
-      const bool vec = vec_buf && ((uintptr_t)a.packed % 16) == 0;
-      unsigned long long n_hc = 0, n_hi = 0, n_rej = 0, n_bytes = 0;
-      unsigned long long running = before;
-      for (uint32_t t = lo; t < hi; t += kThreads) {
-        const uint32_t i = t + threadIdx.x;
-        const bool valid = i < hi;
-        const uint32_t r = valid ? ldcg_u32(&a.res[i]) : 0u;
-        const bool miss = valid && (r & kResLeader);
-        const bool hit = valid && (r & (kResHit0 | kResDup));
-        const uint32_t mb = __ballot_sync(0xffffffffu, miss);
-        const uint32_t hb = __ballot_sync(0xffffffffu, hit);
-        const uint32_t g = t + w * 32;
-        if (lane == 0 && g < hi) a.mask[g >> 5] = hb;
-        if (lane == 0) warp_cnt[w] = __popc(mb);
-        __syncthreads();
-        if (threadIdx.x == 0) {
-          uint32_t acc = 0;
-          for (int k = 0; k < kWarps; ++k) {
-            warp_off[k] = acc;
-            acc += warp_cnt[k];
-          }
-          warp_cnt[0] = acc;  // tile total (read after the next barrier)
-        }
-        __syncthreads();
-        const uint32_t tile_total = warp_cnt[0];
-        if (miss) {
-          const uint32_t local = warp_off[w] + __popc(mb & ((1u << lane) - 1u));
-          const unsigned long long rank = running + local;
-          a.miss_idx[rank] = i;
-          list_i[local] = i;
-          list_r[local] = (uint32_t)(rank - before);
-          const uint32_t len = chunk_len(a, i);
-          n_bytes += len;
-          if ((r & kResRoundMask) > 1 || a.status[i] == kMissCand) ++n_rej;
-        }
-        if (valid && (r & kResHit0)) ++n_hc;
-        if (valid && (r & kResDup)) ++n_hi;
-        __syncthreads();
-        for (uint32_t k = w; k < tile_total; k += kWarps) {
-          const uint32_t ci = list_i[k];
-          const unsigned long long rank = before + list_r[k];
-          const uint32_t len = chunk_len(a, ci);
-          const unsigned long long slot = slots0 + rank;
-          warp_copy2(a.packed + rank * a.C, a.arena + slot * a.C, a.buf + (uint64_t)ci * a.C,
-                     len, vec);
-          if (lane == 0) {
-            a.slot_len[slot] = len;
-            if (!index_insert(a.index, a.index_mask, a.key[ci], (uint32_t)slot, len))
-              atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-          }
-        }
-        running += tile_total;
-        __syncthreads();
-      }
-      n_hc = block_sum<unsigned long long>(n_hc, red64);
-      n_hi = block_sum<unsigned long long>(n_hi, red64);
-      n_rej = block_sum<unsigned long long>(n_rej, red64);
-      n_bytes = block_sum<unsigned long long>(n_bytes, red64);
+    }
+  }
+  if (ok) {
+    unsigned long long running = before;
+    for (uint32_t t = lo; t < hi; t += kThreads) {
+      const uint32_t g = t + threadIdx.x;
+      const bool valid = g < hi;
+      const bool miss = valid && (ldcg_u32(&ch.res[g]) & kResLeader);
+      const uint32_t mb = __ballot_sync(0xffffffffu, miss);
+      if (lane == 0) warp_cnt[w] = __popc(mb);
+      __syncthreads();
       if (threadIdx.x == 0) {
-        atomicAdd(&a.ctl->acc_hits_cache, n_hc);
-        atomicAdd(&a.ctl->acc_hits_intra, n_hi);
-        atomicAdd(&a.ctl->acc_rejects, n_rej);
-        atomicAdd(&a.ctl->acc_miss_bytes, n_bytes);
-        if (blockIdx.x == 0) atomicExch(&a.ctl->acc_misses, total);
+        uint32_t acc = 0;
+        for (int k = 0; k < kWarps; ++k) {
+          warp_off[k] = acc;
+          acc += warp_cnt[k];
+        }
+        warp_cnt[0] = acc;
       }
+      __syncthreads();
+      if (valid) {
+        const uint32_t r = (uint32_t)(running + warp_off[w] + __popc(mb & ((1u << lane) - 1u)));
+        ch.rank[g] = r;
+        const uint32_t p = ch.pidx[g];
+        if (g == desc(a, p).chunk_base) a.pstart[p] = r;
+      }
+      running += warp_cnt[0];
+      __syncthreads();
+    }
+    ok = grid_barrier(a.ctl, G, a.wait_ns, false);
+  }
+  // ---- D3: hit masks, miss indices, packed bytes, arena copies, inserts -----
+  if (ok) {
+    unsigned long long n_hc = 0, n_hi = 0, n_rej = 0, n_bytes = 0;
+    for (uint32_t t = lo; t < hi; t += kThreads) {
+      const uint32_t g = t + threadIdx.x;
+      const bool valid = g < hi;
+      const uint32_t r = valid ? ldcg_u32(&ch.res[g]) : 0u;
+      const uint32_t p = valid ? ch.pidx[g] : 0xFFFFFFFFu;
+      const bool miss = valid && (r & kResLeader);
+      bool hc = false, hi2 = false, rej = false;
+      uint32_t len = 0;
+      if (valid) {
+        const PayloadDesc& P = desc(a, p);
+        const unsigned long long i = g - P.chunk_base;
+        if (r & kResHit0) hc = true;
+        if (r & kResDup) {
+          if (ch.pidx[ch.ent[g]] == p) hi2 = true;  // leader in the same payload
+          else hc = true;                           // inserted by an earlier payload
+        }
+        if (hc || hi2) atomicOr(P.mask + (i >> 5), 1u << (i & 31));
+        if (miss) {
+          len = ch.len[g];
+          P.miss_idx[ch.rank[g] - __ldcg(&a.pstart[p])] = (uint32_t)i;
+          rej = (r & kResRoundMask) > 1 || ch.status[g] == kMissCand;
+        }
+      }
+      n_hc += hc;
+      n_hi += hi2;
+      n_rej += rej;
+      n_bytes += len;
+      // per-payload result counters
+      const bool has_res = valid && desc(a, p).result != nullptr;
+      gleam_result_t* res = has_res ? desc(a, p).result : nullptr;
+      add_by_key(has_res ? (unsigned long long*)&res->n_hit_cache : nullptr, p, hc, has_res);
+      add_by_key(has_res ? (unsigned long long*)&res->n_hit_intra : nullptr, p, hi2, has_res);
+      add_by_key(has_res ? (unsigned long long*)&res->n_miss : nullptr, p, miss, has_res);
+      add_by_key(has_res ? (unsigned long long*)&res->verify_rejects : nullptr, p, rej, has_res);
+      add_by_key(has_res ? (unsigned long long*)&res->miss_bytes : nullptr, p, len, has_res);
+      // the tile's misses, copied by whole warps
+      const uint32_t mb = __ballot_sync(0xffffffffu, miss);
+      if (lane == 0) warp_cnt[w] = __popc(mb);
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        uint32_t acc = 0;
+        for (int k = 0; k < kWarps; ++k) {
+          warp_off[k] = acc;
+          acc += warp_cnt[k];
+        }
+        warp_cnt[0] = acc;
+      }
+      __syncthreads();
+      if (miss) list_g[warp_off[w] + __popc(mb & ((1u << lane) - 1u))] = g;
+      const uint32_t tile_total = warp_cnt[0];
+      __syncthreads();
+      for (uint32_t k = w; k < tile_total; k += kWarps) {
+        const uint32_t gg = list_g[k];
+        const uint32_t pp = ch.pidx[gg];
+        const PayloadDesc& P = desc(a, pp);
+        const uint32_t rk = ch.rank[gg];
+        const unsigned long long rp = rk - __ldcg(&a.pstart[pp]);
+        const uint32_t ln = ch.len[gg];
+        const unsigned long long slot = slots0 + rk;
+        const uint8_t* src = reinterpret_cast<const uint8_t*>(ch.src[gg]);
+        uint8_t* d1 = P.packed + rp * a.C;
+        uint8_t* d2 = a.arena + slot * a.C;
+        const bool vec = (((uintptr_t)src | (uintptr_t)d1 | (uintptr_t)d2) & 15) == 0;
+        warp_copy2(d1, d2, src, ln, vec);
+        if (lane == 0) {
+          a.slot_len[slot] = ln;
+          if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
+            atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+        }
+      }
+      __syncthreads();
+    }
+    n_hc = block_sum<unsigned long long>(n_hc, red64);
+    n_hi = block_sum<unsigned long long>(n_hi, red64);
+    n_rej = block_sum<unsigned long long>(n_rej, red64);
+    n_bytes = block_sum<unsigned long long>(n_bytes, red64);
+    if (threadIdx.x == 0) {
+      atomicAdd(&a.ctl->acc_hits_cache, n_hc);
+      atomicAdd(&a.ctl->acc_hits_intra, n_hi);
+      atomicAdd(&a.ctl->acc_rejects, n_rej);
+      atomicAdd(&a.ctl->acc_miss_bytes, n_bytes);
+      if (blockIdx.x == 0) atomicExch(&a.ctl->acc_misses, total);
     }
   }
 
   // ---- epilogue: the last block publishes ----------------------------------
+  __shared__ int s_last;
   __syncthreads();
   if (threadIdx.x == 0) {
     __threadfence();
-    const unsigned int ticket = atomicAdd(&a.ctl->done, 1u);
-    if (ticket == G - 1) {
-      __threadfence();
-      const int err = ld_volatile_s32(&a.ctl->err);
-      const unsigned long long misses = __ldcg(&a.ctl->acc_misses);
-      const unsigned long long hc = __ldcg(&a.ctl->acc_hits_cache);
-      const unsigned long long hi2 = __ldcg(&a.ctl->acc_hits_intra);
-      const unsigned long long rej = __ldcg(&a.ctl->acc_rejects);
-      const unsigned long long mbytes = __ldcg(&a.ctl->acc_miss_bytes);
-      if (err == 0) {
-        a.dstats[ST_CALLS] += 1;
-        a.dstats[ST_CHUNKS] += N;
-        a.dstats[ST_HITS_CACHE] += hc;
-        a.dstats[ST_HITS_INTRA] += hi2;
-        a.dstats[ST_MISSES] += misses;
-        a.dstats[ST_INSERTS] += misses;
-        a.dstats[ST_REJECTS] += rej;
-        a.dstats[ST_SLOTS_USED] = slots0 + misses;
-        a.dstats[ST_BYTES_USED] += mbytes;
-      }
-      if (a.result != nullptr) {
-        a.result->status = err;
-        a.result->n_miss = err ? 0 : misses;
-        a.result->n_hit_cache = err ? 0 : hc;
-        a.result->n_hit_intra = err ? 0 : hi2;
-        a.result->verify_rejects = err ? 0 : rej;
-        a.result->miss_bytes = err ? 0 : mbytes;
-      }
-      __threadfence();
+    s_last = atomicAdd(&a.ctl->done, 1u) == G - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const int err = ld_volatile_s32(&a.ctl->err);
+  if (threadIdx.x == 0) {
+    const unsigned long long misses = __ldcg(&a.ctl->acc_misses);
+    const unsigned long long hc = __ldcg(&a.ctl->acc_hits_cache);
+    const unsigned long long hi2 = __ldcg(&a.ctl->acc_hits_intra);
+    const unsigned long long rej = __ldcg(&a.ctl->acc_rejects);
+    const unsigned long long mbytes = __ldcg(&a.ctl->acc_miss_bytes);
+    if (err == 0) {
+      a.dstats[ST_CALLS] += a.ncalls;
+      a.dstats[ST_CHUNKS] += N;
+      a.dstats[ST_HITS_CACHE] += hc;
+      a.dstats[ST_HITS_INTRA] += hi2;
+      a.dstats[ST_MISSES] += misses;
+      a.dstats[ST_INSERTS] += misses;
+      a.dstats[ST_REJECTS] += rej;
+      a.dstats[ST_SLOTS_USED] = slots0 + misses;
+      a.dstats[ST_BYTES_USED] += mbytes;
+    }
+    gleam_result_t* t = a.total;
+    t->status = err;
+    t->n_miss = err ? 0 : misses;
+    t->n_hit_cache = err ? 0 : hc;
+    t->n_hit_intra = err ? 0 : hi2;
+    t->verify_rejects = err ? 0 : rej;
+    t->miss_bytes = err ? 0 : mbytes;
+  }
+  for (uint32_t p = threadIdx.x; p < a.count; p += kThreads) {
+    gleam_result_t* r = desc(a, p).result;
+    if (!r) continue;
+    r->status = err;
+    if (err) {
+      r->n_miss = 0;
+      r->n_hit_cache = 0;
+      r->n_hit_intra = 0;
+      r->verify_rejects = 0;
+      r->miss_bytes = 0;
     }
   }
+  __threadfence();
 }
 
 __global__ void k_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,

@@ -2,6 +2,8 @@
 // cache object (arena, index, counters, per-call workspace) and the launch
 // sequence of one dedup call.  Every step of the path runs in the kernels of
 // hash_probe.cu and dedup_compact.cu; nothing here touches payload bytes.
+#include <cuda.h>
+
 #include <algorithm>
 #include <cstdint>
 #include <cstring>
@@ -26,15 +28,19 @@ struct gleam_cache {
   uint32_t* slot_len = nullptr;
   unsigned long long* dstats = nullptr;
 
-  // per-call workspace
+  // per-call workspace (per chunk, by global chunk number)
   uint64_t ws_chunks = 0;
   void* ws = nullptr;
-  uint8_t* status = nullptr;
-  unsigned long long* key = nullptr;
-  uint32_t* res = nullptr;
-  uint32_t* ent = nullptr;
+  ChunkArrays ch{};
   CallEntry* tbl = nullptr;
   uint64_t tbl_cap = 0;
+
+  // payload tables of multi-payload calls
+  uint64_t tab_cap = 0;
+  PayloadDesc* d_table = nullptr;
+  PayloadDesc* h_table = nullptr;  // pinned staging for the table copy
+  uint32_t* d_pstart = nullptr;
+  cudaEvent_t table_copied = nullptr;
 
   DevCtl* ctl = nullptr;
   uint32_t* bcount = nullptr;
@@ -66,6 +72,7 @@ namespace {
 
 constexpr uint64_t kMinChunk = 32;
 constexpr uint64_t kMaxChunk = 16ull << 20;
+constexpr uint64_t kMaxChunks = 0xFFFFFFFEull;  // chunk numbers are 32-bit
 
 class DeviceGuard {
  public:
@@ -96,53 +103,141 @@ int cuda_err(cudaError_t e) {
   return e == cudaErrorMemoryAllocation ? GLEAM_ERR_NOMEM : GLEAM_ERR_CUDA;
 }
 
-// GLEAM_OK iff p is device memory of `device` (or managed memory).
-int check_device_ptr(const void* p, int device) {
-  if (p == nullptr) return GLEAM_ERR_INVALID_ARG;
-  cudaPointerAttributes at;
-  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-    cudaGetLastError();
-    return GLEAM_ERR_NOT_DEVICE_PTR;
-  }
-  if (at.type == cudaMemoryTypeManaged) return GLEAM_OK;
-  if (at.type == cudaMemoryTypeDevice && at.device == device) return GLEAM_OK;
-  return GLEAM_ERR_NOT_DEVICE_PTR;
+// ---- device pointer checks -------------------------------------------------
+//
+// A pointer is accepted iff the runtime reports device memory of the cache's
+// GPU (or managed memory).  When the driver reports the allocation's address
+// range, the accessed span must lie inside it; the range is then remembered
+// for the rest of the same call, so that payloads and outputs carved from one
+// buffer are checked with a single query.
+typedef CUresult (*PtrAttrsFn)(unsigned int, CUpointer_attribute*, void**, CUdeviceptr);
+
+PtrAttrsFn driver_ptr_attrs() {
+  static PtrAttrsFn fn = []() -> PtrAttrsFn {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuPointerGetAttributes", &f, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+      cudaGetLastError();
+      return nullptr;
+    }
+    return reinterpret_cast<PtrAttrsFn>(f);
+  }();
+  return fn;
 }
+
+class PtrChecker {
+ public:
+  explicit PtrChecker(int device) : device_(device) {}
+
+  // GLEAM_OK iff [p, p + bytes) is device memory of the device.
+  int check(const void* p, uint64_t bytes) {
+    if (p == nullptr) return GLEAM_ERR_INVALID_ARG;
+    const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+    const uintptr_t b = a + bytes;
+    for (int k = 0; k < kRanges; ++k)
+      if (hi_[k] > lo_[k] && a >= lo_[k] && b <= hi_[k]) return GLEAM_OK;
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+      cudaGetLastError();
+      return GLEAM_ERR_NOT_DEVICE_PTR;
+    }
+    const bool ok = at.type == cudaMemoryTypeManaged ||
+                    (at.type == cudaMemoryTypeDevice && at.device == device_);
+    if (!ok) return GLEAM_ERR_NOT_DEVICE_PTR;
+    if (PtrAttrsFn fn = driver_ptr_attrs()) {
+      CUpointer_attribute attrs[2] = {CU_POINTER_ATTRIBUTE_RANGE_START_ADDR,
+                                      CU_POINTER_ATTRIBUTE_RANGE_SIZE};
+      CUdeviceptr start = 0;
+      size_t size = 0;
+      void* data[2] = {&start, &size};
+      if (fn(2, attrs, data, (CUdeviceptr)a) == CUDA_SUCCESS && size > 0) {
+        if (a < start || b > start + size) return GLEAM_ERR_INVALID_ARG;  // span overruns
+        lo_[next_] = start;
+        hi_[next_] = start + size;
+        next_ = (next_ + 1) % kRanges;
+      }
+    }
+    return GLEAM_OK;
+  }
+
+ private:
+  static constexpr int kRanges = 8;
+  int device_;
+  uintptr_t lo_[kRanges] = {};
+  uintptr_t hi_[kRanges] = {};
+  int next_ = 0;
+};
 
 void free_ws(gleam_cache* c) {
   if (c->ws) cudaFree(c->ws);
   c->ws = nullptr;
   c->ws_chunks = 0;
   c->tbl_cap = 0;
+  c->ch = ChunkArrays{};
+  c->tbl = nullptr;
 }
 
-// Grows the per-call workspace to hold `nchunks` chunks (synchronises `s`).
-int ensure_ws(gleam_cache* c, uint64_t nchunks, cudaStream_t s) {
+// Grows the per-chunk workspace to hold `nchunks` chunks.  Waits for the
+// cache's previous work first (it may still be using the old workspace).
+int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   if (nchunks <= c->ws_chunks) return GLEAM_OK;
   uint64_t cap = std::max<uint64_t>({nchunks, 2 * c->ws_chunks, 4096});
-  cap = std::min<uint64_t>(cap, 0xFFFFFFFFull);
+  cap = std::min<uint64_t>(cap, kMaxChunks);
   if (cap < nchunks) cap = nchunks;
   const uint64_t tcap = next_pow2(2 * cap);
-  const uint64_t sz_status = align256(cap);
-  const uint64_t sz_key = align256(cap * 8);
-  const uint64_t sz_res = align256(cap * 4);
-  const uint64_t sz_ent = align256(cap * 4);
-  const uint64_t sz_tbl = align256(tcap * sizeof(CallEntry));
-  if (s != nullptr) cudaStreamSynchronize(s);
-  cudaStreamSynchronize(nullptr);
+  const uint64_t sz[9] = {align256(cap),     align256(cap * 8), align256(cap * 4),
+                          align256(cap * 8), align256(cap * 4), align256(cap * 4),
+                          align256(cap * 4), align256(cap * 4), align256(tcap * sizeof(CallEntry))};
+  uint64_t total = 0;
+  for (uint64_t x : sz) total += x;
+  int rc = cuda_err(cudaEventSynchronize(c->done));
+  if (rc != GLEAM_OK) return rc;
   free_ws(c);
   void* p = nullptr;
-  int rc = cuda_err(cudaMalloc(&p, sz_status + sz_key + sz_res + sz_ent + sz_tbl));
-  if (rc != GLEAM_OK) return rc;
+  if ((rc = cuda_err(cudaMalloc(&p, total))) != GLEAM_OK) return rc;
   uint8_t* b = static_cast<uint8_t*>(p);
   c->ws = p;
-  c->status = b;
-  c->key = reinterpret_cast<unsigned long long*>(b + sz_status);
-  c->res = reinterpret_cast<uint32_t*>(b + sz_status + sz_key);
-  c->ent = reinterpret_cast<uint32_t*>(b + sz_status + sz_key + sz_res);
-  c->tbl = reinterpret_cast<CallEntry*>(b + sz_status + sz_key + sz_res + sz_ent);
+  c->ch.status = b;
+  b += sz[0];
+  c->ch.key = reinterpret_cast<unsigned long long*>(b);
+  b += sz[1];
+  c->ch.len = reinterpret_cast<uint32_t*>(b);
+  b += sz[2];
+  c->ch.src = reinterpret_cast<unsigned long long*>(b);
+  b += sz[3];
+  c->ch.pidx = reinterpret_cast<uint32_t*>(b);
+  b += sz[4];
+  c->ch.res = reinterpret_cast<uint32_t*>(b);
+  b += sz[5];
+  c->ch.ent = reinterpret_cast<uint32_t*>(b);
+  b += sz[6];
+  c->ch.rank = reinterpret_cast<uint32_t*>(b);
+  b += sz[7];
+  c->tbl = reinterpret_cast<CallEntry*>(b);
   c->tbl_cap = tcap;
   c->ws_chunks = cap;
+  return GLEAM_OK;
+}
+
+// Grows the payload tables to `count` payloads.
+int ensure_tables(gleam_cache* c, uint64_t count) {
+  if (count <= c->tab_cap) return GLEAM_OK;
+  const uint64_t cap = std::max<uint64_t>({count, 2 * c->tab_cap, 64});
+  int rc = cuda_err(cudaEventSynchronize(c->done));
+  if (rc != GLEAM_OK) return rc;
+  if (c->d_table) cudaFree(c->d_table);
+  if (c->h_table) cudaFreeHost(c->h_table);
+  if (c->d_pstart) cudaFree(c->d_pstart);
+  c->d_table = nullptr;
+  c->h_table = nullptr;
+  c->d_pstart = nullptr;
+  c->tab_cap = 0;
+  if ((rc = cuda_err(cudaMalloc(&c->d_table, cap * sizeof(PayloadDesc)))) != GLEAM_OK) return rc;
+  if ((rc = cuda_err(cudaMallocHost(&c->h_table, cap * sizeof(PayloadDesc)))) != GLEAM_OK) return rc;
+  if ((rc = cuda_err(cudaMalloc(&c->d_pstart, cap * sizeof(uint32_t)))) != GLEAM_OK) return rc;
+  c->tab_cap = cap;
   return GLEAM_OK;
 }
 
@@ -160,6 +255,10 @@ void destroy_cache(gleam_cache* c) {
     if (c->bcount) cudaFree(c->bcount);
     if (c->d_result) cudaFree(c->d_result);
     if (c->h_result) cudaFreeHost(c->h_result);
+    if (c->d_table) cudaFree(c->d_table);
+    if (c->h_table) cudaFreeHost(c->h_table);
+    if (c->d_pstart) cudaFree(c->d_pstart);
+    if (c->table_copied) cudaEventDestroy(c->table_copied);
     if (c->done) cudaEventDestroy(c->done);
     for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
     cudaGetLastError();
@@ -167,43 +266,89 @@ void destroy_cache(gleam_cache* c) {
   delete c;
 }
 
-int wait_done(const gleam_cache* c) {
-  return cuda_err(cudaEventSynchronize(c->done));
+int wait_done(const gleam_cache* c) { return cuda_err(cudaEventSynchronize(c->done)); }
+
+// Validates one payload and fills its device descriptor (chunk_base left 0).
+int describe(gleam_cache* c, PtrChecker& chk, const gleam_payload_t& p, PayloadDesc* d) {
+  const uint64_t N = (p.n + c->C - 1) / c->C;
+  if (N > kMaxChunks) return GLEAM_ERR_INVALID_ARG;
+  d->buf = static_cast<const uint8_t*>(p.d_buf);
+  d->n = p.n;
+  d->chunk_base = 0;
+  d->nchunks = N;
+  d->mask = p.d_hit_mask;
+  d->miss_idx = p.d_miss_idx;
+  d->packed = static_cast<uint8_t*>(p.d_miss_bytes);
+  d->result = p.d_result;
+  int rc;
+  if (p.d_result && (rc = chk.check(p.d_result, sizeof(gleam_result_t))) != GLEAM_OK) return rc;
+  if (p.n == 0) return GLEAM_OK;
+  if ((rc = chk.check(p.d_buf, p.n)) != GLEAM_OK) return rc;
+  if ((rc = chk.check(p.d_hit_mask, ((N + 31) / 32) * 4)) != GLEAM_OK) return rc;
+  if ((rc = chk.check(p.d_miss_idx, N * 4)) != GLEAM_OK) return rc;
+  if ((rc = chk.check(p.d_miss_bytes, p.n)) != GLEAM_OK) return rc;
+  return GLEAM_OK;
 }
 
-// Enqueues one dedup call on stream s.  Caller holds c->mu and the device.
-int enqueue_dedup(gleam_cache* c, const void* d_buf, size_t n, uint32_t* d_hit_mask,
-                  uint32_t* d_miss_idx, void* d_miss_bytes, gleam_result_t* d_result,
-                  cudaStream_t s) {
-  const uint64_t N = (n + c->C - 1) / c->C;
-  if (N >= 0xFFFFFFFFull) return GLEAM_ERR_INVALID_ARG;
+// Enqueues one dedup call over `count` payloads on stream s, ordered after
+// the cache's previous call.  Caller holds c->mu and the device.
+int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
+            gleam_result_t* d_total, cudaStream_t s) {
+  if (count == 0) return GLEAM_OK;
+  if (count > 0xFFFFFFFEull) return GLEAM_ERR_INVALID_ARG;
+  PtrChecker chk(c->device);
   int rc;
-  if ((rc = check_device_ptr(d_buf, c->device)) != GLEAM_OK) return rc;
-  if ((rc = check_device_ptr(d_hit_mask, c->device)) != GLEAM_OK) return rc;
-  if ((rc = check_device_ptr(d_miss_idx, c->device)) != GLEAM_OK) return rc;
-  if ((rc = check_device_ptr(d_miss_bytes, c->device)) != GLEAM_OK) return rc;
-  if (d_result && (rc = check_device_ptr(d_result, c->device)) != GLEAM_OK) return rc;
-  if ((rc = ensure_ws(c, N, s)) != GLEAM_OK) return rc;
+  if (d_total && (rc = chk.check(d_total, sizeof(gleam_result_t))) != GLEAM_OK) return rc;
 
-  const uint64_t tcap = std::min<uint64_t>(c->tbl_cap, next_pow2(std::max<uint64_t>(64, 2 * N)));
+  PayloadDesc one{};
+  if (count > 1) {
+    if ((rc = ensure_tables(c, count)) != GLEAM_OK) return rc;
+    // the staging buffer may still feed the previous call's table copy
+    if ((rc = cuda_err(cudaEventSynchronize(c->table_copied))) != GLEAM_OK) return rc;
+  }
+  uint64_t Ntot = 0, ncalls = 0;
+  bool aligned = true;
+  for (uint64_t k = 0; k < count; ++k) {
+    PayloadDesc* d = count > 1 ? &c->h_table[k] : &one;
+    if ((rc = describe(c, chk, payloads[k], d)) != GLEAM_OK) return rc;
+    d->chunk_base = Ntot;
+    Ntot += d->nchunks;
+    if (Ntot > kMaxChunks) return GLEAM_ERR_INVALID_ARG;
+    if (d->n) {
+      ++ncalls;
+      aligned = aligned && (reinterpret_cast<uintptr_t>(d->buf) % 16 == 0);
+    }
+  }
+  if ((rc = ensure_ws(c, std::max<uint64_t>(Ntot, 1))) != GLEAM_OK) return rc;
+
+  if ((rc = cuda_err(cudaStreamWaitEvent(s, c->done, 0))) != GLEAM_OK) return rc;
+  if (count > 1) {
+    if ((rc = cuda_err(cudaMemcpyAsync(c->d_table, c->h_table, count * sizeof(PayloadDesc),
+                                       cudaMemcpyHostToDevice, s))) != GLEAM_OK)
+      return rc;
+    if ((rc = cuda_err(cudaEventRecord(c->table_copied, s))) != GLEAM_OK) return rc;
+  }
+  const uint64_t tcap =
+      std::min<uint64_t>(c->tbl_cap, next_pow2(std::max<uint64_t>(64, 2 * Ntot)));
   if ((rc = cuda_err(cudaMemsetAsync(c->ctl, 0, sizeof(DevCtl), s))) != GLEAM_OK) return rc;
   if ((rc = cuda_err(cudaMemsetAsync(c->tbl, 0, tcap * sizeof(CallEntry), s))) != GLEAM_OK)
     return rc;
 
   HashArgs h{};
-  h.buf = static_cast<const uint8_t*>(d_buf);
-  h.n = n;
+  h.table = c->d_table;
+  h.one = one;
+  h.count = (uint32_t)count;
+  h.Ntot = Ntot;
   h.C = c->C;
-  h.N = (uint32_t)N;
   h.fp_out = nullptr;
   h.index = c->index;
   h.index_mask = c->index_cap - 1;
   h.arena = c->arena;
   h.dstats = c->dstats;
   h.key16 = (c->flags & GLEAM_KEY16) ? 1u : 0u;
-  h.status = c->status;
-  h.key_out = c->key;
+  h.ch = c->ch;
   h.ctl = c->ctl;
+
   cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
   if (c->profile) {
     while (c->ev_pool.size() < c->ev_used + 3) {
@@ -215,38 +360,35 @@ int enqueue_dedup(gleam_cache* c, const void* d_buf, size_t n, uint32_t* d_hit_m
     c->ev_used += 3;
     cudaEventRecord(ev[0], s);
   }
-  if ((rc = cuda_err(launch_hash(h, s))) != GLEAM_OK) return rc;
+  if ((rc = cuda_err(launch_hash(h, aligned, s))) != GLEAM_OK) return rc;
   if (ev[1]) cudaEventRecord(ev[1], s);
 
   DedupArgs d{};
-  d.buf = h.buf;
-  d.n = n;
+  d.table = c->d_table;
+  d.one = one;
+  d.count = (uint32_t)count;
+  d.Ntot = Ntot;
   d.C = c->C;
-  d.N = (uint32_t)N;
-  d.mask = d_hit_mask;
-  d.miss_idx = d_miss_idx;
-  d.packed = static_cast<uint8_t*>(d_miss_bytes);
   d.arena = c->arena;
   d.index = c->index;
   d.index_mask = c->index_cap - 1;
   d.nslots = c->nslots;
   d.slot_len = c->slot_len;
   d.dstats = c->dstats;
-  d.status = c->status;
-  d.key = c->key;
-  d.res = c->res;
-  d.ent = c->ent;
+  d.ch = c->ch;
+  d.pstart = count > 1 ? c->d_pstart : c->bcount + c->coop_max_blocks;
   d.tbl = c->tbl;
   d.tbl_mask = tcap - 1;
   d.bcount = c->bcount;
   d.ctl = c->ctl;
-  d.result = d_result ? d_result : c->d_result;
+  d.total = d_total ? d_total : c->d_result;
+  d.ncalls = ncalls;
   d.wait_ns = c->wait_ns;
   d.skip_block = c->skip_block;
   c->skip_block = -1;  // the hook applies to one call
   const int per_block = 4 * dedup_threads();
   int grid = (int)std::max<uint64_t>(
-      1, std::min<uint64_t>(c->coop_max_blocks, (N + per_block - 1) / per_block));
+      1, std::min<uint64_t>(c->coop_max_blocks, (Ntot + per_block - 1) / per_block));
   if (d.skip_block >= 0) {
     grid = std::max(grid, std::min(2, c->coop_max_blocks));  // someone must be left waiting
     if (d.skip_block >= grid) d.skip_block = grid - 1;
@@ -254,6 +396,18 @@ int enqueue_dedup(gleam_cache* c, const void* d_buf, size_t n, uint32_t* d_hit_m
   if ((rc = cuda_err(launch_dedup(d, grid, s))) != GLEAM_OK) return rc;
   if (ev[2]) cudaEventRecord(ev[2], s);
   return cuda_err(cudaEventRecord(c->done, s));
+}
+
+gleam_payload_t make_payload(const void* d_buf, size_t n, uint32_t* d_hit_mask,
+                             uint32_t* d_miss_idx, void* d_miss_bytes, gleam_result_t* d_result) {
+  gleam_payload_t p;
+  p.d_buf = d_buf;
+  p.n = n;
+  p.d_hit_mask = d_hit_mask;
+  p.d_miss_idx = d_miss_idx;
+  p.d_miss_bytes = d_miss_bytes;
+  p.d_result = d_result;
+  return p;
 }
 
 }  // namespace
@@ -309,6 +463,7 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   step(cudaMalloc(&c->d_result, sizeof(gleam_result_t)));
   step(cudaMallocHost(&c->h_result, sizeof(gleam_result_t)));
   step(cudaEventCreateWithFlags(&c->done, cudaEventDisableTiming));
+  step(cudaEventCreateWithFlags(&c->table_copied, cudaEventDisableTiming));
   if (rc == GLEAM_OK) {
     int sms = 0;
     step(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device));
@@ -316,12 +471,14 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     c->coop_max_blocks = sms * per_sm;
     if (c->coop_max_blocks <= 0) rc = GLEAM_ERR_CUDA;
   }
-  if (rc == GLEAM_OK) step(cudaMalloc(&c->bcount, c->coop_max_blocks * sizeof(uint32_t)));
+  // block counts, followed by one word used as the single payload's start rank
+  if (rc == GLEAM_OK) step(cudaMalloc(&c->bcount, (c->coop_max_blocks + 1) * sizeof(uint32_t)));
   if (rc == GLEAM_OK) {
     step(cudaMemset(c->index, 0xFF, c->index_cap * sizeof(IndexEntry)));
     step(cudaMemset(c->dstats, 0, ST_COUNT * sizeof(unsigned long long)));
     step(cudaMemset(c->ctl, 0, sizeof(DevCtl)));
     step(cudaEventRecord(c->done, nullptr));
+    step(cudaEventRecord(c->table_copied, nullptr));
     step(cudaDeviceSynchronize());
   }
   if (rc != GLEAM_OK) {
@@ -339,12 +496,10 @@ int gleam_cache_create(size_t capacity_bytes, size_t chunk_bytes, gleam_cache_t*
 void gleam_cache_destroy(gleam_cache_t* cache) { destroy_cache(cache); }
 
 int gleam_cache_reserve(gleam_cache_t* c, uint64_t max_chunks) {
-  if (!c || max_chunks >= 0xFFFFFFFFull) return GLEAM_ERR_INVALID_ARG;
+  if (!c || max_chunks > kMaxChunks) return GLEAM_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> lk(c->mu);
   DeviceGuard g(c->device);
-  int rc = wait_done(c);
-  if (rc != GLEAM_OK) return rc;
-  return ensure_ws(c, max_chunks, nullptr);
+  return ensure_ws(c, max_chunks);
 }
 
 int gleam_fingerprint(const void* d_buf, size_t n, size_t chunk_bytes, uint64_t* d_out,
@@ -352,9 +507,6 @@ int gleam_fingerprint(const void* d_buf, size_t n, size_t chunk_bytes, uint64_t*
   if (d_out == nullptr || (n > 0 && d_buf == nullptr)) return GLEAM_ERR_INVALID_ARG;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return cuda_err(cudaErrorUnknown);
-  int rc;
-  if ((rc = check_device_ptr(d_out, dev)) != GLEAM_OK) return rc;
-  if (n > 0 && (rc = check_device_ptr(d_buf, dev)) != GLEAM_OK) return rc;
   uint64_t N, C;
   if (chunk_bytes == 0) {
     N = 1;
@@ -364,14 +516,30 @@ int gleam_fingerprint(const void* d_buf, size_t n, size_t chunk_bytes, uint64_t*
     C = chunk_bytes;
   }
   if (N == 0) return GLEAM_OK;
-  if (N >= 0xFFFFFFFFull || C > 0xFFFFFFFFull) return GLEAM_ERR_INVALID_ARG;
+  if (N > kMaxChunks || C > 0xFFFFFFFFull) return GLEAM_ERR_INVALID_ARG;
+  PtrChecker chk(dev);
+  int rc;
+  if ((rc = chk.check(d_out, N * 8)) != GLEAM_OK) return rc;
+  if (n > 0 && (rc = chk.check(d_buf, n)) != GLEAM_OK) return rc;
   HashArgs h{};
-  h.buf = static_cast<const uint8_t*>(d_buf);
-  h.n = n;
+  h.one.buf = static_cast<const uint8_t*>(d_buf);
+  h.one.n = n;
+  h.one.chunk_base = 0;
+  h.one.nchunks = N;
+  h.count = 1;
+  h.Ntot = N;
   h.C = C;
-  h.N = (uint32_t)N;
   h.fp_out = reinterpret_cast<unsigned long long*>(d_out);
-  return cuda_err(launch_hash(h, reinterpret_cast<cudaStream_t>(stream)));
+  const bool aligned = (reinterpret_cast<uintptr_t>(d_buf) % 16 == 0) && (N == 1 || C % 16 == 0);
+  return cuda_err(launch_hash(h, aligned, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int gleam_dedup_copy_batch(gleam_cache_t* c, const gleam_payload_t* payloads, size_t count,
+                           gleam_result_t* d_total, gleam_stream_t stream) {
+  if (!c || (count > 0 && !payloads)) return GLEAM_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(c->mu);
+  DeviceGuard g(c->device);
+  return enqueue(c, payloads, count, d_total, reinterpret_cast<cudaStream_t>(stream));
 }
 
 int gleam_dedup_copy_async(gleam_cache_t* c, const void* d_buf, size_t n, uint32_t* d_hit_mask,
@@ -381,8 +549,8 @@ int gleam_dedup_copy_async(gleam_cache_t* c, const void* d_buf, size_t n, uint32
   if (n == 0) return GLEAM_OK;
   std::lock_guard<std::mutex> lk(c->mu);
   DeviceGuard g(c->device);
-  return enqueue_dedup(c, d_buf, n, d_hit_mask, d_miss_idx, d_miss_bytes, d_result,
-                       reinterpret_cast<cudaStream_t>(stream));
+  const gleam_payload_t p = make_payload(d_buf, n, d_hit_mask, d_miss_idx, d_miss_bytes, d_result);
+  return enqueue(c, &p, 1, nullptr, reinterpret_cast<cudaStream_t>(stream));
 }
 
 int64_t gleam_dedup_copy(gleam_cache_t* c, const void* d_buf, size_t n, uint32_t* d_hit_mask,
@@ -391,7 +559,8 @@ int64_t gleam_dedup_copy(gleam_cache_t* c, const void* d_buf, size_t n, uint32_t
   if (n == 0) return 0;
   std::lock_guard<std::mutex> lk(c->mu);
   DeviceGuard g(c->device);
-  int rc = enqueue_dedup(c, d_buf, n, d_hit_mask, d_miss_idx, d_miss_bytes, c->d_result, nullptr);
+  const gleam_payload_t p = make_payload(d_buf, n, d_hit_mask, d_miss_idx, d_miss_bytes, nullptr);
+  int rc = enqueue(c, &p, 1, c->d_result, nullptr);
   if (rc != GLEAM_OK) return rc;
   rc = cuda_err(cudaMemcpyAsync(c->h_result, c->d_result, sizeof(gleam_result_t),
                                 cudaMemcpyDeviceToHost, nullptr));
@@ -470,7 +639,8 @@ int gleam_cache_debug_insert(gleam_cache_t* c, uint64_t key, const void* d_bytes
   if (!c || len == 0 || len > c->C) return GLEAM_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> lk(c->mu);
   DeviceGuard g(c->device);
-  int rc = check_device_ptr(d_bytes, c->device);
+  PtrChecker chk(c->device);
+  int rc = chk.check(d_bytes, len);
   if (rc != GLEAM_OK) return rc;
   if ((rc = wait_done(c)) != GLEAM_OK) return rc;
   unsigned long long used = 0;
@@ -562,8 +732,8 @@ int gleam_cache_snapshot(gleam_cache_t* c, gleam_snapshot_t** out) {
   return GLEAM_OK;
 }
 
-// Stream-ordered on the legacy default stream: it orders after earlier work
-// on every blocking stream, and later calls there see the restored state.
+// Stream-ordered on the legacy default stream: it orders after the cache's
+// previous call, and later calls on blocking streams see the restored state.
 int gleam_cache_restore(gleam_cache_t* c, const gleam_snapshot_t* s) {
   if (!c || !s || s->owner != c || s->index_cap != c->index_cap) return GLEAM_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> lk(c->mu);

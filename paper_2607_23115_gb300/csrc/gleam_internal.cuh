@@ -78,51 +78,74 @@ __host__ __device__ __forceinline__ unsigned long long mix64(unsigned long long 
 // Kernel argument blocks and launchers (defined in the kernel TUs)
 // ---------------------------------------------------------------------------
 
-struct HashArgs {
+// One payload of a call (a batch of calls has one per payload), as the
+// device sees it.  Chunks of all payloads are numbered consecutively:
+// payload p owns global chunks [chunk_base, chunk_base + nchunks).
+struct __align__(16) PayloadDesc {
   const uint8_t* buf;
-  uint64_t n;
-  uint64_t C;                  // chunk length (bytes)
-  uint32_t N;                  // number of chunks
+  unsigned long long n;
+  unsigned long long chunk_base;
+  unsigned long long nchunks;
+  uint32_t* mask;
+  uint32_t* miss_idx;
+  uint8_t* packed;
+  gleam_result_t* result;  // may be null
+};
+
+// Per-chunk workspace, indexed by global chunk number.
+struct ChunkArrays {
+  uint8_t* status;           // kHit0 / kMissCand / kMissNoCand
+  unsigned long long* key;   // index key (XXH64, or its low 16 bits)
+  uint32_t* len;             // true length
+  unsigned long long* src;   // device address of the chunk's first byte
+  uint32_t* pidx;            // payload number
+  uint32_t* res;             // resolution word (kRes*)
+  uint32_t* ent;             // group-table entry; the leader's number once a duplicate
+  uint32_t* rank;            // exclusive count of misses before the chunk
+};
+
+struct HashArgs {
+  const PayloadDesc* table;  // count > 1
+  PayloadDesc one;           // count == 1
+  uint32_t count;
+  unsigned long long Ntot;   // chunks of all payloads
+  unsigned long long C;      // chunk length (bytes)
   unsigned long long* fp_out;  // optional: XXH64 per chunk
   // probe + verify (index == nullptr: fingerprint only)
   const IndexEntry* index;
-  uint64_t index_mask;
+  unsigned long long index_mask;
   const uint8_t* arena;
   const unsigned long long* dstats;
   uint32_t key16;
-  uint8_t* status;
-  unsigned long long* key_out;
+  ChunkArrays ch;
   DevCtl* ctl;
 };
 
 struct DedupArgs {
-  const uint8_t* buf;
-  uint64_t n;
-  uint64_t C;
-  uint32_t N;
-  uint32_t* mask;
-  uint32_t* miss_idx;
-  uint8_t* packed;
+  const PayloadDesc* table;
+  PayloadDesc one;
+  uint32_t count;
+  unsigned long long Ntot;
+  unsigned long long C;
   uint8_t* arena;
   IndexEntry* index;
-  uint64_t index_mask;
-  uint64_t nslots;
+  unsigned long long index_mask;
+  unsigned long long nslots;
   uint32_t* slot_len;
   unsigned long long* dstats;
-  const uint8_t* status;
-  const unsigned long long* key;
-  uint32_t* res;
-  uint32_t* ent;
+  ChunkArrays ch;
+  uint32_t* pstart;          // per payload: misses before its first chunk
   CallEntry* tbl;
-  uint64_t tbl_mask;
+  unsigned long long tbl_mask;
   uint32_t* bcount;
   DevCtl* ctl;
-  gleam_result_t* result;
+  gleam_result_t* total;     // result of the whole call (never null)
+  unsigned long long ncalls; // payloads with n > 0
   unsigned long long wait_ns;
   int skip_block;
 };
 
-cudaError_t launch_hash(const HashArgs& a, cudaStream_t s);
+cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s);
 cudaError_t launch_dedup(const DedupArgs& a, int grid, cudaStream_t s);
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
                                 unsigned long long* dstats, unsigned long long key,
@@ -185,6 +208,19 @@ __device__ __forceinline__ bool grid_barrier(DevCtl* ctl, unsigned int nblocks,
   if (threadIdx.x == 0) s_ok = (!skip && ld_volatile_s32(&ctl->err) == 0) ? 1 : 0;
   __syncthreads();
   return s_ok != 0;
+}
+
+// Payload owning global chunk g: the last p with chunk_base <= g (empty
+// payloads share their base with the next one and are never chosen).
+__device__ __forceinline__ uint32_t find_payload(const PayloadDesc* table, uint32_t count,
+                                                 unsigned long long g) {
+  uint32_t lo = 0, hi = count;
+  while (hi - lo > 1) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (__ldg(&table[mid].chunk_base) <= g) lo = mid;
+    else hi = mid;
+  }
+  return lo;
 }
 
 #endif  // __CUDACC__

@@ -98,16 +98,28 @@ __device__ __forceinline__ bool group_equal(const uint8_t* p, const uint8_t* q, 
 
 template <bool kAligned, bool kProbe>
 __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
-  const uint64_t gtid = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const uint64_t chunk = gtid >> 2;
-  if (chunk >= a.N) return;  // whole groups leave together
+  const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
+  if (g >= a.Ntot) return;  // whole groups leave together
   const uint32_t lane = threadIdx.x & 3;
   const int gbase = threadIdx.x & 28;
   const unsigned gmask = 0xFu << gbase;
 
-  const uint64_t start = chunk * a.C;
-  const uint32_t len = (uint32_t)min(a.C, a.n - start);
-  const uint8_t* p = a.buf + start;
+  uint32_t pid = 0;
+  const uint8_t* buf;
+  unsigned long long n, base;
+  if (a.count > 1) {
+    pid = find_payload(a.table, a.count, g);
+    buf = a.table[pid].buf;
+    n = a.table[pid].n;
+    base = a.table[pid].chunk_base;
+  } else {
+    buf = a.one.buf;
+    n = a.one.n;
+    base = a.one.chunk_base;
+  }
+  const unsigned long long start = (g - base) * a.C;
+  const uint32_t len = (uint32_t)min(a.C, n - start);
+  const uint8_t* p = buf + start;
   const uint32_t ns = len >> 5;
 
   unsigned long long h;
@@ -124,14 +136,14 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
   h += len;
   h = xfinish(h, p + (uint64_t)ns * 32, len & 31);
 
-  if (a.fp_out != nullptr && lane == 0) a.fp_out[chunk] = h;
+  if (a.fp_out != nullptr && lane == 0) a.fp_out[g] = h;
   if (!kProbe) return;
 
   const unsigned long long key = a.key16 ? (h & 0xFFFFULL) : h;
   const unsigned long long slots_used = a.dstats[ST_SLOTS_USED];
-  uint64_t pos = mix64(key) & a.index_mask;
+  unsigned long long pos = mix64(key) & a.index_mask;
   bool hit = false, cand = false;
-  for (uint64_t probe = 0; probe <= a.index_mask; ++probe) {
+  for (unsigned long long probe = 0; probe <= a.index_mask; ++probe) {
     const IndexEntry e = a.index[pos];
     if (e.slot == kEmptySlot) break;
     if (e.key == key && e.len == len) {
@@ -147,18 +159,20 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
     pos = (pos + 1) & a.index_mask;
   }
   if (lane == 0) {
-    a.status[chunk] = hit ? kHit0 : (cand ? kMissCand : kMissNoCand);
-    a.key_out[chunk] = key;
+    a.ch.status[g] = hit ? kHit0 : (cand ? kMissCand : kMissNoCand);
+    a.ch.key[g] = key;
+    a.ch.len[g] = len;
+    a.ch.src[g] = (unsigned long long)p;
+    a.ch.pidx[g] = pid;
   }
 }
 
 }  // namespace
 
-cudaError_t launch_hash(const HashArgs& a, cudaStream_t s) {
-  if (a.N == 0) return cudaSuccess;
-  const uint64_t threads = (uint64_t)a.N * 4;
+cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
+  if (a.Ntot == 0) return cudaSuccess;
+  const unsigned long long threads = a.Ntot * 4;
   const unsigned grid = (unsigned)((threads + kHashThreads - 1) / kHashThreads);
-  const bool aligned = ((uintptr_t)a.buf % 16 == 0) && (a.N == 1 || a.C % 16 == 0);
   const bool probe = a.index != nullptr;
   if (aligned && probe) k_hash_probe<true, true><<<grid, kHashThreads, 0, s>>>(a);
   else if (aligned) k_hash_probe<true, false><<<grid, kHashThreads, 0, s>>>(a);
