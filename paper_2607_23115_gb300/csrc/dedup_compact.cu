@@ -397,6 +397,9 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
           a.slot_len[slot] = ln;
           if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
             atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+          if (ln >= kPrefixBytes &&
+              !index_insert(a.hints, a.index_mask, ch.hint[gg], (uint32_t)slot, ln))
+            atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
         }
       }
       __syncthreads();

@@ -24,6 +24,7 @@ struct gleam_cache {
 
   uint8_t* arena = nullptr;
   IndexEntry* index = nullptr;
+  IndexEntry* hints = nullptr;  // prefix-hint table, index_cap entries
   uint64_t index_cap = 0;  // power of two >= 2 * nslots
   uint32_t* slot_len = nullptr;
   unsigned long long* dstats = nullptr;
@@ -64,6 +65,7 @@ struct gleam_snapshot {
   int device = 0;
   const gleam_cache* owner = nullptr;
   IndexEntry* index = nullptr;
+  IndexEntry* hints = nullptr;
   uint64_t index_cap = 0;
   unsigned long long* dstats = nullptr;
 };
@@ -187,9 +189,10 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   cap = std::min<uint64_t>(cap, kMaxChunks);
   if (cap < nchunks) cap = nchunks;
   const uint64_t tcap = next_pow2(2 * cap);
-  const uint64_t sz[9] = {align256(cap),     align256(cap * 8), align256(cap * 4),
-                          align256(cap * 8), align256(cap * 4), align256(cap * 4),
-                          align256(cap * 4), align256(cap * 4), align256(tcap * sizeof(CallEntry))};
+  const uint64_t sz[10] = {align256(cap),     align256(cap * 8), align256(cap * 4),
+                           align256(cap * 8), align256(cap * 4), align256(cap * 4),
+                           align256(cap * 4), align256(cap * 4), align256(cap * 8),
+                           align256(tcap * sizeof(CallEntry))};
   uint64_t total = 0;
   for (uint64_t x : sz) total += x;
   int rc = cuda_err(cudaEventSynchronize(c->done));
@@ -215,6 +218,8 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   b += sz[6];
   c->ch.rank = reinterpret_cast<uint32_t*>(b);
   b += sz[7];
+  c->ch.hint = reinterpret_cast<unsigned long long*>(b);
+  b += sz[8];
   c->tbl = reinterpret_cast<CallEntry*>(b);
   c->tbl_cap = tcap;
   c->ws_chunks = cap;
@@ -249,6 +254,7 @@ void destroy_cache(gleam_cache* c) {
     free_ws(c);
     if (c->arena) cudaFree(c->arena);
     if (c->index) cudaFree(c->index);
+    if (c->hints) cudaFree(c->hints);
     if (c->slot_len) cudaFree(c->slot_len);
     if (c->dstats) cudaFree(c->dstats);
     if (c->ctl) cudaFree(c->ctl);
@@ -343,6 +349,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   h.fp_out = nullptr;
   h.index = c->index;
   h.index_mask = c->index_cap - 1;
+  h.hints = c->hints;
   h.arena = c->arena;
   h.dstats = c->dstats;
   h.key16 = (c->flags & GLEAM_KEY16) ? 1u : 0u;
@@ -372,6 +379,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   d.arena = c->arena;
   d.index = c->index;
   d.index_mask = c->index_cap - 1;
+  d.hints = c->hints;
   d.nslots = c->nslots;
   d.slot_len = c->slot_len;
   d.dstats = c->dstats;
@@ -457,6 +465,7 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   };
   step(cudaMalloc(&c->arena, nslots * chunk_bytes));
   step(cudaMalloc(&c->index, c->index_cap * sizeof(IndexEntry)));
+  step(cudaMalloc(&c->hints, c->index_cap * sizeof(IndexEntry)));
   step(cudaMalloc(&c->slot_len, nslots * sizeof(uint32_t)));
   step(cudaMalloc(&c->dstats, ST_COUNT * sizeof(unsigned long long)));
   step(cudaMalloc(&c->ctl, sizeof(DevCtl)));
@@ -475,6 +484,7 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   if (rc == GLEAM_OK) step(cudaMalloc(&c->bcount, (c->coop_max_blocks + 1) * sizeof(uint32_t)));
   if (rc == GLEAM_OK) {
     step(cudaMemset(c->index, 0xFF, c->index_cap * sizeof(IndexEntry)));
+    step(cudaMemset(c->hints, 0xFF, c->index_cap * sizeof(IndexEntry)));
     step(cudaMemset(c->dstats, 0, ST_COUNT * sizeof(unsigned long long)));
     step(cudaMemset(c->ctl, 0, sizeof(DevCtl)));
     step(cudaEventRecord(c->done, nullptr));
@@ -717,9 +727,13 @@ int gleam_cache_snapshot(gleam_cache_t* c, gleam_snapshot_t** out) {
   s->owner = c;
   s->index_cap = c->index_cap;
   rc = cuda_err(cudaMalloc(&s->index, c->index_cap * sizeof(IndexEntry)));
+  if (rc == GLEAM_OK) rc = cuda_err(cudaMalloc(&s->hints, c->index_cap * sizeof(IndexEntry)));
   if (rc == GLEAM_OK) rc = cuda_err(cudaMalloc(&s->dstats, ST_COUNT * sizeof(unsigned long long)));
   if (rc == GLEAM_OK)
     rc = cuda_err(cudaMemcpy(s->index, c->index, c->index_cap * sizeof(IndexEntry),
+                             cudaMemcpyDeviceToDevice));
+  if (rc == GLEAM_OK)
+    rc = cuda_err(cudaMemcpy(s->hints, c->hints, c->index_cap * sizeof(IndexEntry),
                              cudaMemcpyDeviceToDevice));
   if (rc == GLEAM_OK)
     rc = cuda_err(cudaMemcpy(s->dstats, c->dstats, ST_COUNT * sizeof(unsigned long long),
@@ -743,6 +757,9 @@ int gleam_cache_restore(gleam_cache_t* c, const gleam_snapshot_t* s) {
     rc = cuda_err(cudaMemcpyAsync(c->index, s->index, c->index_cap * sizeof(IndexEntry),
                                   cudaMemcpyDeviceToDevice, nullptr));
   if (rc == GLEAM_OK)
+    rc = cuda_err(cudaMemcpyAsync(c->hints, s->hints, c->index_cap * sizeof(IndexEntry),
+                                  cudaMemcpyDeviceToDevice, nullptr));
+  if (rc == GLEAM_OK)
     rc = cuda_err(cudaMemcpyAsync(c->dstats, s->dstats, ST_COUNT * sizeof(unsigned long long),
                                   cudaMemcpyDeviceToDevice, nullptr));
   if (rc == GLEAM_OK) rc = cuda_err(cudaEventRecord(c->done, nullptr));
@@ -754,6 +771,7 @@ void gleam_snapshot_destroy(gleam_snapshot_t* s) {
   DeviceGuard g(s->device);
   cudaDeviceSynchronize();
   if (s->index) cudaFree(s->index);
+  if (s->hints) cudaFree(s->hints);
   if (s->dstats) cudaFree(s->dstats);
   cudaGetLastError();
   delete s;

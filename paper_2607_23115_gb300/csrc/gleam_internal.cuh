@@ -102,7 +102,18 @@ struct ChunkArrays {
   uint32_t* res;             // resolution word (kRes*)
   uint32_t* ent;             // group-table entry; the leader's number once a duplicate
   uint32_t* rank;            // exclusive count of misses before the chunk
+  unsigned long long* hint;  // prefix hint (chunks of at least kPrefixBytes)
 };
+
+// Speculative verify.  After the first kPrefixBytes of a chunk the four XXH64
+// lane accumulators are folded into a 64-bit prefix hint; a second table
+// (same layout as the index, key = hint) maps it to the slot of a cached chunk
+// that began with the same bytes.  The rest of the chunk is then hashed and
+// compared against that slot in the same pass, so a hit reads the payload
+// once.  The hint only chooses what to compare against: a chunk is a hit only
+// if the index (keyed by the full XXH64) lists the slot, and every other
+// key+length candidate is still compared byte for byte.
+constexpr uint32_t kPrefixBytes = 512;
 
 struct HashArgs {
   const PayloadDesc* table;  // count > 1
@@ -114,6 +125,7 @@ struct HashArgs {
   // probe + verify (index == nullptr: fingerprint only)
   const IndexEntry* index;
   unsigned long long index_mask;
+  const IndexEntry* hints;   // prefix-hint table (same size as the index)
   const uint8_t* arena;
   const unsigned long long* dstats;
   uint32_t key16;
@@ -130,6 +142,7 @@ struct DedupArgs {
   uint8_t* arena;
   IndexEntry* index;
   unsigned long long index_mask;
+  IndexEntry* hints;
   unsigned long long nslots;
   uint32_t* slot_len;
   unsigned long long* dstats;

@@ -7,8 +7,12 @@
 // each 32-byte stripe straight from HBM (8 loads in flight per thread, the
 // next batch issued before the current one is folded in).  A warp therefore
 // streams 8 chunks at once and every 32-byte sector it touches is used whole.
-// The group then probes the index and compares each key+length candidate
-// with the cached copy, 8 bytes per thread per stripe.
+// After the first 512 bytes the group looks its prefix hint up and, if a
+// cached chunk began the same way, streams that copy alongside the payload
+// and compares as it hashes (speculative verify).  The group then probes the
+// index with the full fingerprint; the hinted slot is a hit if it is a
+// key+length candidate and compared equal, and any other candidate is
+// compared by re-reading both copies.
 #include "gleam_internal.cuh"
 #include "xxh64_device.cuh"
 
@@ -68,6 +72,76 @@ __device__ __forceinline__ unsigned long long lane_stripes(unsigned long long ac
   return acc;
 }
 
+// Lane accumulator over stripes [s0, s1) while comparing every payload word
+// with the cached copy's word at q (p, q already offset by 8*lane).  `cmp`
+// turns off, for the whole group, as soon as any word differs; diff then
+// stays non-zero.  Loads of the next batch are issued before the current one
+// is folded in.
+template <bool kAligned>
+__device__ __forceinline__ unsigned long long lane_stripes_cmp(
+    unsigned long long acc, const uint8_t* p, const uint8_t* q, uint32_t s0, uint32_t s1,
+    unsigned long long& diff, bool& cmp, unsigned gmask) {
+  constexpr int B = kBatch;
+  unsigned long long x[B], y[B];
+  uint32_t s = s0;
+  uint32_t m = min((uint32_t)B, s1 - s);
+#pragma unroll
+  for (int u = 0; u < B; ++u) {
+    x[u] = (uint32_t)u < m ? load_word<kAligned>(p + (uint64_t)(s + u) * 32) : 0ULL;
+    y[u] = (cmp && (uint32_t)u < m) ? load_arena_word(q + (uint64_t)(s + u) * 32) : x[u];
+  }
+  while (s < s1) {
+    const uint32_t sn = s + m;
+    const uint32_t mn = sn < s1 ? min((uint32_t)B, s1 - sn) : 0u;
+    unsigned long long xn[B], yn[B];
+#pragma unroll
+    for (int u = 0; u < B; ++u) {
+      xn[u] = (uint32_t)u < mn ? load_word<kAligned>(p + (uint64_t)(sn + u) * 32) : 0ULL;
+      yn[u] = (cmp && (uint32_t)u < mn) ? load_arena_word(q + (uint64_t)(sn + u) * 32) : xn[u];
+    }
+    unsigned long long d = 0;
+#pragma unroll
+    for (int u = 0; u < B; ++u) {
+      if ((uint32_t)u < m) {
+        acc = xstep(acc, x[u]);
+        d |= x[u] ^ y[u];
+      }
+    }
+    if (cmp) {
+      diff |= d;
+      unsigned long long g = diff;
+      g |= __shfl_xor_sync(gmask, g, 1);
+      g |= __shfl_xor_sync(gmask, g, 2);
+      if (g) {
+        cmp = false;
+        diff = 1;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < B; ++u) {
+      x[u] = xn[u];
+      y[u] = yn[u];
+    }
+    s = sn;
+    m = mn;
+  }
+  return acc;
+}
+
+// Slot of a cached chunk of length len whose prefix hint is h, or kEmptySlot.
+__device__ __forceinline__ uint32_t hint_lookup(const IndexEntry* t, unsigned long long mask,
+                                                unsigned long long h, uint32_t len,
+                                                unsigned long long slots_used) {
+  unsigned long long pos = mix64(h) & mask;
+  for (unsigned long long probe = 0; probe <= mask; ++probe) {
+    const IndexEntry e = t[pos];
+    if (e.slot == kEmptySlot) return kEmptySlot;
+    if (e.key == h && e.len == len && e.slot < slots_used) return e.slot;
+    pos = (pos + 1) & mask;
+  }
+  return kEmptySlot;
+}
+
 // Byte equality of payload chunk p and cached chunk q over len bytes, by the
 // 4-thread group; leaves early once any word differs.
 template <bool kAligned>
@@ -122,9 +196,45 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
   const uint8_t* p = buf + start;
   const uint32_t ns = len >> 5;
 
+  const bool speculate = kProbe && len >= kPrefixBytes;
+  const unsigned long long slots_used = kProbe ? a.dstats[ST_SLOTS_USED] : 0ULL;
+  unsigned long long hint = 0, diff = 0;
+  uint32_t hint_slot = kEmptySlot;
+  bool cmp = false;
+
   unsigned long long h;
   if (ns) {
-    const unsigned long long acc = lane_stripes<kAligned>(xlane_start(lane), p + 8 * lane, ns);
+    unsigned long long acc = xlane_start(lane);
+    if (speculate) {
+      constexpr uint32_t kPre = kPrefixBytes / 32;
+      acc = lane_stripes<kAligned>(acc, p + 8 * lane, kPre);
+      const unsigned long long b0 = group_shfl(acc, gmask, gbase + 0);
+      const unsigned long long b1 = group_shfl(acc, gmask, gbase + 1);
+      const unsigned long long b2 = group_shfl(acc, gmask, gbase + 2);
+      const unsigned long long b3 = group_shfl(acc, gmask, gbase + 3);
+      hint = b0 ^ xrotl(b1, 16) ^ xrotl(b2, 32) ^ xrotl(b3, 48);
+      hint_slot = hint_lookup(a.hints, a.index_mask, hint, len, slots_used);
+      const uint8_t* q = a.arena + (unsigned long long)hint_slot * a.C;
+      cmp = hint_slot != kEmptySlot;
+      if (cmp) {  // the prefix, already hashed, is compared once (payload words from L2)
+        unsigned long long d = 0;
+#pragma unroll 4
+        for (uint32_t s = 0; s < kPre; ++s) {
+          const uint64_t off = (uint64_t)s * 32 + 8 * lane;
+          d |= load_word<kAligned>(p + off) ^ load_arena_word(q + off);
+        }
+        d |= __shfl_xor_sync(gmask, d, 1);
+        d |= __shfl_xor_sync(gmask, d, 2);
+        if (d) {
+          cmp = false;
+          diff = 1;
+        }
+      }
+      acc = lane_stripes_cmp<kAligned>(acc, p + 8 * lane, q + 8 * lane, kPre, ns, diff, cmp,
+                                       gmask);
+    } else {
+      acc = lane_stripes<kAligned>(acc, p + 8 * lane, ns);
+    }
     const unsigned long long a0 = group_shfl(acc, gmask, gbase + 0);
     const unsigned long long a1 = group_shfl(acc, gmask, gbase + 1);
     const unsigned long long a2 = group_shfl(acc, gmask, gbase + 2);
@@ -139,8 +249,20 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
   if (a.fp_out != nullptr && lane == 0) a.fp_out[g] = h;
   if (!kProbe) return;
 
+  // the bytes after the last full stripe, for the speculative compare
+  bool spec_equal = false;
+  if (speculate && hint_slot != kEmptySlot) {
+    unsigned long long d = diff;
+    if (cmp && lane == 0) {
+      const uint8_t* q = a.arena + (unsigned long long)hint_slot * a.C;
+      for (uint32_t k = ns * 32; k < len; ++k) d |= (unsigned long long)(p[k] ^ q[k]);
+    }
+    d |= __shfl_xor_sync(gmask, d, 1);
+    d |= __shfl_xor_sync(gmask, d, 2);
+    spec_equal = d == 0;
+  }
+
   const unsigned long long key = a.key16 ? (h & 0xFFFFULL) : h;
-  const unsigned long long slots_used = a.dstats[ST_SLOTS_USED];
   unsigned long long pos = mix64(key) & a.index_mask;
   bool hit = false, cand = false;
   for (unsigned long long probe = 0; probe <= a.index_mask; ++probe) {
@@ -151,6 +273,11 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
       if (e.slot >= slots_used) {
         // an entry pointing past the used slots: report, never read it
         if (lane == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+      } else if (e.slot == hint_slot) {
+        if (spec_equal) {  // compared in the streaming pass
+          hit = true;
+          break;
+        }
       } else if (group_equal<kAligned>(p, a.arena + (uint64_t)e.slot * a.C, len, lane, gmask)) {
         hit = true;
         break;
@@ -164,6 +291,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
     a.ch.len[g] = len;
     a.ch.src[g] = (unsigned long long)p;
     a.ch.pidx[g] = pid;
+    a.ch.hint[g] = hint;
   }
 }
 

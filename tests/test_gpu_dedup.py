@@ -216,3 +216,20 @@ def test_snapshot_restore_repeats_identically():
         assert n1 == n2 and gc.stats() == st1
         assert torch.equal(o1.hit_mask, o2.hit_mask) and torch.equal(o1.miss_idx[:n1], o2.miss_idx[:n2])
         snap.close()
+
+
+@pytest.mark.parametrize("key16", [False, True])
+def test_prefix_hint_pointing_at_the_wrong_chunk(key16):
+    """Cached chunks A = X|Y1 and B = X|Y2 share their first 2 KiB, so the
+    prefix hint of X|Y2 may name A; the result must still be a hit on B, and
+    X|Y3 a miss.  Also covers tails longer than the prefix."""
+    C = 4 * KiB
+    flags = B.GLEAM_KEY16 if key16 else 0
+    gc, oc = _pair(64 * C, C, flags)
+    X = W.random_bytes(2 * KiB, seed=41)
+    Y = [W.random_bytes(2 * KiB, seed=42 + k) for k in range(4)]
+    with gc:
+        dedup_both(gc, oc, torch.cat([X, Y[0], X, Y[1]]))
+        dedup_both(gc, oc, torch.cat([X, Y[1], X, Y[2], X, Y[0], X[:1000]]))
+        dedup_both(gc, oc, torch.cat([X, Y[3], X, Y[2], X[:1000]]))
+        compare_cache(gc, oc)
