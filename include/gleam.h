@@ -176,6 +176,34 @@ int gleam_dedup_copy_async(gleam_cache_t* cache, const void* d_buf, size_t n,
 int gleam_dedup_copy_batch(gleam_cache_t* cache, const gleam_payload_t* payloads, size_t count,
                            gleam_result_t* d_total, gleam_stream_t stream);
 
+/* ---- dedup without allocation -------------------------------------------
+ * No counterpart in the paper: an addition for callers that cannot allocate
+ * device memory while they run, e.g. code executing inside an intercepted CUDA
+ * call (the server side of an API-remoting layer handling a host-to-device
+ * copy), where a cudaMalloc would re-enter the interception or disturb the
+ * memory map it keeps for the application.
+ *
+ * Same operation, outputs and cache update as gleam_dedup_copy_async, but the
+ * per-call workspace is one fixed array of about 4.3 MiB in the library's
+ * device image instead of memory allocated by the cache; the call itself only
+ * enqueues memsets and kernels and allocates nothing.  Every GPU that loads
+ * the library holds that array until the process exits.
+ *  - Payloads of more than GLEAM_NOALLOC_MAX_CHUNKS chunks (ceil(n / C)) are
+ *    rejected with GLEAM_ERR_INVALID_ARG; use gleam_dedup_copy_async for them.
+ *  - The first call on a device looks the array's device address up (which
+ *    may load the library's device code on that GPU); make that first call
+ *    before any stream capture.
+ *  - All calls on a GPU, from every cache, share the one array and it keeps
+ *    the last call's contents (the call clears what must start at zero).
+ *    Calls that overlap on the GPU race and give wrong results: order them
+ *    (one stream, or events).  Calls on one cache are ordered automatically.
+ *  - d_result (device, may be NULL) receives the outcome, as for
+ *    gleam_dedup_copy_async; n == 0 returns GLEAM_OK and does nothing. */
+#define GLEAM_NOALLOC_MAX_CHUNKS 65536
+int gleam_dedup_copy_noalloc(gleam_cache_t* cache, const void* d_buf, size_t n,
+                             uint32_t* d_hit_mask, uint32_t* d_miss_idx, void* d_miss_bytes,
+                             gleam_result_t* d_result, gleam_stream_t stream);
+
 /* Copies the cache's counters to *out (host struct).  Waits for the cache's
  * outstanding work on the device. */
 int gleam_cache_stats(const gleam_cache_t* cache, gleam_stats_t* out);

@@ -31,7 +31,8 @@ GLEAM_DEBUG_SKIP_ARRIVE = 2
 EXPORTS = (
     "gleam_cache_create", "gleam_cache_create_ex", "gleam_cache_destroy",
     "gleam_cache_reserve", "gleam_fingerprint", "gleam_dedup_copy",
-    "gleam_dedup_copy_async", "gleam_dedup_copy_batch", "gleam_cache_stats", "gleam_cache_export",
+    "gleam_dedup_copy_async", "gleam_dedup_copy_batch", "gleam_dedup_copy_noalloc",
+    "gleam_cache_stats", "gleam_cache_export",
     "gleam_cache_read_slot", "gleam_cache_debug_insert", "gleam_cache_debug_set",
     "gleam_cache_snapshot", "gleam_cache_restore", "gleam_snapshot_destroy",
     "gleam_cache_profile", "gleam_cache_profile_read", "gleam_status_string",
@@ -85,6 +86,7 @@ def lib() -> ctypes.CDLL:
         "gleam_dedup_copy": (ctypes.c_int64, [vp, vp, sz, vp, vp, vp]),
         "gleam_dedup_copy_async": (i32, [vp, vp, sz, vp, vp, vp, vp, vp]),
         "gleam_dedup_copy_batch": (i32, [vp, ctypes.POINTER(gleam_payload_t), sz, vp, vp]),
+        "gleam_dedup_copy_noalloc": (i32, [vp, vp, sz, vp, vp, vp, vp, vp]),
         "gleam_cache_stats": (i32, [vp, ctypes.POINTER(gleam_stats_t)]),
         "gleam_cache_export": (i32, [vp, vp, vp, u64, ctypes.POINTER(u64)]),
         "gleam_cache_read_slot": (i32, [vp, u64, vp, u64, ctypes.POINTER(u64)]),
@@ -165,6 +167,19 @@ def gleam_dedup_copy_async(cache, d_buf, n: int, d_hit_mask, d_miss_idx, d_miss_
     return lib().gleam_dedup_copy_async(cache, _ptr(d_buf), n, _ptr(d_hit_mask),
                                         _ptr(d_miss_idx), _ptr(d_miss_bytes), _ptr(d_result),
                                         _stream(stream))
+
+
+GLEAM_NOALLOC_MAX_CHUNKS = 65536
+
+
+def gleam_dedup_copy_noalloc(cache, d_buf, n: int, d_hit_mask, d_miss_idx, d_miss_bytes,
+                             d_result=None, stream=None) -> int:
+    """The dedup call for callers that cannot allocate: a fixed library-owned
+    scratch array replaces the cache's workspace (at most
+    GLEAM_NOALLOC_MAX_CHUNKS chunks per call)."""
+    return lib().gleam_dedup_copy_noalloc(cache, _ptr(d_buf), n, _ptr(d_hit_mask),
+                                          _ptr(d_miss_idx), _ptr(d_miss_bytes), _ptr(d_result),
+                                          _stream(stream))
 
 
 def payload_array(payloads):

@@ -778,3 +778,152 @@ void gleam_snapshot_destroy(gleam_snapshot_t* s) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Dedup without allocation (gleam_dedup_copy_noalloc)
+//
+// For callers that must not allocate device memory while they run -- typically
+// code that executes inside an intercepted CUDA call, such as the server side
+// of an API-remoting layer handling a host-to-device copy, where calling
+// cudaMalloc again would re-enter the interception or disturb the memory map
+// it keeps for the application.  The per-call workspace of the normal path
+// (grown with cudaMalloc on demand) is replaced here by one fixed array in the
+// library's device image, so a call only launches kernels and memsets.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr uint64_t kNaChunks = GLEAM_NOALLOC_MAX_CHUNKS;  // chunks per call, at most
+constexpr uint64_t kNaTable = 2 * kNaChunks;               // group-table entries (power of 2)
+constexpr uint64_t kNaBlocks = 4096;                       // block-count words
+
+constexpr uint64_t na_align(uint64_t x) { return (x + 255) & ~255ull; }
+constexpr uint64_t kNaOffStatus = 0;
+constexpr uint64_t kNaOffKey = kNaOffStatus + na_align(kNaChunks);
+constexpr uint64_t kNaOffLen = kNaOffKey + na_align(kNaChunks * 8);
+constexpr uint64_t kNaOffSrc = kNaOffLen + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffPidx = kNaOffSrc + na_align(kNaChunks * 8);
+constexpr uint64_t kNaOffRes = kNaOffPidx + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffEnt = kNaOffRes + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffRank = kNaOffEnt + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffHint = kNaOffRank + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffTbl = kNaOffHint + na_align(kNaChunks * 8);
+constexpr uint64_t kNaOffCtl = kNaOffTbl + na_align(kNaTable * sizeof(CallEntry));
+constexpr uint64_t kNaOffBcount = kNaOffCtl + na_align(sizeof(DevCtl));
+constexpr uint64_t kNaOffResult = kNaOffBcount + na_align((kNaBlocks + 1) * 4);
+constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~4.3 MiB
+
+}  // namespace
+
+// The scratch of every gleam_dedup_copy_noalloc call on this GPU.  Host code
+// must not use this name as an address: it stands for the host-side shadow.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNaBytes];
+
+namespace {
+
+constexpr int kNaMaxDevices = 128;
+std::mutex g_na_mu;
+uint8_t* g_na_ptr[kNaMaxDevices] = {};
+
+// Device address of g_noalloc_scratch on `device` (which must be current),
+// looked up once per device.
+int noalloc_scratch(int device, uint8_t** out) {
+  if (device < 0 || device >= kNaMaxDevices) return GLEAM_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(g_na_mu);
+  if (g_na_ptr[device] == nullptr) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || p == nullptr) return cuda_err(e == cudaSuccess ? cudaErrorUnknown : e);
+    g_na_ptr[device] = static_cast<uint8_t*>(p);
+  }
+  *out = g_na_ptr[device];
+  return GLEAM_OK;
+}
+
+}  // namespace
+
+extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, size_t n,
+                                        uint32_t* d_hit_mask, uint32_t* d_miss_idx,
+                                        void* d_miss_bytes, gleam_result_t* d_result,
+                                        gleam_stream_t stream) {
+  if (!c) return GLEAM_ERR_INVALID_ARG;
+  if (n == 0) return GLEAM_OK;
+  const uint64_t N = (n + c->C - 1) / c->C;
+  if (N > kNaChunks) return GLEAM_ERR_INVALID_ARG;  // beyond the fixed scratch
+  std::lock_guard<std::mutex> lk(c->mu);
+  DeviceGuard g(c->device);
+  if ((uint64_t)c->coop_max_blocks + 1 > kNaBlocks) return GLEAM_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint8_t* base = nullptr;
+  int rc = noalloc_scratch(c->device, &base);
+  if (rc != GLEAM_OK) return rc;
+
+  const gleam_payload_t p = make_payload(d_buf, n, d_hit_mask, d_miss_idx, d_miss_bytes, d_result);
+  PtrChecker chk(c->device);
+  PayloadDesc one{};
+  if ((rc = describe(c, chk, p, &one)) != GLEAM_OK) return rc;
+  const bool aligned = reinterpret_cast<uintptr_t>(one.buf) % 16 == 0;
+
+  ChunkArrays ch{};
+  ch.status = base + kNaOffStatus;
+  ch.key = reinterpret_cast<unsigned long long*>(base + kNaOffKey);
+  ch.len = reinterpret_cast<uint32_t*>(base + kNaOffLen);
+  ch.src = reinterpret_cast<unsigned long long*>(base + kNaOffSrc);
+  ch.pidx = reinterpret_cast<uint32_t*>(base + kNaOffPidx);
+  ch.res = reinterpret_cast<uint32_t*>(base + kNaOffRes);
+  ch.ent = reinterpret_cast<uint32_t*>(base + kNaOffEnt);
+  ch.rank = reinterpret_cast<uint32_t*>(base + kNaOffRank);
+  ch.hint = reinterpret_cast<unsigned long long*>(base + kNaOffHint);
+  CallEntry* tbl = reinterpret_cast<CallEntry*>(base + kNaOffTbl);
+  DevCtl* ctl = reinterpret_cast<DevCtl*>(base + kNaOffCtl);
+  uint32_t* bcount = reinterpret_cast<uint32_t*>(base + kNaOffBcount);
+  gleam_result_t* total = reinterpret_cast<gleam_result_t*>(base + kNaOffResult);
+  const uint64_t tcap = std::min<uint64_t>(kNaTable, next_pow2(std::max<uint64_t>(64, 2 * N)));
+
+  // the array keeps the previous call's contents: clear what must start at zero
+  if ((rc = cuda_err(cudaStreamWaitEvent(s, c->done, 0))) != GLEAM_OK) return rc;
+  if ((rc = cuda_err(cudaMemsetAsync(ctl, 0, sizeof(DevCtl), s))) != GLEAM_OK) return rc;
+  if ((rc = cuda_err(cudaMemsetAsync(tbl, 0, tcap * sizeof(CallEntry), s))) != GLEAM_OK) return rc;
+
+  HashArgs h{};
+  h.one = one;
+  h.count = 1;
+  h.Ntot = N;
+  h.C = c->C;
+  h.index = c->index;
+  h.index_mask = c->index_cap - 1;
+  h.hints = c->hints;
+  h.arena = c->arena;
+  h.dstats = c->dstats;
+  h.key16 = (c->flags & GLEAM_KEY16) ? 1u : 0u;
+  h.ch = ch;
+  h.ctl = ctl;
+  if ((rc = cuda_err(launch_hash(h, aligned, s))) != GLEAM_OK) return rc;
+
+  DedupArgs d{};
+  d.one = one;
+  d.count = 1;
+  d.Ntot = N;
+  d.C = c->C;
+  d.arena = c->arena;
+  d.index = c->index;
+  d.index_mask = c->index_cap - 1;
+  d.hints = c->hints;
+  d.nslots = c->nslots;
+  d.slot_len = c->slot_len;
+  d.dstats = c->dstats;
+  d.ch = ch;
+  d.pstart = bcount + kNaBlocks;
+  d.tbl = tbl;
+  d.tbl_mask = tcap - 1;
+  d.bcount = bcount;
+  d.ctl = ctl;
+  d.total = total;
+  d.ncalls = 1;
+  d.wait_ns = c->wait_ns;
+  d.skip_block = -1;
+  const int per_block = 4 * dedup_threads();
+  const int grid = (int)std::max<uint64_t>(
+      1, std::min<uint64_t>(c->coop_max_blocks, (N + per_block - 1) / per_block));
+  if ((rc = cuda_err(launch_dedup(d, grid, s))) != GLEAM_OK) return rc;
+  return cuda_err(cudaEventRecord(c->done, s));
+}
