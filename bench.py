@@ -48,7 +48,7 @@ def parse_args():
     p.add_argument("--steps", type=int, default=100)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["gleam", "reference"], default="gleam")
-    p.add_argument("--workload", choices=["llama3-8b", "llama3-8b-layer", "gpt2-small"], default="llama3-8b")
+    p.add_argument("--workload", choices=["llama3-8b", "llama3-8b-layer", "llama3-8b-4layers", "gpt2-small"], default="llama3-8b")
     p.add_argument("--cpu-sample-bytes", type=int, default=3 * GiB,
                    help="payload bytes of the oracle's bounded CPU sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -76,6 +76,11 @@ def workload_spec(name):
                     dtype=torch.bfloat16, C=64 * KiB, capacity=512 * MiB, flip_frac=0.10,
                     desc="one Llama-3-8B layer (9 bf16 tensors, 436 MB): the small case of "
                          "the llama3-8b workload for ncu captures")
+    if name == "llama3-8b-4layers":
+        return dict(name="llama3-8b-bf16-four-layers", shapes=W.llama3_8b_shapes()[1:37],
+                    dtype=torch.bfloat16, C=64 * KiB, capacity=2 * GiB, flip_frac=0.10,
+                    desc="four Llama-3-8B layers (36 bf16 tensors, 1.74 GB): a few-GB case "
+                         "of the llama3-8b workload for ncu captures")
     if name == "gpt2-small":
         return dict(name="gpt2-small-fp32-per-tensor-second-pass", shapes=W.gpt2_small_shapes(),
                     dtype=torch.float32, C=4 * KiB, capacity=1 * GiB, flip_frac=0.0,

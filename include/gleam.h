@@ -184,7 +184,7 @@ int gleam_dedup_copy_batch(gleam_cache_t* cache, const gleam_payload_t* payloads
  * memory map it keeps for the application.
  *
  * Same operation, outputs and cache update as gleam_dedup_copy_async, but the
- * per-call workspace is one fixed array of about 4.3 MiB in the library's
+ * per-call workspace is one fixed array of about 4.6 MiB in the library's
  * device image instead of memory allocated by the cache; the call itself only
  * enqueues memsets and kernels and allocates nothing.  Every GPU that loads
  * the library holds that array until the process exits.

@@ -35,6 +35,16 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
+#ifndef GLEAM_COPY_VEC
+#define GLEAM_COPY_VEC 8
+#endif
+#ifndef GLEAM_DEDUP_BLOCKS_PER_SM
+#define GLEAM_DEDUP_BLOCKS_PER_SM 3
+#endif
+#ifndef GLEAM_DEDUP_CHUNKS_PER_BLOCK
+#define GLEAM_DEDUP_CHUNKS_PER_BLOCK 1024
+#endif
+constexpr int kCopyVec = GLEAM_COPY_VEC;  // 16-byte vectors per lane in flight while copying
 
 __device__ __forceinline__ uint32_t ldcg_u32(const uint32_t* p) { return __ldcg(p); }
 
@@ -80,15 +90,15 @@ __device__ void warp_copy2(uint8_t* d1, uint8_t* d2, const uint8_t* s, uint32_t 
     const uint4* sv = reinterpret_cast<const uint4*>(s);
     uint4* d1v = reinterpret_cast<uint4*>(d1);
     uint4* d2v = reinterpret_cast<uint4*>(d2);
-    for (uint32_t k0 = 0; k0 < nv; k0 += 128) {
-      uint4 u[4];
+    for (uint32_t k0 = 0; k0 < nv; k0 += 32 * kCopyVec) {
+      uint4 u[kCopyVec];
 #pragma unroll
-      for (int r = 0; r < 4; ++r) {
+      for (int r = 0; r < kCopyVec; ++r) {
         const uint32_t k = k0 + r * 32 + lane;
         if (k < nv) u[r] = __ldcs(sv + k);
       }
 #pragma unroll
-      for (int r = 0; r < 4; ++r) {
+      for (int r = 0; r < kCopyVec; ++r) {
         const uint32_t k = k0 + r * 32 + lane;
         if (k < nv) {
           __stcs(d1v + k, u[r]);
@@ -167,8 +177,6 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ uint32_t warp_cnt[kWarps];
   __shared__ uint32_t warp_off[kWarps];
-  __shared__ uint32_t list_g[kThreads];
-  __shared__ uint32_t list_r[kThreads];
   __shared__ unsigned long long s_slots0;
 
   const uint32_t G = gridDim.x;
@@ -318,6 +326,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       if (valid) {
         const uint32_t r = (uint32_t)(running + warp_off[w] + __popc(mb & ((1u << lane) - 1u)));
         ch.rank[g] = r;
+        if (miss) ch.order[r] = g;
         const uint32_t p = ch.pidx[g];
         if (g == desc(a, p).chunk_base) a.pstart[p] = r;
       }
@@ -364,45 +373,29 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       add_by_key(has_res ? (unsigned long long*)&res->n_miss : nullptr, p, miss, has_res);
       add_by_key(has_res ? (unsigned long long*)&res->verify_rejects : nullptr, p, rej, has_res);
       add_by_key(has_res ? (unsigned long long*)&res->miss_bytes : nullptr, p, len, has_res);
-      // the tile's misses, copied by whole warps
-      const uint32_t mb = __ballot_sync(0xffffffffu, miss);
-      if (lane == 0) warp_cnt[w] = __popc(mb);
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        uint32_t acc = 0;
-        for (int k = 0; k < kWarps; ++k) {
-          warp_off[k] = acc;
-          acc += warp_cnt[k];
-        }
-        warp_cnt[0] = acc;
+    }
+    // every miss, by rank, copied by whole warps of the whole grid
+    const uint32_t gw = blockIdx.x * kWarps + w, nw = G * kWarps;
+    for (unsigned long long r = gw; r < total; r += nw) {
+      const uint32_t gg = __ldcg(&ch.order[r]);
+      const uint32_t pp = ch.pidx[gg];
+      const PayloadDesc& P = desc(a, pp);
+      const unsigned long long rp = r - __ldcg(&a.pstart[pp]);
+      const uint32_t ln = ch.len[gg];
+      const unsigned long long slot = slots0 + r;
+      const uint8_t* src = reinterpret_cast<const uint8_t*>(ch.src[gg]);
+      uint8_t* d1 = P.packed + rp * a.C;
+      uint8_t* d2 = a.arena + slot * a.C;
+      const bool vec = (((uintptr_t)src | (uintptr_t)d1 | (uintptr_t)d2) & 15) == 0;
+      warp_copy2(d1, d2, src, ln, vec);
+      if (lane == 0) {
+        a.slot_len[slot] = ln;
+        if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
+          atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+        if (ln >= kPrefixBytes &&
+            !index_insert(a.hints, a.index_mask, ch.hint[gg], (uint32_t)slot, ln))
+          atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       }
-      __syncthreads();
-      if (miss) list_g[warp_off[w] + __popc(mb & ((1u << lane) - 1u))] = g;
-      const uint32_t tile_total = warp_cnt[0];
-      __syncthreads();
-      for (uint32_t k = w; k < tile_total; k += kWarps) {
-        const uint32_t gg = list_g[k];
-        const uint32_t pp = ch.pidx[gg];
-        const PayloadDesc& P = desc(a, pp);
-        const uint32_t rk = ch.rank[gg];
-        const unsigned long long rp = rk - __ldcg(&a.pstart[pp]);
-        const uint32_t ln = ch.len[gg];
-        const unsigned long long slot = slots0 + rk;
-        const uint8_t* src = reinterpret_cast<const uint8_t*>(ch.src[gg]);
-        uint8_t* d1 = P.packed + rp * a.C;
-        uint8_t* d2 = a.arena + slot * a.C;
-        const bool vec = (((uintptr_t)src | (uintptr_t)d1 | (uintptr_t)d2) & 15) == 0;
-        warp_copy2(d1, d2, src, ln, vec);
-        if (lane == 0) {
-          a.slot_len[slot] = ln;
-          if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
-            atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-          if (ln >= kPrefixBytes &&
-              !index_insert(a.hints, a.index_mask, ch.hint[gg], (uint32_t)slot, ln))
-            atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-        }
-      }
-      __syncthreads();
     }
     n_hc = block_sum<unsigned long long>(n_hc, red64);
     n_hi = block_sum<unsigned long long>(n_hi, red64);
@@ -486,11 +479,14 @@ __global__ void k_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t*
 
 int dedup_threads() { return kThreads; }
 
+int dedup_chunks_per_block() { return GLEAM_DEDUP_CHUNKS_PER_BLOCK; }
+
+// Co-resident blocks per SM for the cooperative launch (capped).
 int dedup_blocks_per_sm() {
   int nb = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_dedup, kThreads, 0) != cudaSuccess)
     return 0;
-  return nb;
+  return nb < GLEAM_DEDUP_BLOCKS_PER_SM ? nb : GLEAM_DEDUP_BLOCKS_PER_SM;
 }
 
 cudaError_t launch_dedup(const DedupArgs& a, int grid, cudaStream_t s) {

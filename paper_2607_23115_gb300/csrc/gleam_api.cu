@@ -189,10 +189,10 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   cap = std::min<uint64_t>(cap, kMaxChunks);
   if (cap < nchunks) cap = nchunks;
   const uint64_t tcap = next_pow2(2 * cap);
-  const uint64_t sz[10] = {align256(cap),     align256(cap * 8), align256(cap * 4),
+  const uint64_t sz[11] = {align256(cap),     align256(cap * 8), align256(cap * 4),
                            align256(cap * 8), align256(cap * 4), align256(cap * 4),
                            align256(cap * 4), align256(cap * 4), align256(cap * 8),
-                           align256(tcap * sizeof(CallEntry))};
+                           align256(cap * 4), align256(tcap * sizeof(CallEntry))};
   uint64_t total = 0;
   for (uint64_t x : sz) total += x;
   int rc = cuda_err(cudaEventSynchronize(c->done));
@@ -220,6 +220,8 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   b += sz[7];
   c->ch.hint = reinterpret_cast<unsigned long long*>(b);
   b += sz[8];
+  c->ch.order = reinterpret_cast<uint32_t*>(b);
+  b += sz[9];
   c->tbl = reinterpret_cast<CallEntry*>(b);
   c->tbl_cap = tcap;
   c->ws_chunks = cap;
@@ -296,6 +298,18 @@ int describe(gleam_cache* c, PtrChecker& chk, const gleam_payload_t& p, PayloadD
   return GLEAM_OK;
 }
 
+// Blocks of the cooperative dedup launch: enough for its per-chunk phases
+// (chunks / dedup_chunks_per_block) and for its miss copies (one block per
+// kBytesPerDedupBlock of payload), at most the co-resident maximum.
+constexpr uint64_t kBytesPerDedupBlock = 2ull << 20;
+
+int dedup_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
+  const uint64_t per_block = dedup_chunks_per_block();
+  const uint64_t want = std::max<uint64_t>((nchunks + per_block - 1) / per_block,
+                                           (nbytes + kBytesPerDedupBlock - 1) / kBytesPerDedupBlock);
+  return (int)std::max<uint64_t>(1, std::min<uint64_t>(c->coop_max_blocks, want));
+}
+
 // Enqueues one dedup call over `count` payloads on stream s, ordered after
 // the cache's previous call.  Caller holds c->mu and the device.
 int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
@@ -312,7 +326,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     // the staging buffer may still feed the previous call's table copy
     if ((rc = cuda_err(cudaEventSynchronize(c->table_copied))) != GLEAM_OK) return rc;
   }
-  uint64_t Ntot = 0, ncalls = 0;
+  uint64_t Ntot = 0, ncalls = 0, nbytes = 0;
   bool aligned = true;
   for (uint64_t k = 0; k < count; ++k) {
     PayloadDesc* d = count > 1 ? &c->h_table[k] : &one;
@@ -322,6 +336,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     if (Ntot > kMaxChunks) return GLEAM_ERR_INVALID_ARG;
     if (d->n) {
       ++ncalls;
+      nbytes += d->n;
       aligned = aligned && (reinterpret_cast<uintptr_t>(d->buf) % 16 == 0);
     }
   }
@@ -394,9 +409,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   d.wait_ns = c->wait_ns;
   d.skip_block = c->skip_block;
   c->skip_block = -1;  // the hook applies to one call
-  const int per_block = 4 * dedup_threads();
-  int grid = (int)std::max<uint64_t>(
-      1, std::min<uint64_t>(c->coop_max_blocks, (Ntot + per_block - 1) / per_block));
+  int grid = dedup_grid(c, Ntot, nbytes);
   if (d.skip_block >= 0) {
     grid = std::max(grid, std::min(2, c->coop_max_blocks));  // someone must be left waiting
     if (d.skip_block >= grid) d.skip_block = grid - 1;
@@ -476,7 +489,7 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   if (rc == GLEAM_OK) {
     int sms = 0;
     step(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device));
-    const int per_sm = std::min(2, dedup_blocks_per_sm());
+    const int per_sm = dedup_blocks_per_sm();
     c->coop_max_blocks = sms * per_sm;
     if (c->coop_max_blocks <= 0) rc = GLEAM_ERR_CUDA;
   }
@@ -806,11 +819,12 @@ constexpr uint64_t kNaOffRes = kNaOffPidx + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffEnt = kNaOffRes + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffRank = kNaOffEnt + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffHint = kNaOffRank + na_align(kNaChunks * 4);
-constexpr uint64_t kNaOffTbl = kNaOffHint + na_align(kNaChunks * 8);
+constexpr uint64_t kNaOffOrder = kNaOffHint + na_align(kNaChunks * 8);
+constexpr uint64_t kNaOffTbl = kNaOffOrder + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffCtl = kNaOffTbl + na_align(kNaTable * sizeof(CallEntry));
 constexpr uint64_t kNaOffBcount = kNaOffCtl + na_align(sizeof(DevCtl));
 constexpr uint64_t kNaOffResult = kNaOffBcount + na_align((kNaBlocks + 1) * 4);
-constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~4.3 MiB
+constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~4.6 MiB
 
 }  // namespace
 
@@ -873,6 +887,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   ch.ent = reinterpret_cast<uint32_t*>(base + kNaOffEnt);
   ch.rank = reinterpret_cast<uint32_t*>(base + kNaOffRank);
   ch.hint = reinterpret_cast<unsigned long long*>(base + kNaOffHint);
+  ch.order = reinterpret_cast<uint32_t*>(base + kNaOffOrder);
   CallEntry* tbl = reinterpret_cast<CallEntry*>(base + kNaOffTbl);
   DevCtl* ctl = reinterpret_cast<DevCtl*>(base + kNaOffCtl);
   uint32_t* bcount = reinterpret_cast<uint32_t*>(base + kNaOffBcount);
@@ -921,9 +936,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.ncalls = 1;
   d.wait_ns = c->wait_ns;
   d.skip_block = -1;
-  const int per_block = 4 * dedup_threads();
-  const int grid = (int)std::max<uint64_t>(
-      1, std::min<uint64_t>(c->coop_max_blocks, (N + per_block - 1) / per_block));
+  const int grid = dedup_grid(c, N, n);
   if ((rc = cuda_err(launch_dedup(d, grid, s))) != GLEAM_OK) return rc;
   return cuda_err(cudaEventRecord(c->done, s));
 }

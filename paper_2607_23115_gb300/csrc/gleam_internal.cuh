@@ -103,6 +103,7 @@ struct ChunkArrays {
   uint32_t* ent;             // group-table entry; the leader's number once a duplicate
   uint32_t* rank;            // exclusive count of misses before the chunk
   unsigned long long* hint;  // prefix hint (chunks of at least kPrefixBytes)
+  uint32_t* order;           // order[r] = chunk number of the miss of rank r
 };
 
 // Speculative verify.  After the first kPrefixBytes of a chunk the four XXH64
@@ -164,6 +165,7 @@ cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t
                                 unsigned long long* dstats, unsigned long long key,
                                 uint32_t slot, uint32_t len, DevCtl* ctl, cudaStream_t s);
 int dedup_threads();
+int dedup_chunks_per_block();
 int dedup_blocks_per_sm();
 
 // ---------------------------------------------------------------------------

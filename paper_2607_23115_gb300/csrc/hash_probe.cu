@@ -19,8 +19,14 @@
 namespace gleam {
 namespace {
 
-constexpr int kHashThreads = 256;
-constexpr int kBatch = 8;  // stripes per thread in flight
+#ifndef GLEAM_HASH_BATCH
+#define GLEAM_HASH_BATCH 8
+#endif
+#ifndef GLEAM_HASH_THREADS
+#define GLEAM_HASH_THREADS 256
+#endif
+constexpr int kHashThreads = GLEAM_HASH_THREADS;
+constexpr int kBatch = GLEAM_HASH_BATCH;  // stripes per thread in flight
 
 // 8-byte load of read-only payload bytes, no L1 allocation, L2 fetches 256 B.
 template <bool kAligned>
