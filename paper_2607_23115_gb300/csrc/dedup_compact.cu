@@ -35,6 +35,9 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
+#ifndef GLEAM_COPY_STREAMING_STORES
+#define GLEAM_COPY_STREAMING_STORES 1
+#endif
 #ifndef GLEAM_COPY_VEC
 #define GLEAM_COPY_VEC 8
 #endif
@@ -95,14 +98,19 @@ __device__ void warp_copy2(uint8_t* d1, uint8_t* d2, const uint8_t* s, uint32_t 
 #pragma unroll
       for (int r = 0; r < kCopyVec; ++r) {
         const uint32_t k = k0 + r * 32 + lane;
-        if (k < nv) u[r] = __ldcs(sv + k);
+        if (k < nv) u[r] = __ldg(sv + k);
       }
 #pragma unroll
       for (int r = 0; r < kCopyVec; ++r) {
         const uint32_t k = k0 + r * 32 + lane;
         if (k < nv) {
+#if GLEAM_COPY_STREAMING_STORES
           __stcs(d1v + k, u[r]);
           __stcs(d2v + k, u[r]);
+#else
+          d1v[k] = u[r];
+          d2v[k] = u[r];
+#endif
         }
       }
     }
