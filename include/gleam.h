@@ -176,6 +176,21 @@ int gleam_dedup_copy_async(gleam_cache_t* cache, const void* d_buf, size_t n,
 int gleam_dedup_copy_batch(gleam_cache_t* cache, const gleam_payload_t* payloads, size_t count,
                            gleam_result_t* d_total, gleam_stream_t stream);
 
+/* Host-resident payloads (paper Sec. 4.1.2 in its own order: the sender
+ * decides what to send before anything is copied).  The payload stays in
+ * page-locked host memory (cudaHostAlloc, or cudaHostRegister of existing
+ * memory); the kernels read it in place over the CPU-GPU link, so the whole
+ * payload is never written to device memory: only the misses are, to the
+ * packed output and the arena.  h_buf / payload d_buf fields: page-locked
+ * host memory (other host memory and device memory are rejected with
+ * GLEAM_ERR_NOT_DEVICE_PTR); outputs: device memory.  Semantics, results and
+ * ordering are those of gleam_dedup_copy_async / gleam_dedup_copy_batch. */
+int gleam_dedup_copy_host_async(gleam_cache_t* cache, const void* h_buf, size_t n,
+                                uint32_t* d_hit_mask, uint32_t* d_miss_idx, void* d_miss_bytes,
+                                gleam_result_t* d_result, gleam_stream_t stream);
+int gleam_dedup_copy_host_batch(gleam_cache_t* cache, const gleam_payload_t* payloads,
+                                size_t count, gleam_result_t* d_total, gleam_stream_t stream);
+
 /* ---- dedup without allocation -------------------------------------------
  * No counterpart in the paper: an addition for callers that cannot allocate
  * device memory while they run, e.g. code executing inside an intercepted CUDA

@@ -32,6 +32,7 @@ EXPORTS = (
     "gleam_cache_create", "gleam_cache_create_ex", "gleam_cache_destroy",
     "gleam_cache_reserve", "gleam_fingerprint", "gleam_dedup_copy",
     "gleam_dedup_copy_async", "gleam_dedup_copy_batch", "gleam_dedup_copy_noalloc",
+    "gleam_dedup_copy_host_async", "gleam_dedup_copy_host_batch",
     "gleam_cache_stats", "gleam_cache_export",
     "gleam_cache_read_slot", "gleam_cache_debug_insert", "gleam_cache_debug_set",
     "gleam_cache_snapshot", "gleam_cache_restore", "gleam_snapshot_destroy",
@@ -87,6 +88,8 @@ def lib() -> ctypes.CDLL:
         "gleam_dedup_copy_async": (i32, [vp, vp, sz, vp, vp, vp, vp, vp]),
         "gleam_dedup_copy_batch": (i32, [vp, ctypes.POINTER(gleam_payload_t), sz, vp, vp]),
         "gleam_dedup_copy_noalloc": (i32, [vp, vp, sz, vp, vp, vp, vp, vp]),
+        "gleam_dedup_copy_host_async": (i32, [vp, vp, sz, vp, vp, vp, vp, vp]),
+        "gleam_dedup_copy_host_batch": (i32, [vp, ctypes.POINTER(gleam_payload_t), sz, vp, vp]),
         "gleam_cache_stats": (i32, [vp, ctypes.POINTER(gleam_stats_t)]),
         "gleam_cache_export": (i32, [vp, vp, vp, u64, ctypes.POINTER(u64)]),
         "gleam_cache_read_slot": (i32, [vp, u64, vp, u64, ctypes.POINTER(u64)]),
@@ -196,6 +199,20 @@ def gleam_dedup_copy_batch(cache, payloads, d_total=None, stream=None) -> int:
     """payloads: a payload_array(), or a sequence of tuples for it."""
     arr = payloads if hasattr(payloads, "count") else payload_array(payloads)
     return lib().gleam_dedup_copy_batch(cache, arr, arr.count, _ptr(d_total), _stream(stream))
+
+
+def gleam_dedup_copy_host_async(cache, h_buf, n: int, d_hit_mask, d_miss_idx, d_miss_bytes,
+                                d_result=None, stream=None) -> int:
+    return lib().gleam_dedup_copy_host_async(cache, _ptr(h_buf), n, _ptr(d_hit_mask),
+                                             _ptr(d_miss_idx), _ptr(d_miss_bytes),
+                                             _ptr(d_result), _stream(stream))
+
+
+def gleam_dedup_copy_host_batch(cache, payloads, d_total=None, stream=None) -> int:
+    """payloads: a payload_array() whose buffers are page-locked host memory."""
+    arr = payloads if hasattr(payloads, "count") else payload_array(payloads)
+    return lib().gleam_dedup_copy_host_batch(cache, arr, arr.count, _ptr(d_total),
+                                             _stream(stream))
 
 
 def gleam_cache_stats(cache):

@@ -108,6 +108,20 @@ class Cache:
         _check(B.gleam_dedup_copy_batch(self.handle, items, total, stream),
                "gleam_dedup_copy_batch")
 
+    def dedup_host(self, hbuf: torch.Tensor, out: DedupOutputs, result=None, stream=None):
+        """Async dedup of a payload in page-locked host memory (read in place)."""
+        n = hbuf.numel() * hbuf.element_size()
+        _check(B.gleam_dedup_copy_host_async(self.handle, hbuf, n, out.hit_mask, out.miss_idx,
+                                             out.miss_bytes, result, stream),
+               "gleam_dedup_copy_host_async")
+
+    def dedup_host_batch(self, hbufs=None, outs=None, results=None, total=None, stream=None,
+                         items=None):
+        if items is None:
+            items = self.batch_items(hbufs, outs, results)
+        _check(B.gleam_dedup_copy_host_batch(self.handle, items, total, stream),
+               "gleam_dedup_copy_host_batch")
+
     def stats(self) -> dict:
         rc, st = B.gleam_cache_stats(self.handle)
         _check(rc, "gleam_cache_stats")

@@ -133,6 +133,33 @@ class PtrChecker {
  public:
   explicit PtrChecker(int device) : device_(device) {}
 
+  // GLEAM_OK iff [p, p + bytes) is page-locked host memory (cudaHostAlloc or
+  // cudaHostRegister) that the device can read; *dev receives the address to
+  // use in device code.
+  int check_host(const void* p, uint64_t bytes, const void** dev) {
+    if (p == nullptr) return GLEAM_ERR_INVALID_ARG;
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+      cudaGetLastError();
+      return GLEAM_ERR_NOT_DEVICE_PTR;
+    }
+    if (at.type != cudaMemoryTypeHost || at.devicePointer == nullptr)
+      return GLEAM_ERR_NOT_DEVICE_PTR;
+    *dev = at.devicePointer;
+    if (PtrAttrsFn fn = driver_ptr_attrs()) {
+      CUpointer_attribute attrs[2] = {CU_POINTER_ATTRIBUTE_RANGE_START_ADDR,
+                                      CU_POINTER_ATTRIBUTE_RANGE_SIZE};
+      CUdeviceptr start = 0;
+      size_t size = 0;
+      void* data[2] = {&start, &size};
+      const uintptr_t a = reinterpret_cast<uintptr_t>(*dev);
+      if (fn(2, attrs, data, (CUdeviceptr)a) == CUDA_SUCCESS && size > 0 &&
+          (a < start || a + bytes > start + size))
+        return GLEAM_ERR_INVALID_ARG;  // span overruns the registration
+    }
+    return GLEAM_OK;
+  }
+
   // GLEAM_OK iff [p, p + bytes) is device memory of the device.
   int check(const void* p, uint64_t bytes) {
     if (p == nullptr) return GLEAM_ERR_INVALID_ARG;
@@ -277,7 +304,8 @@ void destroy_cache(gleam_cache* c) {
 int wait_done(const gleam_cache* c) { return cuda_err(cudaEventSynchronize(c->done)); }
 
 // Validates one payload and fills its device descriptor (chunk_base left 0).
-int describe(gleam_cache* c, PtrChecker& chk, const gleam_payload_t& p, PayloadDesc* d) {
+int describe(gleam_cache* c, PtrChecker& chk, const gleam_payload_t& p, PayloadDesc* d,
+             bool host_payload = false) {
   const uint64_t N = (p.n + c->C - 1) / c->C;
   if (N > kMaxChunks) return GLEAM_ERR_INVALID_ARG;
   d->buf = static_cast<const uint8_t*>(p.d_buf);
@@ -291,7 +319,13 @@ int describe(gleam_cache* c, PtrChecker& chk, const gleam_payload_t& p, PayloadD
   int rc;
   if (p.d_result && (rc = chk.check(p.d_result, sizeof(gleam_result_t))) != GLEAM_OK) return rc;
   if (p.n == 0) return GLEAM_OK;
-  if ((rc = chk.check(p.d_buf, p.n)) != GLEAM_OK) return rc;
+  if (host_payload) {
+    const void* dev = nullptr;
+    if ((rc = chk.check_host(p.d_buf, p.n, &dev)) != GLEAM_OK) return rc;
+    d->buf = static_cast<const uint8_t*>(dev);
+  } else if ((rc = chk.check(p.d_buf, p.n)) != GLEAM_OK) {
+    return rc;
+  }
   if ((rc = chk.check(p.d_hit_mask, ((N + 31) / 32) * 4)) != GLEAM_OK) return rc;
   if ((rc = chk.check(p.d_miss_idx, N * 4)) != GLEAM_OK) return rc;
   if ((rc = chk.check(p.d_miss_bytes, p.n)) != GLEAM_OK) return rc;
@@ -313,7 +347,7 @@ int dedup_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
 // Enqueues one dedup call over `count` payloads on stream s, ordered after
 // the cache's previous call.  Caller holds c->mu and the device.
 int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
-            gleam_result_t* d_total, cudaStream_t s) {
+            gleam_result_t* d_total, cudaStream_t s, bool host_payloads = false) {
   if (count == 0) return GLEAM_OK;
   if (count > 0xFFFFFFFEull) return GLEAM_ERR_INVALID_ARG;
   PtrChecker chk(c->device);
@@ -330,7 +364,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   bool aligned = true;
   for (uint64_t k = 0; k < count; ++k) {
     PayloadDesc* d = count > 1 ? &c->h_table[k] : &one;
-    if ((rc = describe(c, chk, payloads[k], d)) != GLEAM_OK) return rc;
+    if ((rc = describe(c, chk, payloads[k], d, host_payloads)) != GLEAM_OK) return rc;
     d->chunk_base = Ntot;
     Ntot += d->nchunks;
     if (Ntot > kMaxChunks) return GLEAM_ERR_INVALID_ARG;
@@ -591,6 +625,25 @@ int64_t gleam_dedup_copy(gleam_cache_t* c, const void* d_buf, size_t n, uint32_t
   if (rc != GLEAM_OK) return rc;
   if (c->h_result->status != 0) return c->h_result->status;
   return (int64_t)c->h_result->n_miss;
+}
+
+int gleam_dedup_copy_host_batch(gleam_cache_t* c, const gleam_payload_t* payloads, size_t count,
+                                gleam_result_t* d_total, gleam_stream_t stream) {
+  if (!c || (count > 0 && !payloads)) return GLEAM_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(c->mu);
+  DeviceGuard g(c->device);
+  return enqueue(c, payloads, count, d_total, reinterpret_cast<cudaStream_t>(stream), true);
+}
+
+int gleam_dedup_copy_host_async(gleam_cache_t* c, const void* h_buf, size_t n,
+                                uint32_t* d_hit_mask, uint32_t* d_miss_idx, void* d_miss_bytes,
+                                gleam_result_t* d_result, gleam_stream_t stream) {
+  if (!c) return GLEAM_ERR_INVALID_ARG;
+  if (n == 0) return GLEAM_OK;
+  std::lock_guard<std::mutex> lk(c->mu);
+  DeviceGuard g(c->device);
+  const gleam_payload_t p = make_payload(h_buf, n, d_hit_mask, d_miss_idx, d_miss_bytes, d_result);
+  return enqueue(c, &p, 1, nullptr, reinterpret_cast<cudaStream_t>(stream), true);
 }
 
 int gleam_cache_stats(const gleam_cache_t* c, gleam_stats_t* out) {
