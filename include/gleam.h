@@ -99,6 +99,10 @@ typedef struct gleam_payload {
   uint32_t* d_miss_idx;
   void* d_miss_bytes;
   gleam_result_t* d_result;
+  /* optional (may be NULL), device u32[N]: the arena slot that holds chunk i's
+   * bytes after the call -- the byte-equal cached chunk for a hit, the new
+   * slot for a miss.  Records for gleam_block_check come from here. */
+  uint32_t* d_chunk_slot;
 } gleam_payload_t;
 
 /* ---- cache lifetime ---------------------------------------------------- */
@@ -218,6 +222,24 @@ int gleam_dedup_copy_host_batch(gleam_cache_t* cache, const gleam_payload_t* pay
 int gleam_dedup_copy_noalloc(gleam_cache_t* cache, const void* d_buf, size_t n,
                              uint32_t* d_hit_mask, uint32_t* d_miss_idx, void* d_miss_bytes,
                              gleam_result_t* d_result, gleam_stream_t stream);
+
+/* Weight-block identification at cudaFree time (paper Sec. 4.1.1): a block
+ * (one cudaMalloc) is kept as weights only if every chunk written into it by
+ * host-to-device copies is unchanged when it is freed.  Record r says that the
+ * block's bytes at d_offsets[r] were written with the chunk now stored in
+ * cache slot d_slots[r] (from d_chunk_slot of the dedup call that handled the
+ * copy; for segments written more than once, keep the first write's records).
+ * Each record is compared byte for byte with the block's current bytes.
+ *   d_block: device memory of block_bytes bytes; d_offsets u64[nrec] and
+ *   d_slots u32[nrec]: device arrays; d_mismatch: device u8[nrec] or NULL,
+ *   receives 1 for a record whose bytes differ, that does not fit in the
+ *   block, or that names an unused slot, else 0; d_count: device u64, receives
+ *   the number of such records (0 = the block still holds its weights).
+ * Asynchronous on `stream`, ordered after the cache's previous call; reads
+ * the cache, changes nothing. */
+int gleam_block_check(const gleam_cache_t* cache, const void* d_block, size_t block_bytes,
+                      const uint64_t* d_offsets, const uint32_t* d_slots, size_t nrec,
+                      uint8_t* d_mismatch, uint64_t* d_count, gleam_stream_t stream);
 
 /* Copies the cache's counters to *out (host struct).  Waits for the cache's
  * outstanding work on the device. */

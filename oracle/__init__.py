@@ -63,7 +63,9 @@ def lib():
         l.oracle_cache_destroy.restype = None
         l.oracle_cache_destroy.argtypes = [vp]
         l.oracle_dedup.restype = ctypes.c_int64
-        l.oracle_dedup.argtypes = [vp, vp, sz, vp, vp, vp]
+        l.oracle_dedup.argtypes = [vp, vp, sz, vp, vp, vp, vp]
+        l.oracle_block_check.restype = ctypes.c_int64
+        l.oracle_block_check.argtypes = [vp, vp, u64, vp, vp, u64, vp]
         l.oracle_debug_insert.restype = ctypes.c_int
         l.oracle_debug_insert.argtypes = [vp, u64, vp, sz]
         l.oracle_cache_stats.restype = None
@@ -117,8 +119,9 @@ class OracleCache:
     def __del__(self):
         self.close()
 
-    def dedup(self, data):
-        """Returns (rc, hit_mask u32[], miss_idx u32[n_miss], packed u8[packed_bytes])."""
+    def dedup(self, data, chunk_slots: bool = False):
+        """Returns (rc, hit_mask u32[], miss_idx u32[n_miss], packed u8[packed_bytes]),
+        plus the slot holding every chunk's bytes (u32[N]) if chunk_slots."""
         a = _u8(data)
         n = a.size
         C = self.chunk_bytes
@@ -126,8 +129,19 @@ class OracleCache:
         mask = np.zeros(max(1, (nch + 31) // 32), dtype=np.uint32)
         miss = np.zeros(max(1, nch), dtype=np.uint32)
         packed = np.zeros(max(1, n), dtype=np.uint8)
+        slots = np.zeros(max(1, nch), dtype=np.uint32) if chunk_slots else None
         rc = int(lib().oracle_dedup(self._h, a.ctypes.data, n, mask.ctypes.data,
-                                    miss.ctypes.data, packed.ctypes.data))
+                                    miss.ctypes.data, packed.ctypes.data,
+                                    slots.ctypes.data if chunk_slots else None))
+        if chunk_slots:
+            if rc < 0:
+                return rc, None, None, None, None
+            r = self._finish(rc, n, nch, mask, miss, packed)
+            return r + (slots[:nch].copy(),)
+        return self._finish(rc, n, nch, mask, miss, packed)
+
+    def _finish(self, rc, n, nch, mask, miss, packed):
+        C = self.chunk_bytes
         if rc < 0:
             return rc, None, None, None
         miss = miss[:rc].copy()
@@ -137,6 +151,16 @@ class OracleCache:
             tail = n - last * C if last == nch - 1 else C
             nbytes = (rc - 1) * C + min(C, tail)
         return rc, mask[: (nch + 31) // 32].copy(), miss, packed[:nbytes].copy()
+
+    def block_check(self, block, offsets, slots):
+        """(number of mismatching records, mismatch flags u8[nrec])."""
+        b = _u8(block)
+        offs = np.ascontiguousarray(offsets, dtype=np.uint64)
+        sl = np.ascontiguousarray(slots, dtype=np.uint32)
+        flags = np.zeros(max(1, offs.size), dtype=np.uint8)
+        bad = int(lib().oracle_block_check(self._h, b.ctypes.data, b.size, offs.ctypes.data,
+                                           sl.ctypes.data, offs.size, flags.ctypes.data))
+        return bad, flags[: offs.size]
 
     def debug_insert(self, key: int, data) -> int:
         a = _u8(data)

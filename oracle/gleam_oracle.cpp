@@ -200,7 +200,7 @@ void oracle_cache_destroy(void* cache) { delete static_cast<Cache*>(cache); }
 // Returns the number of misses, or a negative error code.  The cache is only
 // changed when the whole call succeeds.
 int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
-                     uint32_t* miss_idx, uint8_t* packed) {
+                     uint32_t* miss_idx, uint8_t* packed, uint32_t* chunk_slot) {
   Cache* c = static_cast<Cache*>(cache);
   const uint8_t* p = static_cast<const uint8_t*>(buf);
   if (c == nullptr || (n > 0 && buf == nullptr)) return kErrInvalidArg;
@@ -223,6 +223,7 @@ int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
     const uint64_t key = key_of(*c, xxh64(chunk, len, 0));
 
     bool candidate = false, hit = false, hit_is_fresh = false;
+    uint32_t hit_slot = 0;
     auto look = [&](const std::unordered_multimap<uint64_t, Entry>& idx,
                     const std::vector<std::vector<uint8_t>>& store, uint64_t slot_base,
                     bool fresh) {
@@ -233,6 +234,7 @@ int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
         if (bytes_equal(store[it->second.slot - slot_base], chunk, len)) {
           hit = true;
           hit_is_fresh = fresh;
+          hit_slot = it->second.slot;
         }
       }
     };
@@ -242,11 +244,13 @@ int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
     if (hit) {
       hit_mask[i / 32] |= 1u << (i % 32);
       if (hit_is_fresh) ++hits_intra; else ++hits_cache;
+      if (chunk_slot) chunk_slot[i] = hit_slot;
       continue;
     }
     if (candidate) ++rejects;
     if (slots0 + rank >= c->nslots) return kErrCapacity;  // nothing committed
     miss_idx[rank] = static_cast<uint32_t>(i);
+    if (chunk_slot) chunk_slot[i] = static_cast<uint32_t>(slots0 + rank);
     std::memcpy(packed + rank * C, chunk, len);
     Entry e{key, static_cast<uint32_t>(len), static_cast<uint32_t>(slots0 + rank)};
     fresh_index.emplace(key, e);
@@ -268,6 +272,31 @@ int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
   c->inserts += rank;
   c->verify_rejects += rejects;
   return static_cast<int64_t>(rank);
+}
+
+// Weight-block identification at cudaFree time (paper Sec. 4.1.1): record r says
+// that the block's bytes at offsets[r] were written by a host-to-device copy of
+// the chunk stored in slots[r].  The block still holds weights iff every record
+// matches the block's current bytes.  Writes mismatch[r] (1 = differs, or the
+// record does not fit the block / names no stored slot) and returns how many
+// records mismatch.
+int64_t oracle_block_check(const void* cache, const void* block, uint64_t block_bytes,
+                           const uint64_t* offsets, const uint32_t* slots, uint64_t nrec,
+                           uint8_t* mismatch) {
+  const Cache* c = static_cast<const Cache*>(cache);
+  const uint8_t* b = static_cast<const uint8_t*>(block);
+  int64_t bad = 0;
+  for (uint64_t r = 0; r < nrec; ++r) {
+    bool differs = true;
+    if (slots[r] < c->slot_bytes.size()) {
+      const std::vector<uint8_t>& stored = c->slot_bytes[slots[r]];
+      if (offsets[r] <= block_bytes && stored.size() <= block_bytes - offsets[r])
+        differs = !stored.empty() && std::memcmp(b + offsets[r], stored.data(), stored.size()) != 0;
+    }
+    mismatch[r] = differs ? 1 : 0;
+    bad += differs ? 1 : 0;
+  }
+  return bad;
 }
 
 // Test hook: store `bytes` under an arbitrary key (crafted collisions).

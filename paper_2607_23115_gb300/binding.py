@@ -32,7 +32,7 @@ EXPORTS = (
     "gleam_cache_create", "gleam_cache_create_ex", "gleam_cache_destroy",
     "gleam_cache_reserve", "gleam_fingerprint", "gleam_dedup_copy",
     "gleam_dedup_copy_async", "gleam_dedup_copy_batch", "gleam_dedup_copy_noalloc",
-    "gleam_dedup_copy_host_async", "gleam_dedup_copy_host_batch",
+    "gleam_dedup_copy_host_async", "gleam_dedup_copy_host_batch", "gleam_block_check",
     "gleam_cache_stats", "gleam_cache_export",
     "gleam_cache_read_slot", "gleam_cache_debug_insert", "gleam_cache_debug_set",
     "gleam_cache_snapshot", "gleam_cache_restore", "gleam_snapshot_destroy",
@@ -50,7 +50,8 @@ class gleam_stats_t(ctypes.Structure):
 class gleam_payload_t(ctypes.Structure):
     _fields_ = [("d_buf", ctypes.c_void_p), ("n", ctypes.c_size_t),
                 ("d_hit_mask", ctypes.c_void_p), ("d_miss_idx", ctypes.c_void_p),
-                ("d_miss_bytes", ctypes.c_void_p), ("d_result", ctypes.c_void_p)]
+                ("d_miss_bytes", ctypes.c_void_p), ("d_result", ctypes.c_void_p),
+                ("d_chunk_slot", ctypes.c_void_p)]
 
 
 RESULT_FIELDS = ("status", "n_miss", "n_hit_cache", "n_hit_intra", "verify_rejects",
@@ -90,6 +91,7 @@ def lib() -> ctypes.CDLL:
         "gleam_dedup_copy_noalloc": (i32, [vp, vp, sz, vp, vp, vp, vp, vp]),
         "gleam_dedup_copy_host_async": (i32, [vp, vp, sz, vp, vp, vp, vp, vp]),
         "gleam_dedup_copy_host_batch": (i32, [vp, ctypes.POINTER(gleam_payload_t), sz, vp, vp]),
+        "gleam_block_check": (i32, [vp, vp, sz, vp, vp, sz, vp, vp, vp]),
         "gleam_cache_stats": (i32, [vp, ctypes.POINTER(gleam_stats_t)]),
         "gleam_cache_export": (i32, [vp, vp, vp, u64, ctypes.POINTER(u64)]),
         "gleam_cache_read_slot": (i32, [vp, u64, vp, u64, ctypes.POINTER(u64)]),
@@ -187,10 +189,13 @@ def gleam_dedup_copy_noalloc(cache, d_buf, n: int, d_hit_mask, d_miss_idx, d_mis
 
 def payload_array(payloads):
     """ctypes gleam_payload_t[] from (d_buf, n, d_hit_mask, d_miss_idx,
-    d_miss_bytes, d_result) tuples; reusable across calls."""
+    d_miss_bytes, d_result[, d_chunk_slot]) tuples; reusable across calls."""
     arr = (gleam_payload_t * max(1, len(payloads)))()
-    for k, (buf, n, mask, idx, packed, res) in enumerate(payloads):
-        arr[k] = gleam_payload_t(_ptr(buf), n, _ptr(mask), _ptr(idx), _ptr(packed), _ptr(res))
+    for k, t in enumerate(payloads):
+        buf, n, mask, idx, packed, res = t[:6]
+        slots = t[6] if len(t) > 6 else None
+        arr[k] = gleam_payload_t(_ptr(buf), n, _ptr(mask), _ptr(idx), _ptr(packed), _ptr(res),
+                                 _ptr(slots))
     arr.count = len(payloads)
     return arr
 
@@ -213,6 +218,13 @@ def gleam_dedup_copy_host_batch(cache, payloads, d_total=None, stream=None) -> i
     arr = payloads if hasattr(payloads, "count") else payload_array(payloads)
     return lib().gleam_dedup_copy_host_batch(cache, arr, arr.count, _ptr(d_total),
                                              _stream(stream))
+
+
+def gleam_block_check(cache, d_block, block_bytes: int, d_offsets, d_slots, nrec: int,
+                      d_mismatch, d_count, stream=None) -> int:
+    return lib().gleam_block_check(cache, _ptr(d_block), block_bytes, _ptr(d_offsets),
+                                   _ptr(d_slots), nrec, _ptr(d_mismatch), _ptr(d_count),
+                                   _stream(stream))
 
 
 def gleam_cache_stats(cache):

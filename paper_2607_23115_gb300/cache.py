@@ -90,14 +90,26 @@ class Cache:
                "gleam_dedup_copy_async")
 
     @staticmethod
-    def batch_items(bufs, outs, results=None):
+    def batch_items(bufs, outs, results=None, chunk_slots=None):
         """Payload array for dedup_batch (build once, reuse for repeated calls)."""
         items = []
         for k, (b, o) in enumerate(zip(bufs, outs)):
             n = b.numel() * b.element_size()
             r = results[k] if results is not None else None
-            items.append((b, n, o.hit_mask, o.miss_idx, o.miss_bytes, r))
+            sl = chunk_slots[k] if chunk_slots is not None else None
+            items.append((b, n, o.hit_mask, o.miss_idx, o.miss_bytes, r, sl))
         return B.payload_array(items)
+
+    def block_check(self, block: torch.Tensor, offsets: torch.Tensor, slots: torch.Tensor,
+                    mismatch: Optional[torch.Tensor] = None, count: Optional[torch.Tensor] = None,
+                    stream=None) -> torch.Tensor:
+        """Device int64[1] count of records whose bytes no longer match (async)."""
+        if count is None:
+            count = torch.zeros(1, dtype=torch.int64, device=block.device)
+        _check(B.gleam_block_check(self.handle, block, block.numel() * block.element_size(),
+                                   offsets, slots, offsets.numel(), mismatch, count, stream),
+               "gleam_block_check")
+        return count
 
     def dedup_batch(self, bufs, outs=None, results=None, total: Optional[torch.Tensor] = None,
                     stream=None, items=None):

@@ -363,6 +363,13 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
           else hc = true;                           // inserted by an earlier payload
         }
         if (hc || hi2) atomicOr(P.mask + (i >> 5), 1u << (i & 31));
+        if (P.chunk_slot) {
+          uint32_t sl;
+          if (r & kResHit0) sl = ch.ent[g];                                   // matched slot
+          else if (r & kResDup) sl = (uint32_t)(slots0 + __ldcg(&ch.rank[ch.ent[g]]));  // leader's
+          else sl = (uint32_t)(slots0 + ch.rank[g]);                          // its own new slot
+          P.chunk_slot[i] = sl;
+        }
         if (miss) {
           len = ch.len[g];
           P.miss_idx[ch.rank[g] - __ldcg(&a.pstart[p])] = (uint32_t)i;
@@ -469,6 +476,34 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   __threadfence();
 }
 
+// One warp per record: does the block still hold the recorded chunk's bytes?
+__global__ void __launch_bounds__(kThreads) k_block_check(BlockCheckArgs a) {
+  const uint32_t lane = threadIdx.x & 31;
+  const unsigned long long warp = ((unsigned long long)blockIdx.x * kThreads + threadIdx.x) >> 5;
+  const unsigned long long nwarps = ((unsigned long long)gridDim.x * kThreads) >> 5;
+  const unsigned long long used = a.dstats[ST_SLOTS_USED];
+  uint32_t bad = 0;
+  for (unsigned long long r = warp; r < a.nrec; r += nwarps) {
+    const unsigned long long off = a.offsets[r];
+    const uint32_t slot = a.slots[r];
+    bool differs = true;
+    if (slot < used) {
+      const uint32_t len = a.slot_len[slot];
+      if (off <= a.block_bytes && len <= a.block_bytes - off) {
+        const uint8_t* x = a.block + off;
+        const uint8_t* y = a.arena + (unsigned long long)slot * a.C;
+        const bool vec = (((uintptr_t)x | (uintptr_t)y) & 15) == 0;
+        differs = !warp_equal(x, y, len, vec);
+      }
+    }
+    if (lane == 0) {
+      if (a.mismatch) a.mismatch[r] = differs ? 1 : 0;
+      bad += differs;
+    }
+  }
+  if (lane == 0 && bad) atomicAdd(a.count, (unsigned long long)bad);
+}
+
 __global__ void k_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
                                unsigned long long* dstats, unsigned long long key, uint32_t slot,
                                uint32_t len, DevCtl* ctl) {
@@ -501,6 +536,14 @@ cudaError_t launch_dedup(const DedupArgs& a, int grid, cudaStream_t s) {
   DedupArgs copy = a;
   void* args[] = {&copy};
   return cudaLaunchCooperativeKernel((void*)k_dedup, dim3(grid), dim3(kThreads), args, 0, s);
+}
+
+cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s) {
+  if (a.nrec == 0) return cudaSuccess;
+  const unsigned long long warps = a.nrec < (1ull << 20) ? a.nrec : (1ull << 20);
+  const unsigned grid = (unsigned)((warps * 32 + kThreads - 1) / kThreads);
+  k_block_check<<<grid, kThreads, 0, s>>>(a);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,

@@ -316,8 +316,10 @@ int describe(gleam_cache* c, PtrChecker& chk, const gleam_payload_t& p, PayloadD
   d->miss_idx = p.d_miss_idx;
   d->packed = static_cast<uint8_t*>(p.d_miss_bytes);
   d->result = p.d_result;
+  d->chunk_slot = p.d_chunk_slot;
   int rc;
   if (p.d_result && (rc = chk.check(p.d_result, sizeof(gleam_result_t))) != GLEAM_OK) return rc;
+  if (p.d_chunk_slot && N && (rc = chk.check(p.d_chunk_slot, N * 4)) != GLEAM_OK) return rc;
   if (p.n == 0) return GLEAM_OK;
   if (host_payload) {
     const void* dev = nullptr;
@@ -462,6 +464,7 @@ gleam_payload_t make_payload(const void* d_buf, size_t n, uint32_t* d_hit_mask,
   p.d_miss_idx = d_miss_idx;
   p.d_miss_bytes = d_miss_bytes;
   p.d_result = d_result;
+  p.d_chunk_slot = nullptr;
   return p;
 }
 
@@ -644,6 +647,38 @@ int gleam_dedup_copy_host_async(gleam_cache_t* c, const void* h_buf, size_t n,
   DeviceGuard g(c->device);
   const gleam_payload_t p = make_payload(h_buf, n, d_hit_mask, d_miss_idx, d_miss_bytes, d_result);
   return enqueue(c, &p, 1, nullptr, reinterpret_cast<cudaStream_t>(stream), true);
+}
+
+int gleam_block_check(const gleam_cache_t* c, const void* d_block, size_t block_bytes,
+                      const uint64_t* d_offsets, const uint32_t* d_slots, size_t nrec,
+                      uint8_t* d_mismatch, uint64_t* d_count, gleam_stream_t stream) {
+  if (!c || !d_count) return GLEAM_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  PtrChecker chk(c->device);
+  int rc;
+  if ((rc = chk.check(d_count, sizeof(uint64_t))) != GLEAM_OK) return rc;
+  if (nrec > 0) {
+    if (block_bytes > 0 && (rc = chk.check(d_block, block_bytes)) != GLEAM_OK) return rc;
+    if ((rc = chk.check(d_offsets, nrec * 8)) != GLEAM_OK) return rc;
+    if ((rc = chk.check(d_slots, nrec * 4)) != GLEAM_OK) return rc;
+    if (d_mismatch && (rc = chk.check(d_mismatch, nrec)) != GLEAM_OK) return rc;
+  }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((rc = cuda_err(cudaStreamWaitEvent(s, c->done, 0))) != GLEAM_OK) return rc;
+  if ((rc = cuda_err(cudaMemsetAsync(d_count, 0, sizeof(uint64_t), s))) != GLEAM_OK) return rc;
+  BlockCheckArgs a{};
+  a.block = static_cast<const uint8_t*>(d_block);
+  a.block_bytes = block_bytes;
+  a.offsets = reinterpret_cast<const unsigned long long*>(d_offsets);
+  a.slots = d_slots;
+  a.nrec = nrec;
+  a.mismatch = d_mismatch;
+  a.count = reinterpret_cast<unsigned long long*>(d_count);
+  a.arena = c->arena;
+  a.slot_len = c->slot_len;
+  a.dstats = c->dstats;
+  a.C = c->C;
+  return cuda_err(launch_block_check(a, s));
 }
 
 int gleam_cache_stats(const gleam_cache_t* c, gleam_stats_t* out) {

@@ -90,6 +90,7 @@ struct __align__(16) PayloadDesc {
   uint32_t* miss_idx;
   uint8_t* packed;
   gleam_result_t* result;  // may be null
+  uint32_t* chunk_slot;    // may be null: slot holding each chunk's bytes
 };
 
 // Per-chunk workspace, indexed by global chunk number.
@@ -100,7 +101,8 @@ struct ChunkArrays {
   unsigned long long* src;   // device address of the chunk's first byte
   uint32_t* pidx;            // payload number
   uint32_t* res;             // resolution word (kRes*)
-  uint32_t* ent;             // group-table entry; the leader's number once a duplicate
+  uint32_t* ent;             // cache hit: matched slot; else group-table entry, and
+                             // the leader's number once a duplicate
   uint32_t* rank;            // exclusive count of misses before the chunk
   unsigned long long* hint;  // prefix hint (chunks of at least kPrefixBytes)
   uint32_t* order;           // order[r] = chunk number of the miss of rank r
@@ -164,6 +166,21 @@ cudaError_t launch_dedup(const DedupArgs& a, int grid, cudaStream_t s);
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
                                 unsigned long long* dstats, unsigned long long key,
                                 uint32_t slot, uint32_t len, DevCtl* ctl, cudaStream_t s);
+struct BlockCheckArgs {
+  const uint8_t* block;
+  unsigned long long block_bytes;
+  const unsigned long long* offsets;
+  const uint32_t* slots;
+  unsigned long long nrec;
+  uint8_t* mismatch;             // may be null
+  unsigned long long* count;
+  const uint8_t* arena;
+  const uint32_t* slot_len;
+  const unsigned long long* dstats;
+  unsigned long long C;
+};
+
+cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s);
 int dedup_threads();
 int dedup_chunks_per_block();
 int dedup_blocks_per_sm();

@@ -295,6 +295,7 @@ __global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
   const unsigned long long key = a.key16 ? (h & 0xFFFFULL) : h;
   unsigned long long pos = mix64(key) & a.index_mask;
   bool hit = false, cand = false;
+  uint32_t hit_slot = kEmptySlot;
   for (unsigned long long probe = 0; probe <= a.index_mask; ++probe) {
     const IndexEntry e = a.index[pos];
     if (e.slot == kEmptySlot) break;
@@ -306,10 +307,12 @@ __global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
       } else if (e.slot == hint_slot) {
         if (spec_equal) {  // compared in the streaming pass
           hit = true;
+          hit_slot = e.slot;
           break;
         }
       } else if (group_equal<kAligned>(p, a.arena + (uint64_t)e.slot * a.C, len, lane, gmask)) {
         hit = true;
+        hit_slot = e.slot;
         break;
       }
     }
@@ -322,6 +325,7 @@ __global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
     a.ch.src[g] = (unsigned long long)p;
     a.ch.pidx[g] = pid;
     a.ch.hint[g] = hint;
+    if (hit) a.ch.ent[g] = hit_slot;
   }
 }
 

@@ -92,7 +92,7 @@ class BruteCache:
         N = (n + C - 1) // C
         staged = list(self.items)
         slots0 = len(staged)
-        mask, miss, packed = [0] * ((N + 31) // 32), [], bytearray()
+        mask, miss, packed, slots = [0] * ((N + 31) // 32), [], bytearray(), []
         hits_cache = hits_intra = rejects = 0
         for i in range(N):
             c = payload[i * C:(i + 1) * C]
@@ -103,6 +103,7 @@ class BruteCache:
                     break
             if found is not None:
                 mask[i // 32] |= 1 << (i % 32)
+                slots.append(found)
                 if found < slots0:
                     hits_cache += 1
                 else:
@@ -114,8 +115,9 @@ class BruteCache:
             if len(staged) >= self.nslots:
                 return -4, None
             miss.append(i)
+            slots.append(len(staged))
             packed += c
             staged.append((key, c))
         self.items = staged
         return len(miss), dict(mask=mask, miss=miss, packed=bytes(packed), hits_cache=hits_cache,
-                               hits_intra=hits_intra, rejects=rejects)
+                               hits_intra=hits_intra, rejects=rejects, slots=slots)

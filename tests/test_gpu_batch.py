@@ -20,7 +20,10 @@ def _batch_vs_oracle(gc, oc, payloads_host, offsets=None, expect_rc=None):
     outs = [DedupOutputs.alloc(h.numel(), C, DEV) for h in payloads_host]
     res = torch.zeros(len(bufs), B.RESULT_WORDS, dtype=torch.int64, device=DEV)
     total = torch.zeros(B.RESULT_WORDS, dtype=torch.int64, device=DEV)
-    gc.dedup_batch(bufs, outs, [res[k] for k in range(len(bufs))], total)
+    slots = [torch.full((max(1, (h.numel() + C - 1) // C),), -1, dtype=torch.int32, device=DEV)
+             for h in payloads_host]
+    items = gc.batch_items(bufs, outs, [res[k] for k in range(len(bufs))], slots)
+    gc.dedup_batch(None, items=items, total=total)
     torch.cuda.synchronize()
     tot = result_dict(total)
     if expect_rc is not None:
@@ -30,7 +33,8 @@ def _batch_vs_oracle(gc, oc, payloads_host, offsets=None, expect_rc=None):
     sums = dict(n_miss=0, n_hit_cache=0, n_hit_intra=0, verify_rejects=0, miss_bytes=0)
     for k, h in enumerate(payloads_host):
         before = oc.stats()
-        rc, mask_o, miss_o, packed_o = oc.dedup(h.numpy())
+        out_o = oc.dedup(h.numpy(), chunk_slots=True)
+        rc, mask_o, miss_o, packed_o, slots_o = out_o
         after = oc.stats()
         r = result_dict(res[k])
         assert r["status"] == 0 and r["n_miss"] == rc, (k, r, rc)
@@ -46,6 +50,8 @@ def _batch_vs_oracle(gc, oc, payloads_host, offsets=None, expect_rc=None):
         assert np.array_equal(o.hit_mask.cpu().numpy().view(np.uint32)[: len(mask_o)], mask_o), k
         assert np.array_equal(o.miss_idx.cpu().numpy().view(np.uint32)[:rc], miss_o), k
         assert np.array_equal(o.miss_bytes.cpu().numpy()[: len(packed_o)], packed_o), k
+        nch = (h.numel() + C - 1) // C
+        assert np.array_equal(slots[k].cpu().numpy().view(np.uint32)[:nch], slots_o), k
     for f in sums:
         assert tot[f] == sums[f], f
     return tot

@@ -22,15 +22,18 @@ def _payload_from_alphabet(rng, alphabet, nchunks, C, tail):
 
 
 def _check_against_brute(oc: oracle.OracleCache, bc: BruteCache, payload: bytes, C: int):
-    rc, mask, miss, packed = oc.dedup(payload)
+    out = oc.dedup(payload, chunk_slots=True)
+    rc = out[0]
     brc, b = bc.dedup(payload, C)
     assert rc == brc
     if rc < 0:
         return rc
+    _, mask, miss, packed, slots = out
     N = (len(payload) + C - 1) // C
     assert _mask_bits(mask, N) == _mask_bits(b["mask"], N)
     assert miss.tolist() == b["miss"]
     assert packed.tobytes() == b["packed"]
+    assert slots.tolist() == b["slots"]
     return rc, b
 
 
@@ -221,3 +224,35 @@ def test_adversarial_miss_count_closed_form():
     rc16, mask16, miss16, packed16 = oc16.dedup(buf)
     assert rc16 == rc and (miss16 == miss).all() and (packed16 == packed).all()
     assert oc16.stats()["verify_rejects"] >= 64
+
+
+def test_block_check_matches_brute_force():
+    """Weight-block identification (paper Sec. 4.1.1): a block still holds
+    weights iff every chunk recorded from its host-to-device writes matches."""
+    rng = np.random.default_rng(21)
+    C = 64
+    oc = oracle.OracleCache(1000 * C, C)
+    block = bytearray(rng.integers(0, 256, 40 * C + 17, dtype=np.uint8).tobytes())
+    # two "HtoD writes" into the block at offsets 0 and 20*C (+ ragged tail)
+    offs, slots = [], []
+    for base, length in ((0, 20 * C), (20 * C, 20 * C + 17)):
+        _, _, _, _, sl = oc.dedup(bytes(block[base:base + length]), chunk_slots=True)
+        offs += [base + i * C for i in range(len(sl))]
+        slots += sl.tolist()
+    bad, flags = oc.block_check(bytes(block), offs, slots)
+    assert bad == 0 and not flags.any()
+    # change one byte in record 7 and one in the tail record: exactly those differ
+    block[7 * C + 5] ^= 0x10
+    block[40 * C + 3] ^= 0x01
+    bad, flags = oc.block_check(bytes(block), offs, slots)
+    expect = [0] * len(offs)
+    expect[7] = 1
+    expect[len(offs) - 1] = 1
+    assert bad == 2 and flags.tolist() == expect
+    # brute force over the same records: compare stored bytes with the block
+    for r, (o, s_) in enumerate(zip(offs, slots)):
+        stored = oc.slot_bytes(s_)
+        assert (bytes(block[o:o + len(stored)]) != stored) == bool(flags[r])
+    # a record past the block's end, or naming no stored slot, mismatches
+    bad, flags = oc.block_check(bytes(block[: 10 * C]), [9 * C + 1, 0], [0, 10**6])
+    assert bad == 2
