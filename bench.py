@@ -265,7 +265,8 @@ def run_gleam(args, rank, world, local_rank):
     results = torch.zeros(nt, B.RESULT_WORDS, dtype=torch.int64, device=dev)
 
     bufs = [up.payload(k) for k in range(nt)]
-    items = cache.batch_items(bufs, outs, [results[k] for k in range(nt)])
+    chunk_slots = [torch.zeros((s + C - 1) // C, dtype=torch.int32, device=dev) for s in up.sizes]
+    items = cache.batch_items(bufs, outs, [results[k] for k in range(nt)], chunk_slots)
     total_res = torch.zeros(B.RESULT_WORDS, dtype=torch.int64, device=dev)
 
     def one_pass():
@@ -395,6 +396,9 @@ def run_gleam(args, rank, world, local_rank):
         "clocks": clk,
     }
 
+    if not args.profile_launches:
+        line["block_check"] = run_block_check(up, cache, chunk_slots, C, hbm)
+
     if do_cpu:
         nbytes, dt, ntens = oracle_sample(spec, base_host, pert_host, args.cpu_sample_bytes)
         line["cpu_baseline"] = {
@@ -412,6 +416,35 @@ def run_gleam(args, rank, world, local_rank):
 
     cache.close()
     return line
+
+
+def run_block_check(up, cache, chunk_slots, C, hbm):
+    """Weight-block identification at cudaFree time over the whole upload as
+    one block: every chunk's record (offset, slot from the last pass) is
+    compared with the block's bytes; algorithmic bytes = block + cached copies
+    read once = 2 x payload."""
+    import torch
+    offs = torch.cat([torch.arange(len(cs), dtype=torch.int64, device=cs.device) * C + o
+                      for cs, o in zip(chunk_slots, up.offsets)])
+    slots = torch.cat(chunk_slots)
+    cnt = cache.block_check(up.buf, offs, slots)
+    torch.cuda.synchronize()
+    reps = 10
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        cache.block_check(up.buf, offs, slots, count=cnt)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    # the last pass's misses were inserted with the flipped bytes, so every
+    # record matches the current block
+    assert int(cnt.item()) == 0
+    gbs = 2 * up.total_bytes / (ms * 1e-3) / 1e9
+    return {"records": int(offs.numel()), "ms": round(ms, 4), "achieved_gbs": round(gbs, 1),
+            "frac_of_measured_hbm": round(gbs / hbm, 4),
+            "how": "gleam_block_check over the whole upload as one block, records from the "
+                   "timed pass's chunk slots; 2 x payload bytes / CUDA-event time"}
 
 
 def run_e2e_host(args, up, host, cache, snap, outs, results, miss_bytes):
