@@ -340,10 +340,16 @@ __global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
 // second buffer.  The lanes then hash and compare their words from shared
 // memory.  Stage 0 is exactly the prefix used for the hint.
 // ---------------------------------------------------------------------------
+#ifndef GLEAM_STAGE_DEPTH
+#define GLEAM_STAGE_DEPTH 3
+#endif
+#ifndef GLEAM_STAGED_THREADS
+#define GLEAM_STAGED_THREADS 256
+#endif
 constexpr int kStage = 512;                                 // bytes per stage
-constexpr int kDepth = 3;                                   // stages in flight
+constexpr int kDepth = GLEAM_STAGE_DEPTH;                   // stages in flight
 constexpr int kGroupBytes = kDepth * 2 * kStage + 32;       // +32: bank skew
-constexpr int kStagedThreads = 256;
+constexpr int kStagedThreads = GLEAM_STAGED_THREADS;
 constexpr int kStagedSmem = (kStagedThreads / 4) * kGroupBytes;
 static_assert(kStage == (int)kPrefixBytes, "stage 0 must be the hinted prefix");
 
@@ -428,8 +434,12 @@ __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a
     // groups committed so far, oldest first: prologue stages, then one per
     // iteration, plus (at t = 0) one holding the cached copy of stages
     // 1 .. kDepth-1, issued late because the hint is known only then
-    if (t == 1) cp_wait<1>();  // stage 1 and that late group; stage kDepth may pend
-    else cp_wait<kDepth - 1>();
+    // stage t needs everything up to the late group while t < kDepth - 1
+    // (at most t newer groups may pend), else up to its own group
+    if (t == 0 || t >= (uint32_t)kDepth - 1) cp_wait<kDepth - 1>();
+    else if (t == 1) cp_wait<1>();
+    else if (t == 2) cp_wait<2>();
+    else cp_wait<0>();
     __syncwarp(gmask);
     const uint8_t* sp = pay_p(t);
     const uint32_t sst = sbytes(t) >> 5;
