@@ -48,7 +48,8 @@ def parse_args():
     p.add_argument("--steps", type=int, default=100)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["gleam", "reference"], default="gleam")
-    p.add_argument("--workload", choices=["llama3-8b", "llama3-8b-layer", "llama3-8b-4layers", "gpt2-small"], default="llama3-8b")
+    p.add_argument("--workload", default="llama3-8b",
+                   help="one of: " + ", ".join(WORKLOADS))
     p.add_argument("--cpu-sample-bytes", type=int, default=3 * GiB,
                    help="payload bytes of the oracle's bounded CPU sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -63,45 +64,173 @@ def parse_args():
 # workloads
 # ---------------------------------------------------------------------------
 
-def workload_spec(name):
+class Workload:
+    """One benchmark configuration: the payloads of one step (one batch call),
+    what the cache holds before the first step, and bounded host samples for
+    the CPU oracle."""
+
+    def __init__(self, name, desc, C, capacity, flags=0):
+        self.name, self.desc, self.C, self.capacity, self.flags = name, desc, C, capacity, flags
+        self.up = None             # workloads.Upload: the step's payloads
+        self.prefill = []          # lists of device tensors, one batch call each
+        self.after_prefill = None  # run once after the prefill (perturbation)
+        self.crafted = []          # (device bytes whose XXH64 is the key, device bytes stored)
+        self.expect_misses = None  # closed form, checked at full size
+        self.flush_l2 = False      # inputs smaller than L2: flush between timed steps
+        self._sample = None        # (budget, offset) -> (prefill [np], payloads [np], text)
+
+    def sample(self, budget, offset=0):
+        return self._sample(budget, offset)
+
+
+def _np_list(tensors):
+    return [t.cpu().numpy().copy() for t in tensors]
+
+
+def _first_payloads(up, budget, offset):
+    ks, tot, k = [], 0, offset
+    while tot < budget and len(ks) < len(up.sizes):
+        ks.append(k % len(up.sizes))
+        tot += up.sizes[k % len(up.sizes)]
+        k += 1
+    return ks
+
+
+def build_workload(name, dev, sample_budget):
     import torch
     from paper_2607_23115_gb300 import workloads as W
-    if name == "llama3-8b":
-        return dict(name="llama3-8b-bf16-per-tensor", shapes=W.llama3_8b_shapes(),
-                    dtype=torch.bfloat16, C=64 * KiB, capacity=24 * GiB, flip_frac=0.10,
-                    desc="Llama-3-8B-shaped bf16 upload, 291 tensors, ~N(0,0.02); cache "
-                         "prefilled with the base weights; 10% of 64 KiB chunks bit-flipped")
-    if name == "llama3-8b-layer":
-        return dict(name="llama3-8b-bf16-one-layer", shapes=W.llama3_8b_shapes()[1:10],
-                    dtype=torch.bfloat16, C=64 * KiB, capacity=512 * MiB, flip_frac=0.10,
-                    desc="one Llama-3-8B layer (9 bf16 tensors, 436 MB): the small case of "
-                         "the llama3-8b workload for ncu captures")
-    if name == "llama3-8b-4layers":
-        return dict(name="llama3-8b-bf16-four-layers", shapes=W.llama3_8b_shapes()[1:37],
-                    dtype=torch.bfloat16, C=64 * KiB, capacity=2 * GiB, flip_frac=0.10,
-                    desc="four Llama-3-8B layers (36 bf16 tensors, 1.74 GB): a few-GB case "
-                         "of the llama3-8b workload for ncu captures")
-    if name == "gpt2-small":
-        return dict(name="gpt2-small-fp32-per-tensor-second-pass", shapes=W.gpt2_small_shapes(),
-                    dtype=torch.float32, C=4 * KiB, capacity=1 * GiB, flip_frac=0.0,
-                    desc="GPT-2-small-shaped fp32 upload, 148 tensors, ~N(0,0.02); second "
-                         "identical pass (all hits) after a first pass filled the cache")
-    raise ValueError(name)
+    from paper_2607_23115_gb300.workloads import Upload
+
+    if name.startswith("llama3-8b"):
+        shapes = W.llama3_8b_shapes()
+        variants = {"llama3-8b": (shapes, 24 * GiB, "Llama-3-8B-shaped bf16 upload, 291 tensors"),
+                    "llama3-8b-layer": (shapes[1:10], 512 * MiB, "one Llama-3-8B layer, 9 bf16 "
+                                        "tensors (the small case for ncu captures)"),
+                    "llama3-8b-4layers": (shapes[1:37], 2 * GiB, "four Llama-3-8B layers, 36 "
+                                          "bf16 tensors (the few-GB case for ncu captures)")}
+        shp, cap, what = variants[name]
+        wl = Workload({"llama3-8b": "llama3-8b-bf16-per-tensor",
+                       "llama3-8b-layer": "llama3-8b-bf16-one-layer",
+                       "llama3-8b-4layers": "llama3-8b-bf16-four-layers"}[name],
+                      what + ", ~N(0,0.02); cache prefilled with the base weights; 10% of "
+                      "64 KiB chunks bit-flipped", 64 * KiB, cap)
+        up = W.weight_upload(shp, torch.bfloat16, device=dev)
+        wl.up = up
+        wl.prefill = [[up.payload(k) for k in range(len(up.sizes))]]
+        base = {k: up.payload(k).cpu().numpy().copy()
+                for k in _first_payloads(up, sample_budget, 0)}
+
+        def perturb():
+            chunks = up.chunks(wl.C)
+            ids = W.select_chunks(len(chunks), 0.10)
+            W.flip_one_bit_per_chunk(up.buf, chunks, ids)
+            wl.expect_misses = len(ids)
+        wl.after_prefill = perturb
+
+        def sample(budget, offset):
+            ks = _first_payloads(up, budget, offset)
+            pre = [base[k] if k in base else None for k in ks]
+            if any(x is None for x in pre):
+                raise ValueError("sample outside the captured base tensors")
+            return pre, _np_list(up.payload(k) for k in ks), \
+                "%d tensors (%.2f GB) of the upload; oracle prefilled with their base bytes " \
+                "(untimed), timed over their perturbed bytes" % (len(ks), sum(p.size for p in pre) / 1e9)
+        wl._sample = sample
+        return wl
+
+    if name in ("gpt2-small", "gpt2-small-pass1"):
+        pass2 = name == "gpt2-small"
+        wl = Workload("gpt2-small-fp32-per-tensor-" + ("second-pass" if pass2 else "first-pass"),
+                      "GPT-2-small-shaped fp32 upload, 148 tensors, ~N(0,0.02); " +
+                      ("second identical pass (all hits) after a first pass filled the cache"
+                       if pass2 else "first pass on an empty cache (all misses, inserts)"),
+                      4 * KiB, 1 * GiB)
+        up = W.weight_upload(W.gpt2_small_shapes(), torch.float32, device=dev)
+        wl.up = up
+        nch = len(up.chunks(wl.C))
+        if pass2:
+            wl.prefill = [[up.payload(k) for k in range(len(up.sizes))]]
+        wl.expect_misses = 0 if pass2 else nch
+
+        def sample(budget, offset):
+            ks = _first_payloads(up, budget, offset)
+            pays = _np_list(up.payload(k) for k in ks)
+            return (pays if pass2 else []), pays, \
+                "%d tensors (%.2f GB) of the upload%s" % (len(ks), sum(p.size for p in pays) / 1e9,
+                                                          "; oracle prefilled with them (untimed)"
+                                                          if pass2 else "")
+        wl._sample = sample
+        return wl
+
+    if name == "fp16-64m":
+        C = 4 * KiB
+        wl = Workload("fp16-64mib-half-prefilled", "one 64 MiB payload of fp16 ~N(0,0.02), half of "
+                      "its 4 KiB chunks pre-cached (seeded), 128 MiB cache", C, 128 * MiB)
+        buf = W.fp16_payload(64 * MiB, device=dev)
+        wl.up = Upload(buf, [0], [buf.numel()])
+        sel = W.select_chunks(buf.numel() // C, 0.5)
+        pre = W.gather_chunks(buf, C, sel)
+        wl.prefill = [[pre]]
+        wl.expect_misses = buf.numel() // C - len(sel)
+        wl.flush_l2 = True
+        pre_h, buf_h = pre.cpu().numpy(), buf.cpu().numpy()
+        wl._sample = lambda budget, offset: ([pre_h], [buf_h], "the whole 64 MiB payload, oracle "
+                                             "prefilled with the same half (untimed)")
+        return wl
+
+    if name == "small-calls":
+        C = 4 * KiB
+        wl = Workload("small-call-stream-100k", "100,000 payloads of uniform random bytes, sizes "
+                      "log-uniform in 4 KiB-1 MiB (18.8 GB); cache prefilled with 2 GB of "
+                      "unrelated chunks; 32 GiB cache", C, 32 * GiB)
+        up = W.small_call_upload(100000, device=dev)
+        wl.up = up
+        wl.prefill = [[W.random_bytes(2 * 10**9 // C * C, seed=W.SEED_PREFILL, device=dev)]]
+        wl.expect_misses = sum((s + C - 1) // C for s in up.sizes)
+
+        def sample(budget, offset):
+            ks = _first_payloads(up, budget, offset)
+            pays = _np_list(up.payload(k) for k in ks)
+            return [], pays, "%d payloads (%.2f GB), empty oracle cache (the prefill is " \
+                "unrelated random data)" % (len(ks), sum(p.size for p in pays) / 1e9)
+        wl._sample = sample
+        return wl
+
+    if name.startswith("adversarial-"):
+        parts = name.split("-")
+        C = int(parts[1].rstrip("k")) * KiB
+        key16 = len(parts) > 2 and parts[2] == "key16"
+        from paper_2607_23115_gb300 import binding as B
+        wl = Workload("adversarial-1gib-c%dk%s" % (C // KiB, "-key16" if key16 else ""),
+                      "1 GiB: 25%% zero chunks, 25%% copies of 16 patterns, 50%% random, C = %d "
+                      "KiB%s" % (C // KiB, "; KEY16 test mode with 64 crafted colliding entries"
+                                 if key16 else ""), C, 2 * GiB, B.GLEAM_KEY16 if key16 else 0)
+        adv = W.adversarial_payload(1 * GiB, C, device=dev)
+        wl.up = Upload(adv.buf, [0], [adv.buf.numel()])
+        npat = len(set(adv.pattern_id[adv.kind == 1].tolist()))
+        wl.expect_misses = 1 + npat + int((adv.kind == 2).sum())
+        crafted_h = []
+        if key16:
+            pick, rows = W.crafted_collisions(adv, C, count=64)
+            orig = adv.buf.view(-1, C)[pick.to(adv.buf.device)]
+            wl.crafted = [(orig[i], rows[i]) for i in range(64)]
+            crafted_h = [(orig[i].cpu().numpy(), rows[i].cpu().numpy()) for i in range(64)]
+
+        def sample(budget, offset):
+            nb = min(adv.buf.numel(), max(C, budget // C * C))
+            return [], [adv.buf[:nb].cpu().numpy()], \
+                "the first %.2f GB of the payload (in one call)%s" % (
+                    nb / 1e9, ", the 64 crafted entries inserted first" if key16 else "")
+        wl._sample = sample
+        wl.crafted_host = crafted_h
+        return wl
+
+    raise ValueError("unknown workload %r" % name)
 
 
-def make_upload(spec, device):
-    from paper_2607_23115_gb300 import workloads as W
-    return W.weight_upload(spec["shapes"], spec["dtype"], device=device)
-
-
-def perturb(spec, up):
-    from paper_2607_23115_gb300 import workloads as W
-    if spec["flip_frac"] <= 0:
-        return 0
-    chunks = up.chunks(spec["C"])
-    ids = W.select_chunks(len(chunks), spec["flip_frac"])
-    W.flip_one_bit_per_chunk(up.buf, chunks, ids)
-    return len(ids)
+WORKLOADS = ["llama3-8b", "llama3-8b-layer", "llama3-8b-4layers", "gpt2-small",
+             "gpt2-small-pass1", "fp16-64m", "small-calls"] + \
+    ["adversarial-%dk%s" % (c, m) for c in (1, 4, 16, 64) for m in ("", "-key16")]
 
 
 # ---------------------------------------------------------------------------
@@ -166,37 +295,22 @@ class ClockSampler:
 # the oracle on the host cores (bounded sample)
 # ---------------------------------------------------------------------------
 
-def oracle_sample(spec, up_base_host, up_pert_host, sample_bytes, offset_tensor=0):
-    """Oracle dedup of a bounded sample of tensors: prefill with the base
-    tensors (untimed), then time the pass over the perturbed tensors."""
+def oracle_time(wl, budget, offset=0):
+    """The oracle over a bounded sample of the workload: prefill (untimed), then
+    the timed calls.  Returns (payload bytes, seconds, description)."""
     import oracle
-    ks, tot, k = [], 0, offset_tensor
-    n_t = len(up_base_host)
-    while tot < sample_bytes and len(ks) < n_t:
-        ks.append(k % n_t)
-        tot += up_base_host[k % n_t].size
-        k += 1
-    oc = oracle.OracleCache(spec["capacity"], spec["C"])
-    for kk in ks:
-        oc.dedup(up_base_host[kk])
-    src = up_pert_host if up_pert_host is not None else up_base_host
+    pre, pays, text = wl.sample(budget, offset)
+    oc = oracle.OracleCache(wl.capacity, wl.C, oracle.KEY16 if wl.flags & 1 else 0)
+    for orig, row in getattr(wl, "crafted_host", []):
+        oc.debug_insert(oracle.xxh64(orig), row)
+    for x in pre:
+        oc.dedup(x)
     t0 = time.perf_counter()
-    for kk in ks:
-        oc.dedup(src[kk])
+    for x in pays:
+        oc.dedup(x)
     dt = time.perf_counter() - t0
     oc.close()
-    return tot, dt, len(ks)
-
-
-def host_tensors(up, limit_bytes):
-    """numpy copies of the first tensors of an upload, up to limit_bytes."""
-    out, tot = [], 0
-    for k in range(len(up.sizes)):
-        if tot >= limit_bytes:
-            break
-        out.append(up.payload(k).cpu().numpy().copy())
-        tot += up.sizes[k]
-    return out
+    return sum(x.size for x in pays), dt, text
 
 
 # ---------------------------------------------------------------------------
@@ -246,52 +360,49 @@ def run_gleam(args, rank, world, local_rank):
     import torch.distributed as dist
 
     from paper_2607_23115_gb300 import binding as B
-    from paper_2607_23115_gb300.cache import Cache, DedupOutputs
+    from paper_2607_23115_gb300.cache import Cache, DedupOutputs, fingerprint
 
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    spec = workload_spec(args.workload)
-    C = spec["C"]
-
-    up = make_upload(spec, dev)
+    do_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_launches
+    wl = build_workload(args.workload, dev, args.cpu_sample_bytes if do_cpu else 0)
+    C, up = wl.C, wl.up
     nt = len(up.sizes)
     total = up.total_bytes
-    do_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_launches
-    base_host = host_tensors(up, args.cpu_sample_bytes) if do_cpu else None
+    nchunks = sum((s + C - 1) // C for s in up.sizes)
 
-    cache = Cache(spec["capacity"], C)
-    cache.reserve(max((s + C - 1) // C for s in up.sizes))
+    cache = Cache(wl.capacity, C, wl.flags)
+    cache.reserve(max(nchunks, max((sum(t.numel() for t in b) + C - 1) // C + len(b)
+                                   for b in wl.prefill) if wl.prefill else 1))
     outs = [DedupOutputs.alloc(s, C, dev) for s in up.sizes]
     results = torch.zeros(nt, B.RESULT_WORDS, dtype=torch.int64, device=dev)
-
     bufs = [up.payload(k) for k in range(nt)]
-    chunk_slots = [torch.zeros((s + C - 1) // C, dtype=torch.int32, device=dev) for s in up.sizes]
+    chunk_slots = [torch.zeros(max(1, (s + C - 1) // C), dtype=torch.int32, device=dev)
+                   for s in up.sizes]
     items = cache.batch_items(bufs, outs, [results[k] for k in range(nt)], chunk_slots)
     total_res = torch.zeros(B.RESULT_WORDS, dtype=torch.int64, device=dev)
 
     def one_pass():
         cache.dedup_batch(None, items=items, total=total_res, stream=None)
 
-    def one_pass_calls():
-        for k in range(nt):
-            cache.dedup_async(bufs[k], outs[k], results[k], stream=None)
-
-    # prefill with the base upload (untimed), then perturb
-    one_pass()
-    n_flipped = perturb(spec, up)
+    # cache state before the first step: crafted entries, prefill calls, perturbation
+    for orig, row in wl.crafted:
+        key = int(fingerprint(orig, 0).cpu().numpy().view(np.uint64)[0])
+        cache.debug_insert(key, row)
+    for batch in wl.prefill:
+        pouts = [DedupOutputs.alloc(t.numel(), C, dev) for t in batch]
+        cache.dedup_batch(batch, pouts)
+        torch.cuda.synchronize()
+        del pouts
+    if wl.after_prefill:
+        wl.after_prefill()
     torch.cuda.synchronize()
     snap = cache.snapshot()
-    pert_host = None
-    if do_cpu and spec["flip_frac"] > 0:
-        pert_host = [up.payload(k).cpu().numpy().copy() for k in range(len(base_host))]
+    flush = torch.empty(256 * MiB, dtype=torch.uint8, device=dev) if wl.flush_l2 else None
 
     def step():
         cache.restore(snap)
         one_pass()
-
-    def step_calls():
-        cache.restore(snap)
-        one_pass_calls()
 
     for _ in range(args.warmup):
         step()
@@ -301,8 +412,8 @@ def run_gleam(args, rank, world, local_rank):
     miss_bytes = int(r[:, 5].sum())
     n_miss = int(r[:, 1].sum())
     hit_intra = int(r[:, 3].sum())
-    if spec["flip_frac"] > 0:
-        assert n_miss == n_flipped, (n_miss, n_flipped)
+    if wl.expect_misses is not None:
+        assert n_miss == wl.expect_misses, (n_miss, wl.expect_misses)
     # algorithmic bytes: the fused fingerprint/probe/verify kernel reads the
     # payload once and the cached copy of every cache hit
     hit_cache_bytes = total - miss_bytes - hit_intra * C
@@ -316,34 +427,67 @@ def run_gleam(args, rank, world, local_rank):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    t_start.record()
-    for _ in range(args.steps):
-        step()
-    t_end.record()
-    torch.cuda.synchronize()
+    if flush is None:
+        t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t_start.record()
+        for _ in range(args.steps):
+            step()
+        t_end.record()
+        torch.cuda.synchronize()
+        ms = t_start.elapsed_time(t_end)
+    else:  # inputs fit in L2: flush it between steps, outside each step's events
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(args.steps)]
+        for e0, e1 in ev:
+            flush.fill_(1)
+            e0.record()
+            step()
+            e1.record()
+        torch.cuda.synchronize()
+        ms = sum(e0.elapsed_time(e1) for e0, e1 in ev)
     if world > 1:
         dist.barrier()
-    ms = t_start.elapsed_time(t_end)
     clk = clocks.stop() if not args.profile_launches else None
     rc, kms, klaunch = B.gleam_cache_profile_read(cache.handle, 2)
     B.gleam_cache_profile(cache.handle, False)
 
-    # the same pass as one call per tensor (secondary figure)
-    calls_ms = None
+    # the same pass as one call per payload (secondary figures)
+    per_call = None
     if not args.profile_launches:
-        calls_steps = max(1, min(args.steps, 5))
-        step_calls()
+        calls_steps = 1 if nt > 1000 else max(1, min(args.steps, 5))
+        cache.restore(snap)
+        for k in range(nt):
+            cache.dedup_async(bufs[k], outs[k], results[k], stream=None)
         torch.cuda.synchronize()
         c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        th = time.perf_counter()
         c0.record()
         for _ in range(calls_steps):
-            step_calls()
+            cache.restore(snap)
+            for k in range(nt):
+                cache.dedup_async(bufs[k], outs[k], results[k], stream=None)
         c1.record()
         torch.cuda.synchronize()
+        wall = (time.perf_counter() - th) / calls_steps
         calls_ms = c0.elapsed_time(c1) / calls_steps
         rcall = results.cpu().numpy()
         assert (rcall[:, 0] == 0).all() and int(rcall[:, 1].sum()) == n_miss
+        per_call = {"ms_per_step": round(calls_ms, 3),
+                    "value": round(total / (calls_ms * 1e-3) / 1e9, 2),
+                    "us_per_call": round(calls_ms * 1e3 / nt, 3),
+                    "host_wall_us_per_call": round(wall * 1e6 / nt, 3),
+                    "how": "same step as %d gleam_dedup_copy_async calls (one per payload) "
+                           "instead of one gleam_dedup_copy_batch call" % nt}
+        if nt > 1000:  # synchronous calls, like cudaMemcpy, on the first 2000 payloads
+            from paper_2607_23115_gb300 import binding as BB
+            cache.restore(snap)
+            torch.cuda.synchronize()
+            th = time.perf_counter()
+            for k in range(2000):
+                rcs = BB.gleam_dedup_copy(cache.handle, bufs[k], up.sizes[k], outs[k].hit_mask,
+                                          outs[k].miss_idx, outs[k].miss_bytes)
+                assert rcs >= 0, rcs
+            per_call["sync_us_per_call"] = round((time.perf_counter() - th) * 1e6 / 2000, 3)
     if world > 1:
         t = torch.tensor([ms], dtype=torch.float64, device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -353,10 +497,10 @@ def run_gleam(args, rank, world, local_rank):
 
     hbm, hbm_src = measured_peaks()
     k0_ms = kms[0] / max(1, klaunch[0])
-    k0_bytes = kernel0_bytes  # one launch covers the whole upload
+    k0_bytes = kernel0_bytes  # one launch covers the whole step
     k0_gbs = k0_bytes / (k0_ms * 1e-3) / 1e9
-    traffic = committed_traffic(spec["name"])
-    roofline = {"bound": "hbm", "kernel": "k_hash_probe (fingerprint + probe + verify)",
+    traffic = committed_traffic(wl.name)
+    roofline = {"bound": "hbm", "kernel": "k_hash_probe_staged (fingerprint + probe + verify)",
                 "achieved": round(k0_gbs, 1), "peak": hbm, "peak_source": hbm_src,
                 "unit": "GB/s", "frac": round(k0_gbs / hbm, 4),
                 "traffic": traffic, "algorithmic_bytes_per_launch": round(k0_bytes),
@@ -377,41 +521,40 @@ def run_gleam(args, rank, world, local_rank):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
         "data": "synthetic",
-        "config": {"workload": spec["name"], "description": spec["desc"],
+        "config": {"workload": wl.name, "description": wl.desc,
                    "payload_bytes_per_step": total, "payloads_per_step": nt, "calls_per_step": 1,
-                   "api": "gleam_dedup_copy_batch (one call = %d per-tensor payloads)" % nt, "chunk_bytes": C,
-                   "chunks_per_step": sum((s + C - 1) // C for s in up.sizes),
-                   "misses_per_step": n_miss, "cache_capacity_bytes": spec["capacity"],
-                   "l2": "inputs (%.1f GB per step) far larger than the 129 MB L2; no flush"
-                         % (total / 1e9),
+                   "api": "gleam_dedup_copy_batch (one call = %d payloads)" % nt,
+                   "chunk_bytes": C, "chunks_per_step": nchunks, "misses_per_step": n_miss,
+                   "cache_capacity_bytes": wl.capacity, "key16": bool(wl.flags & 1),
+                   "l2": ("inputs (%.2f GB) fit in the 129 MB L2's reach: a 256 MiB buffer is "
+                          "written between timed steps, outside each step's events"
+                          % (total / 1e9)) if flush is not None else
+                         ("inputs (%.1f GB per step) far larger than the 129 MB L2; no flush"
+                          % (total / 1e9)),
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "pipeline_roofline": pipeline,
         "roofline": roofline,
-        "per_call_async": None if calls_ms is None else {
-            "ms_per_step": round(calls_ms, 3),
-            "value": round(total / (calls_ms * 1e-3) / 1e9, 2),
-            "how": "same step as %d gleam_dedup_copy_async calls (one per tensor) instead "
-                   "of one gleam_dedup_copy_batch call" % nt},
+        "per_call_async": per_call,
         "gpu_launches": 2 * args.steps,
         "clocks": clk,
     }
 
     if not args.profile_launches:
+        step()  # the per-call runs above changed the cache; redo the batch pass
+        torch.cuda.synchronize()
         line["block_check"] = run_block_check(up, cache, chunk_slots, C, hbm)
 
     if do_cpu:
-        nbytes, dt, ntens = oracle_sample(spec, base_host, pert_host, args.cpu_sample_bytes)
+        nbytes, dt, text = oracle_time(wl, args.cpu_sample_bytes)
         line["cpu_baseline"] = {
             "value": round(nbytes / dt / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sample": "first %d tensors (%.2f GB) of the same upload: oracle prefilled with "
-                      "their base bytes (untimed), then timed over their perturbed bytes"
-                      % (ntens, nbytes / 1e9), "host_cpus": os.cpu_count()}
+            "sample": text, "host_cpus": os.cpu_count()}
 
-    if not args.no_e2e and not args.profile_launches:
+    if not args.no_e2e and not args.profile_launches and nt <= 1000:
         host = torch.empty(up.buf.numel(), dtype=torch.uint8, pin_memory=True)
         host.copy_(up.buf)
         line["e2e"] = run_e2e_host(args, up, host, cache, snap, outs, results, miss_bytes)
-        line["e2e_copy_then_dedup"] = run_e2e(args, spec, up, host, cache, snap, outs, results,
+        line["e2e_copy_then_dedup"] = run_e2e(args, up, host, cache, snap, outs, results,
                                               miss_bytes)
 
     cache.close()
@@ -504,7 +647,7 @@ def run_e2e_host(args, up, host, cache, snap, outs, results, miss_bytes):
                    "results, hit masks, miss indices and packed miss bytes; wall clock"}
 
 
-def run_e2e(args, spec, up, host, cache, snap, outs, results, miss_bytes):
+def run_e2e(args, up, host, cache, snap, outs, results, miss_bytes):
     """The same metric through the C ABI with HOST buffers: per step, every
     tensor is copied host->device from pinned memory and deduped, and every
     call's result, hit mask, miss indices and packed miss bytes are read back.
@@ -586,49 +729,39 @@ def run_e2e(args, spec, up, host, cache, snap, outs, results, miss_bytes):
 # ---------------------------------------------------------------------------
 
 def run_reference(args, rank, world):
+    """The reference arm: the oracle, single-threaded on the host cores, on
+    the same workload; each step a bounded sample (about 96 MB of payload)
+    taken at a different offset, on a fresh oracle cache."""
     import torch
-    spec = workload_spec(args.workload)
-    C = spec["C"]
     dev = "cuda" if torch.cuda.is_available() else "cpu"
-    # per step a bounded sample: a ~96 MiB slice of tensors, cycling through
-    # the first tensors of the upload, on a freshly prefilled oracle cache
-    slice_bytes = 96 * MiB
-    from paper_2607_23115_gb300 import workloads as W
-    shapes = spec["shapes"]
-    pool_shapes, acc = [], 0
-    for s in shapes[1:]:
-        pool_shapes.append(s)
-        acc += 1
-        if acc >= 40:
-            break
-    up = W.weight_upload(pool_shapes, spec["dtype"], device=dev)
-    base = [up.payload(k).cpu().numpy().copy() for k in range(len(up.sizes))]
-    perturb(spec, up)
-    pert = [up.payload(k).cpu().numpy().copy() for k in range(len(up.sizes))] \
-        if spec["flip_frac"] > 0 else None
-    times, nbytes = [], 0
+    budget = 96 * MiB
+    ahead = budget * (args.warmup + args.steps + 2)
+    wl = build_workload(args.workload, dev, min(ahead, 8 * GiB))
+    if wl.after_prefill:
+        wl.after_prefill()  # the same perturbation, without our cache
+    times, nbytes, text = [], 0, ""
     for i in range(args.warmup + args.steps):
-        nb, dt, nk = oracle_sample(spec, base, pert, slice_bytes, offset_tensor=3 * i)
+        try:
+            nb, dt, text = oracle_time(wl, budget, offset=3 * i)
+        except ValueError:  # beyond the captured base tensors: wrap around
+            nb, dt, text = oracle_time(wl, budget, offset=0)
         if i >= args.warmup:
             times.append(dt)
             nbytes += nb
     t = sum(times)
     value = nbytes / t / 1e9
-    line = {
+    return {
         "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(t / args.steps * 1e3, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u8", "data": "synthetic",
         "impl": "reference",
-        "config": {"workload": spec["name"], "description": spec["desc"], "chunk_bytes": C},
+        "config": {"workload": wl.name, "description": wl.desc, "chunk_bytes": wl.C},
         "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
-                         "sample": "per step ~96 MiB of whole tensors (layer tensors of the "
-                                   "same upload), oracle cache prefilled with their base bytes "
-                                   "(untimed)", "host_cpus": os.cpu_count()},
+                         "sample": "per step: " + text, "host_cpus": os.cpu_count()},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
-    return line
 
 
 def main():

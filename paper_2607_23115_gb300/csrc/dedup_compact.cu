@@ -222,6 +222,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       const uint32_t e = group_entry(a, g, ch.key[g], ch.len[g]);
       if (e == 0xFFFFFFFFu) {
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+        ch.ent[g] = 0xFFFFFFFFu;
         ch.res[g] = kResLeader | 1u;
         continue;
       }
@@ -293,8 +294,18 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   unsigned long long before = 0, total = 0;
   if (ok) {
     uint32_t cnt = 0;
-    for (uint32_t g = lo + threadIdx.x; g < hi; g += kThreads)
-      cnt += (ldcg_u32(&ch.res[g]) & kResLeader) ? 1u : 0u;
+    for (uint32_t g = lo + threadIdx.x; g < hi; g += kThreads) {
+      if (ldcg_u32(&ch.res[g]) & kResLeader) {
+        ++cnt;
+        // leave the group table zeroed for the next call: every claimed entry
+        // belongs to a group with at least one leader
+        const uint32_t e = ch.ent[g];
+        if (e != 0xFFFFFFFFu) {
+          a.tbl[e].owner = 0u;
+          a.tbl[e].minv = 0u;
+        }
+      }
+    }
     const unsigned long long c = block_sum<unsigned long long>(cnt, red64);
     if (threadIdx.x == 0) a.bcount[blockIdx.x] = (uint32_t)c;
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
@@ -472,6 +483,25 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       r->verify_rejects = 0;
       r->miss_bytes = 0;
     }
+  }
+  // Leave the per-call state as the next call expects it: the group table
+  // (cleared entry by entry by the leaders, or here in full after an error
+  // that may have stopped them) and the control block.
+  if (err)
+    for (unsigned long long e = threadIdx.x; e <= a.tbl_mask; e += kThreads) {
+      a.tbl[e].owner = 0u;
+      a.tbl[e].minv = 0u;
+    }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    DevCtl* c = a.ctl;
+    c->bar_count = 0;
+    c->bar_gen = 0;
+    c->err = 0;
+    c->unres[0] = c->unres[1] = c->unres[2] = 0;
+    c->acc_hits_cache = c->acc_hits_intra = c->acc_rejects = 0;
+    c->acc_misses = c->acc_miss_bytes = 0;
+    c->done = 0;
   }
   __threadfence();
 }

@@ -227,6 +227,10 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   free_ws(c);
   void* p = nullptr;
   if ((rc = cuda_err(cudaMalloc(&p, total))) != GLEAM_OK) return rc;
+  if ((rc = cuda_err(cudaMemset(p, 0, total))) != GLEAM_OK) {
+    cudaFree(p);
+    return rc;
+  }
   uint8_t* b = static_cast<uint8_t*>(p);
   c->ws = p;
   c->ch.status = b;
@@ -337,7 +341,7 @@ int describe(gleam_cache* c, PtrChecker& chk, const gleam_payload_t& p, PayloadD
 // Blocks of the cooperative dedup launch: enough for its per-chunk phases
 // (chunks / dedup_chunks_per_block) and for its miss copies (one block per
 // kBytesPerDedupBlock of payload), at most the co-resident maximum.
-constexpr uint64_t kBytesPerDedupBlock = 2ull << 20;
+constexpr uint64_t kBytesPerDedupBlock = 256ull << 10;
 
 int dedup_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
   const uint64_t per_block = dedup_chunks_per_block();
@@ -387,9 +391,8 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   }
   const uint64_t tcap =
       std::min<uint64_t>(c->tbl_cap, next_pow2(std::max<uint64_t>(64, 2 * Ntot)));
-  if ((rc = cuda_err(cudaMemsetAsync(c->ctl, 0, sizeof(DevCtl), s))) != GLEAM_OK) return rc;
-  if ((rc = cuda_err(cudaMemsetAsync(c->tbl, 0, tcap * sizeof(CallEntry), s))) != GLEAM_OK)
-    return rc;
+  // The group table and the control block start zeroed (at allocation) and
+  // every call's dedup kernel leaves them zeroed for the next one.
 
   HashArgs h{};
   h.table = c->d_table;
@@ -450,7 +453,10 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     grid = std::max(grid, std::min(2, c->coop_max_blocks));  // someone must be left waiting
     if (d.skip_block >= grid) d.skip_block = grid - 1;
   }
-  if ((rc = cuda_err(launch_dedup(d, grid, s))) != GLEAM_OK) return rc;
+  if ((rc = cuda_err(launch_dedup(d, grid, s))) != GLEAM_OK) {
+    cudaMemsetAsync(c->ctl, 0, sizeof(DevCtl), s);  // the hash kernel may have flagged it
+    return rc;
+  }
   if (ev[2]) cudaEventRecord(ev[2], s);
   return cuda_err(cudaEventRecord(c->done, s));
 }
