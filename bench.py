@@ -488,12 +488,8 @@ def run_gleam(args, rank, world, local_rank):
                                           outs[k].miss_idx, outs[k].miss_bytes)
                 assert rcs >= 0, rcs
             per_call["sync_us_per_call"] = round((time.perf_counter() - th) * 1e6 / 2000, 3)
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms, value = replica_timing(ms, total, args.steps, world, dev)
     ms_per_step = ms / args.steps
-    value = world * total / (ms_per_step * 1e-3) / 1e9
 
     hbm, hbm_src = measured_peaks()
     k0_ms = kms[0] / max(1, klaunch[0])
@@ -559,6 +555,21 @@ def run_gleam(args, rank, world, local_rank):
 
     cache.close()
     return line
+
+
+def replica_timing(ms_local, payload_bytes, steps, world, device="cpu"):
+    """Multi-GPU runs are independent replicas (the path does not shard): the
+    job's time is the slowest rank's, and its throughput is every rank's
+    payload over that time.  Returns (max ms over ranks, GB/s of the job)."""
+    import torch
+    ms = float(ms_local)
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * payload_bytes / (ms / steps * 1e-3) / 1e9
+    return ms, value
 
 
 def run_block_check(up, cache, chunk_slots, C, hbm):

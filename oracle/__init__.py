@@ -52,7 +52,13 @@ _lib = None
 def lib():
     global _lib
     if _lib is None:
-        l = ctypes.CDLL(build())
+        _lib = _bind(ctypes.CDLL(build()))
+    return _lib
+
+
+def _bind(l):
+    """Declares the C signatures on a loaded oracle library."""
+    if True:
         u64, sz, vp = ctypes.c_uint64, ctypes.c_size_t, ctypes.c_void_p
         l.oracle_xxh64.restype = u64
         l.oracle_xxh64.argtypes = [vp, sz, u64]
@@ -74,8 +80,7 @@ def lib():
         l.oracle_cache_entries.argtypes = [vp, vp, vp, u64]
         l.oracle_slot_bytes.restype = ctypes.c_int64
         l.oracle_slot_bytes.argtypes = [vp, u64, vp, u64]
-        _lib = l
-    return _lib
+    return l
 
 
 def _u8(buf) -> np.ndarray:

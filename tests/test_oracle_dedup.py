@@ -256,3 +256,27 @@ def test_block_check_matches_brute_force():
     # a record past the block's end, or naming no stored slot, mismatches
     bad, flags = oc.block_check(bytes(block[: 10 * C]), [9 * C + 1, 0], [0, 10**6])
     assert bad == 2
+
+
+def test_length_is_part_of_a_candidate():
+    """An entry with the chunk's key but another length is not a candidate: the
+    chunk is a miss without a verify reject (R6: rejects need key + length)."""
+    rng = np.random.default_rng(31)
+    C = 256
+    chunk = rng.integers(0, 256, C, dtype=np.uint8).tobytes()
+    for key16 in (False, True):
+        oc = oracle.OracleCache(64 * C, C, oracle.KEY16 if key16 else 0)
+        assert oc.debug_insert(xxh64_lib(chunk), chunk[:-1]) == 0   # same key, shorter
+        rc, mask, miss, packed = oc.dedup(chunk)
+        assert rc == 1 and oc.stats()["verify_rejects"] == 0
+        assert oc.debug_insert(xxh64_lib(chunk), bytes(C)) == 0     # same key and length
+        rc, mask, miss, packed = oc.dedup(chunk + chunk[:100])
+        # the first chunk now hits the entry the previous call inserted
+        assert rc == 1 and int(mask[0]) == 1 and oc.stats()["verify_rejects"] == 0
+        other = bytearray(chunk)
+        other[5] ^= 1
+        assert oc.debug_insert(xxh64_lib(bytes(other)), bytes(other)[:-1]) == 0
+        oc2 = oracle.OracleCache(64 * C, C, oracle.KEY16 if key16 else 0)
+        assert oc2.debug_insert(xxh64_lib(bytes(other)), bytes(C)) == 0  # key match, bytes differ
+        rc, _, _, _ = oc2.dedup(bytes(other))
+        assert rc == 1 and oc2.stats()["verify_rejects"] == 1
