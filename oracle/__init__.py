@@ -28,6 +28,8 @@ OK = 0
 ERR_INVALID_ARG = -1
 ERR_CAPACITY = -4
 KEY16 = 1
+PAPER_IDS = 4
+NO_SLOT = 0xFFFFFFFF
 
 STAT_FIELDS = (
     "calls", "chunks", "hits_cache", "hits_intra", "misses", "inserts",
@@ -62,6 +64,8 @@ def _bind(l):
         u64, sz, vp = ctypes.c_uint64, ctypes.c_size_t, ctypes.c_void_p
         l.oracle_xxh64.restype = u64
         l.oracle_xxh64.argtypes = [vp, sz, u64]
+        l.oracle_md5.restype = None
+        l.oracle_md5.argtypes = [vp, sz, vp]
         l.oracle_fingerprint.restype = ctypes.c_int
         l.oracle_fingerprint.argtypes = [vp, sz, sz, vp]
         l.oracle_cache_create.restype = vp
@@ -92,6 +96,20 @@ def _u8(buf) -> np.ndarray:
 def xxh64(data, seed: int = 0) -> int:
     a = _u8(data)
     return int(lib().oracle_xxh64(a.ctypes.data, a.size, seed))
+
+
+def md5(data) -> bytes:
+    a = _u8(data)
+    out = np.zeros(16, dtype=np.uint8)
+    lib().oracle_md5(a.ctypes.data, a.size, out.ctypes.data)
+    return out.tobytes()
+
+
+def paper_key(chunk) -> int:
+    """The paper's identifier (App. B.1): MD5 of the first min(len, 128) bytes,
+    first 8 digest bytes as a little-endian integer."""
+    a = _u8(chunk)
+    return int.from_bytes(md5(a[:128])[:8], "little")
 
 
 def fingerprint(data, chunk_bytes: int) -> np.ndarray:

@@ -32,6 +32,11 @@
 //  R8 miss indices ascending, packed bytes in the same order at rank*C,
 //     hit-mask bit i is bit (i % 32) of 32-bit word i / 32, trailing bits 0.
 //  R10 KEY16 mode keys the index by the low 16 bits of the fingerprint.
+//  R13 paper-identifier mode (App. B.1): the key is MD5 of the chunk's first
+//      min(len, 128) bytes (first 8 digest bytes, little-endian); chunks under
+//      1024 bytes are recorded but never cached: always misses, no slot, no
+//      entry, no in-call dedup.  Verify is kept.
+#include <cmath>
 #include <cstddef>
 #include <cstdint>
 #include <cstring>
@@ -122,11 +127,85 @@ uint64_t xxh64(const uint8_t* p, size_t len, uint64_t seed) {
   return h;
 }
 
+// ---- MD5, RFC 1321 ------------------------------------------------------------
+// Used only for the paper's own identifier (App. B.1: MD5 of a chunk's first
+// 1024 bits).  Per-step constants are floor(2^32 * |sin(i)|), i = 1..64.
+struct Md5 {
+  uint32_t k[64];
+  Md5() {
+    for (int i = 0; i < 64; ++i)
+      k[i] = static_cast<uint32_t>(std::floor(std::fabs(std::sin(static_cast<double>(i + 1))) *
+                                              4294967296.0));
+  }
+};
+
+uint32_t rotl32(uint32_t x, int r) { return (x << r) | (x >> (32 - r)); }
+
+void md5(const uint8_t* p, size_t len, uint8_t out[16]) {
+  static const Md5 tab;
+  static const int shift[4][4] = {{7, 12, 17, 22}, {5, 9, 14, 20}, {4, 11, 16, 23}, {6, 10, 15, 21}};
+  // message + 0x80 + zero padding to 56 mod 64 + 64-bit little-endian bit length
+  std::vector<uint8_t> m(p, p + len);
+  m.push_back(0x80);
+  while (m.size() % 64 != 56) m.push_back(0);
+  const uint64_t bits = static_cast<uint64_t>(len) * 8;
+  for (int k = 0; k < 8; ++k) m.push_back(static_cast<uint8_t>(bits >> (8 * k)));
+  uint32_t a0 = 0x67452301u, b0 = 0xefcdab89u, c0 = 0x98badcfeu, d0 = 0x10325476u;
+  for (size_t blk = 0; blk < m.size(); blk += 64) {
+    uint32_t x[16];
+    for (int j = 0; j < 16; ++j) x[j] = read_le32(&m[blk + 4 * j]);
+    uint32_t a = a0, b = b0, c = c0, d = d0;
+    for (int i = 0; i < 64; ++i) {
+      const int round = i / 16;
+      uint32_t f;
+      int g;
+      if (round == 0) {
+        f = (b & c) | (~b & d);
+        g = i;
+      } else if (round == 1) {
+        f = (d & b) | (~d & c);
+        g = (5 * i + 1) % 16;
+      } else if (round == 2) {
+        f = b ^ c ^ d;
+        g = (3 * i + 5) % 16;
+      } else {
+        f = c ^ (b | ~d);
+        g = (7 * i) % 16;
+      }
+      const uint32_t t = d;
+      d = c;
+      c = b;
+      b = b + rotl32(a + f + tab.k[i] + x[g], shift[round][i % 4]);
+      a = t;
+    }
+    a0 += a;
+    b0 += b;
+    c0 += c;
+    d0 += d;
+  }
+  const uint32_t w[4] = {a0, b0, c0, d0};
+  for (int j = 0; j < 4; ++j)
+    for (int k = 0; k < 4; ++k) out[4 * j + k] = static_cast<uint8_t>(w[j] >> (8 * k));
+}
+
+// The paper's identifier of a chunk: MD5 over its first min(len, 128) bytes,
+// first 8 digest bytes as a little-endian u64.
+uint64_t paper_key(const uint8_t* p, size_t len) {
+  uint8_t d[16];
+  md5(p, len < 128 ? len : 128, d);
+  uint64_t k = 0;
+  for (int i = 0; i < 8; ++i) k |= static_cast<uint64_t>(d[i]) << (8 * i);
+  return k;
+}
+
 // ---- the weight cache -----------------------------------------------------
 const int kOk = 0;
 const int kErrInvalidArg = -1;
 const int kErrCapacity = -4;
 const uint32_t kFlagKey16 = 1u;
+const uint32_t kFlagPaperIds = 4u;  // App. B.1 identifiers and small-chunk rule
+const size_t kPaperMinCached = 1024;
+const uint32_t kNoSlot = 0xFFFFFFFFu;
 
 struct Entry {
   uint64_t key;
@@ -150,6 +229,12 @@ uint64_t key_of(const Cache& c, uint64_t fp) {
   return (c.flags & kFlagKey16) ? (fp & 0xFFFFull) : fp;
 }
 
+// Index key of a chunk: XXH64 of the whole chunk, or in paper mode MD5 of its
+// prefix; then the 16-bit truncation of the KEY16 test mode.
+uint64_t chunk_key(const Cache& c, const uint8_t* p, size_t len) {
+  return key_of(c, (c.flags & kFlagPaperIds) ? paper_key(p, len) : xxh64(p, len, 0));
+}
+
 bool bytes_equal(const std::vector<uint8_t>& stored, const uint8_t* p, size_t len) {
   return stored.size() == len && (len == 0 || std::memcmp(stored.data(), p, len) == 0);
 }
@@ -160,6 +245,10 @@ extern "C" {
 
 uint64_t oracle_xxh64(const void* p, size_t n, uint64_t seed) {
   return xxh64(static_cast<const uint8_t*>(p), n, seed);
+}
+
+void oracle_md5(const void* p, size_t n, uint8_t* out16) {
+  md5(static_cast<const uint8_t*>(p), n, out16);
 }
 
 // out[i] = XXH64 of chunk i; chunk_bytes == 0 -> out[0] = XXH64 of all n bytes.
@@ -180,7 +269,7 @@ int oracle_fingerprint(const void* buf, size_t n, size_t chunk_bytes, uint64_t* 
 
 void* oracle_cache_create(size_t capacity_bytes, size_t chunk_bytes, uint32_t flags, int* err) {
   if (chunk_bytes < 32 || chunk_bytes % 32 != 0 || chunk_bytes > (16u << 20) ||
-      (flags & ~kFlagKey16) != 0 || capacity_bytes / (chunk_bytes ? chunk_bytes : 1) == 0 ||
+      (flags & ~(kFlagKey16 | kFlagPaperIds)) != 0 || capacity_bytes / (chunk_bytes ? chunk_bytes : 1) == 0 ||
       capacity_bytes / chunk_bytes > 0xFFFFFFFEull) {
     if (err) *err = kErrInvalidArg;
     return nullptr;
@@ -213,14 +302,24 @@ int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
   std::unordered_multimap<uint64_t, Entry> fresh_index;
   std::vector<std::vector<uint8_t>> fresh_bytes;
   const uint64_t slots0 = c->slot_bytes.size();
+  const bool paper = (c->flags & kFlagPaperIds) != 0;
   uint64_t rank = 0, hits_cache = 0, hits_intra = 0, rejects = 0;
+  uint64_t stored = 0;  // misses given a slot (all of them, except paper-mode small chunks)
 
   for (uint64_t w = 0; w < (nchunks + 31) / 32; ++w) hit_mask[w] = 0;
 
   for (uint64_t i = 0; i < nchunks; ++i) {
     const uint8_t* chunk = p + i * C;
     const size_t len = (n - i * C < C) ? (n - i * C) : C;
-    const uint64_t key = key_of(*c, xxh64(chunk, len, 0));
+    if (paper && len < kPaperMinCached) {
+      // App. B.1: recorded but never cached -- always sent, never inserted
+      miss_idx[rank] = static_cast<uint32_t>(i);
+      if (chunk_slot) chunk_slot[i] = kNoSlot;
+      std::memcpy(packed + rank * C, chunk, len);
+      ++rank;
+      continue;
+    }
+    const uint64_t key = chunk_key(*c, chunk, len);
 
     bool candidate = false, hit = false, hit_is_fresh = false;
     uint32_t hit_slot = 0;
@@ -248,14 +347,15 @@ int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
       continue;
     }
     if (candidate) ++rejects;
-    if (slots0 + rank >= c->nslots) return kErrCapacity;  // nothing committed
+    if (slots0 + stored >= c->nslots) return kErrCapacity;  // nothing committed
     miss_idx[rank] = static_cast<uint32_t>(i);
-    if (chunk_slot) chunk_slot[i] = static_cast<uint32_t>(slots0 + rank);
+    if (chunk_slot) chunk_slot[i] = static_cast<uint32_t>(slots0 + stored);
     std::memcpy(packed + rank * C, chunk, len);
-    Entry e{key, static_cast<uint32_t>(len), static_cast<uint32_t>(slots0 + rank)};
+    Entry e{key, static_cast<uint32_t>(len), static_cast<uint32_t>(slots0 + stored)};
     fresh_index.emplace(key, e);
     fresh_bytes.emplace_back(chunk, chunk + len);
     ++rank;
+    ++stored;
   }
 
   // Commit.
@@ -269,7 +369,7 @@ int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
   c->hits_cache += hits_cache;
   c->hits_intra += hits_intra;
   c->misses += rank;
-  c->inserts += rank;
+  c->inserts += stored;
   c->verify_rejects += rejects;
   return static_cast<int64_t>(rank);
 }

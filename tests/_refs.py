@@ -79,10 +79,11 @@ class BruteCache:
     """The weight cache by its definition: an ordered list of stored byte
     strings; a chunk is a hit iff byte-equal to a stored one of equal length."""
 
-    def __init__(self, nslots: int, key_fn=None):
+    def __init__(self, nslots: int, key_fn=None, paper_min: int = 0):
         self.nslots = nslots
         self.items = []       # (key, bytes) in slot order
         self.key_fn = key_fn  # bytes -> key, only for counting verify rejects
+        self.paper_min = paper_min  # chunks shorter than this are never cached
 
     def insert(self, key, data: bytes):
         self.items.append((key, bytes(data)))
@@ -96,6 +97,11 @@ class BruteCache:
         hits_cache = hits_intra = rejects = 0
         for i in range(N):
             c = payload[i * C:(i + 1) * C]
+            if len(c) < self.paper_min:  # recorded, never cached
+                miss.append(i)
+                slots.append(0xFFFFFFFF)
+                packed += c
+                continue
             found = None
             for s, (_, b) in enumerate(staged):
                 if b == c:

@@ -24,11 +24,11 @@ MUTANTS = [
     ("length not part of a candidate", "if (it->second.len != len) continue;", ""),
     ("earlier misses of the call not looked up", "look(fresh_index, fresh_bytes, slots0, true);", ""),
     ("reject counted without a candidate", "if (candidate) ++rejects;", "++rejects;"),
-    ("capacity off by one", "if (slots0 + rank >= c->nslots)", "if (slots0 + rank > c->nslots)"),
-    ("miss packed at its chunk offset", "std::memcpy(packed + rank * C, chunk, len);",
-     "std::memcpy(packed + i * C, chunk, len);"),
+    ("capacity off by one", "if (slots0 + stored >= c->nslots)", "if (slots0 + stored > c->nslots)"),
+    ("miss packed at its chunk offset", "std::memcpy(packed + rank * C, chunk, len);\n    Entry e",
+     "std::memcpy(packed + i * C, chunk, len);\n    Entry e"),
     ("hit reports a fresh slot", "if (chunk_slot) chunk_slot[i] = hit_slot;",
-     "if (chunk_slot) chunk_slot[i] = static_cast<uint32_t>(slots0 + rank);"),
+     "if (chunk_slot) chunk_slot[i] = static_cast<uint32_t>(slots0 + stored);"),
 ]
 
 
