@@ -61,6 +61,14 @@ enum gleam_status {
                                    so unrelated chunks collide and every hit
                                    must be separated from them by the verify */
 #define GLEAM_DEBUG_CHECKS 0x2u /* extra device-side index/arena checks      */
+#define GLEAM_PAPER_IDS 0x4u    /* the paper's own identifier (App. B.1): the
+                                   index key is MD5 of a chunk's first
+                                   min(len, 128) bytes (first 8 digest bytes,
+                                   little-endian) instead of XXH64 of the whole
+                                   chunk, and chunks under 1024 bytes are
+                                   recorded but never cached: always misses,
+                                   given no slot, never deduplicated.  Every
+                                   key match is still verified byte for byte. */
 
 /* Cumulative counters of one cache (successful calls only). */
 typedef struct gleam_stats {
@@ -101,7 +109,8 @@ typedef struct gleam_payload {
   gleam_result_t* d_result;
   /* optional (may be NULL), device u32[N]: the arena slot that holds chunk i's
    * bytes after the call -- the byte-equal cached chunk for a hit, the new
-   * slot for a miss.  Records for gleam_block_check come from here. */
+   * slot for a miss, 0xFFFFFFFF for a chunk that is never cached
+   * (GLEAM_PAPER_IDS).  Records for gleam_block_check come from here. */
   uint32_t* d_chunk_slot;
 } gleam_payload_t;
 
@@ -111,7 +120,7 @@ typedef struct gleam_payload {
  * slots of chunk_bytes each and an empty index (paper Sec. 4.1.3: the
  * server-side shareable pool; Sec. 4.1.2: the set of resident identifiers).
  * chunk_bytes: multiple of 32, 32..16 MiB.  The slot count must be 1..2^32-2.
- * flags: 0 or a combination of GLEAM_KEY16 and GLEAM_DEBUG_CHECKS.
+ * flags: 0 or a combination of GLEAM_KEY16, GLEAM_DEBUG_CHECKS and GLEAM_PAPER_IDS.
  * On success *out owns about capacity_bytes + 32 B * slots of device memory.
  * Returns GLEAM_OK, GLEAM_ERR_INVALID_ARG, GLEAM_ERR_NOMEM or GLEAM_ERR_CUDA. */
 int gleam_cache_create(size_t capacity_bytes, size_t chunk_bytes, gleam_cache_t** out);
@@ -203,7 +212,7 @@ int gleam_dedup_copy_host_batch(gleam_cache_t* cache, const gleam_payload_t* pay
  * memory map it keeps for the application.
  *
  * Same operation, outputs and cache update as gleam_dedup_copy_async, but the
- * per-call workspace is one fixed array of about 4.6 MiB in the library's
+ * per-call workspace is one fixed array of about 4.9 MiB in the library's
  * device image instead of memory allocated by the cache; the call itself only
  * enqueues memsets and kernels and allocates nothing.  Every GPU that loads
  * the library holds that array until the process exits.

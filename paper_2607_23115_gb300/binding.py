@@ -24,6 +24,7 @@ GLEAM_ERR_INTERNAL = -7
 
 GLEAM_KEY16 = 0x1
 GLEAM_DEBUG_CHECKS = 0x2
+GLEAM_PAPER_IDS = 0x4
 GLEAM_DEBUG_WAIT_LIMIT_NS = 1
 GLEAM_DEBUG_SKIP_ARRIVE = 2
 

@@ -84,7 +84,8 @@ __device__ bool warp_equal(const uint8_t* x, const uint8_t* y, uint32_t len, boo
   return !__any_sync(0xffffffffu, diff);
 }
 
-// Whole-warp copy of one chunk to the packed output and to its arena slot.
+// Whole-warp copy of one chunk to the packed output and to its arena slot
+// (d2 == nullptr: to the packed output only).
 __device__ void warp_copy2(uint8_t* d1, uint8_t* d2, const uint8_t* s, uint32_t len, bool vec) {
   const uint32_t lane = threadIdx.x & 31;
   uint32_t done = 0;
@@ -106,10 +107,10 @@ __device__ void warp_copy2(uint8_t* d1, uint8_t* d2, const uint8_t* s, uint32_t 
         if (k < nv) {
 #if GLEAM_COPY_STREAMING_STORES
           __stcs(d1v + k, u[r]);
-          __stcs(d2v + k, u[r]);
+          if (d2) __stcs(d2v + k, u[r]);
 #else
           d1v[k] = u[r];
-          d2v[k] = u[r];
+          if (d2) d2v[k] = u[r];
 #endif
         }
       }
@@ -119,7 +120,7 @@ __device__ void warp_copy2(uint8_t* d1, uint8_t* d2, const uint8_t* s, uint32_t 
   for (uint32_t k = done + lane; k < len; k += 32) {
     const uint8_t b = s[k];
     d1[k] = b;
-    d2[k] = b;
+    if (d2) d2[k] = b;
   }
 }
 
@@ -185,6 +186,8 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ uint32_t warp_cnt[kWarps];
   __shared__ uint32_t warp_off[kWarps];
+  __shared__ uint32_t swarp_cnt[kWarps];
+  __shared__ uint32_t swarp_off[kWarps];
   __shared__ unsigned long long s_slots0;
 
   const uint32_t G = gridDim.x;
@@ -217,6 +220,11 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       if ((i & 31) == 0) P.mask[i >> 5] = 0;
       if (ch.status[g] == kHit0) {
         ch.res[g] = kResHit0;
+        continue;
+      }
+      if (ch.status[g] == kUncached) {  // never cached: a miss of its own, in no group
+        ch.ent[g] = 0xFFFFFFFFu;
+        ch.res[g] = kResLeader | kResNoSlot | 1u;
         continue;
       }
       const uint32_t e = group_entry(a, g, ch.key[g], ch.len[g]);
@@ -291,12 +299,14 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   const uint64_t per = (((uint64_t)N + G - 1) / G + 31) & ~31ull;
   const uint32_t lo = (uint32_t)min((uint64_t)N, blockIdx.x * per);
   const uint32_t hi = (uint32_t)min((uint64_t)N, lo + per);
-  unsigned long long before = 0, total = 0;
+  unsigned long long before = 0, total = 0, sbefore = 0, stotal = 0;
   if (ok) {
-    uint32_t cnt = 0;
+    uint32_t cnt = 0, scnt = 0;
     for (uint32_t g = lo + threadIdx.x; g < hi; g += kThreads) {
-      if (ldcg_u32(&ch.res[g]) & kResLeader) {
+      const uint32_t r = ldcg_u32(&ch.res[g]);
+      if (r & kResLeader) {
         ++cnt;
+        if (!(r & kResNoSlot)) ++scnt;
         // leave the group table zeroed for the next call: every claimed entry
         // belongs to a group with at least one leader
         const uint32_t e = ch.ent[g];
@@ -307,56 +317,79 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       }
     }
     const unsigned long long c = block_sum<unsigned long long>(cnt, red64);
-    if (threadIdx.x == 0) a.bcount[blockIdx.x] = (uint32_t)c;
+    const unsigned long long sc = block_sum<unsigned long long>(scnt, red64);
+    if (threadIdx.x == 0) {
+      a.bcount[blockIdx.x] = (uint32_t)c;
+      a.bcount[G + blockIdx.x] = (uint32_t)sc;
+    }
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   }
   // ---- D2: exclusive miss rank of every chunk; per-payload start ranks ------
   if (ok) {
     for (uint32_t j = threadIdx.x; j < G; j += kThreads) {
       const uint32_t v = ldcg_u32(&a.bcount[j]);
+      const uint32_t sv = ldcg_u32(&a.bcount[G + j]);
       total += v;
-      if (j < blockIdx.x) before += v;
+      stotal += sv;
+      if (j < blockIdx.x) {
+        before += v;
+        sbefore += sv;
+      }
     }
     before = block_sum<unsigned long long>(before, red64);
     total = block_sum<unsigned long long>(total, red64);
-    if (slots0 + total > a.nslots) {
+    sbefore = block_sum<unsigned long long>(sbefore, red64);
+    stotal = block_sum<unsigned long long>(stotal, red64);
+    if (slots0 + stotal > a.nslots) {
       if (threadIdx.x == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_CAPACITY);
       ok = false;
     }
   }
   if (ok) {
-    unsigned long long running = before;
+    unsigned long long running = before, srunning = sbefore;
     for (uint32_t t = lo; t < hi; t += kThreads) {
       const uint32_t g = t + threadIdx.x;
       const bool valid = g < hi;
-      const bool miss = valid && (ldcg_u32(&ch.res[g]) & kResLeader);
+      const uint32_t rv = valid ? ldcg_u32(&ch.res[g]) : 0u;
+      const bool miss = valid && (rv & kResLeader);
+      const bool stored = miss && !(rv & kResNoSlot);
       const uint32_t mb = __ballot_sync(0xffffffffu, miss);
-      if (lane == 0) warp_cnt[w] = __popc(mb);
+      const uint32_t sb = __ballot_sync(0xffffffffu, stored);
+      if (lane == 0) {
+        warp_cnt[w] = __popc(mb);
+        swarp_cnt[w] = __popc(sb);
+      }
       __syncthreads();
       if (threadIdx.x == 0) {
-        uint32_t acc = 0;
+        uint32_t acc = 0, sacc = 0;
         for (int k = 0; k < kWarps; ++k) {
           warp_off[k] = acc;
           acc += warp_cnt[k];
+          swarp_off[k] = sacc;
+          sacc += swarp_cnt[k];
         }
         warp_cnt[0] = acc;
+        swarp_cnt[0] = sacc;
       }
       __syncthreads();
+      const uint32_t below = (1u << lane) - 1u;
       if (valid) {
-        const uint32_t r = (uint32_t)(running + warp_off[w] + __popc(mb & ((1u << lane) - 1u)));
+        const uint32_t r = (uint32_t)(running + warp_off[w] + __popc(mb & below));
         ch.rank[g] = r;
         if (miss) ch.order[r] = g;
+        if (stored) ch.srank[g] = (uint32_t)(srunning + swarp_off[w] + __popc(sb & below));
         const uint32_t p = ch.pidx[g];
         if (g == desc(a, p).chunk_base) a.pstart[p] = r;
       }
       running += warp_cnt[0];
+      srunning += swarp_cnt[0];
       __syncthreads();
     }
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   }
   // ---- D3: hit masks, miss indices, packed bytes, arena copies, inserts -----
   if (ok) {
-    unsigned long long n_hc = 0, n_hi = 0, n_rej = 0, n_bytes = 0;
+    unsigned long long n_hc = 0, n_hi = 0, n_rej = 0, n_bytes = 0, n_sbytes = 0;
     for (uint32_t t = lo; t < hi; t += kThreads) {
       const uint32_t g = t + threadIdx.x;
       const bool valid = g < hi;
@@ -376,9 +409,10 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
         if (hc || hi2) atomicOr(P.mask + (i >> 5), 1u << (i & 31));
         if (P.chunk_slot) {
           uint32_t sl;
-          if (r & kResHit0) sl = ch.ent[g];                                   // matched slot
-          else if (r & kResDup) sl = (uint32_t)(slots0 + __ldcg(&ch.rank[ch.ent[g]]));  // leader's
-          else sl = (uint32_t)(slots0 + ch.rank[g]);                          // its own new slot
+          if (r & kResHit0) sl = ch.ent[g];                                      // matched slot
+          else if (r & kResDup) sl = (uint32_t)(slots0 + __ldcg(&ch.srank[ch.ent[g]]));  // leader's
+          else if (r & kResNoSlot) sl = kEmptySlot;                              // never cached
+          else sl = (uint32_t)(slots0 + ch.srank[g]);                            // its new slot
           P.chunk_slot[i] = sl;
         }
         if (miss) {
@@ -391,6 +425,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       n_hi += hi2;
       n_rej += rej;
       n_bytes += len;
+      if (!(r & kResNoSlot)) n_sbytes += len;
       // per-payload result counters
       const bool has_res = valid && desc(a, p).result != nullptr;
       gleam_result_t* res = has_res ? desc(a, p).result : nullptr;
@@ -408,9 +443,13 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       const PayloadDesc& P = desc(a, pp);
       const unsigned long long rp = r - __ldcg(&a.pstart[pp]);
       const uint32_t ln = ch.len[gg];
-      const unsigned long long slot = slots0 + r;
       const uint8_t* src = reinterpret_cast<const uint8_t*>(ch.src[gg]);
       uint8_t* d1 = P.packed + rp * a.C;
+      if (ldcg_u32(&ch.res[gg]) & kResNoSlot) {  // sent, never cached
+        warp_copy2(d1, nullptr, src, ln, (((uintptr_t)src | (uintptr_t)d1) & 15) == 0);
+        continue;
+      }
+      const unsigned long long slot = slots0 + __ldcg(&ch.srank[gg]);
       uint8_t* d2 = a.arena + slot * a.C;
       const bool vec = (((uintptr_t)src | (uintptr_t)d1 | (uintptr_t)d2) & 15) == 0;
       warp_copy2(d1, d2, src, ln, vec);
@@ -418,7 +457,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
         a.slot_len[slot] = ln;
         if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-        if (ln >= kPrefixBytes &&
+        if (!a.paper && ln >= kPrefixBytes &&
             !index_insert(a.hints, a.index_mask, ch.hint[gg], (uint32_t)slot, ln))
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       }
@@ -427,12 +466,17 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     n_hi = block_sum<unsigned long long>(n_hi, red64);
     n_rej = block_sum<unsigned long long>(n_rej, red64);
     n_bytes = block_sum<unsigned long long>(n_bytes, red64);
+    n_sbytes = block_sum<unsigned long long>(n_sbytes, red64);
     if (threadIdx.x == 0) {
       atomicAdd(&a.ctl->acc_hits_cache, n_hc);
       atomicAdd(&a.ctl->acc_hits_intra, n_hi);
       atomicAdd(&a.ctl->acc_rejects, n_rej);
       atomicAdd(&a.ctl->acc_miss_bytes, n_bytes);
-      if (blockIdx.x == 0) atomicExch(&a.ctl->acc_misses, total);
+      atomicAdd(&a.ctl->acc_stored_bytes, n_sbytes);
+      if (blockIdx.x == 0) {
+        atomicExch(&a.ctl->acc_misses, total);
+        atomicExch(&a.ctl->acc_stored, stotal);
+      }
     }
   }
 
@@ -453,16 +497,18 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     const unsigned long long hi2 = __ldcg(&a.ctl->acc_hits_intra);
     const unsigned long long rej = __ldcg(&a.ctl->acc_rejects);
     const unsigned long long mbytes = __ldcg(&a.ctl->acc_miss_bytes);
+    const unsigned long long stored = __ldcg(&a.ctl->acc_stored);
+    const unsigned long long sbytes = __ldcg(&a.ctl->acc_stored_bytes);
     if (err == 0) {
       a.dstats[ST_CALLS] += a.ncalls;
       a.dstats[ST_CHUNKS] += N;
       a.dstats[ST_HITS_CACHE] += hc;
       a.dstats[ST_HITS_INTRA] += hi2;
       a.dstats[ST_MISSES] += misses;
-      a.dstats[ST_INSERTS] += misses;
+      a.dstats[ST_INSERTS] += stored;
       a.dstats[ST_REJECTS] += rej;
-      a.dstats[ST_SLOTS_USED] = slots0 + misses;
-      a.dstats[ST_BYTES_USED] += mbytes;
+      a.dstats[ST_SLOTS_USED] = slots0 + stored;
+      a.dstats[ST_BYTES_USED] += sbytes;
     }
     gleam_result_t* t = a.total;
     t->status = err;
@@ -501,6 +547,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     c->unres[0] = c->unres[1] = c->unres[2] = 0;
     c->acc_hits_cache = c->acc_hits_intra = c->acc_rejects = 0;
     c->acc_misses = c->acc_miss_bytes = 0;
+    c->acc_stored = c->acc_stored_bytes = 0;
     c->done = 0;
   }
   __threadfence();

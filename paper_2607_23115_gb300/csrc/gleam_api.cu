@@ -216,10 +216,11 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   cap = std::min<uint64_t>(cap, kMaxChunks);
   if (cap < nchunks) cap = nchunks;
   const uint64_t tcap = next_pow2(2 * cap);
-  const uint64_t sz[11] = {align256(cap),     align256(cap * 8), align256(cap * 4),
+  const uint64_t sz[12] = {align256(cap),     align256(cap * 8), align256(cap * 4),
                            align256(cap * 8), align256(cap * 4), align256(cap * 4),
                            align256(cap * 4), align256(cap * 4), align256(cap * 8),
-                           align256(cap * 4), align256(tcap * sizeof(CallEntry))};
+                           align256(cap * 4), align256(cap * 4),
+                           align256(tcap * sizeof(CallEntry))};
   uint64_t total = 0;
   for (uint64_t x : sz) total += x;
   int rc = cuda_err(cudaEventSynchronize(c->done));
@@ -253,6 +254,8 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   b += sz[8];
   c->ch.order = reinterpret_cast<uint32_t*>(b);
   b += sz[9];
+  c->ch.srank = reinterpret_cast<uint32_t*>(b);
+  b += sz[10];
   c->tbl = reinterpret_cast<CallEntry*>(b);
   c->tbl_cap = tcap;
   c->ws_chunks = cap;
@@ -407,6 +410,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   h.arena = c->arena;
   h.dstats = c->dstats;
   h.key16 = (c->flags & GLEAM_KEY16) ? 1u : 0u;
+  h.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   h.ch = c->ch;
   h.ctl = c->ctl;
 
@@ -438,7 +442,8 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   d.slot_len = c->slot_len;
   d.dstats = c->dstats;
   d.ch = c->ch;
-  d.pstart = count > 1 ? c->d_pstart : c->bcount + c->coop_max_blocks;
+  d.pstart = count > 1 ? c->d_pstart : c->bcount + 2 * c->coop_max_blocks;
+  d.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   d.tbl = c->tbl;
   d.tbl_mask = tcap - 1;
   d.bcount = c->bcount;
@@ -498,7 +503,8 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   *out = nullptr;
   if (chunk_bytes < kMinChunk || chunk_bytes > kMaxChunk || chunk_bytes % 32 != 0)
     return GLEAM_ERR_INVALID_ARG;
-  if ((flags & ~(GLEAM_KEY16 | GLEAM_DEBUG_CHECKS)) != 0) return GLEAM_ERR_INVALID_ARG;
+  if ((flags & ~(GLEAM_KEY16 | GLEAM_DEBUG_CHECKS | GLEAM_PAPER_IDS)) != 0)
+    return GLEAM_ERR_INVALID_ARG;
   const uint64_t nslots = capacity_bytes / chunk_bytes;
   if (nslots == 0 || nslots > 0xFFFFFFFEull) return GLEAM_ERR_INVALID_ARG;
 
@@ -536,8 +542,10 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     c->coop_max_blocks = sms * per_sm;
     if (c->coop_max_blocks <= 0) rc = GLEAM_ERR_CUDA;
   }
-  // block counts, followed by one word used as the single payload's start rank
-  if (rc == GLEAM_OK) step(cudaMalloc(&c->bcount, (c->coop_max_blocks + 1) * sizeof(uint32_t)));
+  // per-block miss and stored-miss counts, then one word used as the single
+  // payload's start rank
+  if (rc == GLEAM_OK)
+    step(cudaMalloc(&c->bcount, (2 * c->coop_max_blocks + 1) * sizeof(uint32_t)));
   if (rc == GLEAM_OK) {
     step(cudaMemset(c->index, 0xFF, c->index_cap * sizeof(IndexEntry)));
     step(cudaMemset(c->hints, 0xFF, c->index_cap * sizeof(IndexEntry)));
@@ -914,11 +922,12 @@ constexpr uint64_t kNaOffEnt = kNaOffRes + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffRank = kNaOffEnt + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffHint = kNaOffRank + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffOrder = kNaOffHint + na_align(kNaChunks * 8);
-constexpr uint64_t kNaOffTbl = kNaOffOrder + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffSrank = kNaOffOrder + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffTbl = kNaOffSrank + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffCtl = kNaOffTbl + na_align(kNaTable * sizeof(CallEntry));
 constexpr uint64_t kNaOffBcount = kNaOffCtl + na_align(sizeof(DevCtl));
-constexpr uint64_t kNaOffResult = kNaOffBcount + na_align((kNaBlocks + 1) * 4);
-constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~4.6 MiB
+constexpr uint64_t kNaOffResult = kNaOffBcount + na_align((2 * kNaBlocks + 1) * 4);
+constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~4.9 MiB
 
 }  // namespace
 
@@ -982,6 +991,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   ch.rank = reinterpret_cast<uint32_t*>(base + kNaOffRank);
   ch.hint = reinterpret_cast<unsigned long long*>(base + kNaOffHint);
   ch.order = reinterpret_cast<uint32_t*>(base + kNaOffOrder);
+  ch.srank = reinterpret_cast<uint32_t*>(base + kNaOffSrank);
   CallEntry* tbl = reinterpret_cast<CallEntry*>(base + kNaOffTbl);
   DevCtl* ctl = reinterpret_cast<DevCtl*>(base + kNaOffCtl);
   uint32_t* bcount = reinterpret_cast<uint32_t*>(base + kNaOffBcount);
@@ -1004,6 +1014,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   h.arena = c->arena;
   h.dstats = c->dstats;
   h.key16 = (c->flags & GLEAM_KEY16) ? 1u : 0u;
+  h.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   h.ch = ch;
   h.ctl = ctl;
   if ((rc = cuda_err(launch_hash(h, aligned, s))) != GLEAM_OK) return rc;
@@ -1021,7 +1032,8 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.slot_len = c->slot_len;
   d.dstats = c->dstats;
   d.ch = ch;
-  d.pstart = bcount + kNaBlocks;
+  d.pstart = bcount + 2 * kNaBlocks;
+  d.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   d.tbl = tbl;
   d.tbl_mask = tcap - 1;
   d.bcount = bcount;

@@ -33,14 +33,15 @@ struct __align__(8) CallEntry {
 };
 
 // Per-chunk outcome of the probe/verify kernel.
-enum : uint8_t { kMissNoCand = 0, kMissCand = 1, kHit0 = 2 };
+enum : uint8_t { kMissNoCand = 0, kMissCand = 1, kHit0 = 2, kUncached = 3 };
 
 // Per-chunk resolution word of the dedup kernel.
 constexpr uint32_t kResUnresolved = 0;
 constexpr uint32_t kResHit0 = 0x20000000u;     // byte-equal to a cached chunk
 constexpr uint32_t kResDup = 0x40000000u;      // byte-equal to an earlier miss
 constexpr uint32_t kResLeader = 0x80000000u;   // | round in which it was resolved
-constexpr uint32_t kResRoundMask = 0x1FFFFFFFu;
+constexpr uint32_t kResNoSlot = 0x10000000u;   // a miss that is never cached
+constexpr uint32_t kResRoundMask = 0x0FFFFFFFu;
 
 // Device counters of one cache, in gleam_stats_t order (first nine fields).
 enum StatIdx {
@@ -48,7 +49,7 @@ enum StatIdx {
   ST_REJECTS, ST_SLOTS_USED, ST_BYTES_USED, ST_COUNT
 };
 
-// Per-call control block, zeroed before every call.
+// Per-call control block; starts zeroed and every dedup kernel leaves it zeroed.
 struct DevCtl {
   unsigned int bar_count;
   unsigned int bar_gen;
@@ -61,6 +62,8 @@ struct DevCtl {
   unsigned long long acc_rejects;
   unsigned long long acc_misses;
   unsigned long long acc_miss_bytes;
+  unsigned long long acc_stored;
+  unsigned long long acc_stored_bytes;
 };
 
 // Position of a key in a power-of-two table: the 64-bit finaliser of
@@ -106,6 +109,7 @@ struct ChunkArrays {
   uint32_t* rank;            // exclusive count of misses before the chunk
   unsigned long long* hint;  // prefix hint (chunks of at least kPrefixBytes)
   uint32_t* order;           // order[r] = chunk number of the miss of rank r
+  uint32_t* srank;           // exclusive count of stored (cached) misses before the chunk
 };
 
 // Speculative verify.  After the first kPrefixBytes of a chunk the four XXH64
@@ -132,6 +136,7 @@ struct HashArgs {
   const uint8_t* arena;
   const unsigned long long* dstats;
   uint32_t key16;
+  uint32_t paper;            // GLEAM_PAPER_IDS: MD5-prefix keys, small chunks uncached
   ChunkArrays ch;
   DevCtl* ctl;
 };
@@ -159,7 +164,11 @@ struct DedupArgs {
   unsigned long long ncalls; // payloads with n > 0
   unsigned long long wait_ns;
   int skip_block;
+  uint32_t paper;            // no prefix hints are kept in GLEAM_PAPER_IDS mode
 };
+
+// Paper-identifier mode (App. B.1): chunks shorter than this get no entry.
+constexpr uint32_t kPaperMinCached = 1024;
 
 cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s);
 cudaError_t launch_dedup(const DedupArgs& a, int grid, cudaStream_t s);

@@ -13,6 +13,8 @@
 // index with the full fingerprint; the hinted slot is a hit if it is a
 // key+length candidate and compared equal, and any other candidate is
 // compared by re-reading both copies.
+#include <cmath>
+
 #include "gleam_internal.cuh"
 #include "xxh64_device.cuh"
 
@@ -555,6 +557,145 @@ __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a
   }
 }
 
+// ---------------------------------------------------------------------------
+// Paper-identifier mode (App. B.1): the key is MD5 (RFC 1321) of the chunk's
+// first min(len, 128) bytes, computed by one lane; candidates are then
+// compared with the payload directly, so no pass over the whole chunk is
+// needed for the key and a chunk without candidates costs only its prefix.
+// ---------------------------------------------------------------------------
+struct Md5Table {
+  uint32_t k[64];  // floor(2^32 * |sin(i + 1)|)
+};
+
+__device__ __forceinline__ uint32_t rotl32(uint32_t x, int r) { return (x << r) | (x >> (32 - r)); }
+
+// First 8 digest bytes (little-endian) of MD5 over p[0, m), m <= 128.
+__device__ unsigned long long md5_prefix_key(const uint8_t* p, uint32_t m, const uint32_t* K) {
+  const uint32_t total = ((m + 8) / 64 + 1) * 64;  // message + 0x80 + padding + length
+  const unsigned long long bits = (unsigned long long)m * 8;
+  uint32_t a0 = 0x67452301u, b0 = 0xefcdab89u, c0 = 0x98badcfeu, d0 = 0x10325476u;
+  for (uint32_t blk = 0; blk < total; blk += 64) {
+    uint32_t x[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      uint32_t w = 0;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t q = blk + 4 * j + k;
+        uint32_t byte;
+        if (q < m) byte = p[q];
+        else if (q == m) byte = 0x80u;
+        else if (q >= total - 8) byte = (uint32_t)(bits >> (8 * (q - (total - 8)))) & 0xFFu;
+        else byte = 0u;
+        w |= byte << (8 * k);
+      }
+      x[j] = w;
+    }
+    uint32_t a = a0, b = b0, c = c0, d = d0;
+#pragma unroll
+    for (int i = 0; i < 64; ++i) {
+      uint32_t f;
+      int g, r;
+      if (i < 16) {
+        f = (b & c) | (~b & d);
+        g = i;
+        r = (i & 3) == 0 ? 7 : (i & 3) == 1 ? 12 : (i & 3) == 2 ? 17 : 22;
+      } else if (i < 32) {
+        f = (d & b) | (~d & c);
+        g = (5 * i + 1) & 15;
+        r = (i & 3) == 0 ? 5 : (i & 3) == 1 ? 9 : (i & 3) == 2 ? 14 : 20;
+      } else if (i < 48) {
+        f = b ^ c ^ d;
+        g = (3 * i + 5) & 15;
+        r = (i & 3) == 0 ? 4 : (i & 3) == 1 ? 11 : (i & 3) == 2 ? 16 : 23;
+      } else {
+        f = c ^ (b | ~d);
+        g = (7 * i) & 15;
+        r = (i & 3) == 0 ? 6 : (i & 3) == 1 ? 10 : (i & 3) == 2 ? 15 : 21;
+      }
+      const uint32_t t = d;
+      d = c;
+      c = b;
+      b = b + rotl32(a + f + K[i] + x[g], r);
+      a = t;
+    }
+    a0 += a;
+    b0 += b;
+    c0 += c;
+    d0 += d;
+  }
+  return (unsigned long long)a0 | ((unsigned long long)b0 << 32);
+}
+
+template <bool kAligned>
+__global__ void __launch_bounds__(kHashThreads) k_probe_paper(HashArgs a, Md5Table tab) {
+  const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
+  if (g >= a.Ntot) return;  // whole groups leave together
+  const uint32_t lane = threadIdx.x & 3;
+  const int gbase = threadIdx.x & 28;
+  const unsigned gmask = 0xFu << gbase;
+
+  uint32_t pid = 0;
+  const uint8_t* buf;
+  unsigned long long n, base;
+  if (a.count > 1) {
+    pid = find_payload(a.table, a.count, g);
+    buf = a.table[pid].buf;
+    n = a.table[pid].n;
+    base = a.table[pid].chunk_base;
+  } else {
+    buf = a.one.buf;
+    n = a.one.n;
+    base = a.one.chunk_base;
+  }
+  const unsigned long long start = (g - base) * a.C;
+  const uint32_t len = (uint32_t)min(a.C, n - start);
+  const uint8_t* p = buf + start;
+
+  unsigned long long key = 0;
+  if (lane == 0) key = md5_prefix_key(p, min(len, 128u), tab.k);
+  key = group_shfl(key, gmask, gbase);
+  if (a.key16) key &= 0xFFFFULL;
+
+  bool hit = false, cand = false;
+  uint32_t hit_slot = kEmptySlot;
+  if (len >= kPaperMinCached) {
+    const unsigned long long slots_used = a.dstats[ST_SLOTS_USED];
+    unsigned long long pos = mix64(key) & a.index_mask;
+    for (unsigned long long probe = 0; probe <= a.index_mask; ++probe) {
+      const IndexEntry e = a.index[pos];
+      if (e.slot == kEmptySlot) break;
+      if (e.key == key && e.len == len) {
+        cand = true;
+        if (e.slot >= slots_used) {
+          if (lane == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+        } else if (group_equal<kAligned>(p, a.arena + (uint64_t)e.slot * a.C, len, lane, gmask)) {
+          hit = true;
+          hit_slot = e.slot;
+          break;
+        }
+      }
+      pos = (pos + 1) & a.index_mask;
+    }
+  }
+  if (lane == 0) {
+    a.ch.status[g] = len < kPaperMinCached ? kUncached : hit ? kHit0 : cand ? kMissCand : kMissNoCand;
+    a.ch.key[g] = key;
+    a.ch.len[g] = len;
+    a.ch.src[g] = (unsigned long long)p;
+    a.ch.pidx[g] = pid;
+    a.ch.hint[g] = 0;
+    if (hit) a.ch.ent[g] = hit_slot;
+  }
+}
+
+Md5Table md5_table() {
+  Md5Table t;
+  for (int i = 0; i < 64; ++i)
+    t.k[i] = (uint32_t)std::floor(std::fabs(std::sin((double)(i + 1))) * 4294967296.0);
+  return t;
+}
+
 }  // namespace
 
 cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
@@ -562,6 +703,12 @@ cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
   const unsigned long long threads = a.Ntot * 4;
   const unsigned grid = (unsigned)((threads + kHashThreads - 1) / kHashThreads);
   const bool probe = a.index != nullptr;
+  if (probe && a.paper) {
+    static const Md5Table tab = md5_table();
+    if (aligned) k_probe_paper<true><<<grid, kHashThreads, 0, s>>>(a, tab);
+    else k_probe_paper<false><<<grid, kHashThreads, 0, s>>>(a, tab);
+    return cudaGetLastError();
+  }
 #if GLEAM_STAGED_HASH
   if (aligned && (a.C % 32 == 0 || a.Ntot == 1)) {
     // per device and cheap: set on every launch
