@@ -101,6 +101,15 @@ def build_workload(name, dev, sample_budget):
     from paper_2607_23115_gb300 import workloads as W
     from paper_2607_23115_gb300.workloads import Upload
 
+    if name == "llama3-8b-paper-ids":
+        from paper_2607_23115_gb300 import binding as B
+        wl = build_workload("llama3-8b", dev, sample_budget)
+        wl.name = "llama3-8b-bf16-per-tensor-paper-ids"
+        wl.desc = wl.desc + "; the paper's identifier (MD5 of each chunk's first 1024 bits) " \
+                            "instead of XXH64, byte verify kept"
+        wl.flags = B.GLEAM_PAPER_IDS
+        return wl
+
     if name.startswith("llama3-8b"):
         shapes = W.llama3_8b_shapes()
         variants = {"llama3-8b": (shapes, 24 * GiB, "Llama-3-8B-shaped bf16 upload, 291 tensors"),
@@ -228,7 +237,8 @@ def build_workload(name, dev, sample_budget):
     raise ValueError("unknown workload %r" % name)
 
 
-WORKLOADS = ["llama3-8b", "llama3-8b-layer", "llama3-8b-4layers", "gpt2-small",
+WORKLOADS = ["llama3-8b", "llama3-8b-paper-ids", "llama3-8b-layer", "llama3-8b-4layers",
+             "gpt2-small",
              "gpt2-small-pass1", "fp16-64m", "small-calls"] + \
     ["adversarial-%dk%s" % (c, m) for c in (1, 4, 16, 64) for m in ("", "-key16")]
 
@@ -300,7 +310,8 @@ def oracle_time(wl, budget, offset=0):
     the timed calls.  Returns (payload bytes, seconds, description)."""
     import oracle
     pre, pays, text = wl.sample(budget, offset)
-    oc = oracle.OracleCache(wl.capacity, wl.C, oracle.KEY16 if wl.flags & 1 else 0)
+    oc = oracle.OracleCache(wl.capacity, wl.C, (oracle.KEY16 if wl.flags & 1 else 0) |
+                            (oracle.PAPER_IDS if wl.flags & 4 else 0))
     for orig, row in getattr(wl, "crafted_host", []):
         oc.debug_insert(oracle.xxh64(orig), row)
     for x in pre:
