@@ -513,7 +513,7 @@ def run_gleam(args, rank, world, local_rank):
                 "traffic": traffic, "algorithmic_bytes_per_launch": round(k0_bytes),
                 "avg_launch_ms": round(k0_ms, 5),
                 "kernel_share_of_step": round((kms[0]) / ms if ms else 0, 4),
-                "k_dedup_avg_launch_ms": round(kms[1] / max(1, klaunch[1]), 5)}
+                "k_dedup_k_pack_avg_ms": round(kms[1] / max(1, klaunch[1]), 5)}
     pipe_gbs = pipeline_bytes / (ms_per_step * 1e-3) / 1e9
     pipeline = {"min_bytes_per_step": pipeline_bytes,
                 "achieved_gbs": round(pipe_gbs, 1),

@@ -387,12 +387,43 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     }
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   }
-  // ---- D3: hit masks, miss indices, packed bytes, arena copies, inserts -----
+  // totals for k_pack (the capacity check above left them unpublished on error)
+  if (ok && blockIdx.x == 0 && threadIdx.x == 0) {
+    a.ctl->acc_misses = total;
+    a.ctl->acc_stored = stotal;
+  }
+}
+
+// Second kernel of the call (a regular launch sized for the copies): hit
+// masks, miss indices, chunk slots, per-payload counters, then every miss by
+// rank copied by whole warps to the packed output and its arena slot and
+// inserted into the index; the last block publishes the counters and results
+// and leaves the per-call state zeroed.  Nothing is written after an error.
+__global__ void __launch_bounds__(kThreads) k_pack(DedupArgs a) {
+  __shared__ unsigned long long red64[kWarps];
+  __shared__ unsigned long long s_slots0, s_total;
+  __shared__ int s_err;
+  const uint32_t G = gridDim.x;
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t N = (uint32_t)a.Ntot;
+  const ChunkArrays& ch = a.ch;
+  if (threadIdx.x == 0) {
+    s_slots0 = *(volatile const unsigned long long*)&a.dstats[ST_SLOTS_USED];
+    s_err = ld_volatile_s32(&a.ctl->err);
+    s_total = __ldcg(&a.ctl->acc_misses);
+  }
+  __syncthreads();
+  const unsigned long long slots0 = s_slots0;
+  const unsigned long long total = s_total;
+  const bool ok = s_err == 0;
+
+  // ---- hit masks, miss indices, chunk slots, counters ------------------------
   if (ok) {
     unsigned long long n_hc = 0, n_hi = 0, n_rej = 0, n_bytes = 0, n_sbytes = 0;
-    for (uint32_t t = lo; t < hi; t += kThreads) {
-      const uint32_t g = t + threadIdx.x;
-      const bool valid = g < hi;
+    for (unsigned long long t = (unsigned long long)blockIdx.x * kThreads; t < N;
+         t += (unsigned long long)G * kThreads) {
+      const uint32_t g = (uint32_t)(t + threadIdx.x);
+      const bool valid = t + threadIdx.x < N;
       const uint32_t r = valid ? ldcg_u32(&ch.res[g]) : 0u;
       const uint32_t p = valid ? ch.pidx[g] : 0xFFFFFFFFu;
       const bool miss = valid && (r & kResLeader);
@@ -473,10 +504,6 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       atomicAdd(&a.ctl->acc_rejects, n_rej);
       atomicAdd(&a.ctl->acc_miss_bytes, n_bytes);
       atomicAdd(&a.ctl->acc_stored_bytes, n_sbytes);
-      if (blockIdx.x == 0) {
-        atomicExch(&a.ctl->acc_misses, total);
-        atomicExch(&a.ctl->acc_stored, stotal);
-      }
     }
   }
 
@@ -609,10 +636,14 @@ int dedup_blocks_per_sm() {
   return nb < GLEAM_DEDUP_BLOCKS_PER_SM ? nb : GLEAM_DEDUP_BLOCKS_PER_SM;
 }
 
-cudaError_t launch_dedup(const DedupArgs& a, int grid, cudaStream_t s) {
+cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s) {
   DedupArgs copy = a;
   void* args[] = {&copy};
-  return cudaLaunchCooperativeKernel((void*)k_dedup, dim3(grid), dim3(kThreads), args, 0, s);
+  cudaError_t e =
+      cudaLaunchCooperativeKernel((void*)k_dedup, dim3(grid), dim3(kThreads), args, 0, s);
+  if (e != cudaSuccess) return e;
+  k_pack<<<pack_grid, kThreads, 0, s>>>(a);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s) {

@@ -48,6 +48,7 @@ struct gleam_cache {
   gleam_result_t* d_result = nullptr;
   gleam_result_t* h_result = nullptr;  // pinned
   int coop_max_blocks = 0;
+  int num_sms = 0;
   cudaEvent_t done = nullptr;
 
   unsigned long long wait_ns = 4000000000ULL;
@@ -353,6 +354,14 @@ int dedup_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
   return (int)std::max<uint64_t>(1, std::min<uint64_t>(c->coop_max_blocks, want));
 }
 
+// Blocks of the pack kernel: one per 256 chunks or per kBytesPerDedupBlock of
+// payload, up to 8 per SM.
+int pack_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
+  const uint64_t want = std::max<uint64_t>((nchunks + 255) / 256,
+                                           (nbytes + kBytesPerDedupBlock - 1) / kBytesPerDedupBlock);
+  return (int)std::max<uint64_t>(1, std::min<uint64_t>(8ull * c->num_sms, want));
+}
+
 // Enqueues one dedup call over `count` payloads on stream s, ordered after
 // the cache's previous call.  Caller holds c->mu and the device.
 int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
@@ -458,7 +467,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     grid = std::max(grid, std::min(2, c->coop_max_blocks));  // someone must be left waiting
     if (d.skip_block >= grid) d.skip_block = grid - 1;
   }
-  if ((rc = cuda_err(launch_dedup(d, grid, s))) != GLEAM_OK) {
+  if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, Ntot, nbytes), s))) != GLEAM_OK) {
     cudaMemsetAsync(c->ctl, 0, sizeof(DevCtl), s);  // the hash kernel may have flagged it
     return rc;
   }
@@ -540,6 +549,7 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     step(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device));
     const int per_sm = dedup_blocks_per_sm();
     c->coop_max_blocks = sms * per_sm;
+    c->num_sms = sms;
     if (c->coop_max_blocks <= 0) rc = GLEAM_ERR_CUDA;
   }
   // per-block miss and stored-miss counts, then one word used as the single
@@ -1043,6 +1053,6 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.wait_ns = c->wait_ns;
   d.skip_block = -1;
   const int grid = dedup_grid(c, N, n);
-  if ((rc = cuda_err(launch_dedup(d, grid, s))) != GLEAM_OK) return rc;
+  if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, N, n), s))) != GLEAM_OK) return rc;
   return cuda_err(cudaEventRecord(c->done, s));
 }

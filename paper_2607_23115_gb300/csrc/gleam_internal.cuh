@@ -171,7 +171,9 @@ struct DedupArgs {
 constexpr uint32_t kPaperMinCached = 1024;
 
 cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s);
-cudaError_t launch_dedup(const DedupArgs& a, int grid, cudaStream_t s);
+// The cooperative resolve/rank kernel on `grid` blocks, then the pack kernel
+// (masks, indices, copies, inserts, publish) on `pack_grid` blocks.
+cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s);
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
                                 unsigned long long* dstats, unsigned long long key,
                                 uint32_t slot, uint32_t len, DevCtl* ctl, cudaStream_t s);
