@@ -187,14 +187,21 @@ def build_workload(name, dev, sample_budget):
                                              "prefilled with the same half (untimed)")
         return wl
 
-    if name == "small-calls":
+    if name in ("small-calls", "small-calls-10k"):
         C = 4 * KiB
-        wl = Workload("small-call-stream-100k", "100,000 payloads of uniform random bytes, sizes "
-                      "log-uniform in 4 KiB-1 MiB (18.8 GB); cache prefilled with 2 GB of "
-                      "unrelated chunks; 32 GiB cache", C, 32 * GiB)
-        up = W.small_call_upload(100000, device=dev)
+        count = 100000 if name == "small-calls" else 10000
+        if count == 100000:
+            wl = Workload("small-call-stream-100k", "100,000 payloads of uniform random bytes, "
+                          "sizes log-uniform in 4 KiB-1 MiB (18.8 GB); cache prefilled with 2 GB "
+                          "of unrelated chunks; 32 GiB cache", C, 32 * GiB)
+        else:
+            wl = Workload("small-call-stream-10k", "10,000 payloads of uniform random bytes, "
+                          "sizes log-uniform in 4 KiB-1 MiB (1.9 GB); cache prefilled with 0.2 GB "
+                          "of unrelated chunks; 4 GiB cache (a profiling-size case)", C, 4 * GiB)
+        up = W.small_call_upload(count, device=dev)
         wl.up = up
-        wl.prefill = [[W.random_bytes(2 * 10**9 // C * C, seed=W.SEED_PREFILL, device=dev)]]
+        pre_bytes = 2 * 10**9 if count == 100000 else 2 * 10**8
+        wl.prefill = [[W.random_bytes(pre_bytes // C * C, seed=W.SEED_PREFILL, device=dev)]]
         wl.expect_misses = sum((s + C - 1) // C for s in up.sizes)
 
         def sample(budget, offset):
@@ -239,7 +246,7 @@ def build_workload(name, dev, sample_budget):
 
 WORKLOADS = ["llama3-8b", "llama3-8b-paper-ids", "llama3-8b-layer", "llama3-8b-4layers",
              "gpt2-small",
-             "gpt2-small-pass1", "fp16-64m", "small-calls"] + \
+             "gpt2-small-pass1", "fp16-64m", "small-calls", "small-calls-10k"] + \
     ["adversarial-%dk%s" % (c, m) for c in (1, 4, 16, 64) for m in ("", "-key16")]
 
 

@@ -14,7 +14,8 @@
 //   * a leader counts as a verify reject iff the cache had a key+length
 //     candidate for it, or an earlier leader of the call has its key+length.
 //
-// One cooperative launch does it all, separated by bounded grid barriers:
+// Two launches follow the hash kernel.  k_dedup, cooperative, with phases
+// separated by bounded grid barriers:
 //   A  outputs are cleared; every non-resident chunk claims the entry of its
 //      (key, length) in a per-call table and posts its number as the group
 //      minimum;
@@ -24,10 +25,13 @@
 //      one key: a true 64-bit collision, or KEY16 test mode);
 //   C  group minima of the remaining chunks are reset and re-posted (A);
 //   D  leaders are counted per contiguous block range; the exclusive rank of
-//      every chunk follows from the block totals plus warp ballots; then hit
-//      masks, miss indices, packed bytes, arena copies and index entries are
-//      written.
-// The last block to finish publishes the counters and the results.
+//      every chunk (and of every stored miss) follows from the block totals
+//      plus warp ballots.
+// k_pack, a regular launch of one wave, then writes hit masks, miss indices,
+// chunk slots and per-payload counters, copies every miss by rank to the
+// packed output and its arena slot and inserts it into the index; its last
+// block publishes the counters and results and leaves the per-call state
+// zeroed for the next call.
 #include "gleam_internal.cuh"
 
 namespace gleam {
@@ -46,6 +50,14 @@ constexpr int kWarps = kThreads / 32;
 #endif
 #ifndef GLEAM_DEDUP_CHUNKS_PER_BLOCK
 #define GLEAM_DEDUP_CHUNKS_PER_BLOCK 1024
+#endif
+#ifndef GLEAM_PACK_MINBLOCKS
+#define GLEAM_PACK_MINBLOCKS 3
+#endif
+#if GLEAM_PACK_MINBLOCKS > 1
+#define GLEAM_PACK_BOUNDS __launch_bounds__(kThreads, GLEAM_PACK_MINBLOCKS)
+#else
+#define GLEAM_PACK_BOUNDS __launch_bounds__(kThreads)
 #endif
 constexpr int kCopyVec = GLEAM_COPY_VEC;  // 16-byte vectors per lane in flight while copying
 
@@ -174,12 +186,11 @@ __device__ __forceinline__ T block_sum(T v, T* red) {
   return t;
 }
 
-// Adds v to *dst once per group of lanes that share `key` (warp-aggregated).
-__device__ __forceinline__ void add_by_key(unsigned long long* dst, uint32_t key, uint32_t v,
-                                           bool active) {
-  const unsigned peers = __match_any_sync(0xffffffffu, active ? key : 0xFFFFFFFFu);
-  const uint32_t sum = __reduce_add_sync(peers, active ? v : 0u);
-  if (active && (threadIdx.x & 31) == (uint32_t)(__ffs(peers) - 1) && sum) atomicAdd(dst, sum);
+// Sum of v over the lanes of `peers`, added to *dst by the one lane of the
+// group whose dst is not null.
+__device__ __forceinline__ void add_in_group(unsigned long long* dst, unsigned peers, uint32_t v) {
+  const uint32_t sum = __reduce_add_sync(peers, v);
+  if (dst && sum) atomicAdd(dst, sum);
 }
 
 __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
@@ -399,7 +410,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
 // rank copied by whole warps to the packed output and its arena slot and
 // inserted into the index; the last block publishes the counters and results
 // and leaves the per-call state zeroed.  Nothing is written after an error.
-__global__ void __launch_bounds__(kThreads) k_pack(DedupArgs a) {
+__global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ unsigned long long s_slots0, s_total;
   __shared__ int s_err;
@@ -428,16 +439,22 @@ __global__ void __launch_bounds__(kThreads) k_pack(DedupArgs a) {
       const uint32_t p = valid ? ch.pidx[g] : 0xFFFFFFFFu;
       const bool miss = valid && (r & kResLeader);
       bool hc = false, hi2 = false, rej = false;
-      uint32_t len = 0;
+      uint32_t len = 0, bit = 0;
+      unsigned long long mw = 0;  // address of the chunk's hit-mask word, if a hit
+      gleam_result_t* res = nullptr;
       if (valid) {
         const PayloadDesc& P = desc(a, p);
         const unsigned long long i = g - P.chunk_base;
+        res = P.result;
         if (r & kResHit0) hc = true;
         if (r & kResDup) {
           if (ch.pidx[ch.ent[g]] == p) hi2 = true;  // leader in the same payload
           else hc = true;                           // inserted by an earlier payload
         }
-        if (hc || hi2) atomicOr(P.mask + (i >> 5), 1u << (i & 31));
+        if (hc || hi2) {
+          mw = (unsigned long long)(P.mask + (i >> 5));
+          bit = 1u << (i & 31);
+        }
         if (P.chunk_slot) {
           uint32_t sl;
           if (r & kResHit0) sl = ch.ent[g];                                      // matched slot
@@ -457,34 +474,55 @@ __global__ void __launch_bounds__(kThreads) k_pack(DedupArgs a) {
       n_rej += rej;
       n_bytes += len;
       if (!(r & kResNoSlot)) n_sbytes += len;
-      // per-payload result counters
-      const bool has_res = valid && desc(a, p).result != nullptr;
-      gleam_result_t* res = has_res ? desc(a, p).result : nullptr;
-      add_by_key(has_res ? (unsigned long long*)&res->n_hit_cache : nullptr, p, hc, has_res);
-      add_by_key(has_res ? (unsigned long long*)&res->n_hit_intra : nullptr, p, hi2, has_res);
-      add_by_key(has_res ? (unsigned long long*)&res->n_miss : nullptr, p, miss, has_res);
-      add_by_key(has_res ? (unsigned long long*)&res->verify_rejects : nullptr, p, rej, has_res);
-      add_by_key(has_res ? (unsigned long long*)&res->miss_bytes : nullptr, p, len, has_res);
+      // hit-mask words and per-payload result counters: one atomic per group
+      // of lanes that share the word or the payload
+      const unsigned mpeers = __match_any_sync(0xffffffffu, mw);
+      const uint32_t bits = __reduce_or_sync(mpeers, bit);
+      if (mw && lane == (uint32_t)(__ffs(mpeers) - 1)) atomicOr((uint32_t*)mw, bits);
+      const unsigned peers = __match_any_sync(0xffffffffu, res ? p : 0xFFFFFFFFu);
+      const bool lead = res && lane == (uint32_t)(__ffs(peers) - 1);
+      add_in_group((unsigned long long*)(lead ? &res->n_hit_cache : nullptr), peers, hc);
+      add_in_group((unsigned long long*)(lead ? &res->n_hit_intra : nullptr), peers, hi2);
+      add_in_group((unsigned long long*)(lead ? &res->n_miss : nullptr), peers, miss);
+      add_in_group((unsigned long long*)(lead ? &res->verify_rejects : nullptr), peers, rej);
+      add_in_group((unsigned long long*)(lead ? &res->miss_bytes : nullptr), peers, len);
     }
-    // every miss, by rank, copied by whole warps of the whole grid
-    const uint32_t gw = blockIdx.x * kWarps + w, nw = G * kWarps;
-    for (unsigned long long r = gw; r < total; r += nw) {
-      const uint32_t gg = __ldcg(&ch.order[r]);
-      const uint32_t pp = ch.pidx[gg];
-      const PayloadDesc& P = desc(a, pp);
-      const unsigned long long rp = r - __ldcg(&a.pstart[pp]);
-      const uint32_t ln = ch.len[gg];
-      const uint8_t* src = reinterpret_cast<const uint8_t*>(ch.src[gg]);
-      uint8_t* d1 = P.packed + rp * a.C;
-      if (ldcg_u32(&ch.res[gg]) & kResNoSlot) {  // sent, never cached
-        warp_copy2(d1, nullptr, src, ln, (((uintptr_t)src | (uintptr_t)d1) & 15) == 0);
-        continue;
+    // Every miss, by rank.  Warp gw owns the contiguous ranks [lo, hi): its
+    // lanes fetch the metadata of 32 ranks at once, the whole warp copies the
+    // 32 chunks one after the other to the packed output and their arena
+    // slots, then each lane inserts its own chunk (32 independent probes).
+    const unsigned long long nw = (unsigned long long)G * kWarps;
+    const unsigned long long gw = (unsigned long long)blockIdx.x * kWarps + w;
+    const unsigned long long lo = total * gw / nw, hi = total * (gw + 1) / nw;
+    for (unsigned long long base = lo; base < hi; base += 32) {
+      const unsigned long long r = base + lane;
+      const bool have = r < hi;
+      uint32_t gg = 0, ln = 0;
+      bool cached = false;
+      unsigned long long slot = 0, src = 0, d1 = 0, d2 = 0;
+      if (have) {
+        gg = ch.order[r];
+        const uint32_t pp = ch.pidx[gg];
+        const PayloadDesc& P = desc(a, pp);
+        ln = ch.len[gg];
+        src = ch.src[gg];
+        d1 = (unsigned long long)(P.packed + (r - a.pstart[pp]) * a.C);
+        cached = !(ch.res[gg] & kResNoSlot);  // else sent, never cached
+        if (cached) {
+          slot = slots0 + ch.srank[gg];
+          d2 = (unsigned long long)(a.arena + slot * a.C);
+        }
       }
-      const unsigned long long slot = slots0 + __ldcg(&ch.srank[gg]);
-      uint8_t* d2 = a.arena + slot * a.C;
-      const bool vec = (((uintptr_t)src | (uintptr_t)d1 | (uintptr_t)d2) & 15) == 0;
-      warp_copy2(d1, d2, src, ln, vec);
-      if (lane == 0) {
+      const uint32_t m = (uint32_t)((hi - base) < 32ull ? (hi - base) : 32ull);
+      for (uint32_t j = 0; j < m; ++j) {
+        const unsigned long long sj = __shfl_sync(0xffffffffu, src, j);
+        const unsigned long long xj = __shfl_sync(0xffffffffu, d1, j);
+        const unsigned long long yj = __shfl_sync(0xffffffffu, d2, j);
+        const uint32_t lj = __shfl_sync(0xffffffffu, ln, j);
+        warp_copy2(reinterpret_cast<uint8_t*>(xj), reinterpret_cast<uint8_t*>(yj),
+                   reinterpret_cast<const uint8_t*>(sj), lj, ((sj | xj | yj) & 15) == 0);
+      }
+      if (have && cached) {
         a.slot_len[slot] = ln;
         if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
@@ -627,6 +665,14 @@ __global__ void k_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t*
 int dedup_threads() { return kThreads; }
 
 int dedup_chunks_per_block() { return GLEAM_DEDUP_CHUNKS_PER_BLOCK; }
+
+// Co-resident blocks per SM of the pack kernel.
+int pack_blocks_per_sm() {
+  int nb = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_pack, kThreads, 0) != cudaSuccess)
+    return 0;
+  return nb;
+}
 
 // Co-resident blocks per SM for the cooperative launch (capped).
 int dedup_blocks_per_sm() {

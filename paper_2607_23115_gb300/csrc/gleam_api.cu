@@ -48,7 +48,7 @@ struct gleam_cache {
   gleam_result_t* d_result = nullptr;
   gleam_result_t* h_result = nullptr;  // pinned
   int coop_max_blocks = 0;
-  int num_sms = 0;
+  int pack_max_blocks = 0;  // pack kernel: all co-resident blocks
   cudaEvent_t done = nullptr;
 
   unsigned long long wait_ns = 4000000000ULL;
@@ -355,11 +355,11 @@ int dedup_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
 }
 
 // Blocks of the pack kernel: one per 256 chunks or per kBytesPerDedupBlock of
-// payload, up to 8 per SM.
+// payload, up to one full wave of co-resident blocks.
 int pack_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
   const uint64_t want = std::max<uint64_t>((nchunks + 255) / 256,
                                            (nbytes + kBytesPerDedupBlock - 1) / kBytesPerDedupBlock);
-  return (int)std::max<uint64_t>(1, std::min<uint64_t>(8ull * c->num_sms, want));
+  return (int)std::max<uint64_t>(1, std::min<uint64_t>(c->pack_max_blocks, want));
 }
 
 // Enqueues one dedup call over `count` payloads on stream s, ordered after
@@ -549,8 +549,8 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     step(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c->device));
     const int per_sm = dedup_blocks_per_sm();
     c->coop_max_blocks = sms * per_sm;
-    c->num_sms = sms;
-    if (c->coop_max_blocks <= 0) rc = GLEAM_ERR_CUDA;
+    c->pack_max_blocks = sms * pack_blocks_per_sm();
+    if (c->coop_max_blocks <= 0 || c->pack_max_blocks <= 0) rc = GLEAM_ERR_CUDA;
   }
   // per-block miss and stored-miss counts, then one word used as the single
   // payload's start rank

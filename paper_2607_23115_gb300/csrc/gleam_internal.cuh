@@ -195,6 +195,7 @@ cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s);
 int dedup_threads();
 int dedup_chunks_per_block();
 int dedup_blocks_per_sm();
+int pack_blocks_per_sm();
 
 // ---------------------------------------------------------------------------
 // Device helpers
