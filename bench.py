@@ -549,7 +549,9 @@ def run_gleam(args, rank, world, local_rank):
         "pipeline_roofline": pipeline,
         "roofline": roofline,
         "per_call_async": per_call,
-        "gpu_launches": 2 * args.steps,
+        # the library's kernels in the timed region, counted by its profile
+        # events: one hash launch and one k_dedup + k_pack pair per call
+        "gpu_launches": int(klaunch[0]) + 2 * int(klaunch[1]),
         "clocks": clk,
     }
 
