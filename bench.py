@@ -3,10 +3,11 @@
 
 One step = one pass of the whole path (fingerprint, probe, verify, in-call
 dedup, compaction, packing, insertion) over one upload: every tensor of the
-workload is one gleam_dedup_copy_async call, as one cudaMemcpy per tensor
-would be.  The cache is restored from a device snapshot at the start of each
-step (16 MiB index copy, inside the timed region), so every step does the
-same work.  Inputs (16 GB for the default workload) are resident in HBM and
+workload is one payload (as one cudaMemcpy per tensor would be), all of them
+in one gleam_dedup_copy_batch call; the same pass as one
+gleam_dedup_copy_async call per tensor is reported beside it.  The cache is
+restored from a device snapshot at the start of each step (index and hint
+table copies, inside the timed region), so every step does the same work.  Inputs (16 GB for the default workload) are resident in HBM and
 far larger than L2, so no L2 flush is needed between steps.
 
 Default workload: a Llama-3-8B-shaped bf16 weight upload (291 tensors,

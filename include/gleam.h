@@ -289,10 +289,11 @@ int gleam_cache_restore(gleam_cache_t* cache, const gleam_snapshot_t* snap);
 void gleam_snapshot_destroy(gleam_snapshot_t* snap);
 
 /* Kernel timing for benchmarks.  While enabled, every dedup call records CUDA
- * events on its own stream around its two kernels: kernel 0 fingerprints,
- * probes and verifies; kernel 1 resolves duplicates, compacts, packs and
- * inserts.  gleam_cache_profile_read waits for the recorded calls, writes the
- * summed device time (ms) and launch count of kernel k to h_ms[k] and
+ * events on its own stream around its two phases: phase 0 is the kernel that
+ * fingerprints, probes and verifies; phase 1 is the two kernels that resolve
+ * duplicates and rank the misses, then compact, pack and insert.
+ * gleam_cache_profile_read waits for the recorded calls, writes the summed
+ * device time (ms) and count of calls of phase k to h_ms[k] and
  * h_launches[k] for k < nkernels (host arrays), and starts a new tally. */
 int gleam_cache_profile(gleam_cache_t* cache, int enable);
 int gleam_cache_profile_read(gleam_cache_t* cache, double* h_ms, uint64_t* h_launches,

@@ -19,7 +19,7 @@
 //    "xxhash_spec" document): four accumulators over 32-byte stripes,
 //    convergence, merge rounds, length, 8/4/1-byte tails, avalanche.
 //
-// Readings taken where the paper is silent (each also listed in the design doc):
+// Readings taken where the paper is silent:
 //  R1 identifier = XXH64(seed 0) of the whole chunk, as a native u64.
 //  R2 chunks are fixed C bytes; chunk_bytes == 0 in oracle_fingerprint means
 //     one hash over the whole payload (the paper's per-payload identifier).
