@@ -29,13 +29,15 @@ ERR_INVALID_ARG = -1
 ERR_CAPACITY = -4
 KEY16 = 1
 PAPER_IDS = 4
+EVICT_LRU = 8
 NO_SLOT = 0xFFFFFFFF
 
 STAT_FIELDS = (
     "calls", "chunks", "hits_cache", "hits_intra", "misses", "inserts",
     "verify_rejects", "slots_used", "bytes_used", "capacity_bytes", "nslots",
-    "chunk_bytes",
+    "chunk_bytes", "evictions",
 )
+RESULT_FIELDS = ("n_miss", "n_hit_cache", "n_hit_intra", "verify_rejects", "miss_bytes")
 
 
 def build(force: bool = False) -> str:
@@ -74,6 +76,8 @@ def _bind(l):
         l.oracle_cache_destroy.argtypes = [vp]
         l.oracle_dedup.restype = ctypes.c_int64
         l.oracle_dedup.argtypes = [vp, vp, sz, vp, vp, vp, vp]
+        l.oracle_dedup_batch.restype = ctypes.c_int64
+        l.oracle_dedup_batch.argtypes = [vp, sz, vp, vp, vp, vp, vp, vp, vp]
         l.oracle_block_check.restype = ctypes.c_int64
         l.oracle_block_check.argtypes = [vp, vp, u64, vp, vp, u64, vp]
         l.oracle_debug_insert.restype = ctypes.c_int
@@ -162,6 +166,37 @@ class OracleCache:
             r = self._finish(rc, n, nch, mask, miss, packed)
             return r + (slots[:nch].copy(),)
         return self._finish(rc, n, nch, mask, miss, packed)
+
+    def dedup_batch(self, datas, chunk_slots: bool = False):
+        """One call over several payloads (a batch).  Returns (rc, outs, results):
+        outs[k] = (hit_mask, miss_idx, packed[, chunk_slots]) of payload k and
+        results[k] = dict of RESULT_FIELDS; (rc, None, None) on an error."""
+        C = self.chunk_bytes
+        arrs = [_u8(d) for d in datas]
+        count = len(arrs)
+        nch = [(a.size + C - 1) // C for a in arrs]
+        masks = [np.zeros(max(1, (m + 31) // 32), dtype=np.uint32) for m in nch]
+        misses = [np.zeros(max(1, m), dtype=np.uint32) for m in nch]
+        packeds = [np.zeros(max(1, a.size), dtype=np.uint8) for a in arrs]
+        slots = [np.zeros(max(1, m), dtype=np.uint32) for m in nch] if chunk_slots else None
+        P = ctypes.c_void_p * max(1, count)
+        bufs = P(*[a.ctypes.data for a in arrs])
+        ns = (ctypes.c_size_t * max(1, count))(*[a.size for a in arrs])
+        res = np.zeros(max(1, 5 * count), dtype=np.uint64)
+        rc = int(lib().oracle_dedup_batch(
+            self._h, count, bufs, ns, P(*[m.ctypes.data for m in masks]),
+            P(*[m.ctypes.data for m in misses]), P(*[m.ctypes.data for m in packeds]),
+            P(*[m.ctypes.data for m in slots]) if chunk_slots else None, res.ctypes.data))
+        if rc < 0:
+            return rc, None, None
+        outs, results = [], []
+        for k in range(count):
+            r = {f: int(res[5 * k + j]) for j, f in enumerate(RESULT_FIELDS)}
+            _, mk, mi, pk = self._finish(r["n_miss"], arrs[k].size, nch[k], masks[k], misses[k],
+                                         packeds[k])
+            outs.append((mk, mi, pk) + ((slots[k][:nch[k]].copy(),) if chunk_slots else ()))
+            results.append(r)
+        return rc, outs, results
 
     def _finish(self, rc, n, nch, mask, miss, packed):
         C = self.chunk_bytes

@@ -36,10 +36,25 @@
 //      min(len, 128) bytes (first 8 digest bytes, little-endian); chunks under
 //      1024 bytes are recorded but never cached: always misses, no slot, no
 //      entry, no in-call dedup.  Verify is kept.
+//  R12 a batch of payloads is its calls made in order (a chunk equal to an
+//      earlier payload's miss is a cache hit for its own payload), except that
+//      running out of slots fails the whole batch.
+//  R16 LRU eviction (Sec. 4.1.3; caches created with the LRU flag): every call
+//      (a batch counts as one call) takes the next value of a clock; the slots
+//      it hits or fills get that value as their last use.  Hits and misses are
+//      decided as without eviction.  If the call's stored misses exceed the
+//      never-used slots, it evicts the missing number of slots among those it
+//      did not hit, least recent last use first, ties by lower slot number;
+//      if too few exist it fails with CAPACITY and changes nothing.  Evicted
+//      slots lose their index entries; the call's new entries take the
+//      evicted slots and then never-used ones, in ascending slot order, in the
+//      order of the misses.
+#include <algorithm>
 #include <cmath>
 #include <cstddef>
 #include <cstdint>
 #include <cstring>
+#include <iterator>
 #include <unordered_map>
 #include <vector>
 
@@ -204,6 +219,7 @@ const int kErrInvalidArg = -1;
 const int kErrCapacity = -4;
 const uint32_t kFlagKey16 = 1u;
 const uint32_t kFlagPaperIds = 4u;  // App. B.1 identifiers and small-chunk rule
+const uint32_t kFlagEvictLru = 8u;  // Sec. 4.1.3 LRU eviction instead of CAPACITY
 const size_t kPaperMinCached = 1024;
 const uint32_t kNoSlot = 0xFFFFFFFFu;
 
@@ -220,9 +236,22 @@ struct Cache {
   uint32_t flags = 0;
   std::unordered_multimap<uint64_t, Entry> index;  // key -> entries
   std::vector<std::vector<uint8_t>> slot_bytes;    // slot -> stored bytes
+  std::vector<uint64_t> last_use;                  // slot -> clock of its last use
+  uint64_t clock = 0;                              // one tick per call
   // statistics, same meaning as the CUDA library's
   uint64_t calls = 0, chunks = 0, hits_cache = 0, hits_intra = 0, misses = 0,
-           inserts = 0, verify_rejects = 0, bytes_used = 0;
+           inserts = 0, verify_rejects = 0, bytes_used = 0, evictions = 0;
+};
+
+// One payload of a call: its bytes, its outputs and its results.
+struct Payload {
+  const uint8_t* p;
+  size_t n;
+  uint32_t* hit_mask;
+  uint32_t* miss_idx;
+  uint8_t* packed;
+  uint32_t* chunk_slot;  // may be null
+  uint64_t n_miss = 0, hits_cache = 0, hits_intra = 0, rejects = 0, miss_bytes = 0;
 };
 
 uint64_t key_of(const Cache& c, uint64_t fp) {
@@ -269,7 +298,7 @@ int oracle_fingerprint(const void* buf, size_t n, size_t chunk_bytes, uint64_t* 
 
 void* oracle_cache_create(size_t capacity_bytes, size_t chunk_bytes, uint32_t flags, int* err) {
   if (chunk_bytes < 32 || chunk_bytes % 32 != 0 || chunk_bytes > (16u << 20) ||
-      (flags & ~(kFlagKey16 | kFlagPaperIds)) != 0 || capacity_bytes / (chunk_bytes ? chunk_bytes : 1) == 0 ||
+      (flags & ~(kFlagKey16 | kFlagPaperIds | kFlagEvictLru)) != 0 || capacity_bytes / (chunk_bytes ? chunk_bytes : 1) == 0 ||
       capacity_bytes / chunk_bytes > 0xFFFFFFFEull) {
     if (err) *err = kErrInvalidArg;
     return nullptr;
@@ -285,93 +314,207 @@ void* oracle_cache_create(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
 
 void oracle_cache_destroy(void* cache) { delete static_cast<Cache*>(cache); }
 
-// The sequential dedup of one payload (paper Sec. 4.1.2 with readings R1-R8).
-// Returns the number of misses, or a negative error code.  The cache is only
-// changed when the whole call succeeds.
+}  // extern "C"
+
+namespace {
+
+// The dedup of one call over `count` payloads (paper Sec. 4.1.2 with
+// readings R1-R8, R12, R13, R16): chunks are decided one at a time, payload
+// after payload, in ascending order.  Returns the number of misses, or a
+// negative error code.  The cache is only changed when the whole call
+// succeeds; on an error the outputs are unspecified.
+int64_t dedup_calls(Cache* c, Payload* pays, size_t count) {
+  const size_t C = c->chunk;
+  uint64_t total_chunks = 0;
+  for (size_t k = 0; k < count; ++k) {
+    if (pays[k].n > 0 && pays[k].p == nullptr) return kErrInvalidArg;
+    total_chunks += (pays[k].n + C - 1) / C;
+  }
+  if (total_chunks > 0xFFFFFFFEull) return kErrInvalidArg;
+  if (total_chunks == 0) return 0;
+  const uint64_t now = ++c->clock;
+
+  // Entries inserted by this call, kept aside until the call commits.  Their
+  // Entry.slot holds the insertion number r; the slot is decided at the end.
+  std::unordered_multimap<uint64_t, Entry> fresh_index;
+  std::vector<std::vector<uint8_t>> fresh_bytes;
+  std::vector<size_t> fresh_payload;                      // payload that inserted r
+  std::vector<std::pair<uint32_t*, uint64_t>> fresh_refs;  // chunk_slot cells naming r
+  const uint64_t slots0 = c->slot_bytes.size();
+  std::vector<char> used(slots0, 0);  // cached slots hit by this call
+  const bool paper = (c->flags & kFlagPaperIds) != 0;
+  uint64_t stored = 0;  // misses given a slot (all of them, except paper-mode small chunks)
+
+  for (size_t k = 0; k < count; ++k) {
+    Payload& P = pays[k];
+    if (P.n == 0) continue;
+    const uint64_t nchunks = (P.n + C - 1) / C;
+    for (uint64_t w = 0; w < (nchunks + 31) / 32; ++w) P.hit_mask[w] = 0;
+    uint64_t rank = 0;
+    for (uint64_t i = 0; i < nchunks; ++i) {
+      const uint8_t* chunk = P.p + i * C;
+      const size_t len = (P.n - i * C < C) ? (P.n - i * C) : C;
+      if (paper && len < kPaperMinCached) {
+        // App. B.1: recorded but never cached -- always sent, never inserted
+        P.miss_idx[rank] = static_cast<uint32_t>(i);
+        if (P.chunk_slot) P.chunk_slot[i] = kNoSlot;
+        std::memcpy(P.packed + rank * C, chunk, len);
+        P.miss_bytes += len;
+        ++rank;
+        continue;
+      }
+      const uint64_t key = chunk_key(*c, chunk, len);
+
+      bool candidate = false, hit = false, hit_is_fresh = false;
+      uint64_t hit_slot = 0;
+      auto look = [&](const std::unordered_multimap<uint64_t, Entry>& idx,
+                      const std::vector<std::vector<uint8_t>>& store, bool fresh) {
+        auto range = idx.equal_range(key);
+        for (auto it = range.first; it != range.second; ++it) {
+          if (it->second.len != len) continue;
+          candidate = true;
+          if (bytes_equal(store[it->second.slot], chunk, len)) {
+            hit = true;
+            hit_is_fresh = fresh;
+            hit_slot = it->second.slot;
+          }
+        }
+      };
+      look(c->index, c->slot_bytes, false);
+      look(fresh_index, fresh_bytes, true);
+
+      if (hit) {
+        P.hit_mask[i / 32] |= 1u << (i % 32);
+        if (hit_is_fresh) {
+          // an earlier miss of this payload, or of an earlier payload of the
+          // batch, whose own call would have inserted it (R12)
+          if (fresh_payload[hit_slot] == k) ++P.hits_intra; else ++P.hits_cache;
+          if (P.chunk_slot) fresh_refs.emplace_back(P.chunk_slot + i, hit_slot);
+        } else {
+          ++P.hits_cache;
+          used[hit_slot] = 1;
+          if (P.chunk_slot) P.chunk_slot[i] = static_cast<uint32_t>(hit_slot);
+        }
+        continue;
+      }
+      if (candidate) ++P.rejects;
+      P.miss_idx[rank] = static_cast<uint32_t>(i);
+      if (P.chunk_slot) fresh_refs.emplace_back(P.chunk_slot + i, stored);
+      std::memcpy(P.packed + rank * C, chunk, len);
+      Entry e{key, static_cast<uint32_t>(len), static_cast<uint32_t>(stored)};
+      fresh_index.emplace(key, e);
+      fresh_bytes.emplace_back(chunk, chunk + len);
+      fresh_payload.push_back(k);
+      P.miss_bytes += len;
+      ++rank;
+      ++stored;
+    }
+    P.n_miss = rank;
+  }
+
+  // Slots for the new entries: never-used slots, and with LRU eviction the
+  // least recently used slots this call did not hit (R7, R16).
+  std::vector<uint64_t> victims;
+  if (stored > c->nslots - slots0) {
+    if (!(c->flags & kFlagEvictLru)) return kErrCapacity;  // nothing committed
+    const uint64_t need = stored - (c->nslots - slots0);
+    std::vector<uint64_t> cand;
+    for (uint64_t s = 0; s < slots0; ++s)
+      if (!used[s]) cand.push_back(s);
+    if (cand.size() < need) return kErrCapacity;
+    std::sort(cand.begin(), cand.end(), [&](uint64_t x, uint64_t y) {
+      return c->last_use[x] != c->last_use[y] ? c->last_use[x] < c->last_use[y] : x < y;
+    });
+    victims.assign(cand.begin(), cand.begin() + need);
+    std::sort(victims.begin(), victims.end());
+  }
+  std::vector<uint64_t> slot_of(stored);
+  for (uint64_t r = 0; r < stored; ++r)
+    slot_of[r] = r < victims.size() ? victims[r] : slots0 + (r - victims.size());
+
+  // Commit: drop the victims' entries, then store the new ones.
+  if (!victims.empty()) {
+    std::vector<char> gone(slots0, 0);
+    for (uint64_t v : victims) {
+      gone[v] = 1;
+      c->bytes_used -= c->slot_bytes[v].size();
+    }
+    for (auto it = c->index.begin(); it != c->index.end();)
+      it = gone[it->second.slot] ? c->index.erase(it) : std::next(it);
+  }
+  for (auto& kv : fresh_index) {
+    Entry e = kv.second;
+    const uint64_t r = e.slot;
+    e.slot = static_cast<uint32_t>(slot_of[r]);
+    c->index.emplace(kv.first, e);
+  }
+  for (uint64_t r = 0; r < stored; ++r) {
+    const uint64_t s = slot_of[r];
+    c->bytes_used += fresh_bytes[r].size();
+    if (s < c->slot_bytes.size()) {
+      c->slot_bytes[s] = std::move(fresh_bytes[r]);
+      c->last_use[s] = now;
+    } else {
+      c->slot_bytes.emplace_back(std::move(fresh_bytes[r]));
+      c->last_use.push_back(now);
+    }
+  }
+  for (uint64_t s = 0; s < slots0; ++s)
+    if (used[s]) c->last_use[s] = now;
+  for (auto& ref : fresh_refs) *ref.first = static_cast<uint32_t>(slot_of[ref.second]);
+
+  uint64_t misses = 0;
+  for (size_t k = 0; k < count; ++k) {
+    const Payload& P = pays[k];
+    if (P.n == 0) continue;
+    c->calls += 1;
+    c->chunks += (P.n + C - 1) / C;
+    c->hits_cache += P.hits_cache;
+    c->hits_intra += P.hits_intra;
+    c->misses += P.n_miss;
+    c->verify_rejects += P.rejects;
+    misses += P.n_miss;
+  }
+  c->inserts += stored;
+  c->evictions += victims.size();
+  return static_cast<int64_t>(misses);
+}
+
+}  // namespace
+
+extern "C" {
+
+// The sequential dedup of one payload: a call of one payload.
 int64_t oracle_dedup(void* cache, const void* buf, size_t n, uint32_t* hit_mask,
                      uint32_t* miss_idx, uint8_t* packed, uint32_t* chunk_slot) {
   Cache* c = static_cast<Cache*>(cache);
-  const uint8_t* p = static_cast<const uint8_t*>(buf);
-  if (c == nullptr || (n > 0 && buf == nullptr)) return kErrInvalidArg;
-  if (n == 0) return 0;
-  const size_t C = c->chunk;
-  const uint64_t nchunks = (n + C - 1) / C;
-  if (nchunks >= (1ull << 32)) return kErrInvalidArg;
+  if (c == nullptr) return kErrInvalidArg;
+  Payload P{static_cast<const uint8_t*>(buf), n, hit_mask, miss_idx, packed, chunk_slot};
+  return dedup_calls(c, &P, 1);
+}
 
-  // Entries inserted by this call, kept aside until the call commits.
-  std::unordered_multimap<uint64_t, Entry> fresh_index;
-  std::vector<std::vector<uint8_t>> fresh_bytes;
-  const uint64_t slots0 = c->slot_bytes.size();
-  const bool paper = (c->flags & kFlagPaperIds) != 0;
-  uint64_t rank = 0, hits_cache = 0, hits_intra = 0, rejects = 0;
-  uint64_t stored = 0;  // misses given a slot (all of them, except paper-mode small chunks)
-
-  for (uint64_t w = 0; w < (nchunks + 31) / 32; ++w) hit_mask[w] = 0;
-
-  for (uint64_t i = 0; i < nchunks; ++i) {
-    const uint8_t* chunk = p + i * C;
-    const size_t len = (n - i * C < C) ? (n - i * C) : C;
-    if (paper && len < kPaperMinCached) {
-      // App. B.1: recorded but never cached -- always sent, never inserted
-      miss_idx[rank] = static_cast<uint32_t>(i);
-      if (chunk_slot) chunk_slot[i] = kNoSlot;
-      std::memcpy(packed + rank * C, chunk, len);
-      ++rank;
-      continue;
+// A batch of payloads in one call.  results: count x 5 u64 (misses,
+// cache hits, in-call hits, verify rejects, miss bytes) per payload.
+int64_t oracle_dedup_batch(void* cache, size_t count, const void* const* bufs, const size_t* ns,
+                           uint32_t* const* hit_masks, uint32_t* const* miss_idxs,
+                           uint8_t* const* packeds, uint32_t* const* chunk_slots,
+                           uint64_t* results) {
+  Cache* c = static_cast<Cache*>(cache);
+  if (c == nullptr || (count > 0 && (bufs == nullptr || ns == nullptr))) return kErrInvalidArg;
+  std::vector<Payload> pays;
+  for (size_t k = 0; k < count; ++k)
+    pays.push_back(Payload{static_cast<const uint8_t*>(bufs[k]), ns[k], hit_masks[k],
+                           miss_idxs[k], packeds[k], chunk_slots ? chunk_slots[k] : nullptr});
+  const int64_t rc = dedup_calls(c, pays.data(), count);
+  if (rc >= 0 && results)
+    for (size_t k = 0; k < count; ++k) {
+      results[5 * k + 0] = pays[k].n_miss;
+      results[5 * k + 1] = pays[k].hits_cache;
+      results[5 * k + 2] = pays[k].hits_intra;
+      results[5 * k + 3] = pays[k].rejects;
+      results[5 * k + 4] = pays[k].miss_bytes;
     }
-    const uint64_t key = chunk_key(*c, chunk, len);
-
-    bool candidate = false, hit = false, hit_is_fresh = false;
-    uint32_t hit_slot = 0;
-    auto look = [&](const std::unordered_multimap<uint64_t, Entry>& idx,
-                    const std::vector<std::vector<uint8_t>>& store, uint64_t slot_base,
-                    bool fresh) {
-      auto range = idx.equal_range(key);
-      for (auto it = range.first; it != range.second; ++it) {
-        if (it->second.len != len) continue;
-        candidate = true;
-        if (bytes_equal(store[it->second.slot - slot_base], chunk, len)) {
-          hit = true;
-          hit_is_fresh = fresh;
-          hit_slot = it->second.slot;
-        }
-      }
-    };
-    look(c->index, c->slot_bytes, 0, false);
-    look(fresh_index, fresh_bytes, slots0, true);
-
-    if (hit) {
-      hit_mask[i / 32] |= 1u << (i % 32);
-      if (hit_is_fresh) ++hits_intra; else ++hits_cache;
-      if (chunk_slot) chunk_slot[i] = hit_slot;
-      continue;
-    }
-    if (candidate) ++rejects;
-    if (slots0 + stored >= c->nslots) return kErrCapacity;  // nothing committed
-    miss_idx[rank] = static_cast<uint32_t>(i);
-    if (chunk_slot) chunk_slot[i] = static_cast<uint32_t>(slots0 + stored);
-    std::memcpy(packed + rank * C, chunk, len);
-    Entry e{key, static_cast<uint32_t>(len), static_cast<uint32_t>(slots0 + stored)};
-    fresh_index.emplace(key, e);
-    fresh_bytes.emplace_back(chunk, chunk + len);
-    ++rank;
-    ++stored;
-  }
-
-  // Commit.
-  for (auto& kv : fresh_index) c->index.emplace(kv.first, kv.second);
-  for (auto& b : fresh_bytes) {
-    c->bytes_used += b.size();
-    c->slot_bytes.emplace_back(std::move(b));
-  }
-  c->calls += 1;
-  c->chunks += nchunks;
-  c->hits_cache += hits_cache;
-  c->hits_intra += hits_intra;
-  c->misses += rank;
-  c->inserts += stored;
-  c->verify_rejects += rejects;
-  return static_cast<int64_t>(rank);
+  return rc;
 }
 
 // Weight-block identification at cudaFree time (paper Sec. 4.1.1): record r says
@@ -408,6 +551,7 @@ int oracle_debug_insert(void* cache, uint64_t key, const void* bytes, size_t len
   Entry e{key_of(*c, key), static_cast<uint32_t>(len), static_cast<uint32_t>(c->slot_bytes.size())};
   c->index.emplace(e.key, e);
   c->slot_bytes.emplace_back(b, b + len);
+  c->last_use.push_back(++c->clock);
   c->bytes_used += len;
   c->inserts += 1;
   return kOk;
@@ -415,7 +559,7 @@ int oracle_debug_insert(void* cache, uint64_t key, const void* bytes, size_t len
 
 // Stats in the CUDA library's field order:
 // calls, chunks, hits_cache, hits_intra, misses, inserts, verify_rejects,
-// slots_used, bytes_used, capacity_bytes, nslots, chunk_bytes.
+// slots_used, bytes_used, capacity_bytes, nslots, chunk_bytes, evictions.
 void oracle_cache_stats(const void* cache, uint64_t* out) {
   const Cache* c = static_cast<const Cache*>(cache);
   out[0] = c->calls;
@@ -430,6 +574,7 @@ void oracle_cache_stats(const void* cache, uint64_t* out) {
   out[9] = c->capacity_bytes;
   out[10] = c->nslots;
   out[11] = c->chunk;
+  out[12] = c->evictions;
 }
 
 // Index contents, ordered by slot: keys[s], lens[s] for s < slots_used.

@@ -79,14 +79,20 @@ class BruteCache:
     """The weight cache by its definition: an ordered list of stored byte
     strings; a chunk is a hit iff byte-equal to a stored one of equal length."""
 
-    def __init__(self, nslots: int, key_fn=None, paper_min: int = 0):
+    def __init__(self, nslots: int, key_fn=None, paper_min: int = 0, lru: bool = False):
         self.nslots = nslots
         self.items = []       # (key, bytes) in slot order
         self.key_fn = key_fn  # bytes -> key, only for counting verify rejects
         self.paper_min = paper_min  # chunks shorter than this are never cached
+        self.lru = lru        # evict least recently used slots instead of failing
+        self.clock = 0
+        self.last_use = []    # per slot: the clock value of the call that last used it
+        self.evictions = 0
 
     def insert(self, key, data: bytes):
         self.items.append((key, bytes(data)))
+        self.clock += 1
+        self.last_use.append(self.clock)
 
     def dedup(self, payload: bytes, C: int):
         n = len(payload)
@@ -127,3 +133,89 @@ class BruteCache:
         self.items = staged
         return len(miss), dict(mask=mask, miss=miss, packed=bytes(packed), hits_cache=hits_cache,
                                hits_intra=hits_intra, rejects=rejects, slots=slots)
+
+    def dedup_batch(self, payloads, C: int):
+        """One call over several payloads, by definition: each chunk, payload
+        after payload, is a hit iff byte-equal to a stored chunk or to an
+        earlier miss of the call.  Then the misses get slots: never-used ones,
+        and (LRU) the least recently used slots the call did not hit, ties by
+        lower slot, in ascending slot order.  Returns (rc, [per-payload dict])."""
+        total = sum((len(p) + C - 1) // C for p in payloads)
+        if total == 0:
+            return 0, [None] * len(payloads)
+        self.clock += 1
+        now = self.clock
+        slots0 = len(self.items)
+        fresh = []   # (bytes, payload number, key) in miss order
+        used = set()
+        outs = []
+        for k, payload in enumerate(payloads):
+            n = len(payload)
+            N = (n + C - 1) // C
+            o = dict(mask=[0] * ((N + 31) // 32), miss=[], packed=bytearray(), slots=[],
+                     hits_cache=0, hits_intra=0, rejects=0)
+            for i in range(N):
+                c = payload[i * C:(i + 1) * C]
+                if len(c) < self.paper_min:
+                    o["miss"].append(i)
+                    o["slots"].append(("none",))
+                    o["packed"] += c
+                    continue
+                found = None
+                for s, (_, b) in enumerate(self.items):
+                    if b == c:
+                        found = ("cache", s)
+                        break
+                if found is None:
+                    for r, (b, kk, _) in enumerate(fresh):
+                        if b == c:
+                            found = ("fresh", r)
+                            break
+                if found is not None:
+                    o["mask"][i // 32] |= 1 << (i % 32)
+                    o["slots"].append(found)
+                    if found[0] == "cache":
+                        used.add(found[1])
+                        o["hits_cache"] += 1
+                    elif fresh[found[1]][1] == k:
+                        o["hits_intra"] += 1
+                    else:
+                        o["hits_cache"] += 1
+                    continue
+                key = self.key_fn(c) if self.key_fn else None
+                if self.key_fn and (any(kk == key and len(b) == len(c) for kk, b in self.items) or
+                                    any(kk == key and len(b) == len(c) for b, _, kk in fresh)):
+                    o["rejects"] += 1
+                o["miss"].append(i)
+                o["slots"].append(("fresh", len(fresh)))
+                o["packed"] += c
+                fresh.append((c, k, key))
+            outs.append(o)
+        M = len(fresh)
+        victims = []
+        if M > self.nslots - slots0:
+            if not self.lru:
+                return -4, None
+            need = M - (self.nslots - slots0)
+            cands = sorted((s for s in range(slots0) if s not in used),
+                           key=lambda s: (self.last_use[s], s))
+            if len(cands) < need:
+                return -4, None
+            victims = sorted(cands[:need])
+        slot_of = victims + list(range(slots0, slots0 + M - len(victims)))
+        for r, (b, _, key) in enumerate(fresh):
+            s = slot_of[r]
+            if s < len(self.items):
+                self.items[s] = (key, b)
+                self.last_use[s] = now
+            else:
+                self.items.append((key, b))
+                self.last_use.append(now)
+        for s in used:
+            self.last_use[s] = now
+        self.evictions += len(victims)
+        for o in outs:
+            o["slots"] = [0xFFFFFFFF if t[0] == "none" else t[1] if t[0] == "cache"
+                          else slot_of[t[1]] for t in o["slots"]]
+            o["packed"] = bytes(o["packed"])
+        return sum(len(o["miss"]) for o in outs), outs

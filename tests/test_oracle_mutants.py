@@ -12,6 +12,7 @@ import pytest
 
 import oracle
 from tests import test_oracle_dedup as D
+from tests import test_oracle_lru as L
 from tests._refs import xxh64_lib
 
 MUTANTS = [
@@ -22,13 +23,25 @@ MUTANTS = [
      "h ^= static_cast<uint64_t>(read_le32(p + off)) * kP2;"),
     ("avalanche shift 29 -> 28", "h ^= h >> 29;", "h ^= h >> 28;"),
     ("length not part of a candidate", "if (it->second.len != len) continue;", ""),
-    ("earlier misses of the call not looked up", "look(fresh_index, fresh_bytes, slots0, true);", ""),
-    ("reject counted without a candidate", "if (candidate) ++rejects;", "++rejects;"),
-    ("capacity off by one", "if (slots0 + stored >= c->nslots)", "if (slots0 + stored > c->nslots)"),
-    ("miss packed at its chunk offset", "std::memcpy(packed + rank * C, chunk, len);\n    Entry e",
-     "std::memcpy(packed + i * C, chunk, len);\n    Entry e"),
-    ("hit reports a fresh slot", "if (chunk_slot) chunk_slot[i] = hit_slot;",
-     "if (chunk_slot) chunk_slot[i] = static_cast<uint32_t>(slots0 + stored);"),
+    ("earlier misses of the call not looked up", "look(fresh_index, fresh_bytes, true);", ""),
+    ("reject counted without a candidate", "if (candidate) ++P.rejects;", "++P.rejects;"),
+    ("capacity off by one", "if (stored > c->nslots - slots0)", "if (stored >= c->nslots - slots0)"),
+    ("miss packed at its chunk offset", "std::memcpy(P.packed + rank * C, chunk, len);\n      Entry e",
+     "std::memcpy(P.packed + i * C, chunk, len);\n      Entry e"),
+    ("hit reports a fresh slot", "if (P.chunk_slot) P.chunk_slot[i] = static_cast<uint32_t>(hit_slot);",
+     "if (P.chunk_slot) P.chunk_slot[i] = static_cast<uint32_t>(slots0 + stored);"),
+    ("LRU evicts the most recently used",
+     "return c->last_use[x] != c->last_use[y] ? c->last_use[x] < c->last_use[y] : x < y;",
+     "return c->last_use[x] != c->last_use[y] ? c->last_use[x] > c->last_use[y] : x < y;"),
+    ("LRU ties go to the higher slot",
+     "return c->last_use[x] != c->last_use[y] ? c->last_use[x] < c->last_use[y] : x < y;",
+     "return c->last_use[x] != c->last_use[y] ? c->last_use[x] < c->last_use[y] : x > y;"),
+    ("a call may evict what it hits", "if (!used[s]) cand.push_back(s);", "cand.push_back(s);"),
+    ("hits do not refresh the last use", "if (used[s]) c->last_use[s] = now;", ""),
+    ("victims keep their index entries",
+     "it = gone[it->second.slot] ? c->index.erase(it) : std::next(it);", "it = std::next(it);"),
+    ("an earlier payload's miss counts as in-call",
+     "if (fresh_payload[hit_slot] == k) ++P.hits_intra; else ++P.hits_cache;", "++P.hits_intra;"),
 ]
 
 
@@ -49,6 +62,11 @@ def _pins_hold() -> bool:
         D.test_tail_length_is_part_of_equality()
         D.test_crafted_collisions_are_rejected()
         D.test_length_is_part_of_a_candidate()
+        for seed in (0, 1):
+            L.test_lru_batches_match_brute_force(seed, False)
+        L.test_lru_batches_match_brute_force(2, True)
+        L.test_worked_example_slots_by_hand()
+        L.test_a_call_never_evicts_what_it_hits()
     except AssertionError:
         return False
     return True
