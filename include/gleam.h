@@ -50,7 +50,8 @@ enum gleam_status {
   GLEAM_ERR_INVALID_ARG = -1,   /* NULL handle/pointer, bad sizes, bad flags   */
   GLEAM_ERR_NOT_DEVICE_PTR = -2,/* a buffer is not device memory of this GPU  */
   GLEAM_ERR_CUDA = -3,          /* a CUDA runtime call failed                 */
-  GLEAM_ERR_CAPACITY = -4,      /* misses do not fit the free slots           */
+  GLEAM_ERR_CAPACITY = -4,      /* misses do not fit the free (or, with
+                                   GLEAM_EVICT_LRU, the evictable) slots      */
   GLEAM_ERR_TIMEOUT = -5,       /* a bounded device-side wait ran out         */
   GLEAM_ERR_NOMEM = -6,         /* device allocation failed                   */
   GLEAM_ERR_INTERNAL = -7       /* a device-side consistency check failed     */
@@ -69,6 +70,14 @@ enum gleam_status {
                                    recorded but never cached: always misses,
                                    given no slot, never deduplicated.  Every
                                    key match is still verified byte for byte. */
+#define GLEAM_EVICT_LRU 0x8u    /* paper Sec. 4.1.3: when a call's misses do not
+                                   fit the never-used slots, evict the least
+                                   recently used slots that the call did not
+                                   hit (last use = the latest call that hit or
+                                   filled the slot; ties: lower slot first),
+                                   instead of failing with GLEAM_ERR_CAPACITY.
+                                   A batch is one call for this.  Costs 9 bytes
+                                   of device memory per slot. */
 
 /* Cumulative counters of one cache (successful calls only). */
 typedef struct gleam_stats {
@@ -86,6 +95,7 @@ typedef struct gleam_stats {
   uint64_t capacity_bytes; /* as passed to create                            */
   uint64_t nslots;         /* capacity_bytes / chunk_bytes                   */
   uint64_t chunk_bytes;    /* C                                              */
+  uint64_t evictions;      /* slots reused by GLEAM_EVICT_LRU                */
 } gleam_stats_t;
 
 /* Written by the device when an asynchronous dedup call completes. */
@@ -120,7 +130,8 @@ typedef struct gleam_payload {
  * slots of chunk_bytes each and an empty index (paper Sec. 4.1.3: the
  * server-side shareable pool; Sec. 4.1.2: the set of resident identifiers).
  * chunk_bytes: multiple of 32, 32..16 MiB.  The slot count must be 1..2^32-2.
- * flags: 0 or a combination of GLEAM_KEY16, GLEAM_DEBUG_CHECKS and GLEAM_PAPER_IDS.
+ * flags: 0 or a combination of GLEAM_KEY16, GLEAM_DEBUG_CHECKS, GLEAM_PAPER_IDS
+ * and GLEAM_EVICT_LRU.
  * On success *out owns about capacity_bytes + 32 B * slots of device memory.
  * Returns GLEAM_OK, GLEAM_ERR_INVALID_ARG, GLEAM_ERR_NOMEM or GLEAM_ERR_CUDA. */
 int gleam_cache_create(size_t capacity_bytes, size_t chunk_bytes, gleam_cache_t** out);
@@ -212,7 +223,7 @@ int gleam_dedup_copy_host_batch(gleam_cache_t* cache, const gleam_payload_t* pay
  * memory map it keeps for the application.
  *
  * Same operation, outputs and cache update as gleam_dedup_copy_async, but the
- * per-call workspace is one fixed array of about 4.9 MiB in the library's
+ * per-call workspace is one fixed array of about 4.6 MiB in the library's
  * device image instead of memory allocated by the cache; the call itself only
  * enqueues memsets and kernels and allocates nothing.  Every GPU that loads
  * the library holds that array until the process exits.
@@ -279,11 +290,19 @@ int gleam_cache_debug_insert(gleam_cache_t* cache, uint64_t key, const void* d_b
  * returns GLEAM_ERR_TIMEOUT with the cache unchanged. */
 #define GLEAM_DEBUG_WAIT_LIMIT_NS 1
 #define GLEAM_DEBUG_SKIP_ARRIVE 2
+/* what = GLEAM_DEBUG_CLOCK: sets the GLEAM_EVICT_LRU clock (the value of the
+ * latest call, 0 .. 2^32-2; the next call takes value + 1), so that tests can
+ * reach clock values of any size.  The clock is 32 bits: a cache that has
+ * served 2^32 - 1 calls no longer orders its slots exactly. */
+#define GLEAM_DEBUG_CLOCK 3
 int gleam_cache_debug_set(gleam_cache_t* cache, int what, int64_t value);
 
-/* Device-side copy of the index, slot count and counters, for restoring the
- * cache between timed repetitions.  Arena bytes past the saved slot count are
- * never read, so they are not copied. */
+/* Device-side copy of the index, slot count and counters (and, for a
+ * GLEAM_EVICT_LRU cache, the slot lengths and last uses), for restoring the
+ * cache between timed repetitions.  Arena bytes are not copied: those past
+ * the saved slot count are never read, and a slot that an eviction reused
+ * after the snapshot keeps its new bytes, so its restored entry no longer
+ * matches them and its chunk misses (every hit is verified). */
 int gleam_cache_snapshot(gleam_cache_t* cache, gleam_snapshot_t** out);
 int gleam_cache_restore(gleam_cache_t* cache, const gleam_snapshot_t* snap);
 void gleam_snapshot_destroy(gleam_snapshot_t* snap);

@@ -25,8 +25,10 @@ GLEAM_ERR_INTERNAL = -7
 GLEAM_KEY16 = 0x1
 GLEAM_DEBUG_CHECKS = 0x2
 GLEAM_PAPER_IDS = 0x4
+GLEAM_EVICT_LRU = 0x8
 GLEAM_DEBUG_WAIT_LIMIT_NS = 1
 GLEAM_DEBUG_SKIP_ARRIVE = 2
+GLEAM_DEBUG_CLOCK = 3
 
 # Every symbol include/gleam.h declares (checked by the ABI test).
 EXPORTS = (
@@ -45,7 +47,7 @@ class gleam_stats_t(ctypes.Structure):
     _fields_ = [(f, ctypes.c_uint64) for f in (
         "calls", "chunks", "hits_cache", "hits_intra", "misses", "inserts",
         "verify_rejects", "slots_used", "bytes_used", "capacity_bytes", "nslots",
-        "chunk_bytes")]
+        "chunk_bytes", "evictions")]
 
 
 class gleam_payload_t(ctypes.Structure):

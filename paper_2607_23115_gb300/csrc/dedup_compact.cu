@@ -193,6 +193,203 @@ __device__ __forceinline__ void add_in_group(unsigned long long* dst, unsigned p
   if (dst && sum) atomicAdd(dst, sum);
 }
 
+// ---- LRU eviction (paper Sec. 4.1.3; reading R16) ---------------------------
+//
+// The K slots to evict are the K smallest (last use, slot number) among the
+// used slots whose last use is before this call (the call's own hits were
+// stamped with its clock value in phase A).  The cut-off stamp is found by a
+// two-pass radix select on its high and low 16 bits; the victims are then the
+// slots older than the cut-off plus the lowest-numbered slots at it.  Their
+// index and hint-table entries are removed without tombstones surviving the
+// call: each is first replaced by a tombstone, then every cluster (maximal
+// run of occupied entries) that holds one is rebuilt by its single owner
+// thread, moving each live entry, in cluster order, to the first hole between
+// its home position and itself, and finally the remaining tombstones become
+// empty.  Clusters shrink but never merge, so owners never meet.
+
+// Rebuilds the cluster that starts at `start` (its predecessor is empty).
+__device__ void compact_cluster(IndexEntry* t, unsigned long long mask, unsigned long long start) {
+  unsigned long long len = 0;
+  bool any = false;
+  for (unsigned long long q = start; len <= mask; q = (q + 1) & mask, ++len) {
+    const uint32_t sl = t[q].slot;
+    if (sl == kEmptySlot) break;
+    any |= sl == kTombSlot;
+  }
+  if (!any) return;
+  for (unsigned long long k = 0; k < len; ++k) {
+    const unsigned long long q = (start + k) & mask;
+    const IndexEntry e = t[q];
+    if (e.slot == kTombSlot) continue;
+    for (unsigned long long j = mix64(e.key) & mask; j != q; j = (j + 1) & mask) {
+      if (t[j].slot == kTombSlot) {
+        t[j] = e;
+        t[q].slot = kTombSlot;
+        break;
+      }
+    }
+  }
+}
+
+// Exclusive block-wide prefix of per-thread flags, in thread order, for one
+// 256-slot step; returns the thread's offset and adds the step's total to
+// *running (shared arrays: kWarps counts + offsets).
+__device__ __forceinline__ uint32_t block_rank(bool f, uint32_t* cnt, uint32_t* off,
+                                               unsigned long long* running_total) {
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const uint32_t b = __ballot_sync(0xffffffffu, f);
+  if (lane == 0) cnt[w] = __popc(b);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t acc = 0;
+    for (int k = 0; k < kWarps; ++k) {
+      off[k] = acc;
+      acc += cnt[k];
+    }
+    cnt[0] = acc;
+  }
+  __syncthreads();
+  const uint32_t r = off[w] + __popc(b & ((1u << lane) - 1u));
+  const uint32_t step = cnt[0];
+  __syncthreads();
+  *running_total += step;
+  return r;
+}
+
+// Selects and removes the K victims; false if a grid barrier failed.
+__device__ bool lru_evict(const DedupArgs& a, unsigned long long slots0, unsigned long long K,
+                          unsigned long long* sred, uint32_t* cnt, uint32_t* off,
+                          unsigned long long* red64) {
+  const uint32_t G = gridDim.x, lane = threadIdx.x & 31;
+  const unsigned long long tid = (unsigned long long)blockIdx.x * kThreads + threadIdx.x;
+  const unsigned long long nth = (unsigned long long)G * kThreads;
+  const uint32_t now = a.epoch;
+
+  // cut-off stamp: radix select on the high, then the low 16 bits
+  uint32_t hi_bin = 0;
+  unsigned long long below = 0;
+  for (int pass = 0; pass < 2; ++pass) {
+    for (unsigned long long base = tid - lane; base < slots0; base += nth) {
+      const unsigned long long sl = base + lane;
+      uint32_t key = 0xFFFFFFFFu;
+      if (sl < slots0) {
+        const uint32_t u = __ldcg(&a.last_use[sl]);
+        if (u != now && (pass == 0 || (u >> 16) == hi_bin)) key = pass == 0 ? (u >> 16) : (u & 0xFFFFu);
+      }
+      const unsigned peers = __match_any_sync(0xffffffffu, key);
+      if (key != 0xFFFFFFFFu && lane == (uint32_t)(__ffs(peers) - 1))
+        atomicAdd(&a.bins[key], (uint32_t)__popc(peers));
+    }
+    if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
+    if (blockIdx.x == 0) {
+      unsigned long long part = 0;
+      for (uint32_t j = 0; j < kLruBins / kThreads; ++j)
+        part += __ldcg(&a.bins[threadIdx.x * (kLruBins / kThreads) + j]);
+      sred[threadIdx.x] = part;
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        const unsigned long long target = K - below;  // >= 1 candidates in this range
+        unsigned long long acc = 0;
+        uint32_t pi = 0;
+        while (pi + 1 < (uint32_t)kThreads && acc + sred[pi] < target) acc += sred[pi++];
+        uint32_t bin = pi * (kLruBins / kThreads);
+        const uint32_t last = bin + kLruBins / kThreads - 1;
+        while (bin < last && acc + __ldcg(&a.bins[bin]) < target) acc += __ldcg(&a.bins[bin++]);
+        if (pass == 0) {
+          a.ctl->lru_hi = bin;
+          a.ctl->lru_below = acc;
+        } else {
+          a.ctl->lru_cut = (hi_bin << 16) | bin;
+          a.ctl->lru_below = below + acc;
+          a.ctl->lru_ties = target - acc;
+        }
+      }
+      __syncthreads();
+      for (uint32_t j = threadIdx.x; j < kLruBins; j += kThreads) a.bins[j] = 0u;
+    }
+    if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
+    hi_bin = __ldcg(&a.ctl->lru_hi);
+    below = __ldcg(&a.ctl->lru_below);
+  }
+  const uint32_t cut = __ldcg(&a.ctl->lru_cut);
+  const unsigned long long ties = __ldcg(&a.ctl->lru_ties);
+
+  // per contiguous slot range: candidates older than the cut-off, and at it
+  const unsigned long long per = ((slots0 + G - 1) / G + 31) & ~31ull;
+  const unsigned long long lo = min(slots0, blockIdx.x * per);
+  const unsigned long long hi = min(slots0, lo + per);
+  {
+    uint32_t nlt = 0, ntie = 0;
+    for (unsigned long long sl = lo + threadIdx.x; sl < hi; sl += kThreads) {
+      const uint32_t u = __ldcg(&a.last_use[sl]);
+      if (u != now) {
+        nlt += u < cut;
+        ntie += u == cut;
+      }
+    }
+    const unsigned long long t_lt = block_sum<unsigned long long>(nlt, red64);
+    const unsigned long long t_tie = block_sum<unsigned long long>(ntie, red64);
+    if (threadIdx.x == 0) {
+      a.bcount[blockIdx.x] = (uint32_t)t_tie;
+      a.bcount[G + blockIdx.x] = (uint32_t)t_lt;
+    }
+  }
+  if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
+  {
+    unsigned long long tie_before = 0, lt_before = 0;
+    for (uint32_t j = threadIdx.x; j < blockIdx.x; j += kThreads) {
+      tie_before += __ldcg(&a.bcount[j]);
+      lt_before += __ldcg(&a.bcount[G + j]);
+    }
+    tie_before = block_sum<unsigned long long>(tie_before, red64);
+    lt_before = block_sum<unsigned long long>(lt_before, red64);
+    unsigned long long vrun = lt_before + min(ties, tie_before), trun = tie_before;
+    unsigned long long vbytes = 0;
+    for (unsigned long long t0 = lo; t0 < hi; t0 += kThreads) {
+      const unsigned long long sl = t0 + threadIdx.x;
+      const uint32_t u = sl < hi ? __ldcg(&a.last_use[sl]) : now;
+      const bool tie = u != now && u == cut;
+      const unsigned long long tb = trun;
+      const uint32_t tr = block_rank(tie, cnt, off, &trun);
+      const bool victim = (u != now && u < cut) || (tie && tb + tr < ties);
+      const unsigned long long vb = vrun;
+      const uint32_t vr = block_rank(victim, cnt, off, &vrun);
+      if (victim && vb + vr < K) {  // always: the counts above add up to K
+        a.victims[vb + vr] = (uint32_t)sl;
+        a.vflag[sl] = 1;
+        vbytes += a.slot_len[sl];
+      }
+    }
+    vbytes = block_sum<unsigned long long>(vbytes, red64);
+    if (threadIdx.x == 0 && vbytes) atomicAdd(&a.ctl->acc_victim_bytes, vbytes);
+  }
+  if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
+
+  // the victims' entries leave the index and the hint table
+  const unsigned long long tsize = a.index_mask + 1;
+  for (unsigned long long q = tid; q < tsize; q += nth) {
+    const uint32_t s1 = a.index[q].slot;
+    if (s1 < slots0 && a.vflag[s1]) a.index[q].slot = kTombSlot;
+    const uint32_t s2 = a.hints[q].slot;
+    if (s2 < slots0 && a.vflag[s2]) a.hints[q].slot = kTombSlot;
+  }
+  if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
+  for (unsigned long long q = tid; q < tsize; q += nth) {
+    const unsigned long long prev = (q + tsize - 1) & a.index_mask;
+    if (a.index[q].slot != kEmptySlot && a.index[prev].slot == kEmptySlot)
+      compact_cluster(a.index, a.index_mask, q);
+    if (a.hints[q].slot != kEmptySlot && a.hints[prev].slot == kEmptySlot)
+      compact_cluster(a.hints, a.index_mask, q);
+  }
+  if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
+  for (unsigned long long q = tid; q < tsize; q += nth) {
+    if (a.index[q].slot == kTombSlot) a.index[q].slot = kEmptySlot;
+    if (a.hints[q].slot == kTombSlot) a.hints[q].slot = kEmptySlot;
+  }
+  for (unsigned long long r = tid; r < K; r += nth) a.vflag[a.victims[r]] = 0;
+  return true;
+}
+
 __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ uint32_t warp_cnt[kWarps];
@@ -200,6 +397,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   __shared__ uint32_t swarp_cnt[kWarps];
   __shared__ uint32_t swarp_off[kWarps];
   __shared__ unsigned long long s_slots0;
+  __shared__ unsigned long long sred[kThreads];
 
   const uint32_t G = gridDim.x;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -213,8 +411,9 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   __syncthreads();
   const unsigned long long slots0 = s_slots0;
 
-  // ---- A: clear outputs, round-1 claims -------------------------------------
-  if (!skip) {
+  // ---- A: clear outputs, round-1 claims; LRU: stamp the slots hit ----------
+  {
+    unsigned long long distinct = 0;
     for (uint32_t p = tid; p < a.count; p += nth) {
       gleam_result_t* r = desc(a, p).result;
       if (r) {
@@ -231,6 +430,11 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       if ((i & 31) == 0) P.mask[i >> 5] = 0;
       if (ch.status[g] == kHit0) {
         ch.res[g] = kResHit0;
+        if (a.lru) {  // the first chunk to stamp a slot keeps its old value
+          const uint32_t old = atomicExch(&a.last_use[ch.ent[g]], a.epoch);
+          ch.old[g] = old;
+          distinct += old != a.epoch;
+        }
         continue;
       }
       if (ch.status[g] == kUncached) {  // never cached: a miss of its own, in no group
@@ -248,6 +452,10 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       ch.ent[g] = e;
       ch.res[g] = kResUnresolved;
       atomicMax(&a.tbl[e].minv, ~g);
+    }
+    if (a.lru) {
+      distinct = block_sum<unsigned long long>(distinct, red64);
+      if (threadIdx.x == 0 && distinct) atomicAdd(&a.ctl->acc_distinct, distinct);
     }
   }
   bool ok = grid_barrier(a.ctl, G, a.wait_ns, skip);
@@ -310,7 +518,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   const uint64_t per = (((uint64_t)N + G - 1) / G + 31) & ~31ull;
   const uint32_t lo = (uint32_t)min((uint64_t)N, blockIdx.x * per);
   const uint32_t hi = (uint32_t)min((uint64_t)N, lo + per);
-  unsigned long long before = 0, total = 0, sbefore = 0, stotal = 0;
+  unsigned long long before = 0, total = 0, sbefore = 0, stotal = 0, evict = 0;
   if (ok) {
     uint32_t cnt = 0, scnt = 0;
     for (uint32_t g = lo + threadIdx.x; g < hi; g += kThreads) {
@@ -351,9 +559,13 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     total = block_sum<unsigned long long>(total, red64);
     sbefore = block_sum<unsigned long long>(sbefore, red64);
     stotal = block_sum<unsigned long long>(stotal, red64);
-    if (slots0 + stotal > a.nslots) {
-      if (threadIdx.x == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_CAPACITY);
-      ok = false;
+    if (stotal > a.nslots - slots0) {
+      // LRU: evict the missing slots among those this call did not hit
+      evict = stotal - (a.nslots - slots0);
+      if (!a.lru || evict > slots0 - __ldcg(&a.ctl->acc_distinct)) {
+        if (threadIdx.x == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_CAPACITY);
+        ok = false;
+      }
     }
   }
   if (ok) {
@@ -398,10 +610,12 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     }
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   }
+  if (ok && evict) ok = lru_evict(a, slots0, evict, sred, warp_cnt, warp_off, red64);
   // totals for k_pack (the capacity check above left them unpublished on error)
   if (ok && blockIdx.x == 0 && threadIdx.x == 0) {
     a.ctl->acc_misses = total;
     a.ctl->acc_stored = stotal;
+    a.ctl->evict_k = evict;
   }
 }
 
@@ -412,7 +626,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
 // and leaves the per-call state zeroed.  Nothing is written after an error.
 __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
   __shared__ unsigned long long red64[kWarps];
-  __shared__ unsigned long long s_slots0, s_total;
+  __shared__ unsigned long long s_slots0, s_total, s_evict;
   __shared__ int s_err;
   const uint32_t G = gridDim.x;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -422,11 +636,25 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
     s_slots0 = *(volatile const unsigned long long*)&a.dstats[ST_SLOTS_USED];
     s_err = ld_volatile_s32(&a.ctl->err);
     s_total = __ldcg(&a.ctl->acc_misses);
+    s_evict = __ldcg(&a.ctl->evict_k);
   }
   __syncthreads();
   const unsigned long long slots0 = s_slots0;
   const unsigned long long total = s_total;
+  const unsigned long long evict = s_evict;
   const bool ok = s_err == 0;
+  // slot of the stored miss of stored rank sr: the evicted slots in ascending
+  // order, then never-used slots
+  auto slot_of = [&](uint32_t sr) -> unsigned long long {
+    return sr < evict ? (unsigned long long)__ldcg(&a.victims[sr]) : slots0 + (sr - evict);
+  };
+
+  // ---- after an error: give the hit slots their last use back (LRU) ---------
+  if (!ok && a.lru) {
+    for (unsigned long long g = (unsigned long long)blockIdx.x * kThreads + threadIdx.x; g < N;
+         g += (unsigned long long)G * kThreads)
+      if (ch.status[g] == kHit0 && ch.old[g] != a.epoch) a.last_use[ch.ent[g]] = ch.old[g];
+  }
 
   // ---- hit masks, miss indices, chunk slots, counters ------------------------
   if (ok) {
@@ -458,9 +686,9 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
         if (P.chunk_slot) {
           uint32_t sl;
           if (r & kResHit0) sl = ch.ent[g];                                      // matched slot
-          else if (r & kResDup) sl = (uint32_t)(slots0 + __ldcg(&ch.srank[ch.ent[g]]));  // leader's
+          else if (r & kResDup) sl = (uint32_t)slot_of(__ldcg(&ch.srank[ch.ent[g]]));  // leader's
           else if (r & kResNoSlot) sl = kEmptySlot;                              // never cached
-          else sl = (uint32_t)(slots0 + ch.srank[g]);                            // its new slot
+          else sl = (uint32_t)slot_of(ch.srank[g]);                              // its new slot
           P.chunk_slot[i] = sl;
         }
         if (miss) {
@@ -509,7 +737,7 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
         d1 = (unsigned long long)(P.packed + (r - a.pstart[pp]) * a.C);
         cached = !(ch.res[gg] & kResNoSlot);  // else sent, never cached
         if (cached) {
-          slot = slots0 + ch.srank[gg];
+          slot = slot_of(ch.srank[gg]);
           d2 = (unsigned long long)(a.arena + slot * a.C);
         }
       }
@@ -524,6 +752,7 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
       }
       if (have && cached) {
         a.slot_len[slot] = ln;
+        if (a.lru) a.last_use[slot] = a.epoch;
         if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
         if (!a.paper && ln >= kPrefixBytes &&
@@ -564,6 +793,7 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
     const unsigned long long mbytes = __ldcg(&a.ctl->acc_miss_bytes);
     const unsigned long long stored = __ldcg(&a.ctl->acc_stored);
     const unsigned long long sbytes = __ldcg(&a.ctl->acc_stored_bytes);
+    const unsigned long long vbytes = __ldcg(&a.ctl->acc_victim_bytes);
     if (err == 0) {
       a.dstats[ST_CALLS] += a.ncalls;
       a.dstats[ST_CHUNKS] += N;
@@ -572,8 +802,9 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
       a.dstats[ST_MISSES] += misses;
       a.dstats[ST_INSERTS] += stored;
       a.dstats[ST_REJECTS] += rej;
-      a.dstats[ST_SLOTS_USED] = slots0 + stored;
-      a.dstats[ST_BYTES_USED] += sbytes;
+      a.dstats[ST_SLOTS_USED] = slots0 + stored - evict;
+      a.dstats[ST_BYTES_USED] += sbytes - vbytes;
+      a.dstats[ST_EVICTIONS] += evict;
     }
     gleam_result_t* t = a.total;
     t->status = err;
@@ -598,11 +829,16 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
   // Leave the per-call state as the next call expects it: the group table
   // (cleared entry by entry by the leaders, or here in full after an error
   // that may have stopped them) and the control block.
-  if (err)
+  if (err) {
     for (unsigned long long e = threadIdx.x; e <= a.tbl_mask; e += kThreads) {
       a.tbl[e].owner = 0u;
       a.tbl[e].minv = 0u;
     }
+    if (a.lru) {  // an eviction that stopped half-way may have left these set
+      for (uint32_t j = threadIdx.x; j < kLruBins; j += kThreads) a.bins[j] = 0u;
+      for (unsigned long long j = threadIdx.x; j < a.nslots; j += kThreads) a.vflag[j] = 0;
+    }
+  }
   __syncthreads();
   if (threadIdx.x == 0) {
     DevCtl* c = a.ctl;
@@ -613,6 +849,8 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
     c->acc_hits_cache = c->acc_hits_intra = c->acc_rejects = 0;
     c->acc_misses = c->acc_miss_bytes = 0;
     c->acc_stored = c->acc_stored_bytes = 0;
+    c->acc_distinct = c->evict_k = c->lru_below = c->lru_ties = c->acc_victim_bytes = 0;
+    c->lru_hi = c->lru_cut = 0;
     c->done = 0;
   }
   __threadfence();
@@ -648,13 +886,14 @@ __global__ void __launch_bounds__(kThreads) k_block_check(BlockCheckArgs a) {
 
 __global__ void k_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
                                unsigned long long* dstats, unsigned long long key, uint32_t slot,
-                               uint32_t len, DevCtl* ctl) {
+                               uint32_t len, DevCtl* ctl, uint32_t* last_use, uint32_t epoch) {
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   if (!index_insert(index, index_mask, key, slot, len)) {
     ctl->err = GLEAM_ERR_INTERNAL;
     return;
   }
   slot_len[slot] = len;
+  if (last_use) last_use[slot] = epoch;
   dstats[ST_SLOTS_USED] = (unsigned long long)slot + 1;
   dstats[ST_INSERTS] += 1;
   dstats[ST_BYTES_USED] += len;
@@ -702,8 +941,10 @@ cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s) {
 
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
                                 unsigned long long* dstats, unsigned long long key,
-                                uint32_t slot, uint32_t len, DevCtl* ctl, cudaStream_t s) {
-  k_debug_insert<<<1, 32, 0, s>>>(index, index_mask, slot_len, dstats, key, slot, len, ctl);
+                                uint32_t slot, uint32_t len, DevCtl* ctl, uint32_t* last_use,
+                                uint32_t epoch, cudaStream_t s) {
+  k_debug_insert<<<1, 32, 0, s>>>(index, index_mask, slot_len, dstats, key, slot, len, ctl,
+                                  last_use, epoch);
   return cudaGetLastError();
 }
 

@@ -29,6 +29,13 @@ struct gleam_cache {
   uint32_t* slot_len = nullptr;
   unsigned long long* dstats = nullptr;
 
+  // LRU eviction (GLEAM_EVICT_LRU)
+  uint32_t* last_use = nullptr;  // per slot
+  uint8_t* vflag = nullptr;      // per slot
+  uint32_t* victims = nullptr;   // per slot
+  uint32_t* bins = nullptr;      // kLruBins
+  uint32_t epoch = 0;            // clock value of the latest call
+
   // per-call workspace (per chunk, by global chunk number)
   uint64_t ws_chunks = 0;
   void* ws = nullptr;
@@ -69,6 +76,9 @@ struct gleam_snapshot {
   IndexEntry* hints = nullptr;
   uint64_t index_cap = 0;
   unsigned long long* dstats = nullptr;
+  uint32_t* slot_len = nullptr;  // LRU caches: slot lengths and last uses too
+  uint32_t* last_use = nullptr;
+  uint64_t nslots = 0;
 };
 
 namespace {
@@ -217,10 +227,10 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   cap = std::min<uint64_t>(cap, kMaxChunks);
   if (cap < nchunks) cap = nchunks;
   const uint64_t tcap = next_pow2(2 * cap);
-  const uint64_t sz[12] = {align256(cap),     align256(cap * 8), align256(cap * 4),
+  const uint64_t sz[13] = {align256(cap),     align256(cap * 8), align256(cap * 4),
                            align256(cap * 8), align256(cap * 4), align256(cap * 4),
                            align256(cap * 4), align256(cap * 4), align256(cap * 8),
-                           align256(cap * 4), align256(cap * 4),
+                           align256(cap * 4), align256(cap * 4), align256(cap * 4),
                            align256(tcap * sizeof(CallEntry))};
   uint64_t total = 0;
   for (uint64_t x : sz) total += x;
@@ -257,6 +267,8 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   b += sz[9];
   c->ch.srank = reinterpret_cast<uint32_t*>(b);
   b += sz[10];
+  c->ch.old = reinterpret_cast<uint32_t*>(b);
+  b += sz[11];
   c->tbl = reinterpret_cast<CallEntry*>(b);
   c->tbl_cap = tcap;
   c->ws_chunks = cap;
@@ -294,6 +306,10 @@ void destroy_cache(gleam_cache* c) {
     if (c->hints) cudaFree(c->hints);
     if (c->slot_len) cudaFree(c->slot_len);
     if (c->dstats) cudaFree(c->dstats);
+    if (c->last_use) cudaFree(c->last_use);
+    if (c->vflag) cudaFree(c->vflag);
+    if (c->victims) cudaFree(c->victims);
+    if (c->bins) cudaFree(c->bins);
     if (c->ctl) cudaFree(c->ctl);
     if (c->bcount) cudaFree(c->bcount);
     if (c->d_result) cudaFree(c->d_result);
@@ -360,6 +376,18 @@ int pack_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
   const uint64_t want = std::max<uint64_t>((nchunks + 255) / 256,
                                            (nbytes + kBytesPerDedupBlock - 1) / kBytesPerDedupBlock);
   return (int)std::max<uint64_t>(1, std::min<uint64_t>(c->pack_max_blocks, want));
+}
+
+// The LRU fields of a call's kernel arguments; takes the call's clock value.
+void set_lru(gleam_cache* c, DedupArgs* d, uint64_t nchunks) {
+  if (!(c->flags & GLEAM_EVICT_LRU)) return;
+  if (nchunks) ++c->epoch;
+  d->lru = 1u;
+  d->epoch = c->epoch;
+  d->last_use = c->last_use;
+  d->vflag = c->vflag;
+  d->victims = c->victims;
+  d->bins = c->bins;
 }
 
 // Enqueues one dedup call over `count` payloads on stream s, ordered after
@@ -460,6 +488,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   d.total = d_total ? d_total : c->d_result;
   d.ncalls = ncalls;
   d.wait_ns = c->wait_ns;
+  set_lru(c, &d, Ntot);
   d.skip_block = c->skip_block;
   c->skip_block = -1;  // the hook applies to one call
   int grid = dedup_grid(c, Ntot, nbytes);
@@ -512,7 +541,7 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   *out = nullptr;
   if (chunk_bytes < kMinChunk || chunk_bytes > kMaxChunk || chunk_bytes % 32 != 0)
     return GLEAM_ERR_INVALID_ARG;
-  if ((flags & ~(GLEAM_KEY16 | GLEAM_DEBUG_CHECKS | GLEAM_PAPER_IDS)) != 0)
+  if ((flags & ~(GLEAM_KEY16 | GLEAM_DEBUG_CHECKS | GLEAM_PAPER_IDS | GLEAM_EVICT_LRU)) != 0)
     return GLEAM_ERR_INVALID_ARG;
   const uint64_t nslots = capacity_bytes / chunk_bytes;
   if (nslots == 0 || nslots > 0xFFFFFFFEull) return GLEAM_ERR_INVALID_ARG;
@@ -539,6 +568,12 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   step(cudaMalloc(&c->hints, c->index_cap * sizeof(IndexEntry)));
   step(cudaMalloc(&c->slot_len, nslots * sizeof(uint32_t)));
   step(cudaMalloc(&c->dstats, ST_COUNT * sizeof(unsigned long long)));
+  if (flags & GLEAM_EVICT_LRU) {
+    step(cudaMalloc(&c->last_use, nslots * sizeof(uint32_t)));
+    step(cudaMalloc(&c->vflag, nslots));
+    step(cudaMalloc(&c->victims, nslots * sizeof(uint32_t)));
+    step(cudaMalloc(&c->bins, kLruBins * sizeof(uint32_t)));
+  }
   step(cudaMalloc(&c->ctl, sizeof(DevCtl)));
   step(cudaMalloc(&c->d_result, sizeof(gleam_result_t)));
   step(cudaMallocHost(&c->h_result, sizeof(gleam_result_t)));
@@ -561,6 +596,11 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     step(cudaMemset(c->hints, 0xFF, c->index_cap * sizeof(IndexEntry)));
     step(cudaMemset(c->dstats, 0, ST_COUNT * sizeof(unsigned long long)));
     step(cudaMemset(c->ctl, 0, sizeof(DevCtl)));
+    if (flags & GLEAM_EVICT_LRU) {
+      step(cudaMemset(c->last_use, 0, nslots * sizeof(uint32_t)));
+      step(cudaMemset(c->vflag, 0, nslots));
+      step(cudaMemset(c->bins, 0, kLruBins * sizeof(uint32_t)));
+    }
     step(cudaEventRecord(c->done, nullptr));
     step(cudaEventRecord(c->table_copied, nullptr));
     step(cudaDeviceSynchronize());
@@ -722,6 +762,7 @@ int gleam_cache_stats(const gleam_cache_t* c, gleam_stats_t* out) {
   out->verify_rejects = s[ST_REJECTS];
   out->slots_used = s[ST_SLOTS_USED];
   out->bytes_used = s[ST_BYTES_USED];
+  out->evictions = s[ST_EVICTIONS];
   out->capacity_bytes = c->capacity_bytes;
   out->nslots = c->nslots;
   out->chunk_bytes = c->C;
@@ -786,7 +827,8 @@ int gleam_cache_debug_insert(gleam_cache_t* c, uint64_t key, const void* d_bytes
   rc = cuda_err(cudaMemcpy(c->arena + used * c->C, d_bytes, len, cudaMemcpyDeviceToDevice));
   if (rc == GLEAM_OK)
     rc = cuda_err(launch_debug_insert(c->index, c->index_cap - 1, c->slot_len, c->dstats, k,
-                                      (uint32_t)used, (uint32_t)len, c->ctl, nullptr));
+                                      (uint32_t)used, (uint32_t)len, c->ctl, c->last_use,
+                                      c->last_use ? ++c->epoch : 0u, nullptr));
   if (rc == GLEAM_OK) rc = cuda_err(cudaDeviceSynchronize());
   if (rc == GLEAM_OK) rc = cuda_err(cudaEventRecord(c->done, nullptr));
   return rc;
@@ -802,6 +844,11 @@ int gleam_cache_debug_set(gleam_cache_t* c, int what, int64_t value) {
   }
   if (what == GLEAM_DEBUG_SKIP_ARRIVE) {
     c->skip_block = (int)value;
+    return GLEAM_OK;
+  }
+  if (what == GLEAM_DEBUG_CLOCK) {
+    if (value < 0 || value > 0xFFFFFFFEll) return GLEAM_ERR_INVALID_ARG;
+    c->epoch = (uint32_t)value;
     return GLEAM_OK;
   }
   return GLEAM_ERR_INVALID_ARG;
@@ -863,6 +910,17 @@ int gleam_cache_snapshot(gleam_cache_t* c, gleam_snapshot_t** out) {
   if (rc == GLEAM_OK)
     rc = cuda_err(cudaMemcpy(s->dstats, c->dstats, ST_COUNT * sizeof(unsigned long long),
                              cudaMemcpyDeviceToDevice));
+  if (rc == GLEAM_OK && c->last_use) {
+    s->nslots = c->nslots;
+    rc = cuda_err(cudaMalloc(&s->slot_len, c->nslots * sizeof(uint32_t)));
+    if (rc == GLEAM_OK) rc = cuda_err(cudaMalloc(&s->last_use, c->nslots * sizeof(uint32_t)));
+    if (rc == GLEAM_OK)
+      rc = cuda_err(cudaMemcpy(s->slot_len, c->slot_len, c->nslots * sizeof(uint32_t),
+                               cudaMemcpyDeviceToDevice));
+    if (rc == GLEAM_OK)
+      rc = cuda_err(cudaMemcpy(s->last_use, c->last_use, c->nslots * sizeof(uint32_t),
+                               cudaMemcpyDeviceToDevice));
+  }
   if (rc != GLEAM_OK) {
     gleam_snapshot_destroy(s);
     return rc;
@@ -887,6 +945,13 @@ int gleam_cache_restore(gleam_cache_t* c, const gleam_snapshot_t* s) {
   if (rc == GLEAM_OK)
     rc = cuda_err(cudaMemcpyAsync(c->dstats, s->dstats, ST_COUNT * sizeof(unsigned long long),
                                   cudaMemcpyDeviceToDevice, nullptr));
+  if (rc == GLEAM_OK && s->last_use) {
+    rc = cuda_err(cudaMemcpyAsync(c->slot_len, s->slot_len, s->nslots * sizeof(uint32_t),
+                                  cudaMemcpyDeviceToDevice, nullptr));
+    if (rc == GLEAM_OK)
+      rc = cuda_err(cudaMemcpyAsync(c->last_use, s->last_use, s->nslots * sizeof(uint32_t),
+                                    cudaMemcpyDeviceToDevice, nullptr));
+  }
   if (rc == GLEAM_OK) rc = cuda_err(cudaEventRecord(c->done, nullptr));
   return rc;
 }
@@ -898,6 +963,8 @@ void gleam_snapshot_destroy(gleam_snapshot_t* s) {
   if (s->index) cudaFree(s->index);
   if (s->hints) cudaFree(s->hints);
   if (s->dstats) cudaFree(s->dstats);
+  if (s->slot_len) cudaFree(s->slot_len);
+  if (s->last_use) cudaFree(s->last_use);
   cudaGetLastError();
   delete s;
 }
@@ -933,11 +1000,12 @@ constexpr uint64_t kNaOffRank = kNaOffEnt + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffHint = kNaOffRank + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffOrder = kNaOffHint + na_align(kNaChunks * 8);
 constexpr uint64_t kNaOffSrank = kNaOffOrder + na_align(kNaChunks * 4);
-constexpr uint64_t kNaOffTbl = kNaOffSrank + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffOld = kNaOffSrank + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffTbl = kNaOffOld + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffCtl = kNaOffTbl + na_align(kNaTable * sizeof(CallEntry));
 constexpr uint64_t kNaOffBcount = kNaOffCtl + na_align(sizeof(DevCtl));
 constexpr uint64_t kNaOffResult = kNaOffBcount + na_align((2 * kNaBlocks + 1) * 4);
-constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~4.9 MiB
+constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~4.6 MiB
 
 }  // namespace
 
@@ -1002,6 +1070,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   ch.hint = reinterpret_cast<unsigned long long*>(base + kNaOffHint);
   ch.order = reinterpret_cast<uint32_t*>(base + kNaOffOrder);
   ch.srank = reinterpret_cast<uint32_t*>(base + kNaOffSrank);
+  ch.old = reinterpret_cast<uint32_t*>(base + kNaOffOld);
   CallEntry* tbl = reinterpret_cast<CallEntry*>(base + kNaOffTbl);
   DevCtl* ctl = reinterpret_cast<DevCtl*>(base + kNaOffCtl);
   uint32_t* bcount = reinterpret_cast<uint32_t*>(base + kNaOffBcount);
@@ -1051,6 +1120,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.total = total;
   d.ncalls = 1;
   d.wait_ns = c->wait_ns;
+  set_lru(c, &d, N);
   d.skip_block = -1;
   const int grid = dedup_grid(c, N, n);
   if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, N, n), s))) != GLEAM_OK) return rc;

@@ -13,6 +13,9 @@ namespace gleam {
 // ---------------------------------------------------------------------------
 
 constexpr uint32_t kEmptySlot = 0xFFFFFFFFu;
+// A removed entry while an eviction rebuilds its cluster; no table holds one
+// between calls.
+constexpr uint32_t kTombSlot = 0xFFFFFFFEu;
 
 // One entry of the cache index: open addressing, linear probing, load <= 1/2.
 // An entry is free iff slot == kEmptySlot; key/len are valid once the insert
@@ -43,10 +46,11 @@ constexpr uint32_t kResLeader = 0x80000000u;   // | round in which it was resolv
 constexpr uint32_t kResNoSlot = 0x10000000u;   // a miss that is never cached
 constexpr uint32_t kResRoundMask = 0x0FFFFFFFu;
 
-// Device counters of one cache, in gleam_stats_t order (first nine fields).
+// Device counters of one cache, in gleam_stats_t order (the fields that
+// change; capacity, slot count and chunk size are host constants).
 enum StatIdx {
   ST_CALLS = 0, ST_CHUNKS, ST_HITS_CACHE, ST_HITS_INTRA, ST_MISSES, ST_INSERTS,
-  ST_REJECTS, ST_SLOTS_USED, ST_BYTES_USED, ST_COUNT
+  ST_REJECTS, ST_SLOTS_USED, ST_BYTES_USED, ST_EVICTIONS, ST_COUNT
 };
 
 // Per-call control block; starts zeroed and every dedup kernel leaves it zeroed.
@@ -64,6 +68,14 @@ struct DevCtl {
   unsigned long long acc_miss_bytes;
   unsigned long long acc_stored;
   unsigned long long acc_stored_bytes;
+  // LRU eviction (caches created with GLEAM_EVICT_LRU)
+  unsigned long long acc_distinct;      // distinct cached slots hit by the call
+  unsigned long long evict_k;           // slots the call evicts
+  unsigned long long lru_below;         // candidates older than the cut-off bin / stamp
+  unsigned long long lru_ties;          // candidates at the cut-off stamp to evict
+  unsigned long long acc_victim_bytes;  // stored bytes of the evicted slots
+  unsigned int lru_hi;                  // high 16 bits of the cut-off stamp
+  unsigned int lru_cut;                 // the cut-off stamp
 };
 
 // Position of a key in a power-of-two table: the 64-bit finaliser of
@@ -110,6 +122,7 @@ struct ChunkArrays {
   unsigned long long* hint;  // prefix hint (chunks of at least kPrefixBytes)
   uint32_t* order;           // order[r] = chunk number of the miss of rank r
   uint32_t* srank;           // exclusive count of stored (cached) misses before the chunk
+  uint32_t* old;             // LRU: last use of a hit's slot before this call stamped it
 };
 
 // Speculative verify.  After the first kPrefixBytes of a chunk the four XXH64
@@ -165,7 +178,16 @@ struct DedupArgs {
   unsigned long long wait_ns;
   int skip_block;
   uint32_t paper;            // no prefix hints are kept in GLEAM_PAPER_IDS mode
+  // LRU eviction (GLEAM_EVICT_LRU; lru == 0: the other fields are unused)
+  uint32_t lru;
+  uint32_t epoch;            // this call's clock value
+  uint32_t* last_use;        // per slot: clock value of its last use
+  uint8_t* vflag;            // per slot: evicted by this call (zero between calls)
+  uint32_t* victims;         // evicted slots in ascending order
+  uint32_t* bins;            // 65536-bin histogram (zero between calls)
 };
+
+constexpr uint32_t kLruBins = 65536;
 
 // Paper-identifier mode (App. B.1): chunks shorter than this get no entry.
 constexpr uint32_t kPaperMinCached = 1024;
@@ -176,7 +198,8 @@ cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s);
 cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s);
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
                                 unsigned long long* dstats, unsigned long long key,
-                                uint32_t slot, uint32_t len, DevCtl* ctl, cudaStream_t s);
+                                uint32_t slot, uint32_t len, DevCtl* ctl, uint32_t* last_use,
+                                uint32_t epoch, cudaStream_t s);
 struct BlockCheckArgs {
   const uint8_t* block;
   unsigned long long block_bytes;

@@ -61,5 +61,11 @@ def test_null_handles_are_rejected(lib):
 
 
 def test_gleam_struct_sizes():
-    assert ctypes.sizeof(B.gleam_stats_t) == 12 * 8
+    """The binding's structs have the header's fields, in the header's order."""
+    with open(HEADER) as f:
+        h = f.read()
+    body = re.search(r"typedef struct gleam_stats \{(.*?)\} gleam_stats_t;", h, re.S).group(1)
+    fields = re.findall(r"uint64_t (\w+);", body)
+    assert [f for f, _ in B.gleam_stats_t._fields_] == fields
+    assert ctypes.sizeof(B.gleam_stats_t) == 8 * len(fields)
     assert B.RESULT_WORDS * 8 == 48
