@@ -111,6 +111,19 @@ def build_workload(name, dev, sample_budget):
         wl.flags = B.GLEAM_PAPER_IDS
         return wl
 
+    if name == "llama3-8b-lru":
+        from paper_2607_23115_gb300 import binding as B
+        wl = build_workload("llama3-8b", dev, sample_budget)
+        nch = len(wl.up.chunks(wl.C))
+        wl.name = "llama3-8b-bf16-per-tensor-lru"
+        wl.capacity = (nch + nch // 20) * wl.C
+        wl.flags = B.GLEAM_EVICT_LRU
+        wl.desc = wl.desc + "; LRU cache (Sec. 4.1.3) of the base's chunks + 5%% slots " \
+                            "(%.2f GiB), so every step evicts half as many slots as it misses" \
+                            % (wl.capacity / GiB)
+        wl.sample_capacity = lambda pre_chunks: (pre_chunks + pre_chunks // 20) * wl.C
+        return wl
+
     if name.startswith("llama3-8b"):
         shapes = W.llama3_8b_shapes()
         variants = {"llama3-8b": (shapes, 24 * GiB, "Llama-3-8B-shaped bf16 upload, 291 tensors"),
@@ -245,7 +258,8 @@ def build_workload(name, dev, sample_budget):
     raise ValueError("unknown workload %r" % name)
 
 
-WORKLOADS = ["llama3-8b", "llama3-8b-paper-ids", "llama3-8b-layer", "llama3-8b-4layers",
+WORKLOADS = ["llama3-8b", "llama3-8b-paper-ids", "llama3-8b-lru", "llama3-8b-layer",
+             "llama3-8b-4layers",
              "gpt2-small",
              "gpt2-small-pass1", "fp16-64m", "small-calls", "small-calls-10k"] + \
     ["adversarial-%dk%s" % (c, m) for c in (1, 4, 16, 64) for m in ("", "-key16")]
@@ -318,8 +332,13 @@ def oracle_time(wl, budget, offset=0):
     the timed calls.  Returns (payload bytes, seconds, description)."""
     import oracle
     pre, pays, text = wl.sample(budget, offset)
-    oc = oracle.OracleCache(wl.capacity, wl.C, (oracle.KEY16 if wl.flags & 1 else 0) |
-                            (oracle.PAPER_IDS if wl.flags & 4 else 0))
+    capacity = wl.capacity
+    if getattr(wl, "sample_capacity", None):  # scaled so that the sample evicts too
+        capacity = wl.sample_capacity(sum((x.size + wl.C - 1) // wl.C for x in pre))
+        text += "; oracle cache of %d slots, so the sample evicts too" % (capacity // wl.C)
+    oc = oracle.OracleCache(capacity, wl.C, (oracle.KEY16 if wl.flags & 1 else 0) |
+                            (oracle.PAPER_IDS if wl.flags & 4 else 0) |
+                            (oracle.EVICT_LRU if wl.flags & 8 else 0))
     for orig, row in getattr(wl, "crafted_host", []):
         oc.debug_insert(oracle.xxh64(orig), row)
     for x in pre:
@@ -423,9 +442,11 @@ def run_gleam(args, rank, world, local_rank):
         cache.restore(snap)
         one_pass()
 
+    ev0 = cache.stats()["evictions"]
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
+    evictions = cache.stats()["evictions"] - ev0  # of the last warm-up step (restored before)
     r = results.cpu().numpy()
     assert (r[:, 0] == 0).all(), "a dedup call failed: %s" % r[r[:, 0] != 0][:3]
     miss_bytes = int(r[:, 5].sum())
@@ -540,6 +561,7 @@ def run_gleam(args, rank, world, local_rank):
                    "payload_bytes_per_step": total, "payloads_per_step": nt, "calls_per_step": 1,
                    "api": "gleam_dedup_copy_batch (one call = %d payloads)" % nt,
                    "chunk_bytes": C, "chunks_per_step": nchunks, "misses_per_step": n_miss,
+                   "evictions_per_step": evictions,
                    "cache_capacity_bytes": wl.capacity, "key16": bool(wl.flags & 1),
                    "l2": ("inputs (%.2f GB) fit in the 129 MB L2's reach: a 256 MiB buffer is "
                           "written between timed steps, outside each step's events"

@@ -260,6 +260,7 @@ __device__ __forceinline__ uint32_t block_rank(bool f, uint32_t* cnt, uint32_t* 
 __device__ bool lru_evict(const DedupArgs& a, unsigned long long slots0, unsigned long long K,
                           unsigned long long* sred, uint32_t* cnt, uint32_t* off,
                           unsigned long long* red64) {
+  static_assert(kLruBins == kThreads * kThreads, "one part of kThreads bins per thread");
   const uint32_t G = gridDim.x, lane = threadIdx.x & 31;
   const unsigned long long tid = (unsigned long long)blockIdx.x * kThreads + threadIdx.x;
   const unsigned long long nth = (unsigned long long)G * kThreads;
@@ -282,19 +283,37 @@ __device__ bool lru_evict(const DedupArgs& a, unsigned long long slots0, unsigne
     }
     if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
     if (blockIdx.x == 0) {
+      // the bin holding the K-th candidate: partial sums of 256 bins per
+      // thread (16-byte loads), the part holding it, then that part's bins
+      constexpr uint32_t kPer = kLruBins / kThreads;
+      const uint4* b4 = reinterpret_cast<const uint4*>(a.bins + threadIdx.x * kPer);
       unsigned long long part = 0;
-      for (uint32_t j = 0; j < kLruBins / kThreads; ++j)
-        part += __ldcg(&a.bins[threadIdx.x * (kLruBins / kThreads) + j]);
+#pragma unroll 16
+      for (uint32_t j = 0; j < kPer / 4; ++j) {
+        const uint4 v = __ldcg(b4 + j);
+        part += (unsigned long long)v.x + v.y + v.z + v.w;
+      }
       sred[threadIdx.x] = part;
       __syncthreads();
+      const unsigned long long target = K - below;  // >= 1 candidates in this range
       if (threadIdx.x == 0) {
-        const unsigned long long target = K - below;  // >= 1 candidates in this range
         unsigned long long acc = 0;
         uint32_t pi = 0;
         while (pi + 1 < (uint32_t)kThreads && acc + sred[pi] < target) acc += sred[pi++];
-        uint32_t bin = pi * (kLruBins / kThreads);
-        const uint32_t last = bin + kLruBins / kThreads - 1;
-        while (bin < last && acc + __ldcg(&a.bins[bin]) < target) acc += __ldcg(&a.bins[bin++]);
+        off[0] = pi;
+        sred[kThreads - 1] = acc;  // candidates before part pi (its own sum is no longer needed)
+      }
+      __syncthreads();
+      const uint32_t pi = off[0];
+      const unsigned long long acc0 = sred[kThreads - 1];
+      __syncthreads();
+      sred[threadIdx.x] = __ldcg(&a.bins[pi * kPer + threadIdx.x]);
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        unsigned long long acc = acc0;
+        uint32_t j = 0;
+        while (j + 1 < kPer && acc + sred[j] < target) acc += sred[j++];
+        const uint32_t bin = pi * kPer + j;
         if (pass == 0) {
           a.ctl->lru_hi = bin;
           a.ctl->lru_below = acc;
@@ -305,7 +324,8 @@ __device__ bool lru_evict(const DedupArgs& a, unsigned long long slots0, unsigne
         }
       }
       __syncthreads();
-      for (uint32_t j = threadIdx.x; j < kLruBins; j += kThreads) a.bins[j] = 0u;
+      uint4* z4 = reinterpret_cast<uint4*>(a.bins);
+      for (uint32_t j = threadIdx.x; j < kLruBins / 4; j += kThreads) z4[j] = make_uint4(0, 0, 0, 0);
     }
     if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
     hi_bin = __ldcg(&a.ctl->lru_hi);
