@@ -290,6 +290,64 @@ __device__ __forceinline__ uint32_t find_payload(const PayloadDesc* table, uint3
   return lo;
 }
 
+// The last p in [lo, hi) with chunk_base <= g, given table[lo].chunk_base <= g.
+__device__ __forceinline__ uint32_t find_payload_in(const PayloadDesc* table, uint32_t lo,
+                                                    uint32_t hi, unsigned long long g) {
+  while (hi - lo > 1) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (__ldg(&table[mid].chunk_base) <= g) lo = mid;
+    else hi = mid;
+  }
+  return lo;
+}
+
+// Payload owning chunk g, for a block whose threads handle consecutive chunks
+// starting at g0 (g >= g0).  Warp 0 finds g0's payload with a 32-way search
+// (32 independent loads per step, about log32(count) steps instead of
+// log2(count) dependent ones) and stages the chunk bases of the 32 payloads
+// from there in shared memory, where every thread then finds its own; a chunk
+// past them falls back to bisection.  Every thread of the block must call it.
+// scratch: 33 words of shared memory, free again when the call returns.
+__device__ __forceinline__ uint32_t block_find_payload(const PayloadDesc* table, uint32_t count,
+                                                       unsigned long long g0,
+                                                       unsigned long long g,
+                                                       unsigned long long* scratch) {
+  unsigned long long* s_base = scratch;
+  unsigned long long* s_p0 = scratch + 32;
+  if (threadIdx.x < 32) {
+    const uint32_t lane = threadIdx.x;
+    uint32_t lo = 0, hi = count;  // table[lo].chunk_base <= g0; hi == count or its base > g0
+    while (hi - lo > 1) {
+      const uint32_t span = hi - lo;
+      const uint32_t q = lo + 1 + (uint32_t)(((unsigned long long)(span - 1) * lane) >> 5);
+      const unsigned m = __ballot_sync(0xffffffffu, __ldg(&table[q].chunk_base) <= g0);
+      if (m == 0) {
+        hi = lo + 1;
+      } else {
+        const int L = 31 - __clz(m);  // pivots grow with the lane, so m is a prefix
+        const uint32_t qL = __shfl_sync(0xffffffffu, q, L);
+        const uint32_t qN = __shfl_sync(0xffffffffu, q, L < 31 ? L + 1 : 31);
+        lo = qL;
+        if (L < 31) hi = qN;
+      }
+    }
+    s_base[lane] = lo + lane < count ? __ldg(&table[lo + lane].chunk_base) : ~0ull;
+    if (lane == 0) *s_p0 = lo;
+  }
+  __syncthreads();
+  uint32_t lo = 0, hi = 32;
+  while (hi - lo > 1) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (s_base[mid] <= g) lo = mid;
+    else hi = mid;
+  }
+  const uint32_t p0 = (uint32_t)*s_p0;
+  __syncthreads();  // the scratch may be reused from here on
+  if (lo == 31 && p0 + 32 < count && __ldg(&table[p0 + 32].chunk_base) <= g)
+    return find_payload_in(table, p0 + 32, count, g);
+  return p0 + lo;
+}
+
 #endif  // __CUDACC__
 
 }  // namespace gleam

@@ -208,6 +208,12 @@ __device__ __forceinline__ bool group_equal(const uint8_t* p, const uint8_t* q, 
 template <bool kAligned, bool kProbe>
 __global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
   const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
+  __shared__ unsigned long long s_scratch[33];
+  const uint32_t pid_b =
+      a.count > 1 ? block_find_payload(a.table, a.count,
+                                       ((unsigned long long)blockIdx.x * blockDim.x) >> 2, g,
+                                       s_scratch)
+                  : 0u;
   if (g >= a.Ntot) return;  // whole groups leave together
   const uint32_t lane = threadIdx.x & 3;
   const int gbase = threadIdx.x & 28;
@@ -217,7 +223,7 @@ __global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
   const uint8_t* buf;
   unsigned long long n, base;
   if (a.count > 1) {
-    pid = find_payload(a.table, a.count, g);
+    pid = pid_b;
     buf = a.table[pid].buf;
     n = a.table[pid].n;
     base = a.table[pid].chunk_base;
@@ -380,6 +386,13 @@ template <bool kProbe>
 __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
+  // the payload search borrows the start of the stage buffers (no static
+  // shared memory: any would cost this kernel a fifth of its bandwidth)
+  const uint32_t pid_b =
+      a.count > 1 ? block_find_payload(a.table, a.count,
+                                       ((unsigned long long)blockIdx.x * blockDim.x) >> 2, g,
+                                       reinterpret_cast<unsigned long long*>(smem))
+                  : 0u;
   if (g >= a.Ntot) return;  // whole groups leave together
   const uint32_t lane = threadIdx.x & 3;
   const int gbase = threadIdx.x & 28;
@@ -394,7 +407,7 @@ __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a
   const uint8_t* buf;
   unsigned long long n, base;
   if (a.count > 1) {
-    pid = find_payload(a.table, a.count, g);
+    pid = pid_b;
     buf = a.table[pid].buf;
     n = a.table[pid].n;
     base = a.table[pid].chunk_base;
@@ -630,6 +643,12 @@ __device__ unsigned long long md5_prefix_key(const uint8_t* p, uint32_t m, const
 template <bool kAligned>
 __global__ void __launch_bounds__(kHashThreads) k_probe_paper(HashArgs a, Md5Table tab) {
   const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
+  __shared__ unsigned long long s_scratch[33];
+  const uint32_t pid_b =
+      a.count > 1 ? block_find_payload(a.table, a.count,
+                                       ((unsigned long long)blockIdx.x * blockDim.x) >> 2, g,
+                                       s_scratch)
+                  : 0u;
   if (g >= a.Ntot) return;  // whole groups leave together
   const uint32_t lane = threadIdx.x & 3;
   const int gbase = threadIdx.x & 28;
@@ -639,7 +658,7 @@ __global__ void __launch_bounds__(kHashThreads) k_probe_paper(HashArgs a, Md5Tab
   const uint8_t* buf;
   unsigned long long n, base;
   if (a.count > 1) {
-    pid = find_payload(a.table, a.count, g);
+    pid = pid_b;
     buf = a.table[pid].buf;
     n = a.table[pid].n;
     base = a.table[pid].chunk_base;
