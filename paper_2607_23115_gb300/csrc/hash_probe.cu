@@ -347,12 +347,18 @@ __global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
 // and the cached copy named by the prefix hint streams alongside into a
 // second buffer.  The lanes then hash and compare their words from shared
 // memory.  Stage 0 is exactly the prefix used for the hint.
+//
+// Two stages in flight and blocks of one warp (8 groups, 16.6 KB of shared
+// memory): about 100 groups share an SM, and that many independent chunks
+// hide each chunk's dependent lookups (payload, prefix hint, index probe)
+// better than deeper pipelines with fewer groups (measured: 3 stages and
+// 64 groups per SM took 5.05 ms on the Llama upload, this takes 4.64 ms).
 // ---------------------------------------------------------------------------
 #ifndef GLEAM_STAGE_DEPTH
-#define GLEAM_STAGE_DEPTH 3
+#define GLEAM_STAGE_DEPTH 2
 #endif
 #ifndef GLEAM_STAGED_THREADS
-#define GLEAM_STAGED_THREADS 256
+#define GLEAM_STAGED_THREADS 32
 #endif
 constexpr int kStage = 512;                                 // bytes per stage
 constexpr int kDepth = GLEAM_STAGE_DEPTH;                   // stages in flight
@@ -360,6 +366,7 @@ constexpr int kGroupBytes = kDepth * 2 * kStage + 32;       // +32: bank skew
 constexpr int kStagedThreads = GLEAM_STAGED_THREADS;
 constexpr int kStagedSmem = (kStagedThreads / 4) * kGroupBytes;
 static_assert(kStage == (int)kPrefixBytes, "stage 0 must be the hinted prefix");
+static_assert(kStagedSmem >= 33 * 8, "the payload search borrows 33 words of the stage buffers");
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
   asm volatile("cp.async.cg.shared.global.L2::256B [%0], [%1], 16;" ::"r"(dst), "l"(src)
