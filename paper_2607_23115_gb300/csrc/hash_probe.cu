@@ -715,6 +715,162 @@ __global__ void __launch_bounds__(kHashThreads) k_probe_paper(HashArgs a, Md5Tab
   }
 }
 
+// Staged variant of the paper-identifier probe for 16-byte-aligned payloads.
+// Stage 0 of the chunk arrives by cp.async; one lane computes the MD5 key
+// from shared memory, the group probes the index, and only if a key+length
+// candidate exists do the rest of the chunk and the candidate's copy stream
+// through two stages in flight and get compared (each lane compares the
+// 16-byte pieces it copied itself, so no cross-lane sync is needed); the
+// first difference ends the streaming.  A chunk without a candidate costs one
+// stage; further candidates after a mismatch are compared by re-reading.
+__global__ void __launch_bounds__(kStagedThreads) k_probe_paper_staged(HashArgs a, Md5Table tab) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
+  const uint32_t pid_b =
+      a.count > 1 ? block_find_payload(a.table, a.count,
+                                       ((unsigned long long)blockIdx.x * blockDim.x) >> 2, g,
+                                       reinterpret_cast<unsigned long long*>(smem))
+                  : 0u;
+  if (g >= a.Ntot) return;  // whole groups leave together
+  const uint32_t lane = threadIdx.x & 3;
+  const int gbase = threadIdx.x & 28;
+  const unsigned gmask = 0xFu << gbase;
+  uint8_t* region = smem + (threadIdx.x >> 2) * kGroupBytes;
+  const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(region);
+
+  uint32_t pid = 0;
+  const uint8_t* buf;
+  unsigned long long n, base;
+  if (a.count > 1) {
+    pid = pid_b;
+    buf = a.table[pid].buf;
+    n = a.table[pid].n;
+    base = a.table[pid].chunk_base;
+  } else {
+    buf = a.one.buf;
+    n = a.one.n;
+    base = a.one.chunk_base;
+  }
+  const unsigned long long start = (g - base) * a.C;
+  const uint32_t len = (uint32_t)min(a.C, n - start);
+  const uint8_t* p = buf + start;
+  const uint32_t full = (len >> 5) * 32;  // bytes in whole stripes
+  const uint32_t nst = (full + kStage - 1) / kStage;
+  auto sbytes = [&](uint32_t t) { return min((uint32_t)kStage, full - t * kStage); };
+
+  unsigned long long key = 0;
+  bool hit = false, cand = false;
+  uint32_t hit_slot = kEmptySlot;
+  if (len < kPaperMinCached) {  // recorded, never cached: only the key
+    if (lane == 0) key = md5_prefix_key(p, min(len, 128u), tab.k);
+    key = group_shfl(key, gmask, gbase);
+    if (a.key16) key &= 0xFFFFULL;
+  } else {
+    // stage 0 (the first 512 bytes) -> MD5 of its first 128 bytes
+    stage_copy(sbase, p, kStage, lane);
+    cp_commit();
+    cp_wait<0>();
+    __syncwarp(gmask);
+    if (lane == 0) key = md5_prefix_key(region, 128u, tab.k);
+    key = group_shfl(key, gmask, gbase);
+    if (a.key16) key &= 0xFFFFULL;
+
+    // the first key+length candidate
+    const unsigned long long slots_used = a.dstats[ST_SLOTS_USED];
+    unsigned long long pos = mix64(key) & a.index_mask;
+    uint32_t first = kEmptySlot;
+    for (unsigned long long probe = 0; probe <= a.index_mask; ++probe) {
+      const IndexEntry e = a.index[pos];
+      if (e.slot == kEmptySlot) break;
+      if (e.key == key && e.len == len) {
+        if (e.slot >= slots_used) {
+          if (lane == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+        } else {
+          first = e.slot;
+          break;
+        }
+      }
+      pos = (pos + 1) & a.index_mask;
+    }
+    if (first != kEmptySlot) {
+      cand = true;
+      const uint8_t* q = a.arena + (unsigned long long)first * a.C;
+      // stream the candidate (and the rest of the payload), two stages in flight
+      stage_copy(sbase + kStage, q, kStage, lane);
+      cp_commit();
+      if (nst > 1) {
+        stage_copy(sbase + 2 * kStage, p + kStage, sbytes(1), lane);
+        stage_copy(sbase + 3 * kStage, q + kStage, sbytes(1), lane);
+      }
+      cp_commit();
+      bool equal = true;
+      for (uint32_t t = 0; t < nst; ++t) {
+        cp_wait<1>();  // stage t's group; the one after it may still be in flight
+        const uint32_t b = (t & 1) * 2 * kStage;
+        unsigned long long d = 0;
+#pragma unroll
+        for (int j = 0; j < kStage / 64; ++j) {
+          const uint32_t off = (uint32_t)j * 64 + lane * 16;
+          if (off < sbytes(t)) {
+            const uint4 x = *reinterpret_cast<const uint4*>(region + b + off);
+            const uint4 y = *reinterpret_cast<const uint4*>(region + b + kStage + off);
+            d |= (unsigned long long)((x.x ^ y.x) | (x.y ^ y.y) | (x.z ^ y.z) | (x.w ^ y.w));
+          }
+        }
+        d |= __shfl_xor_sync(gmask, d, 1);
+        d |= __shfl_xor_sync(gmask, d, 2);
+        if (d) {
+          equal = false;
+          break;
+        }
+        if (t + 2 < nst) {  // into the buffers this lane has just read
+          stage_copy(sbase + b, p + (unsigned long long)(t + 2) * kStage, sbytes(t + 2), lane);
+          stage_copy(sbase + b + kStage, q + (unsigned long long)(t + 2) * kStage, sbytes(t + 2),
+                     lane);
+        }
+        cp_commit();
+      }
+      cp_wait<0>();
+      if (equal) {  // the bytes after the last whole stripe
+        unsigned long long d = 0;
+        if (lane == 0)
+          for (uint32_t k = full; k < len; ++k) d |= (unsigned long long)(p[k] ^ q[k]);
+        d |= __shfl_xor_sync(gmask, d, 1);
+        d |= __shfl_xor_sync(gmask, d, 2);
+        equal = d == 0;
+      }
+      if (equal) {
+        hit = true;
+        hit_slot = first;
+      } else {  // any further candidates, by re-reading both copies
+        pos = (pos + 1) & a.index_mask;
+        for (unsigned long long probe = 0; probe <= a.index_mask && !hit; ++probe) {
+          const IndexEntry e = a.index[pos];
+          if (e.slot == kEmptySlot) break;
+          if (e.key == key && e.len == len) {
+            if (e.slot >= slots_used) {
+              if (lane == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+            } else if (group_equal<true>(p, a.arena + (uint64_t)e.slot * a.C, len, lane, gmask)) {
+              hit = true;
+              hit_slot = e.slot;
+            }
+          }
+          pos = (pos + 1) & a.index_mask;
+        }
+      }
+    }
+  }
+  if (lane == 0) {
+    a.ch.status[g] = len < kPaperMinCached ? kUncached : hit ? kHit0 : cand ? kMissCand : kMissNoCand;
+    a.ch.key[g] = key;
+    a.ch.len[g] = len;
+    a.ch.src[g] = (unsigned long long)p;
+    a.ch.pidx[g] = pid;
+    a.ch.hint[g] = 0;
+    if (hit) a.ch.ent[g] = hit_slot;
+  }
+}
+
 Md5Table md5_table() {
   Md5Table t;
   for (int i = 0; i < 64; ++i)
@@ -731,6 +887,13 @@ cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
   const bool probe = a.index != nullptr;
   if (probe && a.paper) {
     static const Md5Table tab = md5_table();
+#if GLEAM_STAGED_HASH
+    if (aligned && a.C % 32 == 0) {
+      const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
+      k_probe_paper_staged<<<sg, kStagedThreads, kStagedSmem, s>>>(a, tab);
+      return cudaGetLastError();
+    }
+#endif
     if (aligned) k_probe_paper<true><<<grid, kHashThreads, 0, s>>>(a, tab);
     else k_probe_paper<false><<<grid, kHashThreads, 0, s>>>(a, tab);
     return cudaGetLastError();
