@@ -410,6 +410,15 @@ __device__ bool lru_evict(const DedupArgs& a, unsigned long long slots0, unsigne
   return true;
 }
 
+// Posts ~g as a candidate minimum of group entry `e` (0xFFFFFFFF: none), one
+// atomic per group of lanes that share the entry.  Called by the whole warp.
+__device__ __forceinline__ void post_minimum(const DedupArgs& a, uint32_t e, uint32_t g) {
+  const unsigned peers = __match_any_sync(0xffffffffu, e);
+  const uint32_t m = __reduce_max_sync(peers, e != 0xFFFFFFFFu ? ~g : 0u);
+  if (e != 0xFFFFFFFFu && (threadIdx.x & 31) == (uint32_t)(__ffs(peers) - 1))
+    atomicMax(&a.tbl[e].minv, m);
+}
+
 __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ uint32_t warp_cnt[kWarps];
@@ -444,34 +453,39 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
         r->miss_bytes = 0;
       }
     }
-    for (uint32_t g = tid; g < N; g += nth) {
-      const PayloadDesc& P = desc(a, ch.pidx[g]);
-      const unsigned long long i = g - P.chunk_base;
-      if ((i & 31) == 0) P.mask[i >> 5] = 0;
-      if (ch.status[g] == kHit0) {
-        ch.res[g] = kResHit0;
-        if (a.lru) {  // the first chunk to stamp a slot keeps its old value
-          const uint32_t old = atomicExch(&a.last_use[ch.ent[g]], a.epoch);
-          ch.old[g] = old;
-          distinct += old != a.epoch;
+    // warp-uniform steps, so that chunks of one group in a warp post their
+    // minimum with one atomic (all-zero chunks, say, share a group)
+    for (uint32_t base = tid - lane; base < N; base += nth) {
+      const uint32_t g = base + lane;
+      uint32_t post = 0xFFFFFFFFu;  // group entry that gets this chunk's number
+      if (g < N) {
+        const PayloadDesc& P = desc(a, ch.pidx[g]);
+        const unsigned long long i = g - P.chunk_base;
+        if ((i & 31) == 0) P.mask[i >> 5] = 0;
+        if (ch.status[g] == kHit0) {
+          ch.res[g] = kResHit0;
+          if (a.lru) {  // the first chunk to stamp a slot keeps its old value
+            const uint32_t old = atomicExch(&a.last_use[ch.ent[g]], a.epoch);
+            ch.old[g] = old;
+            distinct += old != a.epoch;
+          }
+        } else if (ch.status[g] == kUncached) {  // never cached: a miss of its own, in no group
+          ch.ent[g] = 0xFFFFFFFFu;
+          ch.res[g] = kResLeader | kResNoSlot | 1u;
+        } else {
+          const uint32_t e = group_entry(a, g, ch.key[g], ch.len[g]);
+          if (e == 0xFFFFFFFFu) {
+            atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+            ch.ent[g] = 0xFFFFFFFFu;
+            ch.res[g] = kResLeader | 1u;
+          } else {
+            ch.ent[g] = e;
+            ch.res[g] = kResUnresolved;
+            post = e;
+          }
         }
-        continue;
       }
-      if (ch.status[g] == kUncached) {  // never cached: a miss of its own, in no group
-        ch.ent[g] = 0xFFFFFFFFu;
-        ch.res[g] = kResLeader | kResNoSlot | 1u;
-        continue;
-      }
-      const uint32_t e = group_entry(a, g, ch.key[g], ch.len[g]);
-      if (e == 0xFFFFFFFFu) {
-        atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-        ch.ent[g] = 0xFFFFFFFFu;
-        ch.res[g] = kResLeader | 1u;
-        continue;
-      }
-      ch.ent[g] = e;
-      ch.res[g] = kResUnresolved;
-      atomicMax(&a.tbl[e].minv, ~g);
+      post_minimum(a, post, g);
     }
     if (a.lru) {
       distinct = block_sum<unsigned long long>(distinct, red64);
@@ -528,8 +542,10 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       if (ldcg_u32(&ch.res[g]) == kResUnresolved) a.tbl[ch.ent[g]].minv = 0;
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
     if (!ok) break;
-    for (uint32_t g = tid; g < N; g += nth)
-      if (ldcg_u32(&ch.res[g]) == kResUnresolved) atomicMax(&a.tbl[ch.ent[g]].minv, ~g);
+    for (uint32_t base = tid - lane; base < N; base += nth) {
+      const uint32_t g = base + lane;
+      post_minimum(a, g < N && ldcg_u32(&ch.res[g]) == kResUnresolved ? ch.ent[g] : 0xFFFFFFFFu, g);
+    }
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
     ++round;
   }
