@@ -498,12 +498,16 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   uint32_t round = 1;
   while (ok) {
     if (tid == 0) atomicExch(&a.ctl->unres[(round + 1) % 3], 0u);
+    // W chunks per warp step: 32, or fewer when there are too few chunks to
+    // give every warp a step (large chunks), so the compares spread over the grid
     const uint32_t nwarps = nth / 32;
-    for (uint32_t base = (tid / 32) * 32; base < N; base += nwarps * 32) {
+    uint32_t W = 32;
+    while (W > 1 && (unsigned long long)N < (unsigned long long)nwarps * W) W >>= 1;
+    for (uint32_t base = (tid / 32) * W; base < N; base += nwarps * W) {
       const uint32_t g = base + lane;
       bool need = false;
       uint32_t m = 0;
-      if (g < N && ldcg_u32(&ch.res[g]) == kResUnresolved) {
+      if (lane < W && g < N && ldcg_u32(&ch.res[g]) == kResUnresolved) {
         m = ~ldcg_u32(&a.tbl[ch.ent[g]].minv);
         if (m == g) {
           ch.res[g] = kResLeader | round;
