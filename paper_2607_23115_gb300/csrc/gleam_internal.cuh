@@ -251,6 +251,11 @@ __device__ __forceinline__ bool grid_barrier(DevCtl* ctl, unsigned int nblocks,
                                              unsigned long long wait_ns, bool skip) {
   __shared__ int s_ok;  // the block's verdict, so that every thread agrees
   __syncthreads();
+  if (nblocks == 1) {  // one block: the block barrier already orders its memory accesses
+    if (threadIdx.x == 0) s_ok = (!skip && ld_volatile_s32(&ctl->err) == 0) ? 1 : 0;
+    __syncthreads();
+    return s_ok != 0;
+  }
   if (threadIdx.x == 0 && !skip) {
     const unsigned int gen = ld_acquire_u32(&ctl->bar_gen);
     __threadfence();
