@@ -327,6 +327,19 @@ class ClockSampler:
 # the oracle on the host cores (bounded sample)
 # ---------------------------------------------------------------------------
 
+def cpu_model():
+    """The host CPU's model name (lscpu), or the machine type."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    import platform
+    return platform.machine()
+
+
 def oracle_time(wl, budget, offset=0):
     """The oracle over a bounded sample of the workload: prefill (untimed), then
     the timed calls.  Returns (payload bytes, seconds, description)."""
@@ -516,6 +529,8 @@ def run_gleam(args, rank, world, local_rank):
                     "value": round(total / (calls_ms * 1e-3) / 1e9, 2),
                     "us_per_call": round(calls_ms * 1e3 / nt, 3),
                     "host_wall_us_per_call": round(wall * 1e6 / nt, 3),
+                    "calls_per_s": round(nt / (calls_ms * 1e-3)),
+                    "insert_gbs": round(miss_bytes / (calls_ms * 1e-3) / 1e9, 2),
                     "how": "same step as %d gleam_dedup_copy_async calls (one per payload) "
                            "instead of one gleam_dedup_copy_batch call" % nt}
         if nt > 1000:  # synchronous calls, like cudaMemcpy, on the first 2000 payloads
@@ -587,7 +602,7 @@ def run_gleam(args, rank, world, local_rank):
         nbytes, dt, text = oracle_time(wl, args.cpu_sample_bytes)
         line["cpu_baseline"] = {
             "value": round(nbytes / dt / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sample": text, "host_cpus": os.cpu_count()}
+            "sample": text, "host_cpus": os.cpu_count(), "host_cpu_model": cpu_model()}
 
     if not args.no_e2e and not args.profile_launches and nt <= 1000:
         host = torch.empty(up.buf.numel(), dtype=torch.uint8, pin_memory=True)
@@ -812,7 +827,8 @@ def run_reference(args, rank, world):
         "impl": "reference",
         "config": {"workload": wl.name, "description": wl.desc, "chunk_bytes": wl.C},
         "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
-                         "sample": "per step: " + text, "host_cpus": os.cpu_count()},
+                         "sample": "per step: " + text, "host_cpus": os.cpu_count(),
+                         "host_cpu_model": cpu_model()},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
