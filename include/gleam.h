@@ -207,8 +207,13 @@ int gleam_dedup_copy_batch(gleam_cache_t* cache, const gleam_payload_t* payloads
  * payload is never written to device memory: only the misses are, to the
  * packed output and the arena.  h_buf / payload d_buf fields: page-locked
  * host memory (other host memory and device memory are rejected with
- * GLEAM_ERR_NOT_DEVICE_PTR); outputs: device memory.  Semantics, results and
- * ordering are those of gleam_dedup_copy_async / gleam_dedup_copy_batch. */
+ * GLEAM_ERR_NOT_DEVICE_PTR).  Outputs: device memory; the miss indices, the
+ * packed miss bytes and the chunk slots may also be page-locked host memory,
+ * which the kernels then write over the link directly, so the bytes that must
+ * cross the network land on the host without a separate copy (hit masks and
+ * results stay in device memory: they are updated with atomics).  Semantics,
+ * results and ordering are those of gleam_dedup_copy_async /
+ * gleam_dedup_copy_batch. */
 int gleam_dedup_copy_host_async(gleam_cache_t* cache, const void* h_buf, size_t n,
                                 uint32_t* d_hit_mask, uint32_t* d_miss_idx, void* d_miss_bytes,
                                 gleam_result_t* d_result, gleam_stream_t stream);

@@ -342,8 +342,21 @@ int describe(gleam_cache* c, PtrChecker& chk, const gleam_payload_t& p, PayloadD
   d->result = p.d_result;
   d->chunk_slot = p.d_chunk_slot;
   int rc;
+  // An output that the kernels only store to (no atomics) may, for the host
+  // entries, also be page-locked host memory: *out receives the address the
+  // kernels use.
+  auto check_out = [&](void* ptr, uint64_t bytes, void** out) -> int {
+    int r = chk.check(ptr, bytes);
+    if (r != GLEAM_ERR_NOT_DEVICE_PTR || !host_payload) return r;
+    const void* dev = nullptr;
+    if ((r = chk.check_host(ptr, bytes, &dev)) != GLEAM_OK) return r;
+    *out = const_cast<void*>(dev);
+    return GLEAM_OK;
+  };
   if (p.d_result && (rc = chk.check(p.d_result, sizeof(gleam_result_t))) != GLEAM_OK) return rc;
-  if (p.d_chunk_slot && N && (rc = chk.check(p.d_chunk_slot, N * 4)) != GLEAM_OK) return rc;
+  if (p.d_chunk_slot && N &&
+      (rc = check_out(p.d_chunk_slot, N * 4, reinterpret_cast<void**>(&d->chunk_slot))) != GLEAM_OK)
+    return rc;
   if (p.n == 0) return GLEAM_OK;
   if (host_payload) {
     const void* dev = nullptr;
@@ -353,8 +366,10 @@ int describe(gleam_cache* c, PtrChecker& chk, const gleam_payload_t& p, PayloadD
     return rc;
   }
   if ((rc = chk.check(p.d_hit_mask, ((N + 31) / 32) * 4)) != GLEAM_OK) return rc;
-  if ((rc = chk.check(p.d_miss_idx, N * 4)) != GLEAM_OK) return rc;
-  if ((rc = chk.check(p.d_miss_bytes, p.n)) != GLEAM_OK) return rc;
+  if ((rc = check_out(p.d_miss_idx, N * 4, reinterpret_cast<void**>(&d->miss_idx))) != GLEAM_OK)
+    return rc;
+  if ((rc = check_out(p.d_miss_bytes, p.n, reinterpret_cast<void**>(&d->packed))) != GLEAM_OK)
+    return rc;
   return GLEAM_OK;
 }
 

@@ -115,3 +115,34 @@ def test_pageable_and_device_memory_are_rejected_by_the_host_entry():
                                            out.miss_bytes)
         assert rc == B.GLEAM_ERR_NOT_DEVICE_PTR
         assert gc.stats()["calls"] == 0
+
+
+@pytest.mark.parametrize("offset", [0, 3])
+def test_indices_packed_bytes_and_slots_written_to_pinned_host_memory(offset):
+    """The host entries may put the miss indices, packed miss bytes and chunk
+    slots in page-locked host memory; the kernels write them over the link."""
+    C = 4 * KiB
+    gc, oc = Cache(64 * MiB, C), oracle.OracleCache(64 * MiB, C)
+    host = W.fp16_payload(4 * MiB, seed=1)
+    with gc:
+        for payload in (host[: 2 * MiB], torch.cat([host, host[:1000]]), host[: 3 * MiB + 77]):
+            n = payload.numel()
+            N = (n + C - 1) // C
+            hb = _pinned(payload, offset)
+            mask = torch.zeros((N + 31) // 32, dtype=torch.int32, device=DEV)
+            idx = torch.full((N,), -1, dtype=torch.int32).pin_memory()
+            packed = _pinned(torch.zeros(n, dtype=torch.uint8), offset)
+            slots = torch.full((N,), -1, dtype=torch.int32).pin_memory()
+            res = torch.zeros(B.RESULT_WORDS, dtype=torch.int64, device=DEV)
+            items = B.payload_array([(hb, n, mask, idx, packed, res, slots)])
+            rc = B.gleam_dedup_copy_host_batch(gc.handle, items, None, None)
+            assert rc == 0, rc
+            torch.cuda.synchronize()
+            r = result_dict(res)
+            rc_o, mask_o, miss_o, packed_o, slots_o = oc.dedup(payload.numpy(), chunk_slots=True)
+            assert r["status"] == 0 and r["n_miss"] == rc_o
+            assert np.array_equal(mask.cpu().numpy().view(np.uint32)[: len(mask_o)], mask_o)
+            assert np.array_equal(idx.numpy().view(np.uint32)[:rc_o], miss_o)
+            assert np.array_equal(packed.numpy()[: len(packed_o)], packed_o)
+            assert np.array_equal(slots.numpy().view(np.uint32), slots_o)
+        compare_cache(gc, oc)
