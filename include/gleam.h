@@ -61,7 +61,14 @@ enum gleam_status {
 #define GLEAM_KEY16 0x1u        /* test mode: index key = low 16 bits of XXH64,
                                    so unrelated chunks collide and every hit
                                    must be separated from them by the verify */
-#define GLEAM_DEBUG_CHECKS 0x2u /* extra device-side index/arena checks      */
+#define GLEAM_DEBUG_CHECKS 0x2u /* after every dedup call, check on the device
+                                   that each index entry names a used slot of
+                                   its recorded length, that each used slot has
+                                   exactly one index entry, and that each hint
+                                   entry names a used slot of its length; a
+                                   violation makes the call's statuses (and the
+                                   synchronous return) GLEAM_ERR_INTERNAL.  Costs
+                                   a pass over the index and 4 bytes per slot. */
 #define GLEAM_PAPER_IDS 0x4u    /* the paper's own identifier (App. B.1): the
                                    index key is MD5 of a chunk's first
                                    min(len, 128) bytes (first 8 digest bytes,
@@ -300,6 +307,9 @@ int gleam_cache_debug_insert(gleam_cache_t* cache, uint64_t key, const void* d_b
  * reach clock values of any size.  The clock is 32 bits: a cache that has
  * served 2^32 - 1 calls no longer orders its slots exactly. */
 #define GLEAM_DEBUG_CLOCK 3
+/* what = GLEAM_DEBUG_DROP_ENTRY: removes the index entry of slot `value`
+ * (damages the cache on purpose, to test GLEAM_DEBUG_CHECKS).  Synchronous. */
+#define GLEAM_DEBUG_DROP_ENTRY 4
 int gleam_cache_debug_set(gleam_cache_t* cache, int what, int64_t value);
 
 /* Device-side copy of the index, slot count and counters (and, for a

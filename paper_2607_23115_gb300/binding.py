@@ -29,6 +29,7 @@ GLEAM_EVICT_LRU = 0x8
 GLEAM_DEBUG_WAIT_LIMIT_NS = 1
 GLEAM_DEBUG_SKIP_ARRIVE = 2
 GLEAM_DEBUG_CLOCK = 3
+GLEAM_DEBUG_DROP_ENTRY = 4
 
 # Every symbol include/gleam.h declares (checked by the ABI test).
 EXPORTS = (

@@ -939,7 +939,57 @@ __global__ void k_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t*
   dstats[ST_BYTES_USED] += len;
 }
 
+// ---- GLEAM_DEBUG_CHECKS --------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_check_entries(IndexCheckArgs a) {
+  const unsigned long long used = a.dstats[ST_SLOTS_USED];
+  const unsigned long long n = a.index_mask + 1;
+  bool bad = false;
+  for (unsigned long long q = (unsigned long long)blockIdx.x * kThreads + threadIdx.x; q < n;
+       q += (unsigned long long)gridDim.x * kThreads) {
+    const IndexEntry e = a.index[q];
+    if (e.slot != kEmptySlot) {
+      if (e.slot >= used || e.len != a.slot_len[e.slot]) bad = true;
+      else atomicAdd(&a.count[e.slot], 1u);
+    }
+    const IndexEntry h = a.hints[q];
+    if (h.slot != kEmptySlot && (h.slot >= used || h.len != a.slot_len[h.slot])) bad = true;
+  }
+  if (bad) atomicExch(a.flag, 1u);
+}
+
+__global__ void __launch_bounds__(kThreads) k_check_slots(IndexCheckArgs a) {
+  const unsigned long long used = a.dstats[ST_SLOTS_USED];
+  bool bad = false;
+  for (unsigned long long sl = (unsigned long long)blockIdx.x * kThreads + threadIdx.x; sl < used;
+       sl += (unsigned long long)gridDim.x * kThreads) {
+    bad |= a.count[sl] != 1u;
+    a.count[sl] = 0u;
+  }
+  if (bad) atomicExch(a.flag, 1u);
+}
+
+__global__ void k_check_publish(IndexCheckArgs a) {
+  if (*(volatile uint32_t*)a.flag == 0u) return;
+  for (uint32_t p = threadIdx.x; p < a.npayloads; p += blockDim.x) {
+    gleam_result_t* r = a.npayloads > 1 ? a.table[p].result : a.one.result;
+    if (r) r->status = GLEAM_ERR_INTERNAL;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    a.total->status = GLEAM_ERR_INTERNAL;
+    *a.flag = 0u;
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_index_check(const IndexCheckArgs& a, cudaStream_t s) {
+  const unsigned grid = 1024;
+  k_check_entries<<<grid, kThreads, 0, s>>>(a);
+  k_check_slots<<<grid, kThreads, 0, s>>>(a);
+  k_check_publish<<<1, kThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
 
 int dedup_threads() { return kThreads; }
 

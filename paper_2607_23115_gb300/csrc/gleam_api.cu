@@ -36,6 +36,10 @@ struct gleam_cache {
   uint32_t* bins = nullptr;      // kLruBins
   uint32_t epoch = 0;            // clock value of the latest call
 
+  // GLEAM_DEBUG_CHECKS
+  uint32_t* dbg_count = nullptr;  // per slot
+  uint32_t* dbg_flag = nullptr;
+
   // per-call workspace (per chunk, by global chunk number)
   uint64_t ws_chunks = 0;
   void* ws = nullptr;
@@ -310,6 +314,8 @@ void destroy_cache(gleam_cache* c) {
     if (c->vflag) cudaFree(c->vflag);
     if (c->victims) cudaFree(c->victims);
     if (c->bins) cudaFree(c->bins);
+    if (c->dbg_count) cudaFree(c->dbg_count);
+    if (c->dbg_flag) cudaFree(c->dbg_flag);
     if (c->ctl) cudaFree(c->ctl);
     if (c->bcount) cudaFree(c->bcount);
     if (c->d_result) cudaFree(c->d_result);
@@ -403,6 +409,24 @@ void set_lru(gleam_cache* c, DedupArgs* d, uint64_t nchunks) {
   d->vflag = c->vflag;
   d->victims = c->victims;
   d->bins = c->bins;
+}
+
+// GLEAM_DEBUG_CHECKS: the index consistency check after a call.
+int enqueue_index_check(gleam_cache* c, const DedupArgs& d, cudaStream_t s) {
+  if (!(c->flags & GLEAM_DEBUG_CHECKS)) return GLEAM_OK;
+  IndexCheckArgs k{};
+  k.index = c->index;
+  k.hints = c->hints;
+  k.index_mask = c->index_cap - 1;
+  k.slot_len = c->slot_len;
+  k.dstats = c->dstats;
+  k.count = c->dbg_count;
+  k.flag = c->dbg_flag;
+  k.table = d.table;
+  k.one = d.one;
+  k.npayloads = d.count;
+  k.total = d.total;
+  return cuda_err(launch_index_check(k, s));
 }
 
 // Enqueues one dedup call over `count` payloads on stream s, ordered after
@@ -516,6 +540,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     return rc;
   }
   if (ev[2]) cudaEventRecord(ev[2], s);
+  if ((rc = enqueue_index_check(c, d, s)) != GLEAM_OK) return rc;
   return cuda_err(cudaEventRecord(c->done, s));
 }
 
@@ -583,6 +608,10 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   step(cudaMalloc(&c->hints, c->index_cap * sizeof(IndexEntry)));
   step(cudaMalloc(&c->slot_len, nslots * sizeof(uint32_t)));
   step(cudaMalloc(&c->dstats, ST_COUNT * sizeof(unsigned long long)));
+  if (flags & GLEAM_DEBUG_CHECKS) {
+    step(cudaMalloc(&c->dbg_count, nslots * sizeof(uint32_t)));
+    step(cudaMalloc(&c->dbg_flag, sizeof(uint32_t)));
+  }
   if (flags & GLEAM_EVICT_LRU) {
     step(cudaMalloc(&c->last_use, nslots * sizeof(uint32_t)));
     step(cudaMalloc(&c->vflag, nslots));
@@ -611,6 +640,10 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     step(cudaMemset(c->hints, 0xFF, c->index_cap * sizeof(IndexEntry)));
     step(cudaMemset(c->dstats, 0, ST_COUNT * sizeof(unsigned long long)));
     step(cudaMemset(c->ctl, 0, sizeof(DevCtl)));
+    if (flags & GLEAM_DEBUG_CHECKS) {
+      step(cudaMemset(c->dbg_count, 0, nslots * sizeof(uint32_t)));
+      step(cudaMemset(c->dbg_flag, 0, sizeof(uint32_t)));
+    }
     if (flags & GLEAM_EVICT_LRU) {
       step(cudaMemset(c->last_use, 0, nslots * sizeof(uint32_t)));
       step(cudaMemset(c->vflag, 0, nslots));
@@ -860,6 +893,22 @@ int gleam_cache_debug_set(gleam_cache_t* c, int what, int64_t value) {
   if (what == GLEAM_DEBUG_SKIP_ARRIVE) {
     c->skip_block = (int)value;
     return GLEAM_OK;
+  }
+  if (what == GLEAM_DEBUG_DROP_ENTRY) {  // damage the index on purpose (host side)
+    DeviceGuard g(c->device);
+    int rc = wait_done(c);
+    if (rc != GLEAM_OK) return rc;
+    std::vector<IndexEntry> host(c->index_cap);
+    rc = cuda_err(cudaMemcpy(host.data(), c->index, c->index_cap * sizeof(IndexEntry),
+                             cudaMemcpyDeviceToHost));
+    if (rc != GLEAM_OK) return rc;
+    for (uint64_t q = 0; q < c->index_cap; ++q)
+      if (host[q].slot == (uint64_t)value) {
+        const uint32_t empty = kEmptySlot;
+        return cuda_err(cudaMemcpy(&c->index[q].slot, &empty, sizeof(empty),
+                                   cudaMemcpyHostToDevice));
+      }
+    return GLEAM_ERR_INVALID_ARG;
   }
   if (what == GLEAM_DEBUG_CLOCK) {
     if (value < 0 || value > 0xFFFFFFFEll) return GLEAM_ERR_INVALID_ARG;
@@ -1139,5 +1188,6 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.skip_block = -1;
   const int grid = dedup_grid(c, N, n);
   if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, N, n), s))) != GLEAM_OK) return rc;
+  if ((rc = enqueue_index_check(c, d, s)) != GLEAM_OK) return rc;
   return cuda_err(cudaEventRecord(c->done, s));
 }

@@ -215,6 +215,25 @@ struct BlockCheckArgs {
 };
 
 cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s);
+
+// GLEAM_DEBUG_CHECKS: after a call, every index entry must name a used slot
+// with its recorded length, every used slot must be named by exactly one
+// index entry, and every hint entry must name a used slot of its length; a
+// violation turns the call's statuses into GLEAM_ERR_INTERNAL.
+struct IndexCheckArgs {
+  const IndexEntry* index;
+  const IndexEntry* hints;
+  unsigned long long index_mask;
+  const uint32_t* slot_len;
+  const unsigned long long* dstats;
+  uint32_t* count;           // per slot, zero between checks
+  uint32_t* flag;            // zero between checks
+  const PayloadDesc* table;  // the call's payloads (count > 1), or `one`
+  PayloadDesc one;
+  uint32_t npayloads;
+  gleam_result_t* total;
+};
+cudaError_t launch_index_check(const IndexCheckArgs& a, cudaStream_t s);
 int dedup_threads();
 int dedup_chunks_per_block();
 int dedup_blocks_per_sm();
