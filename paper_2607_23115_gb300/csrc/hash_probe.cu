@@ -3,16 +3,19 @@
 // resident chunks; App. B.1: confirm the match so collisions cannot alias).
 //
 // Mapping: a group of 4 consecutive threads owns one chunk; thread `lane`
-// runs XXH64 accumulator lane `lane`, reading the 8-byte word at 8*lane of
-// each 32-byte stripe straight from HBM (8 loads in flight per thread, the
-// next batch issued before the current one is folded in).  A warp therefore
-// streams 8 chunks at once and every 32-byte sector it touches is used whole.
-// After the first 512 bytes the group looks its prefix hint up and, if a
-// cached chunk began the same way, streams that copy alongside the payload
-// and compares as it hashes (speculative verify).  The group then probes the
-// index with the full fingerprint; the hinted slot is a hit if it is a
-// key+length candidate and compared equal, and any other candidate is
-// compared by re-reading both copies.
+// runs XXH64 accumulator lane `lane` on the 8-byte word at 8*lane of each
+// 32-byte stripe, so a warp works on 8 chunks and every 32-byte sector it
+// touches is used whole.  After the first 512 bytes the group looks its
+// prefix hint up and, if a cached chunk began the same way, streams that copy
+// alongside the payload and compares as it hashes (speculative verify).  The
+// group then probes the index with the full fingerprint; the hinted slot is a
+// hit if it is a key+length candidate and compared equal, and any other
+// candidate is compared by re-reading both copies.
+//
+// Kernels: k_hash_probe_staged (16-byte-aligned payloads: chunks stream
+// through shared memory by cp.async), k_hash_probe (any alignment: direct
+// loads), and for the paper's identifiers k_probe_paper_staged /
+// k_probe_paper (MD5 of the first 128 bytes as the key).
 #include <cmath>
 
 #include "gleam_internal.cuh"
