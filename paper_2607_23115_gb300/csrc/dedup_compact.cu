@@ -136,6 +136,151 @@ __device__ void warp_copy2(uint8_t* d1, uint8_t* d2, const uint8_t* s, uint32_t 
   }
 }
 
+// ---- bulk asynchronous copies (k_pack's miss copies) -------------------------
+//
+// Lane 0 of a warp moves the warp's misses through kPackBufs shared-memory
+// buffers of kPackPiece bytes: a bulk copy (the TMA engine, no registers)
+// brings a piece in and signals an mbarrier with its byte count, then two bulk
+// copies write it to the packed output and the arena slot.  Up to kPackBufs
+// pieces are in flight per warp across chunk boundaries.  Needs 16-byte
+// aligned addresses; a chunk's last len % 16 bytes are copied by its lane.
+#ifndef GLEAM_PACK_BULK
+#define GLEAM_PACK_BULK 1
+#endif
+constexpr uint32_t kPackPiece = 2048;
+constexpr uint32_t kPackBufs = 4;
+struct PackMeta {
+  unsigned long long src, d1, d2;
+  uint32_t len, pad;
+};
+// per warp: the buffers, then the mbarriers (64 B), then the batch's metadata;
+// a multiple of 128 bytes so that every warp's buffers start 128-byte aligned
+constexpr uint32_t kPackWarpBytes =
+    (kPackBufs * kPackPiece + 64 + 32 * (uint32_t)sizeof(PackMeta) + 127) & ~127u;
+constexpr uint32_t kPackSmem = GLEAM_PACK_BULK ? kWarps * kPackWarpBytes : 0;
+
+__device__ __forceinline__ void mbar_init(uint32_t bar) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(done)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+// Waits for the mbarrier's phase of this parity, for at most limit_ns.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
+                                         unsigned long long limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity))
+    if (globaltimer_ns() - t0 > limit_ns) return false;
+  return true;
+}
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,
+                                          uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_store(void* dst, uint32_t src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+template <int N>
+__device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
+}
+// Until at most n (0..3; more waits for 3) newest bulk store groups still read
+// shared memory.
+__device__ __forceinline__ void bulk_wait_read_n(uint32_t n) {
+  if (n == 0) bulk_wait_read<0>();
+  else if (n == 1) bulk_wait_read<1>();
+  else if (n == 2) bulk_wait_read<2>();
+  else bulk_wait_read<3>();
+}
+static_assert(kPackBufs == 4, "bulk_wait_read_n covers up to kPackBufs - 1 pending groups");
+
+// Ring state of one warp's lane 0, kept across its batches of 32 misses.
+struct PackRing {
+  uint32_t issued, consumed, phase;
+};
+
+// Lane 0: the whole-16-byte part of chunks 0..m-1 of `meta`; false if a
+// piece did not arrive within limit_ns (the pieces still in flight have then
+// been waited for, again with the limit).
+__device__ bool bulk_copy_batch(const PackMeta* meta, uint32_t m, uint32_t bufs, uint32_t bars,
+                                PackRing& ring, unsigned long long limit_ns) {
+  auto nbytes = [&](uint32_t j) { return meta[j].len & ~15u; };
+  uint32_t ij = 0, ioff = 0, cj = 0, coff = 0;  // issue and consume cursors
+  while (ij < m && nbytes(ij) == 0) ++ij;
+  cj = ij;
+  while (cj < m) {
+    while (ring.issued - ring.consumed < kPackBufs && ij < m) {
+      const uint32_t b = ring.issued % kPackBufs;
+      // the store that last read buffer b (piece issued - kPackBufs) must be done reading
+      if (ring.issued >= kPackBufs) bulk_wait_read_n(kPackBufs - 1 - (ring.issued - ring.consumed));
+      const uint32_t nb = nbytes(ij);
+      const uint32_t bytes = min(kPackPiece, nb - ioff);
+      mbar_expect_tx(bars + 8 * b, bytes);
+      bulk_load(bufs + b * kPackPiece, reinterpret_cast<const uint8_t*>(meta[ij].src) + ioff, bytes,
+                bars + 8 * b);
+      ++ring.issued;
+      ioff += bytes;
+      if (ioff == nb) {
+        ioff = 0;
+        do ++ij;
+        while (ij < m && nbytes(ij) == 0);
+      }
+    }
+    const uint32_t b = ring.consumed % kPackBufs;
+    if (!mbar_wait(bars + 8 * b, (ring.phase >> b) & 1u, limit_ns)) {
+      for (uint32_t k = ring.consumed; k < ring.issued; ++k) {  // let the loads land
+        const uint32_t bb = k % kPackBufs;
+        mbar_wait(bars + 8 * bb, (ring.phase >> bb) & 1u, limit_ns);
+        ring.phase ^= 1u << bb;
+      }
+      ring.consumed = ring.issued;
+      return false;
+    }
+    ring.phase ^= 1u << b;
+    const uint32_t nb = nbytes(cj);
+    const uint32_t bytes = min(kPackPiece, nb - coff);
+    bulk_store(reinterpret_cast<uint8_t*>(meta[cj].d1) + coff, bufs + b * kPackPiece, bytes);
+    if (meta[cj].d2) bulk_store(reinterpret_cast<uint8_t*>(meta[cj].d2) + coff, bufs + b * kPackPiece, bytes);
+    bulk_commit();
+    ++ring.consumed;
+    coff += bytes;
+    if (coff == nb) {
+      coff = 0;
+      do ++cj;
+      while (cj < m && nbytes(cj) == 0);
+    }
+  }
+  return true;
+}
+
 // Claims a free index entry for (key, slot, len); false if the table is full.
 __device__ bool index_insert(IndexEntry* index, uint64_t mask, unsigned long long key,
                              uint32_t slot, uint32_t len) {
@@ -683,6 +828,20 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
   const unsigned long long total = s_total;
   const unsigned long long evict = s_evict;
   const bool ok = s_err == 0;
+#if GLEAM_PACK_BULK
+  extern __shared__ __align__(128) uint8_t pack_smem[];
+  const uint32_t wbase = (uint32_t)__cvta_generic_to_shared(pack_smem) + w * kPackWarpBytes;
+  const uint32_t bufs = wbase, bars = wbase + kPackBufs * kPackPiece;
+  PackMeta* meta = reinterpret_cast<PackMeta*>(pack_smem + w * kPackWarpBytes +
+                                               kPackBufs * kPackPiece + 64);
+  PackRing ring{0u, 0u, 0u};
+  if (lane == 0) {
+    for (uint32_t b = 0; b < kPackBufs; ++b) mbar_init(bars + 8 * b);
+    mbar_fence_init();
+  }
+  __syncwarp();
+  bool bulk_failed = false;
+#endif
   // slot of the stored miss of stored rank sr: the evicted slots in ascending
   // order, then never-used slots
   auto slot_of = [&](uint32_t sr) -> unsigned long long {
@@ -782,6 +941,29 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
         }
       }
       const uint32_t m = (uint32_t)((hi - base) < 32ull ? (hi - base) : 32ull);
+#if GLEAM_PACK_BULK
+      const bool bulk =
+          !a.plain_copy && __all_sync(0xffffffffu, !have || ((src | d1 | d2) & 15) == 0);
+      if (bulk) {
+        if (have) meta[lane] = PackMeta{src, d1, d2, ln, 0u};
+        __syncwarp();
+        if (lane == 0 && !bulk_failed &&
+            !bulk_copy_batch(meta, m, bufs, bars, ring, a.wait_ns)) {
+          bulk_failed = true;
+          atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_TIMEOUT);
+        }
+        if (have) {  // the last len % 16 bytes
+          const uint8_t* sp = reinterpret_cast<const uint8_t*>(src);
+          uint8_t* x = reinterpret_cast<uint8_t*>(d1);
+          uint8_t* y = reinterpret_cast<uint8_t*>(d2);
+          for (uint32_t k = ln & ~15u; k < ln; ++k) {
+            x[k] = sp[k];
+            if (y) y[k] = sp[k];
+          }
+        }
+        __syncwarp();
+      } else
+#endif
       for (uint32_t j = 0; j < m; ++j) {
         const unsigned long long sj = __shfl_sync(0xffffffffu, src, j);
         const unsigned long long xj = __shfl_sync(0xffffffffu, d1, j);
@@ -800,6 +982,9 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       }
     }
+#if GLEAM_PACK_BULK
+    if (lane == 0) bulk_wait_all<0>();  // every piece written before the block ends
+#endif
     n_hc = block_sum<unsigned long long>(n_hc, red64);
     n_hi = block_sum<unsigned long long>(n_hi, red64);
     n_rej = block_sum<unsigned long long>(n_rej, red64);
@@ -998,7 +1183,12 @@ int dedup_chunks_per_block() { return GLEAM_DEDUP_CHUNKS_PER_BLOCK; }
 // Co-resident blocks per SM of the pack kernel.
 int pack_blocks_per_sm() {
   int nb = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_pack, kThreads, 0) != cudaSuccess)
+  if (kPackSmem > 48 * 1024 &&
+      cudaFuncSetAttribute((const void*)k_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kPackSmem) != cudaSuccess)
+    return 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_pack, kThreads, kPackSmem) !=
+      cudaSuccess)
     return 0;
   return nb;
 }
@@ -1017,7 +1207,10 @@ cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream
   cudaError_t e =
       cudaLaunchCooperativeKernel((void*)k_dedup, dim3(grid), dim3(kThreads), args, 0, s);
   if (e != cudaSuccess) return e;
-  k_pack<<<pack_grid, kThreads, 0, s>>>(a);
+  if (kPackSmem > 48 * 1024)
+    cudaFuncSetAttribute((const void*)k_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         kPackSmem);
+  k_pack<<<pack_grid, kThreads, kPackSmem, s>>>(a);
   return cudaGetLastError();
 }
 

@@ -148,6 +148,9 @@ class PtrChecker {
  public:
   explicit PtrChecker(int device) : device_(device) {}
 
+  // Whether any pointer checked so far was managed memory.
+  bool saw_managed() const { return managed_; }
+
   // GLEAM_OK iff [p, p + bytes) is page-locked host memory (cudaHostAlloc or
   // cudaHostRegister) that the device can read; *dev receives the address to
   // use in device code.
@@ -190,6 +193,7 @@ class PtrChecker {
     const bool ok = at.type == cudaMemoryTypeManaged ||
                     (at.type == cudaMemoryTypeDevice && at.device == device_);
     if (!ok) return GLEAM_ERR_NOT_DEVICE_PTR;
+    managed_ = managed_ || at.type == cudaMemoryTypeManaged;
     if (PtrAttrsFn fn = driver_ptr_attrs()) {
       CUpointer_attribute attrs[2] = {CU_POINTER_ATTRIBUTE_RANGE_START_ADDR,
                                       CU_POINTER_ATTRIBUTE_RANGE_SIZE};
@@ -212,6 +216,7 @@ class PtrChecker {
   uintptr_t lo_[kRanges] = {};
   uintptr_t hi_[kRanges] = {};
   int next_ = 0;
+  bool managed_ = false;
 };
 
 void free_ws(gleam_cache* c) {
@@ -520,6 +525,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   d.ch = c->ch;
   d.pstart = count > 1 ? c->d_pstart : c->bcount + 2 * c->coop_max_blocks;
   d.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
+  d.plain_copy = (host_payloads || chk.saw_managed()) ? 1u : 0u;
   d.tbl = c->tbl;
   d.tbl_mask = tcap - 1;
   d.bcount = c->bcount;
@@ -1184,6 +1190,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.total = total;
   d.ncalls = 1;
   d.wait_ns = c->wait_ns;
+  d.plain_copy = chk.saw_managed() ? 1u : 0u;
   set_lru(c, &d, N);
   d.skip_block = -1;
   const int grid = dedup_grid(c, N, n);

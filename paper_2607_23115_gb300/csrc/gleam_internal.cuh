@@ -178,6 +178,8 @@ struct DedupArgs {
   unsigned long long wait_ns;
   int skip_block;
   uint32_t paper;            // no prefix hints are kept in GLEAM_PAPER_IDS mode
+  uint32_t plain_copy;       // copy misses with loads and stores, not bulk copies
+                             // (payloads or outputs in host or managed memory)
   // LRU eviction (GLEAM_EVICT_LRU; lru == 0: the other fields are unused)
   uint32_t lru;
   uint32_t epoch;            // this call's clock value
