@@ -16,6 +16,7 @@
 // through shared memory by cp.async), k_hash_probe (any alignment: direct
 // loads), and for the paper's identifiers k_probe_paper_staged /
 // k_probe_paper (MD5 of the first 128 bytes as the key).
+#include <algorithm>
 #include <cmath>
 
 #include "gleam_internal.cuh"
@@ -392,15 +393,15 @@ __device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uin
   }
 }
 
+// The chunks of block-sized range vb (kStagedThreads / 4 consecutive chunks).
 template <bool kProbe>
-__global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {
-  extern __shared__ __align__(16) uint8_t smem[];
-  const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
+__device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long long vb,
+                                             uint8_t* smem) {
+  const unsigned long long g = (vb * blockDim.x + threadIdx.x) >> 2;
   // the payload search borrows the start of the stage buffers (no static
   // shared memory: any would cost this kernel a fifth of its bandwidth)
   const uint32_t pid_b =
-      a.count > 1 ? block_find_payload(a.table, a.count,
-                                       ((unsigned long long)blockIdx.x * blockDim.x) >> 2, g,
+      a.count > 1 ? block_find_payload(a.table, a.count, (vb * blockDim.x) >> 2, g,
                                        reinterpret_cast<unsigned long long*>(smem))
                   : 0u;
   if (g >= a.Ntot) return;  // whole groups leave together
@@ -577,6 +578,16 @@ __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a
     a.ch.pidx[g] = pid;
     a.ch.hint[g] = hint;
     if (hit) a.ch.ent[g] = hit_slot;
+  }
+}
+
+template <bool kProbe>
+__global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  const unsigned long long nvb = (a.Ntot * 4 + kStagedThreads - 1) / kStagedThreads;
+  for (unsigned long long vb = blockIdx.x; vb < nvb; vb += gridDim.x) {
+    __syncthreads();  // the previous range's groups are done with the shared memory
+    staged_range<kProbe>(a, vb, smem);
   }
 }
 
