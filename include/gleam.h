@@ -177,7 +177,9 @@ int gleam_fingerprint(const void* d_buf, size_t n, size_t chunk_bytes, uint64_t*
  * Synchronous like cudaMemcpy (runs on the legacy default stream).
  * Returns the number of misses (>= 0) or a negative gleam_status; on
  * GLEAM_ERR_CAPACITY and GLEAM_ERR_TIMEOUT the cache is unchanged and the
- * outputs are unspecified.  n == 0 returns 0 and touches nothing. */
+ * outputs are unspecified.  n == 0 returns 0 and touches nothing.
+ * With GLEAM_EVICT_LRU, misses that do not fit the never-used slots take the
+ * slots of least recently used chunks that this call did not hit. */
 int64_t gleam_dedup_copy(gleam_cache_t* cache, const void* d_buf, size_t n,
                          uint32_t* d_hit_mask, uint32_t* d_miss_idx, void* d_miss_bytes);
 
@@ -198,9 +200,11 @@ int gleam_dedup_copy_async(gleam_cache_t* cache, const void* d_buf, size_t n,
  * host-to-device copy in turn; a chunk equal to an earlier payload's miss is
  * a hit on the cache, as that payload's call would have inserted it).  All
  * chunks of all payloads are processed together, so per-call latency is paid
- * once.  Exception: if the misses of the whole batch do not fit the free
+ * once.  Exceptions: if the misses of the whole batch do not fit the free
  * slots, the batch returns GLEAM_ERR_CAPACITY as a unit and the cache is
- * unchanged.  payloads: host array, read before the call returns (each
+ * unchanged; with GLEAM_EVICT_LRU the batch is one call for eviction (one
+ * clock value, victims chosen once, among the slots no payload of the batch
+ * hit).  payloads: host array, read before the call returns (each
  * entry's buffers as for gleam_dedup_copy).  d_total (device, may be NULL)
  * receives the sums over the batch.  Asynchronous on `stream`; ordered after
  * the cache's previous call whatever its stream. */
