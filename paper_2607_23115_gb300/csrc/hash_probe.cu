@@ -258,7 +258,9 @@ __global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
       const unsigned long long b2 = group_shfl(acc, gmask, gbase + 2);
       const unsigned long long b3 = group_shfl(acc, gmask, gbase + 3);
       hint = b0 ^ xrotl(b1, 16) ^ xrotl(b2, 32) ^ xrotl(b3, 48);
-      hint_slot = hint_lookup(a.hints, a.index_mask, hint, len, slots_used);
+      // an empty cache has no hints to look up
+      hint_slot = slots_used ? hint_lookup(a.hints, a.index_mask, hint, len, slots_used)
+                             : kEmptySlot;
       const uint8_t* q = a.arena + (unsigned long long)hint_slot * a.C;
       cmp = hint_slot != kEmptySlot;
       if (cmp) {  // the prefix, already hashed, is compared once (payload words from L2)
@@ -311,7 +313,7 @@ __global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
   unsigned long long pos = mix64(key) & a.index_mask;
   bool hit = false, cand = false;
   uint32_t hit_slot = kEmptySlot;
-  for (unsigned long long probe = 0; probe <= a.index_mask; ++probe) {
+  for (unsigned long long probe = 0; slots_used && probe <= a.index_mask; ++probe) {
     const IndexEntry e = a.index[pos];
     if (e.slot == kEmptySlot) break;
     if (e.key == key && e.len == len) {
@@ -490,7 +492,9 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
       const unsigned long long b2 = group_shfl(acc, gmask, gbase + 2);
       const unsigned long long b3 = group_shfl(acc, gmask, gbase + 3);
       hint = b0 ^ xrotl(b1, 16) ^ xrotl(b2, 32) ^ xrotl(b3, 48);
-      hint_slot = hint_lookup(a.hints, a.index_mask, hint, len, slots_used);
+      // an empty cache has no hints to look up
+      hint_slot = slots_used ? hint_lookup(a.hints, a.index_mask, hint, len, slots_used)
+                             : kEmptySlot;
       cmp = hint_slot != kEmptySlot;
       if (cmp) {
         q = a.arena + (unsigned long long)hint_slot * a.C;
@@ -549,7 +553,7 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   unsigned long long pos = mix64(key) & a.index_mask;
   bool hit = false, cand = false;
   uint32_t hit_slot = kEmptySlot;
-  for (unsigned long long probe = 0; probe <= a.index_mask; ++probe) {
+  for (unsigned long long probe = 0; slots_used && probe <= a.index_mask; ++probe) {
     const IndexEntry e = a.index[pos];
     if (e.slot == kEmptySlot) break;
     if (e.key == key && e.len == len) {
