@@ -34,20 +34,8 @@ namespace {
 #ifndef GLEAM_STAGED_HASH
 #define GLEAM_STAGED_HASH 1
 #endif
-#ifndef GLEAM_PREFETCH_DIST
-#define GLEAM_PREFETCH_DIST 0
-#endif
-#ifndef GLEAM_HASH_MINBLOCKS
-#define GLEAM_HASH_MINBLOCKS 0
-#endif
 constexpr int kHashThreads = GLEAM_HASH_THREADS;
 constexpr int kBatch = GLEAM_HASH_BATCH;  // stripes per thread in flight
-// Bytes ahead of the current stripe that each group asks L2 to fetch (0: off).
-constexpr uint32_t kPrefetchDist = GLEAM_PREFETCH_DIST;
-
-__device__ __forceinline__ void prefetch_l2(const void* p) {
-  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
-}
 
 // 8-byte load of read-only payload bytes, no L1 allocation, L2 fetches 256 B.
 template <bool kAligned>
@@ -82,8 +70,6 @@ __device__ __forceinline__ unsigned long long lane_stripes(unsigned long long ac
 #pragma unroll
     for (int u = 0; u < kBatch; ++u) x[u] = load_word<kAligned>(p + (uint64_t)u * 32);
     for (; s + 2 * kBatch <= ns; s += kBatch) {
-      if (kPrefetchDist && (uint64_t)(s + kBatch) * 32 + kPrefetchDist < (uint64_t)ns * 32)
-        prefetch_l2(p + (uint64_t)s * 32 + kPrefetchDist);
       unsigned long long y[kBatch];
 #pragma unroll
       for (int u = 0; u < kBatch; ++u)
@@ -122,10 +108,6 @@ __device__ __forceinline__ unsigned long long lane_stripes_cmp(
   while (s < s1) {
     const uint32_t sn = s + m;
     const uint32_t mn = sn < s1 ? min((uint32_t)B, s1 - sn) : 0u;
-    if (kPrefetchDist && (uint64_t)sn * 32 + kPrefetchDist < (uint64_t)s1 * 32) {
-      prefetch_l2(p + (uint64_t)s * 32 + kPrefetchDist);
-      if (cmp) prefetch_l2(q + (uint64_t)s * 32 + kPrefetchDist);
-    }
     unsigned long long xn[B], yn[B];
 #pragma unroll
     for (int u = 0; u < B; ++u) {
@@ -203,14 +185,9 @@ __device__ __forceinline__ bool group_equal(const uint8_t* p, const uint8_t* q, 
   return diff == 0;
 }
 
-#if GLEAM_HASH_MINBLOCKS > 1
-#define GLEAM_HASH_BOUNDS __launch_bounds__(kHashThreads, GLEAM_HASH_MINBLOCKS)
-#else
-#define GLEAM_HASH_BOUNDS __launch_bounds__(kHashThreads)
-#endif
 
 template <bool kAligned, bool kProbe>
-__global__ void GLEAM_HASH_BOUNDS k_hash_probe(HashArgs a) {
+__global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
   const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
   __shared__ unsigned long long s_scratch[33];
   const uint32_t pid_b =
