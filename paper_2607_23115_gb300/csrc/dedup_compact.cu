@@ -659,6 +659,10 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
         } else if (m > g) {  // the group minimum can only be below g: table damaged
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
           ch.res[g] = kResLeader | round;
+        } else if (ch.hint[g] != ch.hint[m]) {
+          // different first 512 bytes (the prefix hints differ), so different
+          // chunks: no byte compare, the chunk waits for a later round
+          atomicAdd(&a.ctl->unres[round % 3], 1u);
         } else {
           need = true;
         }
