@@ -381,7 +381,7 @@ def measured_peaks():
 def kernel_source_digest():
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2607_23115_gb300", "csrc")
-    for f in ("hash_probe.cu", "xxh64_device.cuh", "gleam_internal.cuh"):
+    for f in ("hash_probe.cu", "staged_hash.cuh", "xxh64_device.cuh", "gleam_internal.cuh"):
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]

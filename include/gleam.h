@@ -314,6 +314,10 @@ int gleam_cache_debug_insert(gleam_cache_t* cache, uint64_t key, const void* d_b
 /* what = GLEAM_DEBUG_DROP_ENTRY: removes the index entry of slot `value`
  * (damages the cache on purpose, to test GLEAM_DEBUG_CHECKS).  Synchronous. */
 #define GLEAM_DEBUG_DROP_ENTRY 4
+/* what = GLEAM_DEBUG_SMALL_CALLS: the largest call, in chunks, that may run as
+ * one single-block kernel instead of three launches (default 64; 0 turns that
+ * path off).  Only the speed changes: every output is the same either way. */
+#define GLEAM_DEBUG_SMALL_CALLS 5
 int gleam_cache_debug_set(gleam_cache_t* cache, int what, int64_t value);
 
 /* Device-side copy of the index, slot count and counters (and, for a
@@ -329,7 +333,9 @@ void gleam_snapshot_destroy(gleam_snapshot_t* snap);
 /* Kernel timing for benchmarks.  While enabled, every dedup call records CUDA
  * events on its own stream around its two phases: phase 0 is the kernel that
  * fingerprints, probes and verifies; phase 1 is the two kernels that resolve
- * duplicates and rank the misses, then compact, pack and insert.
+ * duplicates and rank the misses, then compact, pack and insert; a small
+ * call that runs as one single-block kernel (GLEAM_DEBUG_SMALL_CALLS) counts
+ * all of its time in phase 0.
  * gleam_cache_profile_read waits for the recorded calls, writes the summed
  * device time (ms) and count of calls of phase k to h_ms[k] and
  * h_launches[k] for k < nkernels (host arrays), and starts a new tally. */

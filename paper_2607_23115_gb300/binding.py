@@ -30,6 +30,7 @@ GLEAM_DEBUG_WAIT_LIMIT_NS = 1
 GLEAM_DEBUG_SKIP_ARRIVE = 2
 GLEAM_DEBUG_CLOCK = 3
 GLEAM_DEBUG_DROP_ENTRY = 4
+GLEAM_DEBUG_SMALL_CALLS = 5
 
 # Every symbol include/gleam.h declares (checked by the ABI test).
 EXPORTS = (

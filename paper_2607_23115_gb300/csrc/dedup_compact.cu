@@ -32,7 +32,13 @@
 // packed output and its arena slot and inserts it into the index; its last
 // block publishes the counters and results and leaves the per-call state
 // zeroed for the next call.
+//
+// A call with few chunks runs instead as one single-block kernel,
+// k_small_call: the staged hash, then k_dedup's and k_pack's steps with a
+// grid of one block (every grid barrier a block barrier), so that the call
+// costs one launch and no kernel boundary.
 #include "gleam_internal.cuh"
+#include "staged_hash.cuh"
 
 namespace gleam {
 namespace {
@@ -402,12 +408,13 @@ __device__ __forceinline__ uint32_t block_rank(bool f, uint32_t* cnt, uint32_t* 
 }
 
 // Selects and removes the K victims; false if a grid barrier failed.
-__device__ bool lru_evict(const DedupArgs& a, unsigned long long slots0, unsigned long long K,
+__device__ bool lru_evict(const DedupArgs& a, uint32_t G, uint32_t bid,
+                          unsigned long long slots0, unsigned long long K,
                           unsigned long long* sred, uint32_t* cnt, uint32_t* off,
                           unsigned long long* red64) {
   static_assert(kLruBins == kThreads * kThreads, "one part of kThreads bins per thread");
-  const uint32_t G = gridDim.x, lane = threadIdx.x & 31;
-  const unsigned long long tid = (unsigned long long)blockIdx.x * kThreads + threadIdx.x;
+  const uint32_t lane = threadIdx.x & 31;
+  const unsigned long long tid = (unsigned long long)bid * kThreads + threadIdx.x;
   const unsigned long long nth = (unsigned long long)G * kThreads;
   const uint32_t now = a.epoch;
 
@@ -427,7 +434,7 @@ __device__ bool lru_evict(const DedupArgs& a, unsigned long long slots0, unsigne
         atomicAdd(&a.bins[key], (uint32_t)__popc(peers));
     }
     if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
-    if (blockIdx.x == 0) {
+    if (bid == 0) {
       // the bin holding the K-th candidate: partial sums of 256 bins per
       // thread (16-byte loads), the part holding it, then that part's bins
       constexpr uint32_t kPer = kLruBins / kThreads;
@@ -481,7 +488,7 @@ __device__ bool lru_evict(const DedupArgs& a, unsigned long long slots0, unsigne
 
   // per contiguous slot range: candidates older than the cut-off, and at it
   const unsigned long long per = ((slots0 + G - 1) / G + 31) & ~31ull;
-  const unsigned long long lo = min(slots0, blockIdx.x * per);
+  const unsigned long long lo = min(slots0, bid * per);
   const unsigned long long hi = min(slots0, lo + per);
   {
     uint32_t nlt = 0, ntie = 0;
@@ -495,14 +502,14 @@ __device__ bool lru_evict(const DedupArgs& a, unsigned long long slots0, unsigne
     const unsigned long long t_lt = block_sum<unsigned long long>(nlt, red64);
     const unsigned long long t_tie = block_sum<unsigned long long>(ntie, red64);
     if (threadIdx.x == 0) {
-      a.bcount[blockIdx.x] = (uint32_t)t_tie;
-      a.bcount[G + blockIdx.x] = (uint32_t)t_lt;
+      a.bcount[bid] = (uint32_t)t_tie;
+      a.bcount[G + bid] = (uint32_t)t_lt;
     }
   }
   if (!grid_barrier(a.ctl, G, a.wait_ns, false)) return false;
   {
     unsigned long long tie_before = 0, lt_before = 0;
-    for (uint32_t j = threadIdx.x; j < blockIdx.x; j += kThreads) {
+    for (uint32_t j = threadIdx.x; j < bid; j += kThreads) {
       tie_before += __ldcg(&a.bcount[j]);
       lt_before += __ldcg(&a.bcount[G + j]);
     }
@@ -564,7 +571,9 @@ __device__ __forceinline__ void post_minimum(const DedupArgs& a, uint32_t e, uin
     atomicMax(&a.tbl[e].minv, m);
 }
 
-__global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
+// The first-occurrence resolution and miss ranks of a call, run by block
+// `bid` of a grid of G co-resident blocks.
+__device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uint32_t bid) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ uint32_t warp_cnt[kWarps];
   __shared__ uint32_t warp_off[kWarps];
@@ -573,12 +582,11 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
   __shared__ unsigned long long s_slots0;
   __shared__ unsigned long long sred[kThreads];
 
-  const uint32_t G = gridDim.x;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const uint32_t tid = blockIdx.x * kThreads + threadIdx.x;
+  const uint32_t tid = bid * kThreads + threadIdx.x;
   const uint32_t nth = G * kThreads;
   const uint32_t N = (uint32_t)a.Ntot;
-  const bool skip = (int)blockIdx.x == a.skip_block;
+  const bool skip = (int)bid == a.skip_block;
   const ChunkArrays& ch = a.ch;
 
   if (threadIdx.x == 0) s_slots0 = *(volatile const unsigned long long*)&a.dstats[ST_SLOTS_USED];
@@ -705,7 +713,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
 
   // ---- D1: misses per contiguous block range --------------------------------
   const uint64_t per = (((uint64_t)N + G - 1) / G + 31) & ~31ull;
-  const uint32_t lo = (uint32_t)min((uint64_t)N, blockIdx.x * per);
+  const uint32_t lo = (uint32_t)min((uint64_t)N, bid * per);
   const uint32_t hi = (uint32_t)min((uint64_t)N, lo + per);
   unsigned long long before = 0, total = 0, sbefore = 0, stotal = 0, evict = 0;
   if (ok) {
@@ -727,8 +735,8 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     const unsigned long long c = block_sum<unsigned long long>(cnt, red64);
     const unsigned long long sc = block_sum<unsigned long long>(scnt, red64);
     if (threadIdx.x == 0) {
-      a.bcount[blockIdx.x] = (uint32_t)c;
-      a.bcount[G + blockIdx.x] = (uint32_t)sc;
+      a.bcount[bid] = (uint32_t)c;
+      a.bcount[G + bid] = (uint32_t)sc;
     }
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   }
@@ -739,7 +747,7 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
       const uint32_t sv = ldcg_u32(&a.bcount[G + j]);
       total += v;
       stotal += sv;
-      if (j < blockIdx.x) {
+      if (j < bid) {
         before += v;
         sbefore += sv;
       }
@@ -799,9 +807,9 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
     }
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   }
-  if (ok && evict) ok = lru_evict(a, slots0, evict, sred, warp_cnt, warp_off, red64);
+  if (ok && evict) ok = lru_evict(a, G, bid, slots0, evict, sred, warp_cnt, warp_off, red64);
   // totals for k_pack (the capacity check above left them unpublished on error)
-  if (ok && blockIdx.x == 0 && threadIdx.x == 0) {
+  if (ok && bid == 0 && threadIdx.x == 0) {
     a.ctl->acc_misses = total;
     a.ctl->acc_stored = stotal;
     a.ctl->evict_k = evict;
@@ -813,11 +821,11 @@ __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
 // rank copied by whole warps to the packed output and its arena slot and
 // inserted into the index; the last block publishes the counters and results
 // and leaves the per-call state zeroed.  Nothing is written after an error.
-__global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
+__device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uint32_t bid,
+                                             uint8_t* pack_smem) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ unsigned long long s_slots0, s_total, s_evict;
   __shared__ int s_err;
-  const uint32_t G = gridDim.x;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const uint32_t N = (uint32_t)a.Ntot;
   const ChunkArrays& ch = a.ch;
@@ -833,7 +841,6 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
   const unsigned long long evict = s_evict;
   const bool ok = s_err == 0;
 #if GLEAM_PACK_BULK
-  extern __shared__ __align__(128) uint8_t pack_smem[];
   const uint32_t wbase = (uint32_t)__cvta_generic_to_shared(pack_smem) + w * kPackWarpBytes;
   const uint32_t bufs = wbase, bars = wbase + kPackBufs * kPackPiece;
   PackMeta* meta = reinterpret_cast<PackMeta*>(pack_smem + w * kPackWarpBytes +
@@ -854,7 +861,7 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
 
   // ---- after an error: give the hit slots their last use back (LRU) ---------
   if (!ok && a.lru) {
-    for (unsigned long long g = (unsigned long long)blockIdx.x * kThreads + threadIdx.x; g < N;
+    for (unsigned long long g = (unsigned long long)bid * kThreads + threadIdx.x; g < N;
          g += (unsigned long long)G * kThreads)
       if (ch.status[g] == kHit0 && ch.old[g] != a.epoch) a.last_use[ch.ent[g]] = ch.old[g];
   }
@@ -862,7 +869,7 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
   // ---- hit masks, miss indices, chunk slots, counters ------------------------
   if (ok) {
     unsigned long long n_hc = 0, n_hi = 0, n_rej = 0, n_bytes = 0, n_sbytes = 0;
-    for (unsigned long long t = (unsigned long long)blockIdx.x * kThreads; t < N;
+    for (unsigned long long t = (unsigned long long)bid * kThreads; t < N;
          t += (unsigned long long)G * kThreads) {
       const uint32_t g = (uint32_t)(t + threadIdx.x);
       const bool valid = t + threadIdx.x < N;
@@ -923,7 +930,7 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
     // 32 chunks one after the other to the packed output and their arena
     // slots, then each lane inserts its own chunk (32 independent probes).
     const unsigned long long nw = (unsigned long long)G * kWarps;
-    const unsigned long long gw = (unsigned long long)blockIdx.x * kWarps + w;
+    const unsigned long long gw = (unsigned long long)bid * kWarps + w;
     const unsigned long long lo = total * gw / nw, hi = total * (gw + 1) / nw;
     for (unsigned long long base = lo; base < hi; base += 32) {
       const unsigned long long r = base + lane;
@@ -1085,6 +1092,36 @@ __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
   __threadfence();
 }
 
+__global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
+  resolve_rank(a, gridDim.x, blockIdx.x);
+}
+
+__global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
+  extern __shared__ __align__(128) uint8_t pack_smem[];
+  pack_publish(a, gridDim.x, blockIdx.x, pack_smem);
+}
+
+// A whole small call in one block: the staged hash of its chunks (kThreads / 4
+// at a time), then the resolution and ranks, then the copies, inserts and
+// publish, separated by block barriers instead of kernel boundaries and grid
+// barriers.  The pack reuses the shared memory of the hash stages.
+constexpr uint32_t kSmallGroups = kThreads / 4;
+constexpr uint32_t kSmallHashSmem = kSmallGroups * (uint32_t)kGroupBytes;
+constexpr uint32_t kSmallSmem = kSmallHashSmem > kPackSmem ? kSmallHashSmem : kPackSmem;
+
+__global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a) {
+  extern __shared__ __align__(128) uint8_t small_smem[];
+  const unsigned long long nvb = (h.Ntot * 4 + kThreads - 1) / kThreads;
+  for (unsigned long long vb = 0; vb < nvb; ++vb) {
+    __syncthreads();  // the previous range's groups are done with the shared memory
+    staged_range<true>(h, vb, small_smem);
+  }
+  __syncthreads();  // every chunk's probe outcome written (and its stage copies landed)
+  resolve_rank(a, 1, 0);
+  __syncthreads();
+  pack_publish(a, 1, 0, small_smem);
+}
+
 // One warp per record: does the block still hold the recorded chunk's bytes?
 __global__ void __launch_bounds__(kThreads) k_block_check(BlockCheckArgs a) {
   const uint32_t lane = threadIdx.x & 31;
@@ -1215,6 +1252,15 @@ cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream
     cudaFuncSetAttribute((const void*)k_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          kPackSmem);
   k_pack<<<pack_grid, kThreads, kPackSmem, s>>>(a);
+  return cudaGetLastError();
+}
+
+uint32_t small_call_groups() { return kSmallGroups; }
+
+cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_t s) {
+  cudaFuncSetAttribute((const void*)k_small_call, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       kSmallSmem);
+  k_small_call<<<1, kThreads, kSmallSmem, s>>>(h, a);
   return cudaGetLastError();
 }
 

@@ -62,6 +62,12 @@ struct gleam_cache {
   int pack_max_blocks = 0;  // pack kernel: all co-resident blocks
   cudaEvent_t done = nullptr;
 
+  // single-block calls: the largest call (in chunks) that runs as one kernel,
+  // and an upper bound of the slots in use (no device read needed), which
+  // tells when a call of an LRU cache cannot need an eviction
+  uint64_t small_max_chunks = 0;
+  uint64_t slots_bound = 0;
+
   unsigned long long wait_ns = 4000000000ULL;
   int skip_block = -1;
 
@@ -83,6 +89,7 @@ struct gleam_snapshot {
   uint32_t* slot_len = nullptr;  // LRU caches: slot lengths and last uses too
   uint32_t* last_use = nullptr;
   uint64_t nslots = 0;
+  uint64_t slots_bound = 0;  // the cache's host-side bound of its used slots
 };
 
 namespace {
@@ -416,6 +423,26 @@ void set_lru(gleam_cache* c, DedupArgs* d, uint64_t nchunks) {
   d->bins = c->bins;
 }
 
+// A call of at most this many payload bytes may run as the single-block kernel.
+constexpr uint64_t kSmallMaxBytes = 256ull << 10;
+
+// Whether a call runs as one single-block kernel instead of three launches:
+// few chunks and bytes (one block then hashes them about as fast as a grid
+// does, and the two kernel boundaries were most of the call's time), payloads
+// the staged hash can read, 64-bit or KEY16 keys, and no possible eviction
+// (an evicting call scans the whole index, which wants the full grid).
+bool small_call(const gleam_cache* c, bool aligned, uint64_t Ntot, uint64_t nbytes,
+                int skip_block) {
+  return Ntot > 0 && Ntot <= c->small_max_chunks && nbytes <= kSmallMaxBytes && aligned &&
+         (c->C % 32 == 0 || Ntot == 1) && !(c->flags & GLEAM_PAPER_IDS) && skip_block < 0 &&
+         (!(c->flags & GLEAM_EVICT_LRU) || c->slots_bound + Ntot <= c->nslots);
+}
+
+// After a call is enqueued: it stores at most Ntot new slots.
+void note_call(gleam_cache* c, uint64_t Ntot) {
+  c->slots_bound = std::min<uint64_t>(c->nslots, c->slots_bound + Ntot);
+}
+
 // GLEAM_DEBUG_CHECKS: the index consistency check after a call.
 int enqueue_index_check(gleam_cache* c, const DedupArgs& d, cudaStream_t s) {
   if (!(c->flags & GLEAM_DEBUG_CHECKS)) return GLEAM_OK;
@@ -495,20 +522,6 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   h.ch = c->ch;
   h.ctl = c->ctl;
 
-  cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
-  if (c->profile) {
-    while (c->ev_pool.size() < c->ev_used + 3) {
-      cudaEvent_t e;
-      if ((rc = cuda_err(cudaEventCreate(&e))) != GLEAM_OK) return rc;
-      c->ev_pool.push_back(e);
-    }
-    for (int k = 0; k < 3; ++k) ev[k] = c->ev_pool[c->ev_used + k];
-    c->ev_used += 3;
-    cudaEventRecord(ev[0], s);
-  }
-  if ((rc = cuda_err(launch_hash(h, aligned, s))) != GLEAM_OK) return rc;
-  if (ev[1]) cudaEventRecord(ev[1], s);
-
   DedupArgs d{};
   d.table = c->d_table;
   d.one = one;
@@ -541,11 +554,32 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     grid = std::max(grid, std::min(2, c->coop_max_blocks));  // someone must be left waiting
     if (d.skip_block >= grid) d.skip_block = grid - 1;
   }
-  if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, Ntot, nbytes), s))) != GLEAM_OK) {
-    cudaMemsetAsync(c->ctl, 0, sizeof(DevCtl), s);  // the hash kernel may have flagged it
-    return rc;
+  const bool fused = small_call(c, aligned, Ntot, nbytes, d.skip_block);
+
+  cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
+  if (c->profile) {
+    while (c->ev_pool.size() < c->ev_used + 3) {
+      cudaEvent_t e;
+      if ((rc = cuda_err(cudaEventCreate(&e))) != GLEAM_OK) return rc;
+      c->ev_pool.push_back(e);
+    }
+    for (int k = 0; k < 3; ++k) ev[k] = c->ev_pool[c->ev_used + k];
+    c->ev_used += 3;
+    cudaEventRecord(ev[0], s);
+  }
+  if (fused) {  // one kernel: all of its time is phase 0
+    if ((rc = cuda_err(launch_small_call(h, d, s))) != GLEAM_OK) return rc;
+    if (ev[1]) cudaEventRecord(ev[1], s);
+  } else {
+    if ((rc = cuda_err(launch_hash(h, aligned, s))) != GLEAM_OK) return rc;
+    if (ev[1]) cudaEventRecord(ev[1], s);
+    if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, Ntot, nbytes), s))) != GLEAM_OK) {
+      cudaMemsetAsync(c->ctl, 0, sizeof(DevCtl), s);  // the hash kernel may have flagged it
+      return rc;
+    }
   }
   if (ev[2]) cudaEventRecord(ev[2], s);
+  note_call(c, Ntot);
   if ((rc = enqueue_index_check(c, d, s)) != GLEAM_OK) return rc;
   return cuda_err(cudaEventRecord(c->done, s));
 }
@@ -635,6 +669,7 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     const int per_sm = dedup_blocks_per_sm();
     c->coop_max_blocks = sms * per_sm;
     c->pack_max_blocks = sms * pack_blocks_per_sm();
+    c->small_max_chunks = small_call_groups();
     if (c->coop_max_blocks <= 0 || c->pack_max_blocks <= 0) rc = GLEAM_ERR_CUDA;
   }
   // per-block miss and stored-miss counts, then one word used as the single
@@ -885,6 +920,7 @@ int gleam_cache_debug_insert(gleam_cache_t* c, uint64_t key, const void* d_bytes
                                       c->last_use ? ++c->epoch : 0u, nullptr));
   if (rc == GLEAM_OK) rc = cuda_err(cudaDeviceSynchronize());
   if (rc == GLEAM_OK) rc = cuda_err(cudaEventRecord(c->done, nullptr));
+  if (rc == GLEAM_OK) note_call(c, 1);
   return rc;
 }
 
@@ -915,6 +951,11 @@ int gleam_cache_debug_set(gleam_cache_t* c, int what, int64_t value) {
                                    cudaMemcpyHostToDevice));
       }
     return GLEAM_ERR_INVALID_ARG;
+  }
+  if (what == GLEAM_DEBUG_SMALL_CALLS) {
+    if (value < 0 || value > (int64_t)kMaxChunks) return GLEAM_ERR_INVALID_ARG;
+    c->small_max_chunks = (uint64_t)value;
+    return GLEAM_OK;
   }
   if (what == GLEAM_DEBUG_CLOCK) {
     if (value < 0 || value > 0xFFFFFFFEll) return GLEAM_ERR_INVALID_ARG;
@@ -968,6 +1009,7 @@ int gleam_cache_snapshot(gleam_cache_t* c, gleam_snapshot_t** out) {
   s->device = c->device;
   s->owner = c;
   s->index_cap = c->index_cap;
+  s->slots_bound = c->slots_bound;
   rc = cuda_err(cudaMalloc(&s->index, c->index_cap * sizeof(IndexEntry)));
   if (rc == GLEAM_OK) rc = cuda_err(cudaMalloc(&s->hints, c->index_cap * sizeof(IndexEntry)));
   if (rc == GLEAM_OK) rc = cuda_err(cudaMalloc(&s->dstats, ST_COUNT * sizeof(unsigned long long)));
@@ -1022,7 +1064,10 @@ int gleam_cache_restore(gleam_cache_t* c, const gleam_snapshot_t* s) {
       rc = cuda_err(cudaMemcpyAsync(c->last_use, s->last_use, s->nslots * sizeof(uint32_t),
                                     cudaMemcpyDeviceToDevice, nullptr));
   }
-  if (rc == GLEAM_OK) rc = cuda_err(cudaEventRecord(c->done, nullptr));
+  if (rc == GLEAM_OK) {
+    c->slots_bound = s->slots_bound;
+    rc = cuda_err(cudaEventRecord(c->done, nullptr));
+  }
   return rc;
 }
 
@@ -1166,7 +1211,6 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   h.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   h.ch = ch;
   h.ctl = ctl;
-  if ((rc = cuda_err(launch_hash(h, aligned, s))) != GLEAM_OK) return rc;
 
   DedupArgs d{};
   d.one = one;
@@ -1193,8 +1237,14 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.plain_copy = chk.saw_managed() ? 1u : 0u;
   set_lru(c, &d, N);
   d.skip_block = -1;
-  const int grid = dedup_grid(c, N, n);
-  if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, N, n), s))) != GLEAM_OK) return rc;
+  if (small_call(c, aligned, N, n, -1)) {
+    if ((rc = cuda_err(launch_small_call(h, d, s))) != GLEAM_OK) return rc;
+  } else {
+    if ((rc = cuda_err(launch_hash(h, aligned, s))) != GLEAM_OK) return rc;
+    const int grid = dedup_grid(c, N, n);
+    if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, N, n), s))) != GLEAM_OK) return rc;
+  }
+  note_call(c, N);
   if ((rc = enqueue_index_check(c, d, s)) != GLEAM_OK) return rc;
   return cuda_err(cudaEventRecord(c->done, s));
 }

@@ -198,6 +198,12 @@ cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s);
 // The cooperative resolve/rank kernel on `grid` blocks, then the pack kernel
 // (masks, indices, copies, inserts, publish) on `pack_grid` blocks.
 cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s);
+// A whole call (hash, resolve and rank, pack) as one single-block kernel, for
+// calls with few chunks whose payloads suit the staged hash (16-byte aligned)
+// outside GLEAM_PAPER_IDS mode; the block hashes small_call_groups() chunks at
+// a time.
+cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_t s);
+uint32_t small_call_groups();
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
                                 unsigned long long* dstats, unsigned long long key,
                                 uint32_t slot, uint32_t len, DevCtl* ctl, uint32_t* last_use,

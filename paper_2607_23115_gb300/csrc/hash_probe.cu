@@ -21,17 +21,11 @@
 
 #include "gleam_internal.cuh"
 #include "xxh64_device.cuh"
-
-// The fingerprint-only instantiations (kProbe = false) see slots_used == 0 as a
-// constant in probe code they never reach.
-#pragma nv_diag_suppress 186
+#include "staged_hash.cuh"
 
 namespace gleam {
 namespace {
 
-#ifndef GLEAM_HASH_BATCH
-#define GLEAM_HASH_BATCH 8
-#endif
 #ifndef GLEAM_HASH_THREADS
 #define GLEAM_HASH_THREADS 256
 #endif
@@ -39,30 +33,7 @@ namespace {
 #define GLEAM_STAGED_HASH 1
 #endif
 constexpr int kHashThreads = GLEAM_HASH_THREADS;
-constexpr int kBatch = GLEAM_HASH_BATCH;  // stripes per thread in flight
 
-// 8-byte load of read-only payload bytes, no L1 allocation, L2 fetches 256 B.
-template <bool kAligned>
-__device__ __forceinline__ unsigned long long load_word(const uint8_t* p) {
-  if (kAligned) {
-    unsigned long long v;
-    asm("ld.global.nc.L1::no_allocate.L2::256B.u64 %0, [%1];" : "=l"(v) : "l"(p));
-    return v;
-  } else {
-    return load_le64_bytes(p);
-  }
-}
-
-__device__ __forceinline__ unsigned long long load_arena_word(const uint8_t* p) {
-  unsigned long long v;
-  asm("ld.global.nc.L1::no_allocate.L2::256B.u64 %0, [%1];" : "=l"(v) : "l"(p));
-  return v;
-}
-
-__device__ __forceinline__ unsigned long long group_shfl(unsigned long long v, unsigned gmask,
-                                                         int src) {
-  return __shfl_sync(gmask, v, src);
-}
 
 // Lane accumulator over `ns` stripes starting at p (p already offset by 8*lane).
 template <bool kAligned>
@@ -147,47 +118,6 @@ __device__ __forceinline__ unsigned long long lane_stripes_cmp(
   return acc;
 }
 
-// Slot of a cached chunk of length len whose prefix hint is h, or kEmptySlot.
-__device__ __forceinline__ uint32_t hint_lookup(const IndexEntry* t, unsigned long long mask,
-                                                unsigned long long h, uint32_t len,
-                                                unsigned long long slots_used) {
-  unsigned long long pos = mix64(h) & mask;
-  for (unsigned long long probe = 0; probe <= mask; ++probe) {
-    const IndexEntry e = t[pos];
-    if (e.slot == kEmptySlot) return kEmptySlot;
-    if (e.key == h && e.len == len && e.slot < slots_used) return e.slot;
-    pos = (pos + 1) & mask;
-  }
-  return kEmptySlot;
-}
-
-// Byte equality of payload chunk p and cached chunk q over len bytes, by the
-// 4-thread group; leaves early once any word differs.
-template <bool kAligned>
-__device__ __forceinline__ bool group_equal(const uint8_t* p, const uint8_t* q, uint32_t len,
-                                            uint32_t lane, unsigned gmask) {
-  const uint32_t ns = len >> 5;
-  unsigned long long diff = 0;
-  for (uint32_t s = 0; s < ns; s += kBatch) {
-    const uint32_t m = min((uint32_t)kBatch, ns - s);
-#pragma unroll
-    for (int u = 0; u < kBatch; ++u) {
-      if ((uint32_t)u < m) {
-        const uint64_t off = (uint64_t)(s + u) * 32 + 8 * lane;
-        diff |= load_word<kAligned>(p + off) ^ load_arena_word(q + off);
-      }
-    }
-    diff |= __shfl_xor_sync(gmask, diff, 1);
-    diff |= __shfl_xor_sync(gmask, diff, 2);
-    if (diff) return false;
-  }
-  if (lane == 0) {
-    for (uint32_t k = ns * 32; k < len; ++k) diff |= (unsigned long long)(p[k] ^ q[k]);
-  }
-  diff |= __shfl_xor_sync(gmask, diff, 1);
-  diff |= __shfl_xor_sync(gmask, diff, 2);
-  return diff == 0;
-}
 
 
 template <bool kAligned, bool kProbe>
@@ -327,244 +257,6 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
   }
 }
 
-// ---------------------------------------------------------------------------
-// Staged variant for 16-byte-aligned payloads.  Each 4-thread group streams
-// its chunk through shared memory in kStage-byte stages with asynchronous
-// 16-byte global->shared copies (kDepth stages in flight, no registers held),
-// and the cached copy named by the prefix hint streams alongside into a
-// second buffer.  The lanes then hash and compare their words from shared
-// memory.  Stage 0 is exactly the prefix used for the hint.
-//
-// Two stages in flight and blocks of one warp (8 groups, 16.6 KB of shared
-// memory): about 100 groups share an SM, and that many independent chunks
-// hide each chunk's dependent lookups (payload, prefix hint, index probe)
-// better than deeper pipelines with fewer groups (measured: 3 stages and
-// 64 groups per SM took 5.05 ms on the Llama upload, this takes 4.64 ms).
-// ---------------------------------------------------------------------------
-#ifndef GLEAM_STAGE_DEPTH
-#define GLEAM_STAGE_DEPTH 2
-#endif
-#ifndef GLEAM_STAGED_THREADS
-#define GLEAM_STAGED_THREADS 32
-#endif
-constexpr int kStage = 512;                                 // bytes per stage
-constexpr int kDepth = GLEAM_STAGE_DEPTH;                   // stages in flight
-constexpr int kGroupBytes = kDepth * 2 * kStage + 32;       // +32: bank skew
-constexpr int kStagedThreads = GLEAM_STAGED_THREADS;
-constexpr int kStagedSmem = (kStagedThreads / 4) * kGroupBytes;
-static_assert(kStage == (int)kPrefixBytes, "stage 0 must be the hinted prefix");
-static_assert(kStagedSmem >= 33 * 8, "the payload search borrows 33 words of the stage buffers");
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global.L2::256B [%0], [%1], 16;" ::"r"(dst), "l"(src)
-               : "memory");
-}
-__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-// This lane's share (4 lanes x 8 x 16 bytes) of one stage of `src` into `dst`;
-// `bytes` (multiple of 32, <= kStage) of the stage exist.
-__device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uint32_t bytes,
-                                           uint32_t lane) {
-#pragma unroll
-  for (int j = 0; j < kStage / 64; ++j) {
-    const uint32_t off = (uint32_t)j * 64 + lane * 16;
-    if (off < bytes) cp_async16(dst + off, src + off);
-  }
-}
-
-// The chunks of block-sized range vb (kStagedThreads / 4 consecutive chunks).
-template <bool kProbe>
-__device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long long vb,
-                                             uint8_t* smem) {
-  const unsigned long long g = (vb * blockDim.x + threadIdx.x) >> 2;
-  // the payload search borrows the start of the stage buffers (no static
-  // shared memory: any would cost this kernel a fifth of its bandwidth)
-  const uint32_t pid_b =
-      a.count > 1 ? block_find_payload(a.table, a.count, (vb * blockDim.x) >> 2, g,
-                                       reinterpret_cast<unsigned long long*>(smem))
-                  : 0u;
-  if (g >= a.Ntot) return;  // whole groups leave together
-  const uint32_t lane = threadIdx.x & 3;
-  const int gbase = threadIdx.x & 28;
-  const unsigned gmask = 0xFu << gbase;
-  uint8_t* region = smem + (threadIdx.x >> 2) * kGroupBytes;
-  const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(region);
-  // stage buffer t % kDepth: payload at [0, kStage), cached copy at [kStage, 2 kStage)
-  auto pay_s = [&](uint32_t t) { return sbase + (t % kDepth) * 2 * kStage; };
-  auto pay_p = [&](uint32_t t) { return region + (t % kDepth) * 2 * kStage; };
-
-  uint32_t pid = 0;
-  const uint8_t* buf;
-  unsigned long long n, base;
-  if (a.count > 1) {
-    pid = pid_b;
-    buf = a.table[pid].buf;
-    n = a.table[pid].n;
-    base = a.table[pid].chunk_base;
-  } else {
-    buf = a.one.buf;
-    n = a.one.n;
-    base = a.one.chunk_base;
-  }
-  const unsigned long long start = (g - base) * a.C;
-  const uint32_t len = (uint32_t)min(a.C, n - start);
-  const uint8_t* p = buf + start;
-  const uint32_t ns = len >> 5;
-  const uint32_t full = ns * 32;                       // bytes in whole stripes
-  const uint32_t nst = (full + kStage - 1) / kStage;   // stages
-  auto sbytes = [&](uint32_t t) { return min((uint32_t)kStage, full - t * kStage); };
-
-  const bool speculate = kProbe && len >= kPrefixBytes;
-  const unsigned long long slots_used = kProbe ? a.dstats[ST_SLOTS_USED] : 0ULL;
-  unsigned long long hint = 0, diff = 0;
-  uint32_t hint_slot = kEmptySlot;
-  const uint8_t* q = nullptr;
-  bool cmp = false;
-
-  unsigned long long acc = xlane_start(lane);
-  // prologue: payload stages 0 .. kDepth-2
-#pragma unroll
-  for (int t = 0; t < kDepth - 1; ++t) {
-    if ((uint32_t)t < nst) stage_copy(pay_s(t), p + t * kStage, sbytes(t), lane);
-    cp_commit();
-  }
-  for (uint32_t t = 0; t < nst; ++t) {
-    // issue stage t + kDepth - 1 into the buffer consumed at t - 1
-    const uint32_t tn = t + kDepth - 1;
-    if (tn < nst) {
-      stage_copy(pay_s(tn), p + (unsigned long long)tn * kStage, sbytes(tn), lane);
-      if (cmp) stage_copy(pay_s(tn) + kStage, q + (unsigned long long)tn * kStage, sbytes(tn), lane);
-    }
-    cp_commit();
-    // groups committed so far, oldest first: prologue stages, then one per
-    // iteration, plus (at t = 0) one holding the cached copy of stages
-    // 1 .. kDepth-1, issued late because the hint is known only then
-    // stage t needs everything up to the late group while t < kDepth - 1
-    // (at most t newer groups may pend), else up to its own group
-    if (t == 0 || t >= (uint32_t)kDepth - 1) cp_wait<kDepth - 1>();
-    else if (t == 1) cp_wait<1>();
-    else if (t == 2) cp_wait<2>();
-    else cp_wait<0>();
-    __syncwarp(gmask);
-    const uint8_t* sp = pay_p(t);
-    const uint32_t sst = sbytes(t) >> 5;
-    unsigned long long d = 0;
-    if (cmp && t > 0) {
-      const uint8_t* sq = sp + kStage;
-#pragma unroll 4
-      for (uint32_t s = 0; s < sst; ++s) {
-        const unsigned long long w = *reinterpret_cast<const unsigned long long*>(sp + s * 32 + lane * 8);
-        const unsigned long long c = *reinterpret_cast<const unsigned long long*>(sq + s * 32 + lane * 8);
-        acc = xstep(acc, w);
-        d |= w ^ c;
-      }
-    } else {
-#pragma unroll 4
-      for (uint32_t s = 0; s < sst; ++s)
-        acc = xstep(acc, *reinterpret_cast<const unsigned long long*>(sp + s * 32 + lane * 8));
-    }
-    if (t == 0 && speculate) {
-      const unsigned long long b0 = group_shfl(acc, gmask, gbase + 0);
-      const unsigned long long b1 = group_shfl(acc, gmask, gbase + 1);
-      const unsigned long long b2 = group_shfl(acc, gmask, gbase + 2);
-      const unsigned long long b3 = group_shfl(acc, gmask, gbase + 3);
-      hint = b0 ^ xrotl(b1, 16) ^ xrotl(b2, 32) ^ xrotl(b3, 48);
-      // an empty cache has no hints to look up
-      hint_slot = slots_used ? hint_lookup(a.hints, a.index_mask, hint, len, slots_used)
-                             : kEmptySlot;
-      cmp = hint_slot != kEmptySlot;
-      if (cmp) {
-        q = a.arena + (unsigned long long)hint_slot * a.C;
-        // the prefix, still in stage buffer 0, against the cached copy's prefix
-#pragma unroll 4
-        for (uint32_t s = 0; s < (uint32_t)kStage / 32; ++s)
-          d |= *reinterpret_cast<const unsigned long long*>(sp + s * 32 + lane * 8) ^
-               load_arena_word(q + s * 32 + lane * 8);
-        // the cached copy of the stages already in flight
-        for (uint32_t tt = 1; tt < (uint32_t)kDepth && tt < nst; ++tt)
-          stage_copy(pay_s(tt) + kStage, q + (unsigned long long)tt * kStage, sbytes(tt), lane);
-      }
-    }
-    if (t == 0) cp_commit();  // the late group (empty without a hint)
-    if (cmp) {
-      diff |= d;
-      unsigned long long gd = diff;
-      gd |= __shfl_xor_sync(gmask, gd, 1);
-      gd |= __shfl_xor_sync(gmask, gd, 2);
-      if (gd) {
-        cmp = false;  // stop streaming the cached copy
-        diff = 1;
-      }
-    }
-    __syncwarp(gmask);  // everyone is done with buffer t before it is refilled
-  }
-  cp_wait<0>();
-
-  unsigned long long h;
-  if (ns) {
-    const unsigned long long a0 = group_shfl(acc, gmask, gbase + 0);
-    const unsigned long long a1 = group_shfl(acc, gmask, gbase + 1);
-    const unsigned long long a2 = group_shfl(acc, gmask, gbase + 2);
-    const unsigned long long a3 = group_shfl(acc, gmask, gbase + 3);
-    h = xconverge(a0, a1, a2, a3);
-  } else {
-    h = kXP5;
-  }
-  h += len;
-  h = xfinish(h, p + full, len & 31);
-
-  if (a.fp_out != nullptr && lane == 0) a.fp_out[g] = h;
-  if (!kProbe) return;
-
-  bool spec_equal = false;
-  if (speculate && hint_slot != kEmptySlot) {
-    unsigned long long dd = diff;
-    if (cmp && lane == 0)
-      for (uint32_t k = full; k < len; ++k) dd |= (unsigned long long)(p[k] ^ q[k]);
-    dd |= __shfl_xor_sync(gmask, dd, 1);
-    dd |= __shfl_xor_sync(gmask, dd, 2);
-    spec_equal = dd == 0;
-  }
-
-  const unsigned long long key = a.key16 ? (h & 0xFFFFULL) : h;
-  unsigned long long pos = mix64(key) & a.index_mask;
-  bool hit = false, cand = false;
-  uint32_t hit_slot = kEmptySlot;
-  for (unsigned long long probe = 0; slots_used && probe <= a.index_mask; ++probe) {
-    const IndexEntry e = a.index[pos];
-    if (e.slot == kEmptySlot) break;
-    if (e.key == key && e.len == len) {
-      cand = true;
-      if (e.slot >= slots_used) {
-        if (lane == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-      } else if (e.slot == hint_slot) {
-        if (spec_equal) {
-          hit = true;
-          hit_slot = e.slot;
-          break;
-        }
-      } else if (group_equal<true>(p, a.arena + (uint64_t)e.slot * a.C, len, lane, gmask)) {
-        hit = true;
-        hit_slot = e.slot;
-        break;
-      }
-    }
-    pos = (pos + 1) & a.index_mask;
-  }
-  if (lane == 0) {
-    a.ch.status[g] = hit ? kHit0 : (cand ? kMissCand : kMissNoCand);
-    a.ch.key[g] = key;
-    a.ch.len[g] = len;
-    a.ch.src[g] = (unsigned long long)p;
-    a.ch.pidx[g] = pid;
-    a.ch.hint[g] = hint;
-    if (hit) a.ch.ent[g] = hit_slot;
-  }
-}
 
 template <bool kProbe>
 __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {

@@ -9,3 +9,26 @@ if ROOT not in sys.path:
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (runs the libgleam.so kernels)")
     config.addinivalue_line("markers", "slow: full-size workload, minutes of work")
+
+
+import pytest  # noqa: E402
+
+
+@pytest.fixture(params=["one-kernel", "three-kernels"])
+def call_path(request, monkeypatch):
+    """Runs a test twice: as the library runs it (a call of at most 64 chunks
+    and 256 KiB as one single-block kernel) and with every call on the
+    three-launch path (hash kernel, cooperative resolve kernel, pack kernel),
+    so that both paths meet every parity case.  Outputs must not differ."""
+    if request.param == "three-kernels":
+        from paper_2607_23115_gb300 import binding as B
+        from paper_2607_23115_gb300.cache import Cache
+
+        init = Cache.__init__
+
+        def init_three_kernels(self, *args, **kwargs):
+            init(self, *args, **kwargs)
+            self.debug_set(B.GLEAM_DEBUG_SMALL_CALLS, 0)
+
+        monkeypatch.setattr(Cache, "__init__", init_three_kernels)
+    return request.param

@@ -10,7 +10,7 @@ from paper_2607_23115_gb300 import workloads as W
 from paper_2607_23115_gb300.cache import Cache, DedupOutputs, result_dict
 from tests._parity import DEV, compare_cache, to_device
 
-pytestmark = pytest.mark.gpu
+pytestmark = [pytest.mark.gpu, pytest.mark.usefixtures("call_path")]
 KiB, MiB = 1024, 1 << 20
 
 

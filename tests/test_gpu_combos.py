@@ -10,7 +10,7 @@ from paper_2607_23115_gb300 import binding as B
 from paper_2607_23115_gb300.cache import Cache, result_dict
 from tests._parity import DEV, compare_cache
 
-pytestmark = pytest.mark.gpu
+pytestmark = [pytest.mark.gpu, pytest.mark.usefixtures("call_path")]
 
 
 def _batch(gc, oc, payloads, host=False, host_out=False):

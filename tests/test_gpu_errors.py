@@ -9,7 +9,7 @@ from paper_2607_23115_gb300 import workloads as W
 from paper_2607_23115_gb300.cache import Cache, DedupOutputs
 from tests._parity import DEV, compare_cache, dedup_both
 
-pytestmark = pytest.mark.gpu
+pytestmark = [pytest.mark.gpu, pytest.mark.usefixtures("call_path")]
 
 
 def test_host_pointers_are_rejected():

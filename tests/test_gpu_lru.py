@@ -11,7 +11,7 @@ from paper_2607_23115_gb300 import binding as B
 from paper_2607_23115_gb300.cache import Cache, DedupOutputs, result_dict
 from tests._parity import DEV, STAT_KEYS, compare_cache, to_device
 
-pytestmark = pytest.mark.gpu
+pytestmark = [pytest.mark.gpu, pytest.mark.usefixtures("call_path")]
 KiB = 1024
 
 

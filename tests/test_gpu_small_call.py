@@ -1,0 +1,80 @@
+"""The single-block kernel that runs a whole small call (hash, resolve and
+rank, pack) against the oracle, at the edges of where the library chooses it
+(64 chunks, 256 KiB) and with the limit raised so that one block hashes
+several ranges of chunks in turn; every case is also run with that path off,
+and both runs must give the same outputs and cache."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_23115_gb300 import binding as B
+from paper_2607_23115_gb300 import workloads as W
+from paper_2607_23115_gb300.cache import Cache
+from tests._parity import compare_cache, dedup_both
+
+pytestmark = pytest.mark.gpu
+KiB, MiB = 1024, 1 << 20
+
+
+def _alphabet_payload(rng, C, nch, alphabet, tail):
+    parts = [alphabet[int(rng.integers(len(alphabet)))] for _ in range(nch)]
+    if tail:
+        parts.append(W.random_bytes(tail, seed=int(rng.integers(1 << 30))))
+    return torch.cat(parts) if parts else torch.zeros(0, dtype=torch.uint8)
+
+
+def _run(limit, C, flags, calls, seed):
+    """The calls on a cache whose single-block limit is `limit` chunks (0: off),
+    each checked against the oracle; returns the cache's export."""
+    gc = Cache(4 * MiB, C, flags)
+    oc = oracle.OracleCache(4 * MiB, C, flags)
+    gc.debug_set(B.GLEAM_DEBUG_SMALL_CALLS, limit)
+    rng = np.random.default_rng(seed)
+    alphabet = [W.random_bytes(C, seed=500 + k) for k in range(24)] + \
+        [torch.zeros(C, dtype=torch.uint8)]
+    with gc:
+        for nch, tail, offset in calls:
+            dedup_both(gc, oc, _alphabet_payload(rng, C, nch, alphabet, tail), offset=offset)
+        compare_cache(gc, oc)
+        keys, lens, count = gc.export()
+        return sorted(zip(keys[:count].tolist(), lens[:count].tolist())), gc.stats()
+
+
+@pytest.mark.parametrize("key16", [False, True])
+def test_edges_of_the_single_block_path(key16):
+    C = 4 * KiB
+    flags = B.GLEAM_KEY16 if key16 else 0
+    # chunks and tail bytes around 64 chunks / 256 KiB; offset 4 is unaligned
+    # (always the three-launch path)
+    calls = [(1, 0, 0), (0, 100, 0), (63, 0, 0), (64, 0, 0), (63, 4095, 0), (64, 1, 0),
+             (65, 0, 0), (2, 0, 4), (40, 17, 0), (64, 0, 0), (16, 0, 0)]
+    on = _run(64, C, flags, calls, seed=1)
+    off = _run(0, C, flags, calls, seed=1)
+    assert on == off
+
+
+@pytest.mark.parametrize("C", [32, 1 * KiB])
+def test_one_block_hashing_several_ranges(C):
+    # with the limit raised, a call of up to 1000 chunks runs in one block that
+    # hashes 64 chunks at a time
+    calls = [(1000, 0, 0), (700, 5, 0), (129, 0, 0), (256, C - 1, 0), (64, 0, 0), (65, 0, 0)]
+    raised = _run(1000, C, 0, calls, seed=C)
+    off = _run(0, C, 0, calls, seed=C)
+    assert raised == off
+
+
+def test_small_calls_near_a_full_lru_cache():
+    # a full LRU cache evicts; the library then runs the three-launch path
+    C = 1 * KiB
+    nslots = 48
+    gc = Cache(nslots * C, C, B.GLEAM_EVICT_LRU)
+    oc = oracle.OracleCache(nslots * C, C, B.GLEAM_EVICT_LRU)
+    rng = np.random.default_rng(7)
+    alphabet = [W.random_bytes(C, seed=900 + k) for k in range(100)]
+    with gc:
+        for call in range(40):
+            nch = int(rng.integers(1, 20))
+            dedup_both(gc, oc, _alphabet_payload(rng, C, nch, alphabet, 0))
+        compare_cache(gc, oc)
+        assert gc.stats()["evictions"] == oc.stats()["evictions"] > 0

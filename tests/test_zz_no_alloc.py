@@ -13,7 +13,7 @@ from paper_2607_23115_gb300 import binding as B
 from paper_2607_23115_gb300 import workloads as W
 from paper_2607_23115_gb300.cache import Cache, DedupOutputs, result_dict
 
-pytestmark = pytest.mark.gpu
+pytestmark = [pytest.mark.gpu, pytest.mark.usefixtures("call_path")]
 DEV = torch.device("cuda:0")
 C = 4096
 
