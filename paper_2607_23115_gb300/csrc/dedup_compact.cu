@@ -581,6 +581,7 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
   __shared__ uint32_t swarp_off[kWarps];
   __shared__ unsigned long long s_slots0;
   __shared__ unsigned long long sred[kThreads];
+  __shared__ int s_err1;
 
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const uint32_t tid = bid * kThreads + threadIdx.x;
@@ -589,9 +590,9 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
   const bool skip = (int)bid == a.skip_block;
   const ChunkArrays& ch = a.ch;
 
-  if (threadIdx.x == 0) s_slots0 = *(volatile const unsigned long long*)&a.dstats[ST_SLOTS_USED];
-  __syncthreads();
-  const unsigned long long slots0 = s_slots0;
+  // thread 0's read of the slot count completes while phase A runs
+  const unsigned long long my_slots0 =
+      threadIdx.x == 0 ? *(volatile const unsigned long long*)&a.dstats[ST_SLOTS_USED] : 0ull;
 
   // ---- A: clear outputs, round-1 claims; LRU: stamp the slots hit ----------
   {
@@ -650,6 +651,7 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
   // ---- B/C: rounds until every chunk is a hit, duplicate or leader ---------
   uint32_t round = 1;
   while (ok) {
+    bool stay = false;  // one of this thread's chunks is left for the next round
     if (tid == 0) atomicExch(&a.ctl->unres[(round + 1) % 3], 0u);
     // W chunks per warp step: 32, or fewer when there are too few chunks to
     // give every warp a step (large chunks), so the compares spread over the grid
@@ -671,6 +673,7 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
           // different first 512 bytes (the prefix hints differ), so different
           // chunks: no byte compare, the chunk waits for a later round
           atomicAdd(&a.ctl->unres[round % 3], 1u);
+          stay = true;
         } else {
           need = true;
         }
@@ -692,13 +695,18 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
             ch.res[gg] = kResDup;
           } else {
             atomicAdd(&a.ctl->unres[round % 3], 1u);
+            stay = true;
           }
         }
       }
     }
-    ok = grid_barrier(a.ctl, G, a.wait_ns, false);
-    if (!ok) break;
-    if (ldcg_u32(&a.ctl->unres[round % 3]) == 0) break;
+    if (G == 1) {  // the block's own count, without the round trip to the counter
+      if (!__syncthreads_or(stay)) break;
+    } else {
+      ok = grid_barrier(a.ctl, G, a.wait_ns, false);
+      if (!ok) break;
+      if (ldcg_u32(&a.ctl->unres[round % 3]) == 0) break;
+    }
     for (uint32_t g = tid; g < N; g += nth)
       if (ldcg_u32(&ch.res[g]) == kResUnresolved) a.tbl[ch.ent[g]].minv = 0;
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
@@ -734,14 +742,22 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
     }
     const unsigned long long c = block_sum<unsigned long long>(cnt, red64);
     const unsigned long long sc = block_sum<unsigned long long>(scnt, red64);
-    if (threadIdx.x == 0) {
-      a.bcount[bid] = (uint32_t)c;
-      a.bcount[G + bid] = (uint32_t)sc;
+    if (G == 1) {
+      total = c;
+      stotal = sc;
+    } else {
+      if (threadIdx.x == 0) {
+        a.bcount[bid] = (uint32_t)c;
+        a.bcount[G + bid] = (uint32_t)sc;
+      }
+      ok = grid_barrier(a.ctl, G, a.wait_ns, false);
     }
-    ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   }
+  if (threadIdx.x == 0) s_slots0 = my_slots0;
+  __syncthreads();
+  const unsigned long long slots0 = s_slots0;
   // ---- D2: exclusive miss rank of every chunk; per-payload start ranks ------
-  if (ok) {
+  if (ok && G > 1) {
     for (uint32_t j = threadIdx.x; j < G; j += kThreads) {
       const uint32_t v = ldcg_u32(&a.bcount[j]);
       const uint32_t sv = ldcg_u32(&a.bcount[G + j]);
@@ -756,6 +772,8 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
     total = block_sum<unsigned long long>(total, red64);
     sbefore = block_sum<unsigned long long>(sbefore, red64);
     stotal = block_sum<unsigned long long>(stotal, red64);
+  }
+  if (ok) {
     if (stotal > a.nslots - slots0) {
       // LRU: evict the missing slots among those this call did not hit
       evict = stotal - (a.nslots - slots0);
@@ -807,6 +825,11 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
     }
     ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   }
+  if (ok && evict && G == 1) {  // its barriers did not read the error word
+    if (threadIdx.x == 0) s_err1 = ld_volatile_s32(&a.ctl->err);
+    __syncthreads();
+    ok = s_err1 == 0;
+  }
   if (ok && evict) ok = lru_evict(a, G, bid, slots0, evict, sred, warp_cnt, warp_off, red64);
   // totals for k_pack (the capacity check above left them unpublished on error)
   if (ok && bid == 0 && threadIdx.x == 0) {
@@ -825,6 +848,8 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
                                              uint8_t* pack_smem) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ unsigned long long s_slots0, s_total, s_evict;
+  // a grid of one block keeps its totals here instead of in the control block
+  __shared__ unsigned long long s_stored, s_vbytes, s_sum[5];
   __shared__ int s_err;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const uint32_t N = (uint32_t)a.Ntot;
@@ -834,6 +859,9 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
     s_err = ld_volatile_s32(&a.ctl->err);
     s_total = __ldcg(&a.ctl->acc_misses);
     s_evict = __ldcg(&a.ctl->evict_k);
+    s_stored = __ldcg(&a.ctl->acc_stored);
+    s_vbytes = __ldcg(&a.ctl->acc_victim_bytes);
+    for (int k = 0; k < 5; ++k) s_sum[k] = 0;
   }
   __syncthreads();
   const unsigned long long slots0 = s_slots0;
@@ -1001,7 +1029,13 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
     n_rej = block_sum<unsigned long long>(n_rej, red64);
     n_bytes = block_sum<unsigned long long>(n_bytes, red64);
     n_sbytes = block_sum<unsigned long long>(n_sbytes, red64);
-    if (threadIdx.x == 0) {
+    if (threadIdx.x == 0 && G == 1) {
+      s_sum[0] = n_hc;
+      s_sum[1] = n_hi;
+      s_sum[2] = n_rej;
+      s_sum[3] = n_bytes;
+      s_sum[4] = n_sbytes;
+    } else if (threadIdx.x == 0) {
       atomicAdd(&a.ctl->acc_hits_cache, n_hc);
       atomicAdd(&a.ctl->acc_hits_intra, n_hi);
       atomicAdd(&a.ctl->acc_rejects, n_rej);
@@ -1014,33 +1048,38 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
   __shared__ int s_last;
   __syncthreads();
   if (threadIdx.x == 0) {
-    __threadfence();
-    s_last = atomicAdd(&a.ctl->done, 1u) == G - 1;
+    if (G == 1) {  // the block barrier already orders the block's own writes
+      s_last = 1;
+    } else {
+      __threadfence();
+      s_last = atomicAdd(&a.ctl->done, 1u) == G - 1;
+    }
   }
   __syncthreads();
   if (!s_last) return;
-  __threadfence();
+  if (G > 1) __threadfence();
   const int err = ld_volatile_s32(&a.ctl->err);
   if (threadIdx.x == 0) {
-    const unsigned long long misses = __ldcg(&a.ctl->acc_misses);
-    const unsigned long long hc = __ldcg(&a.ctl->acc_hits_cache);
-    const unsigned long long hi2 = __ldcg(&a.ctl->acc_hits_intra);
-    const unsigned long long rej = __ldcg(&a.ctl->acc_rejects);
-    const unsigned long long mbytes = __ldcg(&a.ctl->acc_miss_bytes);
-    const unsigned long long stored = __ldcg(&a.ctl->acc_stored);
-    const unsigned long long sbytes = __ldcg(&a.ctl->acc_stored_bytes);
-    const unsigned long long vbytes = __ldcg(&a.ctl->acc_victim_bytes);
-    if (err == 0) {
-      a.dstats[ST_CALLS] += a.ncalls;
-      a.dstats[ST_CHUNKS] += N;
-      a.dstats[ST_HITS_CACHE] += hc;
-      a.dstats[ST_HITS_INTRA] += hi2;
-      a.dstats[ST_MISSES] += misses;
-      a.dstats[ST_INSERTS] += stored;
-      a.dstats[ST_REJECTS] += rej;
+    const bool one = G == 1;
+    const unsigned long long misses = total;
+    const unsigned long long hc = one ? s_sum[0] : __ldcg(&a.ctl->acc_hits_cache);
+    const unsigned long long hi2 = one ? s_sum[1] : __ldcg(&a.ctl->acc_hits_intra);
+    const unsigned long long rej = one ? s_sum[2] : __ldcg(&a.ctl->acc_rejects);
+    const unsigned long long mbytes = one ? s_sum[3] : __ldcg(&a.ctl->acc_miss_bytes);
+    const unsigned long long sbytes = one ? s_sum[4] : __ldcg(&a.ctl->acc_stored_bytes);
+    const unsigned long long stored = s_stored;
+    const unsigned long long vbytes = s_vbytes;
+    if (err == 0) {  // no reads: the counters change by atomic adds
+      atomicAdd(&a.dstats[ST_CALLS], a.ncalls);
+      atomicAdd(&a.dstats[ST_CHUNKS], (unsigned long long)N);
+      atomicAdd(&a.dstats[ST_HITS_CACHE], hc);
+      atomicAdd(&a.dstats[ST_HITS_INTRA], hi2);
+      atomicAdd(&a.dstats[ST_MISSES], misses);
+      atomicAdd(&a.dstats[ST_INSERTS], stored);
+      atomicAdd(&a.dstats[ST_REJECTS], rej);
       a.dstats[ST_SLOTS_USED] = slots0 + stored - evict;
-      a.dstats[ST_BYTES_USED] += sbytes - vbytes;
-      a.dstats[ST_EVICTIONS] += evict;
+      atomicAdd(&a.dstats[ST_BYTES_USED], sbytes - vbytes);
+      atomicAdd(&a.dstats[ST_EVICTIONS], evict);
     }
     gleam_result_t* t = a.total;
     t->status = err;
@@ -1109,8 +1148,22 @@ constexpr uint32_t kSmallGroups = kThreads / 4;
 constexpr uint32_t kSmallHashSmem = kSmallGroups * (uint32_t)kGroupBytes;
 constexpr uint32_t kSmallSmem = kSmallHashSmem > kPackSmem ? kSmallHashSmem : kPackSmem;
 
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
 __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a) {
   extern __shared__ __align__(128) uint8_t small_smem[];
+  // Device-resident payloads (16-byte aligned here) are prefetched into L2 at
+  // once, lane p taking payload p in 16 KiB pieces, so that the hash stages
+  // wait for L2 rather than HBM.
+  constexpr uint32_t kPiece = 16u << 10;
+  if (!a.plain_copy && a.count <= 32 && threadIdx.x < a.count) {
+    const PayloadDesc& P = desc(a, threadIdx.x);
+    const unsigned long long nb = P.n & ~15ull;
+    for (unsigned long long off = 0; off < nb; off += kPiece)
+      prefetch_l2(P.buf + off, (uint32_t)min((unsigned long long)kPiece, nb - off));
+  }
   const unsigned long long nvb = (h.Ntot * 4 + kThreads - 1) / kThreads;
   for (unsigned long long vb = 0; vb < nvb; ++vb) {
     __syncthreads();  // the previous range's groups are done with the shared memory

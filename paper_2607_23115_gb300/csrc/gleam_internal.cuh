@@ -273,16 +273,15 @@ __device__ __forceinline__ int ld_volatile_s32(const int* p) {
 // `wait_ns`: a block that gives up records GLEAM_ERR_TIMEOUT and every block
 // then leaves through its epilogue.  `skip` makes the calling block leave
 // without arriving (test hook for the bounded wait).  Returns true if the
-// whole grid arrived and no error is recorded.
+// whole grid arrived and no error is recorded.  A grid of one block has no
+// one to wait for: the block barrier orders its memory accesses, and it
+// returns !skip without reading the error word (a caller about to make a
+// change that an error must prevent reads it itself).
 __device__ __forceinline__ bool grid_barrier(DevCtl* ctl, unsigned int nblocks,
                                              unsigned long long wait_ns, bool skip) {
   __shared__ int s_ok;  // the block's verdict, so that every thread agrees
   __syncthreads();
-  if (nblocks == 1) {  // one block: the block barrier already orders its memory accesses
-    if (threadIdx.x == 0) s_ok = (!skip && ld_volatile_s32(&ctl->err) == 0) ? 1 : 0;
-    __syncthreads();
-    return s_ok != 0;
-  }
+  if (nblocks == 1) return !skip;
   if (threadIdx.x == 0 && !skip) {
     const unsigned int gen = ld_acquire_u32(&ctl->bar_gen);
     __threadfence();
