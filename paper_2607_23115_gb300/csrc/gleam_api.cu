@@ -403,11 +403,16 @@ int dedup_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
   return (int)std::max<uint64_t>(1, std::min<uint64_t>(c->coop_max_blocks, want));
 }
 
-// Blocks of the pack kernel: one per 256 chunks or per kBytesPerDedupBlock of
+// Blocks of the pack kernel: one per 256 chunks or per kBytesPerPackBlock of
 // payload, up to one full wave of co-resident blocks.
+#ifndef GLEAM_PACK_BYTES_PER_BLOCK
+#define GLEAM_PACK_BYTES_PER_BLOCK (32ull << 10)
+#endif
+constexpr uint64_t kBytesPerPackBlock = GLEAM_PACK_BYTES_PER_BLOCK;
+
 int pack_grid(const gleam_cache* c, uint64_t nchunks, uint64_t nbytes) {
   const uint64_t want = std::max<uint64_t>((nchunks + 255) / 256,
-                                           (nbytes + kBytesPerDedupBlock - 1) / kBytesPerDedupBlock);
+                                           (nbytes + kBytesPerPackBlock - 1) / kBytesPerPackBlock);
   return (int)std::max<uint64_t>(1, std::min<uint64_t>(c->pack_max_blocks, want));
 }
 
