@@ -268,6 +268,17 @@ __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a
   }
 }
 
+template <bool kProbe>
+cudaError_t launch_staged(const HashArgs& a, cudaStream_t s) {
+  // per device and cheap: set on every launch
+  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe>,
+                       cudaFuncAttributeMaxDynamicSharedMemorySize, kStagedSmem);
+  const unsigned long long threads = a.Ntot * 4;
+  const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
+  k_hash_probe_staged<kProbe><<<sg, kStagedThreads, kStagedSmem, s>>>(a);
+  return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------------------
 // Paper-identifier mode (App. B.1): the key is MD5 (RFC 1321) of the chunk's
 // first min(len, 128) bytes, computed by one lane; candidates are then
@@ -590,16 +601,8 @@ cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
     return cudaGetLastError();
   }
 #if GLEAM_STAGED_HASH
-  if (aligned && (a.C % 32 == 0 || a.Ntot == 1)) {
-    // per device and cheap: set on every launch
-    cudaFuncSetAttribute(probe ? (const void*)k_hash_probe_staged<true>
-                               : (const void*)k_hash_probe_staged<false>,
-                         cudaFuncAttributeMaxDynamicSharedMemorySize, kStagedSmem);
-    const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
-    if (probe) k_hash_probe_staged<true><<<sg, kStagedThreads, kStagedSmem, s>>>(a);
-    else k_hash_probe_staged<false><<<sg, kStagedThreads, kStagedSmem, s>>>(a);
-    return cudaGetLastError();
-  }
+  if (aligned && (a.C % 32 == 0 || a.Ntot == 1))
+    return probe ? launch_staged<true>(a, s) : launch_staged<false>(a, s);
 #endif
   if (aligned && probe) k_hash_probe<true, true><<<grid, kHashThreads, 0, s>>>(a);
   else if (aligned) k_hash_probe<true, false><<<grid, kHashThreads, 0, s>>>(a);

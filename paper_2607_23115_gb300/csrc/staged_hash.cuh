@@ -121,6 +121,17 @@ template <int N>
 __device__ __forceinline__ void cp_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
+// Waits until at most min(n, kMax - 1) committed groups are pending (the
+// instruction takes an immediate count).
+template <int kMax>
+__device__ __forceinline__ void cp_wait_upto(uint32_t n) {
+  if constexpr (kMax <= 1) {
+    cp_wait<0>();
+  } else {
+    if (n >= (uint32_t)kMax - 1) cp_wait<kMax - 1>();
+    else cp_wait_upto<kMax - 1>(n);
+  }
+}
 
 // This lane's share (4 lanes x 8 x 16 bytes) of one stage of `src` into `dst`;
 // `bytes` (multiple of 32, <= kStage) of the stage exist.
@@ -133,7 +144,8 @@ __device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uin
   }
 }
 
-// The chunks of block-sized range vb (blockDim.x / 4 consecutive chunks).
+// The chunks of block-sized range vb (blockDim.x / 4 consecutive chunks); the
+// shared memory holds one region of kGroupBytes per group.
 template <bool kProbe>
 __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long long vb,
                                              uint8_t* smem) {
@@ -202,15 +214,30 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
     // 1 .. kDepth-1, issued late because the hint is known only then
     // stage t needs everything up to the late group while t < kDepth - 1
     // (at most t newer groups may pend), else up to its own group
-    if (t == 0 || t >= (uint32_t)kDepth - 1) cp_wait<kDepth - 1>();
-    else if (t == 1) cp_wait<1>();
-    else if (t == 2) cp_wait<2>();
-    else cp_wait<0>();
+    cp_wait_upto<kDepth>((t == 0 || t >= (uint32_t)kDepth - 1) ? (uint32_t)kDepth - 1 : t);
     __syncwarp(gmask);
     const uint8_t* sp = pay_p(t);
     const uint32_t sst = sbytes(t) >> 5;
     unsigned long long d = 0;
-    if (cmp && t > 0) {
+    auto word = [&](const uint8_t* b, uint32_t s) {
+      return *reinterpret_cast<const unsigned long long*>(b + s * 32 + lane * 8);
+    };
+    if (sst == (uint32_t)kStage / 32) {
+      // a whole stage, eight stripes at a time: the loads and the compare
+      // overlap the XXH64 chain instead of waiting in it
+#pragma unroll
+      for (uint32_t h = 0; h < (uint32_t)kStage / 32; h += 8) {
+        unsigned long long w[8];
+#pragma unroll
+        for (uint32_t u = 0; u < 8; ++u) w[u] = word(sp, h + u);
+        if (cmp && t > 0) {
+#pragma unroll
+          for (uint32_t u = 0; u < 8; ++u) d |= w[u] ^ word(sp + kStage, h + u);
+        }
+#pragma unroll
+        for (uint32_t u = 0; u < 8; ++u) acc = xstep(acc, w[u]);
+      }
+    } else if (cmp && t > 0) {
       const uint8_t* sq = sp + kStage;
 #pragma unroll 4
       for (uint32_t s = 0; s < sst; ++s) {
@@ -248,14 +275,11 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
     }
     if (t == 0) cp_commit();  // the late group (empty without a hint)
     if (cmp) {
+      // a lane that found a difference stops streaming its share of the
+      // cached copy; the others may then compare stale words, which can only
+      // add differences to a chunk already known to differ
       diff |= d;
-      unsigned long long gd = diff;
-      gd |= __shfl_xor_sync(gmask, gd, 1);
-      gd |= __shfl_xor_sync(gmask, gd, 2);
-      if (gd) {
-        cmp = false;  // stop streaming the cached copy
-        diff = 1;
-      }
+      if (diff) cmp = false;
     }
     __syncwarp(gmask);  // everyone is done with buffer t before it is refilled
   }
