@@ -6,9 +6,13 @@ dedup, compaction, packing, insertion) over one upload: every tensor of the
 workload is one payload (as one cudaMemcpy per tensor would be), all of them
 in one gleam_dedup_copy_batch call; the same pass as one
 gleam_dedup_copy_async call per tensor is reported beside it.  The cache is
-restored from a device snapshot at the start of each step (index and hint
-table copies, inside the timed region), so every step does the same work.  Inputs (16 GB for the default workload) are resident in HBM and
-far larger than L2, so no L2 flush is needed between steps.
+restored from a device snapshot before each step (index and hint table
+copies), so every step does the same work; each step is timed by its own
+CUDA events, after the restore (the repetitions are restored untimed), and
+the line reports their sum over the K steps and their median.  Inputs (16 GB
+for the default workload) are resident in HBM and far larger than L2, so no
+L2 flush is needed between steps; smaller ones get one before each step,
+outside its events.
 
 Default workload: a Llama-3-8B-shaped bf16 weight upload (291 tensors,
 ~16.06 GB, values ~N(0, 0.02)), chunk C = 64 KiB, a 24 GiB cache pre-filled
@@ -480,24 +484,21 @@ def run_gleam(args, rank, world, local_rank):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    if flush is None:
-        t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        t_start.record()
-        for _ in range(args.steps):
-            step()
-        t_end.record()
-        torch.cuda.synchronize()
-        ms = t_start.elapsed_time(t_end)
-    else:  # inputs fit in L2: flush it between steps, outside each step's events
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(args.steps)]
-        for e0, e1 in ev:
+    # each step restores the cache snapshot first, outside its own events (the
+    # repetitions are restored untimed); inputs that fit in L2 are also flushed
+    # there
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    for e0, e1 in ev:
+        cache.restore(snap)
+        if flush is not None:
             flush.fill_(1)
-            e0.record()
-            step()
-            e1.record()
-        torch.cuda.synchronize()
-        ms = sum(e0.elapsed_time(e1) for e0, e1 in ev)
+        e0.record()
+        one_pass()
+        e1.record()
+    torch.cuda.synchronize()
+    step_ms = [e0.elapsed_time(e1) for e0, e1 in ev]
+    ms = sum(step_ms)
     if world > 1:
         dist.barrier()
     clk = clocks.stop() if not args.profile_launches else None
@@ -570,6 +571,8 @@ def run_gleam(args, rank, world, local_rank):
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
+        "step_ms": {"median": round(statistics.median(step_ms), 4),
+                    "min": round(min(step_ms), 4), "max": round(max(step_ms), 4)},
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
         "data": "synthetic",
         "config": {"workload": wl.name, "description": wl.desc,
@@ -579,8 +582,9 @@ def run_gleam(args, rank, world, local_rank):
                    "evictions_per_step": evictions,
                    "cache_capacity_bytes": wl.capacity, "key16": bool(wl.flags & 1),
                    "l2": ("inputs (%.2f GB) fit in the 129 MB L2's reach: a 256 MiB buffer is "
-                          "written between timed steps, outside each step's events"
-                          % (total / 1e9)) if flush is not None else
+                          "written between timed steps, after the cache snapshot is restored, "
+                          "both outside each step's events" % (total / 1e9))
+                         if flush is not None else
                          ("inputs (%.1f GB per step) far larger than the 129 MB L2; no flush"
                           % (total / 1e9)),
                    "parallelism": "replicas" if world > 1 else "single GPU"},

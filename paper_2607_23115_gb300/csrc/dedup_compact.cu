@@ -1118,7 +1118,6 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
   if (threadIdx.x == 0) {
     DevCtl* c = a.ctl;
     c->bar_count = 0;
-    c->bar_gen = 0;
     c->err = 0;
     c->unres[0] = c->unres[1] = c->unres[2] = 0;
     c->acc_hits_cache = c->acc_hits_intra = c->acc_rejects = 0;

@@ -55,8 +55,8 @@ enum StatIdx {
 
 // Per-call control block; starts zeroed and every dedup kernel leaves it zeroed.
 struct DevCtl {
-  unsigned int bar_count;
-  unsigned int bar_gen;
+  unsigned int bar_count;  // grid-barrier arrivals of the call (nblocks per barrier)
+  unsigned int pad1;
   int err;
   unsigned int done;
   unsigned int unres[3];
@@ -283,22 +283,20 @@ __device__ __forceinline__ bool grid_barrier(DevCtl* ctl, unsigned int nblocks,
   __syncthreads();
   if (nblocks == 1) return !skip;
   if (threadIdx.x == 0 && !skip) {
-    const unsigned int gen = ld_acquire_u32(&ctl->bar_gen);
+    // arrivals only grow during a call: this barrier is passed once the
+    // count reaches the next multiple of nblocks (no reset, no second flag)
     __threadfence();
     const unsigned int arrived = atomicAdd(&ctl->bar_count, 1u);
-    if (arrived == nblocks - 1) {
-      atomicExch(&ctl->bar_count, 0u);
-      __threadfence();
-      atomicAdd(&ctl->bar_gen, 1u);
-    } else {
+    const unsigned int target = (arrived / nblocks + 1) * nblocks;
+    if (arrived + 1 != target) {
       const unsigned long long t0 = globaltimer_ns();
-      while (ld_acquire_u32(&ctl->bar_gen) == gen) {
+      while (ld_acquire_u32(&ctl->bar_count) < target) {
         if (ld_volatile_s32(&ctl->err) != 0) break;
         if (globaltimer_ns() - t0 > wait_ns) {
           atomicCAS(&ctl->err, 0, (int)GLEAM_ERR_TIMEOUT);
           break;
         }
-        __nanosleep(100);
+        __nanosleep(32);
       }
     }
     __threadfence();
