@@ -78,3 +78,24 @@ def test_small_calls_near_a_full_lru_cache():
             dedup_both(gc, oc, _alphabet_payload(rng, C, nch, alphabet, 0))
         compare_cache(gc, oc)
         assert gc.stats()["evictions"] == oc.stats()["evictions"] > 0
+
+
+def test_the_library_takes_the_single_block_path():
+    # a call that runs as one kernel has nothing in the profile's second phase
+    # (its events are recorded back to back); with the path off, the resolve
+    # and pack kernels take several microseconds per call there
+    C = 4 * KiB
+    payloads = [W.random_bytes(16 * C, seed=700 + k).to("cuda") for k in range(20)]
+    phase1 = {}
+    for limit in (64, 0):
+        gc = Cache(4 * MiB, C)
+        gc.debug_set(B.GLEAM_DEBUG_SMALL_CALLS, limit)
+        with gc:
+            B.gleam_cache_profile(gc.handle, True)
+            for p in payloads:
+                gc.dedup(p)
+            rc, ms, n = B.gleam_cache_profile_read(gc.handle, 2)
+            assert rc == 0 and n == [20, 20]
+            phase1[limit] = ms[1] * 1e3 / 20  # us per call
+    assert phase1[64] < 3.0, phase1
+    assert phase1[0] > 5.0, phase1
