@@ -459,11 +459,13 @@ def run_gleam(args, rank, world, local_rank):
         cache.restore(snap)
         one_pass()
 
-    ev0 = cache.stats()["evictions"]
+    st0 = cache.stats()
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
-    evictions = cache.stats()["evictions"] - ev0  # of the last warm-up step (restored before)
+    st1 = cache.stats()  # the last warm-up step's counters (restored before it)
+    evictions = st1["evictions"] - st0["evictions"]
+    spec_chunks = st1["spec_chunks"] - st0["spec_chunks"]
     r = results.cpu().numpy()
     assert (r[:, 0] == 0).all(), "a dedup call failed: %s" % r[r[:, 0] != 0][:3]
     miss_bytes = int(r[:, 5].sum())
@@ -474,7 +476,9 @@ def run_gleam(args, rank, world, local_rank):
     # algorithmic bytes: the fused fingerprint/probe/verify kernel reads the
     # payload once and the cached copy of every cache hit
     hit_cache_bytes = total - miss_bytes - hit_intra * C
-    kernel0_bytes = total + hit_cache_bytes
+    # ... and writes twice every chunk it writes ahead (write-through of
+    # likely misses; C bytes per chunk, a tail counted whole)
+    kernel0_bytes = total + hit_cache_bytes + 2 * spec_chunks * C
     pipeline_bytes = 2 * total  # payload read + hit bytes read + miss bytes written
 
     clocks = ClockSampler(local_rank)
@@ -580,6 +584,7 @@ def run_gleam(args, rank, world, local_rank):
                    "api": "gleam_dedup_copy_batch (one call = %d payloads)" % nt,
                    "chunk_bytes": C, "chunks_per_step": nchunks, "misses_per_step": n_miss,
                    "evictions_per_step": evictions,
+                   "written_ahead_chunks_per_step": spec_chunks,
                    "cache_capacity_bytes": wl.capacity, "key16": bool(wl.flags & 1),
                    "l2": ("inputs (%.2f GB) fit in the 129 MB L2's reach: a 256 MiB buffer is "
                           "written between timed steps, after the cache snapshot is restored, "

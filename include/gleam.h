@@ -103,6 +103,10 @@ typedef struct gleam_stats {
   uint64_t nslots;         /* capacity_bytes / chunk_bytes                   */
   uint64_t chunk_bytes;    /* C                                              */
   uint64_t evictions;      /* slots reused by GLEAM_EVICT_LRU                */
+  uint64_t spec_chunks;    /* chunks the hash kernel also wrote ahead to their
+                              likely packed offset and arena slot
+                              (write-through, GLEAM_DEBUG_SPECULATE); a
+                              speed counter that outputs never depend on     */
 } gleam_stats_t;
 
 /* Written by the device when an asynchronous dedup call completes. */
@@ -173,7 +177,9 @@ int gleam_fingerprint(const void* d_buf, size_t n, size_t chunk_bytes, uint64_t*
  *                bits past N are 0;
  *   d_miss_idx   u32[N]: ascending indices of the misses;
  *   d_miss_bytes u8[n]: the r-th miss's bytes at offset r*C (true length for
- *                the last chunk) -- the bytes that must cross the network.
+ *                the last chunk) -- the bytes that must cross the network;
+ *                bytes past the last miss are unspecified (the call may
+ *                write there).
  * Synchronous like cudaMemcpy (runs on the legacy default stream).
  * Returns the number of misses (>= 0) or a negative gleam_status; on
  * GLEAM_ERR_CAPACITY and GLEAM_ERR_TIMEOUT the cache is unchanged and the
@@ -318,6 +324,16 @@ int gleam_cache_debug_insert(gleam_cache_t* cache, uint64_t key, const void* d_b
  * one single-block kernel instead of three launches (default 64; 0 turns that
  * path off).  Only the speed changes: every output is the same either way. */
 #define GLEAM_DEBUG_SMALL_CALLS 5
+/* what = GLEAM_DEBUG_SPECULATE: the write-through of likely misses.  A chunk
+ * that no cached chunk begins like (no prefix-hint match) is written by the
+ * hash kernel, as it streams by, to packed offset i*C of its payload and to
+ * arena slot slots_used + g (g = its number in the call); the pack step then
+ * skips the copies of every miss whose rank puts it exactly there (a payload,
+ * or a run of payloads, of misses only) and copies the others over.  0 = automatic
+ * (default: on while at least half of the chunks written ahead are used,
+ * retried every 256 calls once off), 1 = always, 2 = never.  Only the speed
+ * changes: every output is the same either way. */
+#define GLEAM_DEBUG_SPECULATE 6
 int gleam_cache_debug_set(gleam_cache_t* cache, int what, int64_t value);
 
 /* Device-side copy of the index, slot count and counters (and, for a
@@ -325,7 +341,9 @@ int gleam_cache_debug_set(gleam_cache_t* cache, int what, int64_t value);
  * cache between timed repetitions.  Arena bytes are not copied: those past
  * the saved slot count are never read, and a slot that an eviction reused
  * after the snapshot keeps its new bytes, so its restored entry no longer
- * matches them and its chunk misses (every hit is verified). */
+ * matches them and its chunk misses (every hit is verified).  The
+ * write-through's automatic state (GLEAM_DEBUG_SPECULATE) is not part of a
+ * snapshot: it follows the calls made. */
 int gleam_cache_snapshot(gleam_cache_t* cache, gleam_snapshot_t** out);
 int gleam_cache_restore(gleam_cache_t* cache, const gleam_snapshot_t* snap);
 void gleam_snapshot_destroy(gleam_snapshot_t* snap);

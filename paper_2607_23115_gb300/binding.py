@@ -31,6 +31,7 @@ GLEAM_DEBUG_SKIP_ARRIVE = 2
 GLEAM_DEBUG_CLOCK = 3
 GLEAM_DEBUG_DROP_ENTRY = 4
 GLEAM_DEBUG_SMALL_CALLS = 5
+GLEAM_DEBUG_SPECULATE = 6
 
 # Every symbol include/gleam.h declares (checked by the ABI test).
 EXPORTS = (
@@ -49,7 +50,7 @@ class gleam_stats_t(ctypes.Structure):
     _fields_ = [(f, ctypes.c_uint64) for f in (
         "calls", "chunks", "hits_cache", "hits_intra", "misses", "inserts",
         "verify_rejects", "slots_used", "bytes_used", "capacity_bytes", "nslots",
-        "chunk_bytes", "evictions")]
+        "chunk_bytes", "evictions", "spec_chunks")]
 
 
 class gleam_payload_t(ctypes.Structure):

@@ -849,7 +849,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
   __shared__ unsigned long long red64[kWarps];
   __shared__ unsigned long long s_slots0, s_total, s_evict;
   // a grid of one block keeps its totals here instead of in the control block
-  __shared__ unsigned long long s_stored, s_vbytes, s_sum[5];
+  __shared__ unsigned long long s_stored, s_vbytes, s_sum[7];
   __shared__ int s_err;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const uint32_t N = (uint32_t)a.Ntot;
@@ -861,7 +861,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
     s_evict = __ldcg(&a.ctl->evict_k);
     s_stored = __ldcg(&a.ctl->acc_stored);
     s_vbytes = __ldcg(&a.ctl->acc_victim_bytes);
-    for (int k = 0; k < 5; ++k) s_sum[k] = 0;
+    for (int k = 0; k < 7; ++k) s_sum[k] = 0;
   }
   __syncthreads();
   const unsigned long long slots0 = s_slots0;
@@ -897,6 +897,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
   // ---- hit masks, miss indices, chunk slots, counters ------------------------
   if (ok) {
     unsigned long long n_hc = 0, n_hi = 0, n_rej = 0, n_bytes = 0, n_sbytes = 0;
+    uint32_t n_spec = 0, n_spec_used = 0;  // write-through: chunks written ahead, used
     for (unsigned long long t = (unsigned long long)bid * kThreads; t < N;
          t += (unsigned long long)G * kThreads) {
       const uint32_t g = (uint32_t)(t + threadIdx.x);
@@ -935,6 +936,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
           rej = (r & kResRoundMask) > 1 || ch.status[g] == kMissCand;
         }
       }
+      n_spec += a.spec_active && valid && ch.spec[g];
       n_hc += hc;
       n_hi += hi2;
       n_rej += rej;
@@ -964,7 +966,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
       const unsigned long long r = base + lane;
       const bool have = r < hi;
       uint32_t gg = 0, ln = 0;
-      bool cached = false;
+      bool cached = false, copy = false;
       unsigned long long slot = 0, src = 0, d1 = 0, d2 = 0;
       if (have) {
         gg = ch.order[r];
@@ -974,24 +976,33 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
         src = ch.src[gg];
         d1 = (unsigned long long)(P.packed + (r - a.pstart[pp]) * a.C);
         cached = !(ch.res[gg] & kResNoSlot);  // else sent, never cached
+        uint32_t sr = 0xFFFFFFFFu;
         if (cached) {
-          slot = slot_of(ch.srank[gg]);
+          sr = ch.srank[gg];
+          slot = slot_of(sr);
           d2 = (unsigned long long)(a.arena + slot * a.C);
         }
+        // written ahead by the hash kernel exactly where it belongs: with no
+        // eviction, stored rank g means every earlier chunk of the call is a
+        // stored miss, so the chunk's packed offset is i*C and its slot
+        // slots_used + g, the places it was written to
+        copy = !(a.spec_active && evict == 0 && sr == gg && ch.spec[gg]);
+        n_spec_used += !copy;
       }
-      const uint32_t m = (uint32_t)((hi - base) < 32ull ? (hi - base) : 32ull);
+      const unsigned cmask = __ballot_sync(0xffffffffu, copy);  // lanes whose chunk is copied
+      const uint32_t m = __popc(cmask);
 #if GLEAM_PACK_BULK
       const bool bulk =
-          !a.plain_copy && __all_sync(0xffffffffu, !have || ((src | d1 | d2) & 15) == 0);
+          !a.plain_copy && __all_sync(0xffffffffu, !copy || ((src | d1 | d2) & 15) == 0);
       if (bulk) {
-        if (have) meta[lane] = PackMeta{src, d1, d2, ln, 0u};
+        if (copy) meta[__popc(cmask & ((1u << lane) - 1u))] = PackMeta{src, d1, d2, ln, 0u};
         __syncwarp();
-        if (lane == 0 && !bulk_failed &&
+        if (lane == 0 && m && !bulk_failed &&
             !bulk_copy_batch(meta, m, bufs, bars, ring, a.wait_ns)) {
           bulk_failed = true;
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_TIMEOUT);
         }
-        if (have) {  // the last len % 16 bytes
+        if (copy) {  // the last len % 16 bytes
           const uint8_t* sp = reinterpret_cast<const uint8_t*>(src);
           uint8_t* x = reinterpret_cast<uint8_t*>(d1);
           uint8_t* y = reinterpret_cast<uint8_t*>(d2);
@@ -1003,7 +1014,8 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
         __syncwarp();
       } else
 #endif
-      for (uint32_t j = 0; j < m; ++j) {
+      for (unsigned todo = cmask; todo; todo &= todo - 1) {
+        const int j = __ffs(todo) - 1;
         const unsigned long long sj = __shfl_sync(0xffffffffu, src, j);
         const unsigned long long xj = __shfl_sync(0xffffffffu, d1, j);
         const unsigned long long yj = __shfl_sync(0xffffffffu, d2, j);
@@ -1029,18 +1041,24 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
     n_rej = block_sum<unsigned long long>(n_rej, red64);
     n_bytes = block_sum<unsigned long long>(n_bytes, red64);
     n_sbytes = block_sum<unsigned long long>(n_sbytes, red64);
+    const unsigned long long b_spec = block_sum<unsigned long long>(n_spec, red64);
+    const unsigned long long b_spec_used = block_sum<unsigned long long>(n_spec_used, red64);
     if (threadIdx.x == 0 && G == 1) {
       s_sum[0] = n_hc;
       s_sum[1] = n_hi;
       s_sum[2] = n_rej;
       s_sum[3] = n_bytes;
       s_sum[4] = n_sbytes;
+      s_sum[5] = b_spec;
+      s_sum[6] = b_spec_used;
     } else if (threadIdx.x == 0) {
       atomicAdd(&a.ctl->acc_hits_cache, n_hc);
       atomicAdd(&a.ctl->acc_hits_intra, n_hi);
       atomicAdd(&a.ctl->acc_rejects, n_rej);
       atomicAdd(&a.ctl->acc_miss_bytes, n_bytes);
       atomicAdd(&a.ctl->acc_stored_bytes, n_sbytes);
+      if (b_spec) atomicAdd(&a.ctl->spec_tried, b_spec);
+      if (b_spec_used) atomicAdd(&a.ctl->spec_used, b_spec_used);
     }
   }
 
@@ -1069,6 +1087,21 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
     const unsigned long long sbytes = one ? s_sum[4] : __ldcg(&a.ctl->acc_stored_bytes);
     const unsigned long long stored = s_stored;
     const unsigned long long vbytes = s_vbytes;
+    const unsigned long long spec = one ? s_sum[5] : __ldcg(&a.ctl->spec_tried);
+    const unsigned long long spec_used = one ? s_sum[6] : __ldcg(&a.ctl->spec_used);
+    if (err == 0 && a.spec_state) {
+      // automatic write-through: stays on while at least half of the chunks
+      // written ahead were used; once off, tried again after 256 calls
+      uint32_t* st = a.spec_state;
+      if (spec) {
+        st[0] = 2 * spec_used >= spec ? 1u : 0u;
+        st[1] = 0;
+      } else if (st[0] == 0 && ++st[1] >= 256) {
+        st[0] = 1;
+        st[1] = 0;
+      }
+      *a.spec_mirror = st[0];
+    }
     if (err == 0) {  // no reads: the counters change by atomic adds
       atomicAdd(&a.dstats[ST_CALLS], a.ncalls);
       atomicAdd(&a.dstats[ST_CHUNKS], (unsigned long long)N);
@@ -1080,6 +1113,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
       a.dstats[ST_SLOTS_USED] = slots0 + stored - evict;
       atomicAdd(&a.dstats[ST_BYTES_USED], sbytes - vbytes);
       atomicAdd(&a.dstats[ST_EVICTIONS], evict);
+      if (spec) atomicAdd(&a.dstats[ST_SPEC_CHUNKS], spec);
     }
     gleam_result_t* t = a.total;
     t->status = err;
@@ -1125,6 +1159,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
     c->acc_stored = c->acc_stored_bytes = 0;
     c->acc_distinct = c->evict_k = c->lru_below = c->lru_ties = c->acc_victim_bytes = 0;
     c->lru_hi = c->lru_cut = 0;
+    c->spec_tried = c->spec_used = 0;
     c->done = 0;
   }
   __threadfence();
@@ -1151,6 +1186,7 @@ __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
+template <bool kSpec>
 __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a) {
   extern __shared__ __align__(128) uint8_t small_smem[];
   // Device-resident payloads (16-byte aligned here) are prefetched into L2 at
@@ -1166,7 +1202,7 @@ __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a
   const unsigned long long nvb = (h.Ntot * 4 + kThreads - 1) / kThreads;
   for (unsigned long long vb = 0; vb < nvb; ++vb) {
     __syncthreads();  // the previous range's groups are done with the shared memory
-    staged_range<true>(h, vb, small_smem);
+    staged_range<true, kSpec>(h, vb, small_smem);
   }
   __syncthreads();  // every chunk's probe outcome written (and its stage copies landed)
   resolve_rank(a, 1, 0);
@@ -1309,11 +1345,16 @@ cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream
 
 uint32_t small_call_groups() { return kSmallGroups; }
 
-cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_t s) {
-  cudaFuncSetAttribute((const void*)k_small_call, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                       kSmallSmem);
-  k_small_call<<<1, kThreads, kSmallSmem, s>>>(h, a);
+template <bool kSpec>
+cudaError_t launch_small(const HashArgs& h, const DedupArgs& a, cudaStream_t s) {
+  cudaFuncSetAttribute((const void*)k_small_call<kSpec>,
+                       cudaFuncAttributeMaxDynamicSharedMemorySize, kSmallSmem);
+  k_small_call<kSpec><<<1, kThreads, kSmallSmem, s>>>(h, a);
   return cudaGetLastError();
+}
+
+cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_t s) {
+  return h.spec_mode ? launch_small<true>(h, a, s) : launch_small<false>(h, a, s);
 }
 
 cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s) {

@@ -68,6 +68,11 @@ struct gleam_cache {
   uint64_t small_max_chunks = 0;
   uint64_t slots_bound = 0;
 
+  // write-through of likely misses (HashArgs::spec_mode)
+  uint32_t* spec_state = nullptr;   // device: [0] on, [1] calls since it went off
+  uint32_t* spec_mirror = nullptr;  // page-locked, mapped: [0] as of the last finished call
+  int spec_hook = 0;                // GLEAM_DEBUG_SPECULATE: 0 auto, 1 always, 2 never
+
   unsigned long long wait_ns = 4000000000ULL;
   int skip_block = -1;
 
@@ -243,11 +248,11 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   cap = std::min<uint64_t>(cap, kMaxChunks);
   if (cap < nchunks) cap = nchunks;
   const uint64_t tcap = next_pow2(2 * cap);
-  const uint64_t sz[13] = {align256(cap),     align256(cap * 8), align256(cap * 4),
+  const uint64_t sz[14] = {align256(cap),     align256(cap * 8), align256(cap * 4),
                            align256(cap * 8), align256(cap * 4), align256(cap * 4),
                            align256(cap * 4), align256(cap * 4), align256(cap * 8),
                            align256(cap * 4), align256(cap * 4), align256(cap * 4),
-                           align256(tcap * sizeof(CallEntry))};
+                           align256(cap),     align256(tcap * sizeof(CallEntry))};
   uint64_t total = 0;
   for (uint64_t x : sz) total += x;
   int rc = cuda_err(cudaEventSynchronize(c->done));
@@ -285,6 +290,8 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   b += sz[10];
   c->ch.old = reinterpret_cast<uint32_t*>(b);
   b += sz[11];
+  c->ch.spec = b;
+  b += sz[12];
   c->tbl = reinterpret_cast<CallEntry*>(b);
   c->tbl_cap = tcap;
   c->ws_chunks = cap;
@@ -329,6 +336,8 @@ void destroy_cache(gleam_cache* c) {
     if (c->dbg_count) cudaFree(c->dbg_count);
     if (c->dbg_flag) cudaFree(c->dbg_flag);
     if (c->ctl) cudaFree(c->ctl);
+    if (c->spec_state) cudaFree(c->spec_state);
+    if (c->spec_mirror) cudaFreeHost(c->spec_mirror);
     if (c->bcount) cudaFree(c->bcount);
     if (c->d_result) cudaFree(c->d_result);
     if (c->h_result) cudaFreeHost(c->h_result);
@@ -449,6 +458,30 @@ void note_call(gleam_cache* c, uint64_t Ntot) {
   c->slots_bound = std::min<uint64_t>(c->nslots, c->slots_bound + Ntot);
 }
 
+// The write-through fields of a call's kernel arguments.  It needs the staged
+// hash (16-byte-aligned payloads, C a multiple of 32), device outputs with
+// 16-byte-aligned packed buffers, and 64-bit or KEY16 keys.  In the automatic
+// mode the host launches the write-through variant of the hash kernel when
+// the page-locked copy of the device state says it is on (as of the last call
+// that finished: a call or two late at most, which a heuristic can afford),
+// and every eligible call feeds the state back.
+void set_spec(gleam_cache* c, HashArgs* h, DedupArgs* d, bool eligible) {
+  h->spec_mode = 0;
+  d->spec_active = 0;
+  d->spec_state = nullptr;
+  d->spec_mirror = nullptr;
+  if (!eligible || c->C % 32 != 0 || (c->flags & GLEAM_PAPER_IDS) || c->spec_hook == 2) return;
+  const bool on = c->spec_hook == 1 || *reinterpret_cast<volatile uint32_t*>(c->spec_mirror);
+  h->spec_mode = on ? 1u : 0u;
+  h->arena_w = c->arena;
+  h->nslots = c->nslots;
+  d->spec_active = h->spec_mode;
+  if (c->spec_hook == 0) {
+    d->spec_state = c->spec_state;
+    d->spec_mirror = c->spec_mirror;
+  }
+}
+
 // GLEAM_DEBUG_CHECKS: the index consistency check after a call.
 int enqueue_index_check(gleam_cache* c, const DedupArgs& d, cudaStream_t s) {
   if (!(c->flags & GLEAM_DEBUG_CHECKS)) return GLEAM_OK;
@@ -484,7 +517,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     if ((rc = cuda_err(cudaEventSynchronize(c->table_copied))) != GLEAM_OK) return rc;
   }
   uint64_t Ntot = 0, ncalls = 0, nbytes = 0;
-  bool aligned = true;
+  bool aligned = true, packed_aligned = true;
   for (uint64_t k = 0; k < count; ++k) {
     PayloadDesc* d = count > 1 ? &c->h_table[k] : &one;
     if ((rc = describe(c, chk, payloads[k], d, host_payloads)) != GLEAM_OK) return rc;
@@ -495,6 +528,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
       ++ncalls;
       nbytes += d->n;
       aligned = aligned && (reinterpret_cast<uintptr_t>(d->buf) % 16 == 0);
+      packed_aligned = packed_aligned && (reinterpret_cast<uintptr_t>(d->packed) % 16 == 0);
     }
   }
   if ((rc = ensure_ws(c, std::max<uint64_t>(Ntot, 1))) != GLEAM_OK) return rc;
@@ -561,6 +595,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     if (d.skip_block >= grid) d.skip_block = grid - 1;
   }
   const bool fused = small_call(c, aligned, Ntot, nbytes, d.skip_block);
+  set_spec(c, &h, &d, aligned && packed_aligned && !d.plain_copy);
 
   cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
   if (c->profile) {
@@ -665,6 +700,8 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     step(cudaMalloc(&c->bins, kLruBins * sizeof(uint32_t)));
   }
   step(cudaMalloc(&c->ctl, sizeof(DevCtl)));
+  step(cudaMalloc(&c->spec_state, 2 * sizeof(uint32_t)));
+  step(cudaHostAlloc(&c->spec_mirror, sizeof(uint32_t), cudaHostAllocMapped));
   step(cudaMalloc(&c->d_result, sizeof(gleam_result_t)));
   step(cudaMallocHost(&c->h_result, sizeof(gleam_result_t)));
   step(cudaEventCreateWithFlags(&c->done, cudaEventDisableTiming));
@@ -687,6 +724,9 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     step(cudaMemset(c->hints, 0xFF, c->index_cap * sizeof(IndexEntry)));
     step(cudaMemset(c->dstats, 0, ST_COUNT * sizeof(unsigned long long)));
     step(cudaMemset(c->ctl, 0, sizeof(DevCtl)));
+    const uint32_t spec0[2] = {1u, 0u};  // automatic write-through starts on
+    step(cudaMemcpy(c->spec_state, spec0, sizeof(spec0), cudaMemcpyHostToDevice));
+    if (rc == GLEAM_OK) *c->spec_mirror = 1u;
     if (flags & GLEAM_DEBUG_CHECKS) {
       step(cudaMemset(c->dbg_count, 0, nslots * sizeof(uint32_t)));
       step(cudaMemset(c->dbg_flag, 0, sizeof(uint32_t)));
@@ -858,6 +898,7 @@ int gleam_cache_stats(const gleam_cache_t* c, gleam_stats_t* out) {
   out->slots_used = s[ST_SLOTS_USED];
   out->bytes_used = s[ST_BYTES_USED];
   out->evictions = s[ST_EVICTIONS];
+  out->spec_chunks = s[ST_SPEC_CHUNKS];
   out->capacity_bytes = c->capacity_bytes;
   out->nslots = c->nslots;
   out->chunk_bytes = c->C;
@@ -957,6 +998,11 @@ int gleam_cache_debug_set(gleam_cache_t* c, int what, int64_t value) {
                                    cudaMemcpyHostToDevice));
       }
     return GLEAM_ERR_INVALID_ARG;
+  }
+  if (what == GLEAM_DEBUG_SPECULATE) {
+    if (value < 0 || value > 2) return GLEAM_ERR_INVALID_ARG;
+    c->spec_hook = (int)value;
+    return GLEAM_OK;
   }
   if (what == GLEAM_DEBUG_SMALL_CALLS) {
     if (value < 0 || value > (int64_t)kMaxChunks) return GLEAM_ERR_INVALID_ARG;
@@ -1122,7 +1168,8 @@ constexpr uint64_t kNaOffHint = kNaOffRank + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffOrder = kNaOffHint + na_align(kNaChunks * 8);
 constexpr uint64_t kNaOffSrank = kNaOffOrder + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffOld = kNaOffSrank + na_align(kNaChunks * 4);
-constexpr uint64_t kNaOffTbl = kNaOffOld + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffSpec = kNaOffOld + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffTbl = kNaOffSpec + na_align(kNaChunks);
 constexpr uint64_t kNaOffCtl = kNaOffTbl + na_align(kNaTable * sizeof(CallEntry));
 constexpr uint64_t kNaOffBcount = kNaOffCtl + na_align(sizeof(DevCtl));
 constexpr uint64_t kNaOffResult = kNaOffBcount + na_align((2 * kNaBlocks + 1) * 4);
@@ -1192,6 +1239,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   ch.order = reinterpret_cast<uint32_t*>(base + kNaOffOrder);
   ch.srank = reinterpret_cast<uint32_t*>(base + kNaOffSrank);
   ch.old = reinterpret_cast<uint32_t*>(base + kNaOffOld);
+  ch.spec = base + kNaOffSpec;
   CallEntry* tbl = reinterpret_cast<CallEntry*>(base + kNaOffTbl);
   DevCtl* ctl = reinterpret_cast<DevCtl*>(base + kNaOffCtl);
   uint32_t* bcount = reinterpret_cast<uint32_t*>(base + kNaOffBcount);
@@ -1243,6 +1291,8 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.plain_copy = chk.saw_managed() ? 1u : 0u;
   set_lru(c, &d, N);
   d.skip_block = -1;
+  set_spec(c, &h, &d,
+           aligned && reinterpret_cast<uintptr_t>(one.packed) % 16 == 0 && !d.plain_copy);
   if (small_call(c, aligned, N, n, -1)) {
     if ((rc = cuda_err(launch_small_call(h, d, s))) != GLEAM_OK) return rc;
   } else {

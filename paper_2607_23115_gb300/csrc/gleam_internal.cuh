@@ -50,7 +50,7 @@ constexpr uint32_t kResRoundMask = 0x0FFFFFFFu;
 // change; capacity, slot count and chunk size are host constants).
 enum StatIdx {
   ST_CALLS = 0, ST_CHUNKS, ST_HITS_CACHE, ST_HITS_INTRA, ST_MISSES, ST_INSERTS,
-  ST_REJECTS, ST_SLOTS_USED, ST_BYTES_USED, ST_EVICTIONS, ST_COUNT
+  ST_REJECTS, ST_SLOTS_USED, ST_BYTES_USED, ST_EVICTIONS, ST_SPEC_CHUNKS, ST_COUNT
 };
 
 // Per-call control block; starts zeroed and every dedup kernel leaves it zeroed.
@@ -76,6 +76,9 @@ struct DevCtl {
   unsigned long long acc_victim_bytes;  // stored bytes of the evicted slots
   unsigned int lru_hi;                  // high 16 bits of the cut-off stamp
   unsigned int lru_cut;                 // the cut-off stamp
+  // write-through of likely misses (HashArgs::spec_mode)
+  unsigned long long spec_tried;        // chunks the hash kernel wrote ahead
+  unsigned long long spec_used;         // misses whose copies that made unnecessary
 };
 
 // Position of a key in a power-of-two table: the 64-bit finaliser of
@@ -123,6 +126,8 @@ struct ChunkArrays {
   uint32_t* order;           // order[r] = chunk number of the miss of rank r
   uint32_t* srank;           // exclusive count of stored (cached) misses before the chunk
   uint32_t* old;             // LRU: last use of a hit's slot before this call stamped it
+  uint8_t* spec;             // 1: the hash kernel wrote the chunk to packed offset
+                             // i*C of its payload and to arena slot slots_used + g
 };
 
 // Speculative verify.  After the first kPrefixBytes of a chunk the four XXH64
@@ -152,6 +157,13 @@ struct HashArgs {
   uint32_t paper;            // GLEAM_PAPER_IDS: MD5-prefix keys, small chunks uncached
   ChunkArrays ch;
   DevCtl* ctl;
+  // write-through of likely misses (the host launches the variant of the
+  // staged hash that does it when spec_mode is 1): a chunk of at least
+  // kPrefixBytes with no prefix-hint match is written to its packed offset and
+  // to arena slot slots_used + g as it streams by
+  uint32_t spec_mode;
+  uint8_t* arena_w;                // the arena, for those writes
+  unsigned long long nslots;
 };
 
 struct DedupArgs {
@@ -187,6 +199,13 @@ struct DedupArgs {
   uint8_t* vflag;            // per slot: evicted by this call (zero between calls)
   uint32_t* victims;         // evicted slots in ascending order
   uint32_t* bins;            // 65536-bin histogram (zero between calls)
+  // write-through: spec_active = the hash kernel of this call did it (ch.spec
+  // is valid); feedback of the automatic mode: spec_state[0] = on, [1] = calls
+  // since it went off (null: no feedback), and a copy of [0] in page-locked
+  // host memory that the host reads when it launches the next call
+  uint32_t spec_active;
+  uint32_t* spec_state;
+  uint32_t* spec_mirror;
 };
 
 constexpr uint32_t kLruBins = 65536;

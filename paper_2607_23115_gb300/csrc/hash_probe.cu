@@ -258,24 +258,24 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
 }
 
 
-template <bool kProbe>
+template <bool kProbe, bool kSpec>
 __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned long long nvb = (a.Ntot * 4 + kStagedThreads - 1) / kStagedThreads;
   for (unsigned long long vb = blockIdx.x; vb < nvb; vb += gridDim.x) {
     __syncthreads();  // the previous range's groups are done with the shared memory
-    staged_range<kProbe>(a, vb, smem);
+    staged_range<kProbe, kSpec>(a, vb, smem);
   }
 }
 
-template <bool kProbe>
+template <bool kProbe, bool kSpec>
 cudaError_t launch_staged(const HashArgs& a, cudaStream_t s) {
   // per device and cheap: set on every launch
-  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe>,
+  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kSpec>,
                        cudaFuncAttributeMaxDynamicSharedMemorySize, kStagedSmem);
   const unsigned long long threads = a.Ntot * 4;
   const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
-  k_hash_probe_staged<kProbe><<<sg, kStagedThreads, kStagedSmem, s>>>(a);
+  k_hash_probe_staged<kProbe, kSpec><<<sg, kStagedThreads, kStagedSmem, s>>>(a);
   return cudaGetLastError();
 }
 
@@ -601,8 +601,10 @@ cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
     return cudaGetLastError();
   }
 #if GLEAM_STAGED_HASH
-  if (aligned && (a.C % 32 == 0 || a.Ntot == 1))
-    return probe ? launch_staged<true>(a, s) : launch_staged<false>(a, s);
+  if (aligned && (a.C % 32 == 0 || a.Ntot == 1)) {
+    if (!probe) return launch_staged<false, false>(a, s);
+    return a.spec_mode ? launch_staged<true, true>(a, s) : launch_staged<true, false>(a, s);
+  }
 #endif
   if (aligned && probe) k_hash_probe<true, true><<<grid, kHashThreads, 0, s>>>(a);
   else if (aligned) k_hash_probe<true, false><<<grid, kHashThreads, 0, s>>>(a);

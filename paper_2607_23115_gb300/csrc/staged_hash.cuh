@@ -145,8 +145,9 @@ __device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uin
 }
 
 // The chunks of block-sized range vb (blockDim.x / 4 consecutive chunks); the
-// shared memory holds one region of kGroupBytes per group.
-template <bool kProbe>
+// shared memory holds one region of kGroupBytes per group.  kSpec: with the
+// write-through of likely misses.
+template <bool kProbe, bool kSpec = false>
 __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long long vb,
                                              uint8_t* smem) {
   const unsigned long long g = (vb * blockDim.x + threadIdx.x) >> 2;
@@ -193,6 +194,11 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   uint32_t hint_slot = kEmptySlot;
   const uint8_t* q = nullptr;
   bool cmp = false;
+  // write-through of a likely miss, decided once the prefix hint is known
+  const bool spec_try = kSpec && speculate && slots_used + g < a.nslots;
+  bool spec = false;
+  uint8_t* spk = nullptr;  // packed offset i*C of the payload
+  uint8_t* sar = nullptr;  // arena slot slots_used + g
 
   unsigned long long acc = xlane_start(lane);
   // prologue: payload stages 0 .. kDepth-2
@@ -261,6 +267,11 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
       hint_slot = slots_used ? hint_lookup(a.hints, a.index_mask, hint, len, slots_used)
                              : kEmptySlot;
       cmp = hint_slot != kEmptySlot;
+      spec = spec_try && !cmp;  // no cached chunk begins like it: a likely miss
+      if (spec) {
+        spk = (a.count > 1 ? a.table[pid].packed : a.one.packed) + (g - base) * a.C;
+        sar = a.arena_w + (slots_used + g) * a.C;
+      }
       if (cmp) {
         q = a.arena + (unsigned long long)hint_slot * a.C;
         // the prefix, still in stage buffer 0, against the cached copy's prefix
@@ -281,9 +292,24 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
       diff |= d;
       if (diff) cmp = false;
     }
+    if (spec) {  // this lane's own pieces of stage t, to both destinations
+      const uint32_t sb = sbytes(t);
+#pragma unroll
+      for (int j = 0; j < kStage / 64; ++j) {
+        const uint32_t off = (uint32_t)j * 64 + lane * 16;
+        if (off < sb) {
+          const uint4 v = *reinterpret_cast<const uint4*>(sp + off);
+          const unsigned long long o = (unsigned long long)t * kStage + off;
+          __stcs(reinterpret_cast<uint4*>(spk + o), v);
+          __stcs(reinterpret_cast<uint4*>(sar + o), v);
+        }
+      }
+    }
     __syncwarp(gmask);  // everyone is done with buffer t before it is refilled
   }
   cp_wait<0>();
+  if (spec && lane == 0)  // the bytes past the last whole stripe
+    for (uint32_t k = full; k < len; ++k) spk[k] = sar[k] = p[k];
 
   unsigned long long h;
   if (ns) {
@@ -343,6 +369,7 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
     a.ch.src[g] = (unsigned long long)p;
     a.ch.pidx[g] = pid;
     a.ch.hint[g] = hint;
+    if (kSpec) a.ch.spec[g] = spec ? 1 : 0;
     if (hit) a.ch.ent[g] = hit_slot;
   }
 }

@@ -38,7 +38,9 @@ def _run(limit, C, flags, calls, seed):
             dedup_both(gc, oc, _alphabet_payload(rng, C, nch, alphabet, tail), offset=offset)
         compare_cache(gc, oc)
         keys, lens, count = gc.export()
-        return sorted(zip(keys[:count].tolist(), lens[:count].tolist())), gc.stats()
+        st = gc.stats()
+        st.pop("spec_chunks")  # a speed counter: how much was written ahead
+        return sorted(zip(keys[:count].tolist(), lens[:count].tolist())), st
 
 
 @pytest.mark.parametrize("key16", [False, True])
@@ -99,3 +101,43 @@ def test_the_library_takes_the_single_block_path():
             phase1[limit] = ms[1] * 1e3 / 20  # us per call
     assert phase1[64] < 3.0, phase1
     assert phase1[0] > 5.0, phase1
+
+
+@pytest.mark.parametrize("C", [1 * KiB, 4 * KiB, 64 * KiB])
+def test_write_through_never_changes_outputs(C):
+    # payloads of misses only (written ahead and used), then payloads mixing
+    # hits, in-call duplicates and misses (written ahead where they land, copied
+    # over elsewhere), under every write-through mode and both call paths
+    rng = np.random.default_rng(C)
+    fresh = iter(range(10_000, 20_000))
+    alphabet = [W.random_bytes(C, seed=300 + k) for k in range(8)]
+    calls = []
+    for k in range(10):
+        nch = int(rng.integers(1, 200))
+        if k % 3 == 0:  # misses only
+            parts = [W.random_bytes(C, seed=next(fresh)) for _ in range(nch)]
+        else:
+            parts = [alphabet[int(rng.integers(len(alphabet)))] if rng.random() < 0.5
+                     else W.random_bytes(C, seed=next(fresh)) for _ in range(nch)]
+        if rng.random() < 0.5:
+            parts.append(W.random_bytes(int(rng.integers(1, C)), seed=next(fresh)))
+        calls.append(torch.cat(parts))
+    exports = []
+    for mode in (0, 1, 2):
+        for small in (64, 0):
+            gc = Cache(4096 * C, C)
+            oc = oracle.OracleCache(4096 * C, C)
+            gc.debug_set(B.GLEAM_DEBUG_SPECULATE, mode)
+            gc.debug_set(B.GLEAM_DEBUG_SMALL_CALLS, small)
+            with gc:
+                for payload in calls:
+                    dedup_both(gc, oc, payload)
+                compare_cache(gc, oc)
+                st = gc.stats()
+                if mode == 1:
+                    assert st["spec_chunks"] > 0
+                if mode == 2:
+                    assert st["spec_chunks"] == 0
+                keys, lens, count = gc.export()
+                exports.append(sorted(zip(keys[:count].tolist(), lens[:count].tolist())))
+    assert all(e == exports[0] for e in exports)

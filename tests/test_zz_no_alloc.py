@@ -62,6 +62,9 @@ def test_noalloc_matches_the_allocating_call_on_two_calls_in_a_row():
         assert torch.cuda.mem_get_info()[0] == free_before  # no device allocation
 
         sa, sb = ca.stats(), cb.stats()
+        # spec_chunks is a speed counter of the write-through, not cache state
+        sa.pop("spec_chunks")
+        sb.pop("spec_chunks")
         assert sa == sb
         ka, la, na = ca.export()
         kb, lb, nb = cb.export()
