@@ -465,7 +465,6 @@ def run_gleam(args, rank, world, local_rank):
     torch.cuda.synchronize()
     st1 = cache.stats()  # the last warm-up step's counters (restored before it)
     evictions = st1["evictions"] - st0["evictions"]
-    spec_chunks = st1["spec_chunks"] - st0["spec_chunks"]
     r = results.cpu().numpy()
     assert (r[:, 0] == 0).all(), "a dedup call failed: %s" % r[r[:, 0] != 0][:3]
     miss_bytes = int(r[:, 5].sum())
@@ -476,9 +475,7 @@ def run_gleam(args, rank, world, local_rank):
     # algorithmic bytes: the fused fingerprint/probe/verify kernel reads the
     # payload once and the cached copy of every cache hit
     hit_cache_bytes = total - miss_bytes - hit_intra * C
-    # ... and writes twice every chunk it writes ahead (write-through of
-    # likely misses; C bytes per chunk, a tail counted whole)
-    kernel0_bytes = total + hit_cache_bytes + 2 * spec_chunks * C
+    kernel0_bytes = total + hit_cache_bytes
     pipeline_bytes = 2 * total  # payload read + hit bytes read + miss bytes written
 
     clocks = ClockSampler(local_rank)
@@ -502,6 +499,12 @@ def run_gleam(args, rank, world, local_rank):
         e1.record()
     torch.cuda.synchronize()
     step_ms = [e0.elapsed_time(e1) for e0, e1 in ev]
+    # the hash kernel also writes twice every chunk it writes ahead (write-
+    # through of likely misses; C bytes per chunk, a tail counted whole), as
+    # counted in the last timed step (each step starts from the snapshot's
+    # counters)
+    spec_chunks = cache.stats()["spec_chunks"] - st0["spec_chunks"]
+    kernel0_bytes += 2 * spec_chunks * C
     ms = sum(step_ms)
     if world > 1:
         dist.barrier()
