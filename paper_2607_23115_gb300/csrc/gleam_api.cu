@@ -459,8 +459,8 @@ void note_call(gleam_cache* c, uint64_t Ntot) {
 }
 
 // The write-through fields of a call's kernel arguments.  It needs the staged
-// hash (16-byte-aligned payloads, C a multiple of 32), device outputs with
-// 16-byte-aligned packed buffers, and 64-bit or KEY16 keys.  In the automatic
+// hash (16-byte-aligned payloads, C a multiple of 32), 16-byte-aligned packed
+// buffers (device or page-locked host memory), and 64-bit or KEY16 keys.  In the automatic
 // mode the host launches the write-through variant of the hash kernel when
 // the page-locked copy of the device state says it is on (as of the last call
 // that finished: a call or two late at most, which a heuristic can afford),
@@ -595,7 +595,9 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     if (d.skip_block >= grid) d.skip_block = grid - 1;
   }
   const bool fused = small_call(c, aligned, Ntot, nbytes, d.skip_block);
-  set_spec(c, &h, &d, aligned && packed_aligned && !d.plain_copy);
+  // host payloads too: a chunk written ahead then spares the pack a second
+  // read over the CPU-GPU link (managed memory stays out)
+  set_spec(c, &h, &d, aligned && packed_aligned && !chk.saw_managed());
 
   cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
   if (c->profile) {
