@@ -1186,7 +1186,7 @@ __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
-template <bool kSpec>
+template <bool kAhead>
 __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a) {
   extern __shared__ __align__(128) uint8_t small_smem[];
   // Device-resident payloads (16-byte aligned here) are prefetched into L2 at
@@ -1202,7 +1202,7 @@ __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a
   const unsigned long long nvb = (h.Ntot * 4 + kThreads - 1) / kThreads;
   for (unsigned long long vb = 0; vb < nvb; ++vb) {
     __syncthreads();  // the previous range's groups are done with the shared memory
-    staged_range<true, kSpec>(h, vb, small_smem);
+    staged_range<true, kAhead>(h, vb, small_smem);
   }
   __syncthreads();  // every chunk's probe outcome written (and its stage copies landed)
   resolve_rank(a, 1, 0);
@@ -1345,11 +1345,11 @@ cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream
 
 uint32_t small_call_groups() { return kSmallGroups; }
 
-template <bool kSpec>
+template <bool kAhead>
 cudaError_t launch_small(const HashArgs& h, const DedupArgs& a, cudaStream_t s) {
-  cudaFuncSetAttribute((const void*)k_small_call<kSpec>,
+  cudaFuncSetAttribute((const void*)k_small_call<kAhead>,
                        cudaFuncAttributeMaxDynamicSharedMemorySize, kSmallSmem);
-  k_small_call<kSpec><<<1, kThreads, kSmallSmem, s>>>(h, a);
+  k_small_call<kAhead><<<1, kThreads, kSmallSmem, s>>>(h, a);
   return cudaGetLastError();
 }
 

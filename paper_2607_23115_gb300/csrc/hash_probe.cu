@@ -258,24 +258,24 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
 }
 
 
-template <bool kProbe, bool kSpec>
+template <bool kProbe, bool kAhead>
 __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned long long nvb = (a.Ntot * 4 + kStagedThreads - 1) / kStagedThreads;
   for (unsigned long long vb = blockIdx.x; vb < nvb; vb += gridDim.x) {
     __syncthreads();  // the previous range's groups are done with the shared memory
-    staged_range<kProbe, kSpec>(a, vb, smem);
+    staged_range<kProbe, kAhead>(a, vb, smem);
   }
 }
 
-template <bool kProbe, bool kSpec>
+template <bool kProbe, bool kAhead>
 cudaError_t launch_staged(const HashArgs& a, cudaStream_t s) {
   // per device and cheap: set on every launch
-  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kSpec>,
+  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kAhead>,
                        cudaFuncAttributeMaxDynamicSharedMemorySize, kStagedSmem);
   const unsigned long long threads = a.Ntot * 4;
   const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
-  k_hash_probe_staged<kProbe, kSpec><<<sg, kStagedThreads, kStagedSmem, s>>>(a);
+  k_hash_probe_staged<kProbe, kAhead><<<sg, kStagedThreads, kStagedSmem, s>>>(a);
   return cudaGetLastError();
 }
 

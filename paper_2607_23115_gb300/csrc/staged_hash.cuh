@@ -145,9 +145,9 @@ __device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uin
 }
 
 // The chunks of block-sized range vb (blockDim.x / 4 consecutive chunks); the
-// shared memory holds one region of kGroupBytes per group.  kSpec: with the
-// write-through of likely misses.
-template <bool kProbe, bool kSpec = false>
+// shared memory holds one region of kGroupBytes per group.  kAhead: with the
+// write-through of likely misses (written ahead of the pack step).
+template <bool kProbe, bool kAhead = false>
 __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long long vb,
                                              uint8_t* smem) {
   const unsigned long long g = (vb * blockDim.x + threadIdx.x) >> 2;
@@ -195,10 +195,10 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   const uint8_t* q = nullptr;
   bool cmp = false;
   // write-through of a likely miss, decided once the prefix hint is known
-  const bool spec_try = kSpec && speculate && slots_used + g < a.nslots;
-  bool spec = false;
-  uint8_t* spk = nullptr;  // packed offset i*C of the payload
-  uint8_t* sar = nullptr;  // arena slot slots_used + g
+  const bool ahead_ok = kAhead && speculate && slots_used + g < a.nslots;
+  bool ahead = false;
+  uint8_t* ahead_pk = nullptr;  // packed offset i*C of the payload
+  uint8_t* ahead_ar = nullptr;  // arena slot slots_used + g
 
   unsigned long long acc = xlane_start(lane);
   // prologue: payload stages 0 .. kDepth-2
@@ -267,10 +267,10 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
       hint_slot = slots_used ? hint_lookup(a.hints, a.index_mask, hint, len, slots_used)
                              : kEmptySlot;
       cmp = hint_slot != kEmptySlot;
-      spec = spec_try && !cmp;  // no cached chunk begins like it: a likely miss
-      if (spec) {
-        spk = (a.count > 1 ? a.table[pid].packed : a.one.packed) + (g - base) * a.C;
-        sar = a.arena_w + (slots_used + g) * a.C;
+      ahead = ahead_ok && !cmp;  // no cached chunk begins like it: a likely miss
+      if (ahead) {
+        ahead_pk = (a.count > 1 ? a.table[pid].packed : a.one.packed) + (g - base) * a.C;
+        ahead_ar = a.arena_w + (slots_used + g) * a.C;
       }
       if (cmp) {
         q = a.arena + (unsigned long long)hint_slot * a.C;
@@ -292,7 +292,7 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
       diff |= d;
       if (diff) cmp = false;
     }
-    if (spec) {  // this lane's own pieces of stage t, to both destinations
+    if (ahead) {  // this lane's own pieces of stage t, to both destinations
       const uint32_t sb = sbytes(t);
 #pragma unroll
       for (int j = 0; j < kStage / 64; ++j) {
@@ -300,16 +300,16 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
         if (off < sb) {
           const uint4 v = *reinterpret_cast<const uint4*>(sp + off);
           const unsigned long long o = (unsigned long long)t * kStage + off;
-          __stcs(reinterpret_cast<uint4*>(spk + o), v);
-          __stcs(reinterpret_cast<uint4*>(sar + o), v);
+          __stcs(reinterpret_cast<uint4*>(ahead_pk + o), v);
+          __stcs(reinterpret_cast<uint4*>(ahead_ar + o), v);
         }
       }
     }
     __syncwarp(gmask);  // everyone is done with buffer t before it is refilled
   }
   cp_wait<0>();
-  if (spec && lane == 0)  // the bytes past the last whole stripe
-    for (uint32_t k = full; k < len; ++k) spk[k] = sar[k] = p[k];
+  if (ahead && lane == 0)  // the bytes past the last whole stripe
+    for (uint32_t k = full; k < len; ++k) ahead_pk[k] = ahead_ar[k] = p[k];
 
   unsigned long long h;
   if (ns) {
@@ -369,7 +369,7 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
     a.ch.src[g] = (unsigned long long)p;
     a.ch.pidx[g] = pid;
     a.ch.hint[g] = hint;
-    if (kSpec) a.ch.spec[g] = spec ? 1 : 0;
+    if (kAhead) a.ch.spec[g] = ahead ? 1 : 0;
     if (hit) a.ch.ent[g] = hit_slot;
   }
 }
