@@ -567,7 +567,10 @@ __device__ bool lru_evict(const DedupArgs& a, uint32_t G, uint32_t bid,
 __device__ __forceinline__ void post_minimum(const DedupArgs& a, uint32_t e, uint32_t g) {
   const unsigned peers = __match_any_sync(0xffffffffu, e);
   const uint32_t m = __reduce_max_sync(peers, e != 0xFFFFFFFFu ? ~g : 0u);
-  if (e != 0xFFFFFFFFu && (threadIdx.x & 31) == (uint32_t)(__ffs(peers) - 1))
+  // a group of many chunks (all-zero chunks, say) would queue its atomics on
+  // one address: skip the atomic when a smaller number is already posted
+  if (e != 0xFFFFFFFFu && (threadIdx.x & 31) == (uint32_t)(__ffs(peers) - 1) &&
+      ldcg_u32(&a.tbl[e].minv) < m)
     atomicMax(&a.tbl[e].minv, m);
 }
 
