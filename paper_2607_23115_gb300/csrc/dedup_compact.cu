@@ -961,7 +961,8 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
     // Every miss, by rank.  Warp gw owns the contiguous ranks [lo, hi): its
     // lanes fetch the metadata of 32 ranks at once, the whole warp copies the
     // 32 chunks one after the other to the packed output and their arena
-    // slots, then each lane inserts its own chunk (32 independent probes).
+    // slots (all but those the hash kernel already wrote there), then each
+    // lane inserts its own chunk (32 independent probes).
     const unsigned long long nw = (unsigned long long)G * kWarps;
     const unsigned long long gw = (unsigned long long)bid * kWarps + w;
     const unsigned long long lo = total * gw / nw, hi = total * (gw + 1) / nw;
