@@ -561,6 +561,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   h.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   h.ch = c->ch;
   h.ctl = c->ctl;
+  h.cache_empty = c->slots_bound == 0 ? 1u : 0u;  // an upper bound of the used slots
 
   DedupArgs d{};
   d.table = c->d_table;
@@ -1267,6 +1268,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   h.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   h.ch = ch;
   h.ctl = ctl;
+  h.cache_empty = c->slots_bound == 0 ? 1u : 0u;
 
   DedupArgs d{};
   d.one = one;

@@ -163,6 +163,7 @@ struct HashArgs {
   // to arena slot slots_used + g as it streams by
   uint32_t spec_mode;
   uint8_t* arena_w;                // the arena, for those writes
+  uint32_t cache_empty;            // the host knows the cache holds no chunk yet
   unsigned long long nslots;
 };
 

@@ -258,24 +258,25 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
 }
 
 
-template <bool kProbe, bool kAhead>
+template <bool kProbe, bool kAhead, bool kVerify>
 __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned long long nvb = (a.Ntot * 4 + kStagedThreads - 1) / kStagedThreads;
   for (unsigned long long vb = blockIdx.x; vb < nvb; vb += gridDim.x) {
     __syncthreads();  // the previous range's groups are done with the shared memory
-    staged_range<kProbe, kAhead>(a, vb, smem);
+    staged_range<kProbe, kAhead, kVerify>(a, vb, smem);
   }
 }
 
-template <bool kProbe, bool kAhead>
+template <bool kProbe, bool kAhead, bool kVerify>
 cudaError_t launch_staged(const HashArgs& a, cudaStream_t s) {
+  constexpr int smem = (kStagedThreads / 4) * group_bytes(kVerify);
   // per device and cheap: set on every launch
-  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kAhead>,
-                       cudaFuncAttributeMaxDynamicSharedMemorySize, kStagedSmem);
+  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kAhead, kVerify>,
+                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   const unsigned long long threads = a.Ntot * 4;
   const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
-  k_hash_probe_staged<kProbe, kAhead><<<sg, kStagedThreads, kStagedSmem, s>>>(a);
+  k_hash_probe_staged<kProbe, kAhead, kVerify><<<sg, kStagedThreads, smem, s>>>(a);
   return cudaGetLastError();
 }
 
@@ -602,8 +603,14 @@ cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
   }
 #if GLEAM_STAGED_HASH
   if (aligned && (a.C % 32 == 0 || a.Ntot == 1)) {
-    if (!probe) return launch_staged<false, false>(a, s);
-    return a.spec_mode ? launch_staged<true, true>(a, s) : launch_staged<true, false>(a, s);
+    // no cached copy can be streamed when only fingerprints are wanted or the
+    // cache is known to be empty: the variant without those buffers
+    if (!probe) return launch_staged<false, false, false>(a, s);
+    if (a.cache_empty)
+      return a.spec_mode ? launch_staged<true, true, false>(a, s)
+                         : launch_staged<true, false, false>(a, s);
+    return a.spec_mode ? launch_staged<true, true, true>(a, s)
+                       : launch_staged<true, false, true>(a, s);
   }
 #endif
   if (aligned && probe) k_hash_probe<true, true><<<grid, kHashThreads, 0, s>>>(a);

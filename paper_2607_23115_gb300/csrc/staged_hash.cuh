@@ -106,7 +106,13 @@ __device__ __forceinline__ bool group_equal(const uint8_t* p, const uint8_t* q, 
 #endif
 constexpr int kStage = 512;                                 // bytes per stage
 constexpr int kDepth = GLEAM_STAGE_DEPTH;                   // stages in flight
-constexpr int kGroupBytes = kDepth * 2 * kStage + 32;       // +32: bank skew
+// A group's stage buffers: kDepth stages of its chunk and, when it may
+// compare against a cached copy (verify), kDepth stages of that copy too
+// (+32: bank skew).
+__host__ __device__ constexpr int group_bytes(bool verify) {
+  return kDepth * (verify ? 2 : 1) * kStage + 32;
+}
+constexpr int kGroupBytes = group_bytes(true);
 constexpr int kStagedThreads = GLEAM_STAGED_THREADS;
 constexpr int kStagedSmem = (kStagedThreads / 4) * kGroupBytes;
 static_assert(kStage == (int)kPrefixBytes, "stage 0 must be the hinted prefix");
@@ -145,9 +151,12 @@ __device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uin
 }
 
 // The chunks of block-sized range vb (blockDim.x / 4 consecutive chunks); the
-// shared memory holds one region of kGroupBytes per group.  kAhead: with the
-// write-through of likely misses (written ahead of the pack step).
-template <bool kProbe, bool kAhead = false>
+// shared memory holds one region of group_bytes(kVerify) per group.  kAhead:
+// with the write-through of likely misses (written ahead of the pack step).
+// kVerify = false: no speculative verify and no buffers for a cached copy
+// (an empty cache has none to stream), so twice as many groups fit an SM; a
+// key+length candidate, if any, is still compared with direct loads.
+template <bool kProbe, bool kAhead = false, bool kVerify = true>
 __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long long vb,
                                              uint8_t* smem) {
   const unsigned long long g = (vb * blockDim.x + threadIdx.x) >> 2;
@@ -161,11 +170,12 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   const uint32_t lane = threadIdx.x & 3;
   const int gbase = threadIdx.x & 28;
   const unsigned gmask = 0xFu << gbase;
-  uint8_t* region = smem + (threadIdx.x >> 2) * kGroupBytes;
+  uint8_t* region = smem + (threadIdx.x >> 2) * group_bytes(kVerify);
   const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(region);
   // stage buffer t % kDepth: payload at [0, kStage), cached copy at [kStage, 2 kStage)
-  auto pay_s = [&](uint32_t t) { return sbase + (t % kDepth) * 2 * kStage; };
-  auto pay_p = [&](uint32_t t) { return region + (t % kDepth) * 2 * kStage; };
+  constexpr uint32_t kBuf = (kVerify ? 2 : 1) * kStage;  // one stage's buffers
+  auto pay_s = [&](uint32_t t) { return sbase + (t % kDepth) * kBuf; };
+  auto pay_p = [&](uint32_t t) { return region + (t % kDepth) * kBuf; };
 
   uint32_t pid = 0;
   const uint8_t* buf;
@@ -264,8 +274,8 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
       const unsigned long long b3 = group_shfl(acc, gmask, gbase + 3);
       hint = b0 ^ xrotl(b1, 16) ^ xrotl(b2, 32) ^ xrotl(b3, 48);
       // an empty cache has no hints to look up
-      hint_slot = slots_used ? hint_lookup(a.hints, a.index_mask, hint, len, slots_used)
-                             : kEmptySlot;
+      hint_slot = kVerify && slots_used ? hint_lookup(a.hints, a.index_mask, hint, len, slots_used)
+                                        : kEmptySlot;
       cmp = hint_slot != kEmptySlot;
       ahead = ahead_ok && !cmp;  // no cached chunk begins like it: a likely miss
       if (ahead) {
