@@ -331,7 +331,8 @@ int gleam_cache_debug_insert(gleam_cache_t* cache, uint64_t key, const void* d_b
  * skips the copies of every miss whose rank puts it exactly there (a payload,
  * or a run of payloads, of misses only) and copies the others over (for
  * payloads in host memory this also spares the second read over the link).
- * It needs 16-byte-aligned payloads and packed buffers.  0 = automatic
+ * It needs 16-byte-aligned payloads and packed buffers, chunks of at least
+ * 512 bytes and 64-bit or KEY16 keys (not GLEAM_PAPER_IDS).  0 = automatic
  * (default: on while at least half of the chunks written ahead are used,
  * retried every 256 calls once off), 1 = always, 2 = never.  Only the speed
  * changes: every output is the same either way. */
