@@ -57,7 +57,8 @@ struct gleam_cache {
   DevCtl* ctl = nullptr;
   uint32_t* bcount = nullptr;
   gleam_result_t* d_result = nullptr;
-  gleam_result_t* h_result = nullptr;  // pinned
+  gleam_result_t* h_result = nullptr;      // page-locked, mapped: gleam_dedup_copy's result
+  gleam_result_t* h_result_dev = nullptr;  // its device address
   int coop_max_blocks = 0;
   int pack_max_blocks = 0;  // pack kernel: all co-resident blocks
   cudaEvent_t done = nullptr;
@@ -503,7 +504,8 @@ int enqueue_index_check(gleam_cache* c, const DedupArgs& d, cudaStream_t s) {
 // Enqueues one dedup call over `count` payloads on stream s, ordered after
 // the cache's previous call.  Caller holds c->mu and the device.
 int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
-            gleam_result_t* d_total, cudaStream_t s, bool host_payloads = false) {
+            gleam_result_t* d_total, cudaStream_t s, bool host_payloads = false,
+            gleam_result_t* own_total = nullptr) {
   if (count == 0) return GLEAM_OK;
   if (count > 0xFFFFFFFEull) return GLEAM_ERR_INVALID_ARG;
   PtrChecker chk(c->device);
@@ -584,7 +586,9 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   d.tbl_mask = tcap - 1;
   d.bcount = c->bcount;
   d.ctl = c->ctl;
-  d.total = d_total ? d_total : c->d_result;
+  // the call's result: the caller's device struct, else the library's own
+  // (for gleam_dedup_copy, its page-locked one: read with no copy back)
+  d.total = d_total ? d_total : own_total ? own_total : c->d_result;
   d.ncalls = ncalls;
   d.wait_ns = c->wait_ns;
   set_lru(c, &d, Ntot);
@@ -706,7 +710,8 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   step(cudaMalloc(&c->spec_state, 2 * sizeof(uint32_t)));
   step(cudaHostAlloc(&c->spec_mirror, sizeof(uint32_t), cudaHostAllocMapped));
   step(cudaMalloc(&c->d_result, sizeof(gleam_result_t)));
-  step(cudaMallocHost(&c->h_result, sizeof(gleam_result_t)));
+  step(cudaHostAlloc(&c->h_result, sizeof(gleam_result_t), cudaHostAllocMapped));
+  step(cudaHostGetDevicePointer(&c->h_result_dev, c->h_result, 0));
   step(cudaEventCreateWithFlags(&c->done, cudaEventDisableTiming));
   step(cudaEventCreateWithFlags(&c->table_copied, cudaEventDisableTiming));
   if (rc == GLEAM_OK) {
@@ -822,14 +827,14 @@ int64_t gleam_dedup_copy(gleam_cache_t* c, const void* d_buf, size_t n, uint32_t
   std::lock_guard<std::mutex> lk(c->mu);
   DeviceGuard g(c->device);
   const gleam_payload_t p = make_payload(d_buf, n, d_hit_mask, d_miss_idx, d_miss_bytes, nullptr);
-  int rc = enqueue(c, &p, 1, c->d_result, nullptr);
+  // the last kernel writes the result straight into page-locked host memory
+  int rc = enqueue(c, &p, 1, nullptr, nullptr, false, c->h_result_dev);
   if (rc != GLEAM_OK) return rc;
-  rc = cuda_err(cudaMemcpyAsync(c->h_result, c->d_result, sizeof(gleam_result_t),
-                                cudaMemcpyDeviceToHost, nullptr));
-  if (rc == GLEAM_OK) rc = cuda_err(cudaStreamSynchronize(nullptr));
+  rc = cuda_err(cudaStreamSynchronize(nullptr));
   if (rc != GLEAM_OK) return rc;
-  if (c->h_result->status != 0) return c->h_result->status;
-  return (int64_t)c->h_result->n_miss;
+  const volatile gleam_result_t* r = c->h_result;
+  if (r->status != 0) return r->status;
+  return (int64_t)r->n_miss;
 }
 
 int gleam_dedup_copy_host_batch(gleam_cache_t* c, const gleam_payload_t* payloads, size_t count,
