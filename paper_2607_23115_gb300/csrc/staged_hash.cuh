@@ -84,6 +84,37 @@ __device__ __forceinline__ bool group_equal(const uint8_t* p, const uint8_t* q, 
   return diff == 0;
 }
 
+// Byte equality of payload chunk p and cached chunk q over len bytes by the
+// nl lanes of wmask (a prefix of the warp; this lane is wl): 8-byte words
+// strided across the lanes, kBatch of them per lane in flight, leaving early
+// once any word differs.  Eight groups' worth of lanes take a 64 KiB compare
+// in 32 rounds of loads where one group's four lanes take 256.
+__device__ __forceinline__ bool lanes_equal(const uint8_t* p, const uint8_t* q, uint32_t len,
+                                            unsigned wmask, uint32_t wl, uint32_t nl) {
+  const uint32_t nw = len >> 3;
+  for (uint32_t w0 = 0; w0 < nw; w0 += kBatch * nl) {
+    unsigned long long diff = 0;
+#pragma unroll
+    for (int u = 0; u < kBatch; ++u) {
+      const uint32_t w = w0 + u * nl + wl;
+      if (w < nw) diff |= load_word<true>(p + 8ull * w) ^ load_arena_word(q + 8ull * w);
+    }
+    if (__any_sync(wmask, diff != 0)) return false;
+  }
+  bool d = false;
+  for (uint32_t k = (nw << 3) + wl; k < len; k += nl) d |= p[k] != q[k];
+  return !__any_sync(wmask, d);
+}
+
+// Lanes of this warp whose groups hold a chunk of range vb (g < Ntot): a
+// prefix of the warp, since chunks are numbered in thread order.  Called by a
+// lane of such a group.
+__device__ __forceinline__ unsigned present_lanes(unsigned long long vb, unsigned long long Ntot) {
+  const unsigned long long t0 = vb * blockDim.x + (threadIdx.x & ~31u);
+  const unsigned long long k = 4 * Ntot - t0;
+  return k >= 32 ? 0xffffffffu : (1u << k) - 1;
+}
+
 // ---------------------------------------------------------------------------
 // Staged variant for 16-byte-aligned payloads.  Each 4-thread group streams
 // its chunk through shared memory in kStage-byte stages with asynchronous
@@ -348,29 +379,63 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   }
 
   const unsigned long long key = a.key16 ? (h & 0xFFFFULL) : h;
-  unsigned long long pos = mix64(key) & a.index_mask;
   bool hit = false, cand = false;
   uint32_t hit_slot = kEmptySlot;
-  for (unsigned long long probe = 0; slots_used && probe <= a.index_mask; ++probe) {
-    const IndexEntry e = a.index[pos];
-    if (e.slot == kEmptySlot) break;
-    if (e.key == key && e.len == len) {
-      cand = true;
-      if (e.slot >= slots_used) {
-        if (lane == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-      } else if (e.slot == hint_slot) {
-        if (spec_equal) {
-          hit = true;
-          hit_slot = e.slot;
+  if (slots_used) {
+    // The linear probe, in order.  A key+length candidate other than the
+    // verified hint is compared by the whole warp: each group walks its probe
+    // up to its next such candidate, then the warp compares the pending ones,
+    // one group's at a time, and the groups whose candidate differs walk on.
+    const unsigned wmask = present_lanes(vb, a.Ntot);
+    const uint32_t wl = threadIdx.x & 31, nl = __popc(wmask);
+    unsigned long long pos = mix64(key) & a.index_mask, probe = 0;
+    bool done = false;
+    for (;;) {
+      uint32_t want = kEmptySlot;  // a candidate for the warp to compare
+      while (!done) {
+        if (probe > a.index_mask) {
+          done = true;
           break;
         }
-      } else if (group_equal<true>(p, a.arena + (uint64_t)e.slot * a.C, len, lane, gmask)) {
-        hit = true;
-        hit_slot = e.slot;
-        break;
+        const IndexEntry e = a.index[pos];
+        if (e.slot == kEmptySlot) {
+          done = true;
+          break;
+        }
+        pos = (pos + 1) & a.index_mask;
+        ++probe;
+        if (e.key == key && e.len == len) {
+          cand = true;
+          if (e.slot >= slots_used) {
+            if (lane == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+          } else if (e.slot == hint_slot) {
+            if (spec_equal) {
+              hit = true;
+              hit_slot = e.slot;
+              done = true;
+            }
+          } else {
+            want = e.slot;
+            break;
+          }
+        }
+      }
+      const unsigned pend = __ballot_sync(wmask, want != kEmptySlot) & 0x11111111u;
+      if (!pend) break;
+      for (unsigned m = pend; m; m &= m - 1) {
+        const int src = __ffs(m) - 1;
+        const uint8_t* ps = reinterpret_cast<const uint8_t*>(
+            __shfl_sync(wmask, reinterpret_cast<unsigned long long>(p), src));
+        const uint32_t slot = __shfl_sync(wmask, want, src);
+        const uint32_t ls = __shfl_sync(wmask, len, src);
+        const bool eq = lanes_equal(ps, a.arena + (uint64_t)slot * a.C, ls, wmask, wl, nl);
+        if (gbase == src && eq) {
+          hit = true;
+          hit_slot = slot;
+          done = true;
+        }
       }
     }
-    pos = (pos + 1) & a.index_mask;
   }
   if (lane == 0) {
     a.ch.status[g] = hit ? kHit0 : (cand ? kMissCand : kMissNoCand);

@@ -224,6 +224,37 @@ def test_snapshot_restore_repeats_identically():
 
 
 @pytest.mark.parametrize("key16", [False, True])
+@pytest.mark.parametrize("C", [1 * KiB, 64 * KiB])
+def test_decoys_ahead_of_the_genuine_entry(C, key16):
+    """Every chunk's probe meets planted decoys first: entries under the
+    chunk's own key whose bytes differ in the first byte, past the prefix or
+    in the last byte (for the ragged tail chunk, in its bytes past the last
+    whole word).  Each decoy must be compared and rejected and the genuine
+    entry, inserted after them, found.  13 whole chunks and a tail leave the
+    last group of chunks of a warp part-filled."""
+    flags = B.GLEAM_KEY16 if key16 else 0
+    m = 13
+    X = [W.random_bytes(C, seed=800 + i) for i in range(m)]
+    tail = W.random_bytes(C // 3, seed=799)
+    gc, oc = _pair(256 * C, C, flags)
+    with gc:
+        for x in X + [tail]:
+            key = oracle.xxh64(x.numpy())
+            for pos in (0, C // 2 + 3, x.numel() - 1):
+                if pos >= x.numel():
+                    continue
+                d = x.clone()
+                d[pos] ^= 0x40
+                assert oc.debug_insert(key, d.numpy()) == 0
+                gc.debug_insert(key, d.to(DEV))
+        assert dedup_both(gc, oc, torch.cat(X + [tail])) == m + 1
+        order = np.random.default_rng(C).permutation(m)
+        assert dedup_both(gc, oc, torch.cat([X[i] for i in order] + [tail])) == 0
+        compare_cache(gc, oc)
+        assert gc.stats()["hits_cache"] == m + 1
+
+
+@pytest.mark.parametrize("key16", [False, True])
 def test_prefix_hint_pointing_at_the_wrong_chunk(key16):
     """Cached chunks A = X|Y1 and B = X|Y2 share their first 2 KiB, so the
     prefix hint of X|Y2 may name A; the result must still be a hit on B, and
