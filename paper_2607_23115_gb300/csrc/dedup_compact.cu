@@ -901,10 +901,33 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
   if (ok) {
     unsigned long long n_hc = 0, n_hi = 0, n_rej = 0, n_bytes = 0, n_sbytes = 0;
     uint32_t n_spec = 0, n_spec_used = 0;  // write-through: chunks written ahead, used
-    for (unsigned long long t = (unsigned long long)bid * kThreads; t < N;
-         t += (unsigned long long)G * kThreads) {
-      const uint32_t g = (uint32_t)(t + threadIdx.x);
-      const bool valid = t + threadIdx.x < N;
+    // Each warp classifies a contiguous range of chunks (whole 32-chunk
+    // steps), so that its steps mostly fall in one payload: the counters of a
+    // payload are summed in the warp over its steps and added once where the
+    // warp leaves the payload, instead of once per step by every warp on the
+    // same few addresses (a one-payload call of a million chunks would queue
+    // ~10^5 atomics on one result).
+    const unsigned long long nsteps = ((unsigned long long)N + 31) / 32;
+    const unsigned long long cw_n = (unsigned long long)G * kWarps;
+    const unsigned long long cw = (unsigned long long)bid * kWarps + w;
+    const unsigned long long c_lo = nsteps * cw / cw_n * 32;
+    const unsigned long long c_hi = min((unsigned long long)N, nsteps * (cw + 1) / cw_n * 32);
+    gleam_result_t* acc_res = nullptr;  // the payload whose counters the warp holds
+    unsigned long long acc_hc = 0, acc_hi = 0, acc_miss = 0, acc_rej = 0, acc_len = 0;
+    auto flush = [&]() {
+      if (acc_res && lane == 0) {
+        if (acc_hc) atomicAdd((unsigned long long*)&acc_res->n_hit_cache, acc_hc);
+        if (acc_hi) atomicAdd((unsigned long long*)&acc_res->n_hit_intra, acc_hi);
+        if (acc_miss) atomicAdd((unsigned long long*)&acc_res->n_miss, acc_miss);
+        if (acc_rej) atomicAdd((unsigned long long*)&acc_res->verify_rejects, acc_rej);
+        if (acc_len) atomicAdd((unsigned long long*)&acc_res->miss_bytes, acc_len);
+      }
+      acc_res = nullptr;
+      acc_hc = acc_hi = acc_miss = acc_rej = acc_len = 0;
+    };
+    for (unsigned long long t = c_lo; t < c_hi; t += 32) {
+      const uint32_t g = (uint32_t)(t + lane);
+      const bool valid = t + lane < c_hi;
       const uint32_t r = valid ? ldcg_u32(&ch.res[g]) : 0u;
       const uint32_t p = valid ? ch.pidx[g] : 0xFFFFFFFFu;
       const bool miss = valid && (r & kResLeader);
@@ -951,13 +974,26 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
       const uint32_t bits = __reduce_or_sync(mpeers, bit);
       if (mw && lane == (uint32_t)(__ffs(mpeers) - 1)) atomicOr((uint32_t*)mw, bits);
       const unsigned peers = __match_any_sync(0xffffffffu, res ? p : 0xFFFFFFFFu);
-      const bool lead = res && lane == (uint32_t)(__ffs(peers) - 1);
-      add_in_group((unsigned long long*)(lead ? &res->n_hit_cache : nullptr), peers, hc);
-      add_in_group((unsigned long long*)(lead ? &res->n_hit_intra : nullptr), peers, hi2);
-      add_in_group((unsigned long long*)(lead ? &res->n_miss : nullptr), peers, miss);
-      add_in_group((unsigned long long*)(lead ? &res->verify_rejects : nullptr), peers, rej);
-      add_in_group((unsigned long long*)(lead ? &res->miss_bytes : nullptr), peers, len);
+      if (peers == 0xffffffffu && res) {  // the whole step in one payload that has a result
+        if (res != acc_res) {
+          flush();
+          acc_res = res;
+        }
+        acc_hc += __reduce_add_sync(0xffffffffu, (uint32_t)hc);
+        acc_hi += __reduce_add_sync(0xffffffffu, (uint32_t)hi2);
+        acc_miss += __reduce_add_sync(0xffffffffu, (uint32_t)miss);
+        acc_rej += __reduce_add_sync(0xffffffffu, (uint32_t)rej);
+        acc_len += __reduce_add_sync(0xffffffffu, len);
+      } else {  // payload boundaries: one atomic per group of lanes per counter
+        const bool lead = res && lane == (uint32_t)(__ffs(peers) - 1);
+        add_in_group((unsigned long long*)(lead ? &res->n_hit_cache : nullptr), peers, hc);
+        add_in_group((unsigned long long*)(lead ? &res->n_hit_intra : nullptr), peers, hi2);
+        add_in_group((unsigned long long*)(lead ? &res->n_miss : nullptr), peers, miss);
+        add_in_group((unsigned long long*)(lead ? &res->verify_rejects : nullptr), peers, rej);
+        add_in_group((unsigned long long*)(lead ? &res->miss_bytes : nullptr), peers, len);
+      }
     }
+    flush();
     // Every miss, by rank.  Warp gw owns the contiguous ranks [lo, hi): its
     // lanes fetch the metadata of 32 ranks at once, the whole warp copies the
     // 32 chunks one after the other to the packed output and their arena
