@@ -31,7 +31,7 @@ def _rank(rank, world, port, out):
 
 def test_two_gloo_replicas_take_the_max_time_and_sum_the_payload():
     world = 2
-    mgr = mp.Manager()
+    mgr = mp.get_context("spawn").Manager()  # no fork of a process that may hold threads
     out = mgr.dict()
     mp.spawn(_rank, args=(world, _free_port(), out), nprocs=world, join=True)
     for r in range(world):
