@@ -20,9 +20,10 @@ with the base weights, and 10% of the chunks carrying one flipped bit (a
 fine-tuned variant), so ~90% of chunks hit and ~10% miss and are inserted.
 
 Printed line: payload GB/s (value), the pipeline's minimal-traffic roofline
-fraction (payload read + cached bytes read for hits + miss bytes written =
-2 x payload), the dominant kernel's roofline, the oracle's CPU rate on a
-bounded sample, the end-to-end rate with host buffers, clocks.
+fraction (payload read + cached bytes read for cache hits + miss bytes
+written: 2 x payload when no chunk repeats within the call), the dominant
+kernel's roofline, the oracle's CPU rate on a bounded sample, the end-to-end
+rate with host buffers, clocks.
 """
 from __future__ import annotations
 
@@ -476,7 +477,10 @@ def run_gleam(args, rank, world, local_rank):
     # payload once and the cached copy of every cache hit
     hit_cache_bytes = total - miss_bytes - hit_intra * C
     kernel0_bytes = total + hit_cache_bytes
-    pipeline_bytes = 2 * total  # payload read + hit bytes read + miss bytes written
+    # the pipeline's minimal traffic: payload read once, the cached copy of
+    # every cache hit read, the miss bytes written once (an in-call duplicate
+    # needs neither: its first occurrence is part of the payload read)
+    pipeline_bytes = total + hit_cache_bytes + miss_bytes
 
     clocks = ClockSampler(local_rank)
     if not args.profile_launches:
