@@ -682,20 +682,27 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
         }
       }
       uint32_t todo = __ballot_sync(0xffffffffu, need);
+      // every lane fetches its own chunk's operands at once, so that each
+      // compare below waits for its bytes only, not for their addresses first
+      unsigned long long xs = 0, ys = 0;
+      uint32_t ln = 0;
+      if (need) {
+        xs = ch.src[g];
+        ys = ch.src[m];
+        ln = ch.len[g];
+      }
       while (todo) {
         const int j = __ffs(todo) - 1;
         todo &= todo - 1;
-        const uint32_t gg = base + j;
-        const uint32_t mm = __shfl_sync(0xffffffffu, m, j);
-        const uint8_t* x = reinterpret_cast<const uint8_t*>(ch.src[gg]);
-        const uint8_t* y = reinterpret_cast<const uint8_t*>(ch.src[mm]);
-        const uint32_t len = ch.len[gg];
+        const uint8_t* x = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, xs, j));
+        const uint8_t* y = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, ys, j));
+        const uint32_t len = __shfl_sync(0xffffffffu, ln, j);
         const bool vec = (((uintptr_t)x | (uintptr_t)y) & 15) == 0;
         const bool eq = warp_equal(x, y, len, vec);
         if (lane == (uint32_t)j) {
           if (eq) {
-            ch.ent[gg] = mm;  // the leader, for the hit's classification
-            ch.res[gg] = kResDup;
+            ch.ent[g] = m;  // the leader, for the hit's classification
+            ch.res[g] = kResDup;
           } else {
             atomicAdd(&a.ctl->unres[round % 3], 1u);
             stay = true;
