@@ -475,6 +475,8 @@ def run_gleam(args, rank, world, local_rank):
         assert n_miss == wl.expect_misses, (n_miss, wl.expect_misses)
     # algorithmic bytes: the fused fingerprint/probe/verify kernel reads the
     # payload once and the cached copy of every cache hit
+    # (in-call duplicates counted as whole chunks: exact for every workload
+    # here, none of which repeats a short last chunk within a call)
     hit_cache_bytes = total - miss_bytes - hit_intra * C
     kernel0_bytes = total + hit_cache_bytes
     # the pipeline's minimal traffic: payload read once, the cached copy of
