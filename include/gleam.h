@@ -251,9 +251,13 @@ int gleam_dedup_copy_host_batch(gleam_cache_t* cache, const gleam_payload_t* pay
  * the library holds that array until the process exits.
  *  - Payloads of more than GLEAM_NOALLOC_MAX_CHUNKS chunks (ceil(n / C)) are
  *    rejected with GLEAM_ERR_INVALID_ARG; use gleam_dedup_copy_async for them.
- *  - The first call on a device looks the array's device address up (which
- *    may load the library's device code on that GPU); make that first call
- *    before any stream capture.
+ *  - gleam_cache_create[_ex] looks the array's device address up, on the
+ *    cache's GPU, while it allocates the cache (the lookup may load the
+ *    library's device code on that GPU, which is when the array is
+ *    allocated), so that no call does any set-up.
+ *  - Test hooks of gleam_cache_debug_set apply as to the other calls; kernel
+ *    timing (gleam_cache_profile) does not cover this call: it records no
+ *    events, so that it creates nothing.
  *  - All calls on a GPU, from every cache, share the one array and it keeps
  *    the last call's contents (the call clears what must start at zero).
  *    Calls that overlap on the GPU race and give wrong results: order them
@@ -351,8 +355,9 @@ int gleam_cache_snapshot(gleam_cache_t* cache, gleam_snapshot_t** out);
 int gleam_cache_restore(gleam_cache_t* cache, const gleam_snapshot_t* snap);
 void gleam_snapshot_destroy(gleam_snapshot_t* snap);
 
-/* Kernel timing for benchmarks.  While enabled, every dedup call records CUDA
- * events on its own stream around its two phases: phase 0 is the kernel that
+/* Kernel timing for benchmarks.  While enabled, every dedup call (except
+ * gleam_dedup_copy_noalloc) records CUDA events on its own stream around its
+ * two phases: phase 0 is the kernel that
  * fingerprints, probes and verifies; phase 1 is the two kernels that resolve
  * duplicates and rank the misses, then compact, pack and insert; a small
  * call that runs as one single-block kernel (GLEAM_DEBUG_SMALL_CALLS) counts

@@ -77,6 +77,10 @@ struct gleam_cache {
   unsigned long long wait_ns = 4000000000ULL;
   int skip_block = -1;
 
+  // device address of the allocation-free call's scratch array on this GPU,
+  // looked up when the cache is created
+  uint8_t* na_scratch = nullptr;
+
   // kernel timing (gleam_cache_profile)
   bool profile = false;
   std::vector<cudaEvent_t> ev_pool;  // 3 events per recorded call
@@ -645,6 +649,10 @@ gleam_payload_t make_payload(const void* d_buf, size_t n, uint32_t* d_hit_mask,
   return p;
 }
 
+// Device address of the allocation-free call's scratch array on the current
+// GPU (defined with the entry point at the end of this file).
+int noalloc_scratch(uint8_t** out);
+
 }  // namespace
 
 extern "C" {
@@ -748,6 +756,11 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     step(cudaEventRecord(c->table_copied, nullptr));
     step(cudaDeviceSynchronize());
   }
+  // The allocation-free call's scratch array is looked up here, where the
+  // device is current and allocating is allowed: the lookup may load this
+  // file's device code on the GPU, which allocates the array.
+  if (rc == GLEAM_OK) rc = noalloc_scratch(&c->na_scratch);
+  if (rc == GLEAM_OK) step(load_hash_kernels());
   if (rc != GLEAM_OK) {
     destroy_cache(c);
     return rc;
@@ -1191,22 +1204,13 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[kNaBytes];
 
 namespace {
 
-constexpr int kNaMaxDevices = 128;
-std::mutex g_na_mu;
-uint8_t* g_na_ptr[kNaMaxDevices] = {};
-
-// Device address of g_noalloc_scratch on `device` (which must be current),
-// looked up once per device.
-int noalloc_scratch(int device, uint8_t** out) {
-  if (device < 0 || device >= kNaMaxDevices) return GLEAM_ERR_INVALID_ARG;
-  std::lock_guard<std::mutex> lk(g_na_mu);
-  if (g_na_ptr[device] == nullptr) {
-    void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess || p == nullptr) return cuda_err(e == cudaSuccess ? cudaErrorUnknown : e);
-    g_na_ptr[device] = static_cast<uint8_t*>(p);
-  }
-  *out = g_na_ptr[device];
+// Looks the array up on the current device.  Every cache keeps its own copy
+// of the address, so nothing outlives the context the cache was made in.
+int noalloc_scratch(uint8_t** out) {
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (e != cudaSuccess || p == nullptr) return cuda_err(e == cudaSuccess ? cudaErrorUnknown : e);
+  *out = static_cast<uint8_t*>(p);
   return GLEAM_OK;
 }
 
@@ -1224,13 +1228,13 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   DeviceGuard g(c->device);
   if ((uint64_t)c->coop_max_blocks + 1 > kNaBlocks) return GLEAM_ERR_INVALID_ARG;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  uint8_t* base = nullptr;
-  int rc = noalloc_scratch(c->device, &base);
-  if (rc != GLEAM_OK) return rc;
+  uint8_t* const base = c->na_scratch;
+  if (base == nullptr) return GLEAM_ERR_INTERNAL;
 
   const gleam_payload_t p = make_payload(d_buf, n, d_hit_mask, d_miss_idx, d_miss_bytes, d_result);
   PtrChecker chk(c->device);
   PayloadDesc one{};
+  int rc;
   if ((rc = describe(c, chk, p, &one)) != GLEAM_OK) return rc;
   const bool aligned = reinterpret_cast<uintptr_t>(one.buf) % 16 == 0;
 
@@ -1299,14 +1303,19 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.wait_ns = c->wait_ns;
   d.plain_copy = chk.saw_managed() ? 1u : 0u;
   set_lru(c, &d, N);
-  d.skip_block = -1;
+  d.skip_block = c->skip_block;  // the test hook applies to this one call, as in enqueue()
+  c->skip_block = -1;
+  int grid = dedup_grid(c, N, n);
+  if (d.skip_block >= 0) {
+    grid = std::max(grid, std::min(2, c->coop_max_blocks));  // someone must be left waiting
+    if (d.skip_block >= grid) d.skip_block = grid - 1;
+  }
   set_spec(c, &h, &d,
            aligned && reinterpret_cast<uintptr_t>(one.packed) % 16 == 0 && !d.plain_copy);
-  if (small_call(c, aligned, N, n, -1)) {
+  if (small_call(c, aligned, N, n, d.skip_block)) {
     if ((rc = cuda_err(launch_small_call(h, d, s))) != GLEAM_OK) return rc;
   } else {
     if ((rc = cuda_err(launch_hash(h, aligned, s))) != GLEAM_OK) return rc;
-    const int grid = dedup_grid(c, N, n);
     if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, N, n), s))) != GLEAM_OK) return rc;
   }
   note_call(c, N);

@@ -215,6 +215,9 @@ constexpr uint32_t kLruBins = 65536;
 constexpr uint32_t kPaperMinCached = 1024;
 
 cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s);
+// Loads the hash kernels' device code on the current GPU (cache creation does
+// it, so that no later call loads code, which allocates device memory).
+cudaError_t load_hash_kernels();
 // The cooperative resolve/rank kernel on `grid` blocks, then the pack kernel
 // (masks, indices, copies, inserts, publish) on `pack_grid` blocks.
 cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s);

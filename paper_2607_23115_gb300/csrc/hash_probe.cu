@@ -583,6 +583,13 @@ Md5Table md5_table() {
 
 }  // namespace
 
+// Loads this file's kernels on the current device (a query of one of them
+// loads the module that holds them all, when the runtime loads modules lazily).
+cudaError_t load_hash_kernels() {
+  cudaFuncAttributes fa;
+  return cudaFuncGetAttributes(&fa, k_hash_probe_staged<true, false, true>);
+}
+
 cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
   if (a.Ntot == 0) return cudaSuccess;
   const unsigned long long threads = a.Ntot * 4;
