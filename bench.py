@@ -63,6 +63,8 @@ def parse_args():
     p.add_argument("--e2e-steps", type=int, default=5)
     p.add_argument("--profile-launches", action="store_true",
                    help="few steps, no baselines: for an ncu launch list")
+    p.add_argument("--no-configs", action="store_true",
+                   help="skip the other configurations (the `configs` object)")
     return p.parse_args()
 
 
@@ -410,159 +412,294 @@ def committed_traffic(workload_name):
 # the GPU arm
 # ---------------------------------------------------------------------------
 
-def run_gleam(args, rank, world, local_rank):
-    import numpy as np
-    import torch
-    import torch.distributed as dist
-
-    from paper_2607_23115_gb300 import binding as B
-    from paper_2607_23115_gb300.cache import Cache, DedupOutputs, fingerprint
-
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    do_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_launches
-    wl = build_workload(args.workload, dev, args.cpu_sample_bytes if do_cpu else 0)
+def workload_config(wl):
+    """The `config` object of both arms: what defines the workload (the
+    calls each arm makes to process it are described under `run`)."""
     C, up = wl.C, wl.up
-    nt = len(up.sizes)
-    total = up.total_bytes
-    nchunks = sum((s + C - 1) // C for s in up.sizes)
+    return {"workload": wl.name, "description": wl.desc,
+            "payload_bytes_per_step": up.total_bytes, "payloads_per_step": len(up.sizes),
+            "chunk_bytes": C, "chunks_per_step": sum((s + C - 1) // C for s in up.sizes),
+            "misses_per_step": wl.expect_misses, "cache_capacity_bytes": wl.capacity,
+            "key16": bool(wl.flags & 1), "paper_ids": bool(wl.flags & 4),
+            "evict_lru": bool(wl.flags & 8)}
 
-    cache = Cache(wl.capacity, C, wl.flags)
-    cache.reserve(max(nchunks, max((sum(t.numel() for t in b) + C - 1) // C + len(b)
-                                   for b in wl.prefill) if wl.prefill else 1))
-    outs = [DedupOutputs.alloc(s, C, dev) for s in up.sizes]
-    results = torch.zeros(nt, B.RESULT_WORDS, dtype=torch.int64, device=dev)
-    bufs = [up.payload(k) for k in range(nt)]
-    chunk_slots = [torch.zeros(max(1, (s + C - 1) // C), dtype=torch.int32, device=dev)
-                   for s in up.sizes]
-    items = cache.batch_items(bufs, outs, [results[k] for k in range(nt)], chunk_slots)
-    total_res = torch.zeros(B.RESULT_WORDS, dtype=torch.int64, device=dev)
 
-    def one_pass():
-        cache.dedup_batch(None, items=items, total=total_res, stream=None)
+class Run:
+    """One workload prepared on the GPU: the cache (crafted entries, prefill
+    calls, perturbation done), the step's payloads and outputs, a snapshot to
+    restore before every step."""
 
-    # cache state before the first step: crafted entries, prefill calls, perturbation
-    for orig, row in wl.crafted:
-        key = int(fingerprint(orig, 0).cpu().numpy().view(np.uint64)[0])
-        cache.debug_insert(key, row)
-    for batch in wl.prefill:
-        pouts = [DedupOutputs.alloc(t.numel(), C, dev) for t in batch]
-        cache.dedup_batch(batch, pouts)
+    def __init__(self, wl, dev, extra_flags=()):
+        import torch
+        from paper_2607_23115_gb300 import binding as B
+        from paper_2607_23115_gb300.cache import DedupOutputs
+
+        self.wl, self.dev = wl, dev
+        C, up = wl.C, wl.up
+        self.nt = len(up.sizes)
+        self.total = up.total_bytes
+        self.nchunks = sum((s + C - 1) // C for s in up.sizes)
+        self.outs = [DedupOutputs.alloc(s, C, dev) for s in up.sizes]
+        self.results = torch.zeros(self.nt, B.RESULT_WORDS, dtype=torch.int64, device=dev)
+        self.bufs = [up.payload(k) for k in range(self.nt)]
+        self.chunk_slots = [torch.zeros(max(1, (s + C - 1) // C), dtype=torch.int32, device=dev)
+                            for s in up.sizes]
+        # the cache, and one more per extra creation flag, all filled before the
+        # perturbation
+        self.cache = self._filled_cache(wl.flags)
+        self.extra = {f: self._filled_cache(wl.flags | f) for f in extra_flags}
+        self.items = self.cache.batch_items(self.bufs, self.outs,
+                                            [self.results[k] for k in range(self.nt)],
+                                            self.chunk_slots)
+        self.total_res = torch.zeros(B.RESULT_WORDS, dtype=torch.int64, device=dev)
+        if wl.after_prefill:
+            wl.after_prefill()
         torch.cuda.synchronize()
-        del pouts
-    if wl.after_prefill:
-        wl.after_prefill()
-    torch.cuda.synchronize()
-    snap = cache.snapshot()
-    flush = torch.empty(256 * MiB, dtype=torch.uint8, device=dev) if wl.flush_l2 else None
+        self.snap = self.cache.snapshot()
+        self.extra_snap = {f: c.snapshot() for f, c in self.extra.items()}
+        self.flush = torch.empty(256 * MiB, dtype=torch.uint8, device=dev) if wl.flush_l2 else None
 
-    def step():
-        cache.restore(snap)
-        one_pass()
+    def _filled_cache(self, flags):
+        """A cache with the crafted entries and the prefill calls done."""
+        import numpy as np
+        import torch
+        from paper_2607_23115_gb300.cache import Cache, DedupOutputs, fingerprint
+        wl, C = self.wl, self.wl.C
+        cache = Cache(wl.capacity, C, flags)
+        cache.reserve(max(self.nchunks, max((sum(t.numel() for t in b) + C - 1) // C + len(b)
+                                            for b in wl.prefill) if wl.prefill else 1))
+        for orig, row in wl.crafted:
+            key = int(fingerprint(orig, 0).cpu().numpy().view(np.uint64)[0])
+            cache.debug_insert(key, row)
+        for batch in wl.prefill:
+            pouts = [DedupOutputs.alloc(t.numel(), C, self.dev) for t in batch]
+            cache.dedup_batch(batch, pouts)
+            torch.cuda.synchronize()
+            del pouts
+        return cache
 
-    st0 = cache.stats()
-    for _ in range(args.warmup):
-        step()
-    torch.cuda.synchronize()
-    st1 = cache.stats()  # the last warm-up step's counters (restored before it)
-    evictions = st1["evictions"] - st0["evictions"]
-    r = results.cpu().numpy()
-    assert (r[:, 0] == 0).all(), "a dedup call failed: %s" % r[r[:, 0] != 0][:3]
-    miss_bytes = int(r[:, 5].sum())
-    n_miss = int(r[:, 1].sum())
-    hit_intra = int(r[:, 3].sum())
-    if wl.expect_misses is not None:
-        assert n_miss == wl.expect_misses, (n_miss, wl.expect_misses)
-    # algorithmic bytes: the fused fingerprint/probe/verify kernel reads the
-    # payload once and the cached copy of every cache hit
-    # (in-call duplicates counted as whole chunks: exact for every workload
-    # here, none of which repeats a short last chunk within a call)
-    hit_cache_bytes = total - miss_bytes - hit_intra * C
-    kernel0_bytes = total + hit_cache_bytes
-    # the pipeline's minimal traffic: payload read once, the cached copy of
-    # every cache hit read, the miss bytes written once (an in-call duplicate
-    # needs neither: its first occurrence is part of the payload read)
-    pipeline_bytes = total + hit_cache_bytes + miss_bytes
+    def one_pass(self, stream=None):
+        self.cache.dedup_batch(None, items=self.items, total=self.total_res, stream=stream)
 
-    clocks = ClockSampler(local_rank)
-    if not args.profile_launches:
-        clocks.start()
-    B.gleam_cache_profile(cache.handle, True)
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    # each step restores the cache snapshot first, outside its own events (the
-    # repetitions are restored untimed); inputs that fit in L2 are also flushed
-    # there
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(args.steps)]
-    for e0, e1 in ev:
-        cache.restore(snap)
-        if flush is not None:
-            flush.fill_(1)
-        e0.record()
-        one_pass()
-        e1.record()
-    torch.cuda.synchronize()
-    step_ms = [e0.elapsed_time(e1) for e0, e1 in ev]
-    # the hash kernel also writes twice every chunk it writes ahead (write-
-    # through of likely misses; C bytes per chunk, a tail counted whole), as
-    # counted in the last timed step (each step starts from the snapshot's
-    # counters)
-    spec_chunks = cache.stats()["spec_chunks"] - st0["spec_chunks"]
-    kernel0_bytes += 2 * spec_chunks * C
-    ms = sum(step_ms)
-    if world > 1:
-        dist.barrier()
-    clk = clocks.stop() if not args.profile_launches else None
-    rc, kms, klaunch = B.gleam_cache_profile_read(cache.handle, 2)
-    B.gleam_cache_profile(cache.handle, False)
+    def step(self):
+        self.cache.restore(self.snap)
+        self.one_pass()
 
-    # the same pass as one call per payload (secondary figures)
-    per_call = None
-    if not args.profile_launches:
-        calls_steps = 1 if nt > 1000 else max(1, min(args.steps, 5))
+    def timed(self, steps, warmup, world=1, clocks=None):
+        """`warmup` untimed steps, then `steps` steps each timed by its own CUDA
+        events after an untimed snapshot restore (and L2 flush for inputs that
+        fit in L2).  Returns the raw figures of the timed steps."""
+        import torch
+        import torch.distributed as dist
+        from paper_2607_23115_gb300 import binding as B
+        cache, C = self.cache, self.wl.C
+        st0 = cache.stats()
+        for _ in range(warmup):
+            self.step()
+        torch.cuda.synchronize()
+        st1 = cache.stats()  # the last warm-up step's counters (restored before it)
+        r = self.results.cpu().numpy()
+        assert (r[:, 0] == 0).all(), "a dedup call failed: %s" % r[r[:, 0] != 0][:3]
+        miss_bytes = int(r[:, 5].sum())
+        n_miss = int(r[:, 1].sum())
+        hit_intra = int(r[:, 3].sum())
+        if self.wl.expect_misses is not None:
+            assert n_miss == self.wl.expect_misses, (n_miss, self.wl.expect_misses)
+        if clocks is not None:
+            clocks.start()
+        B.gleam_cache_profile(cache.handle, True)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps)]
+        for e0, e1 in ev:
+            cache.restore(self.snap)
+            if self.flush is not None:
+                self.flush.fill_(1)
+            e0.record()
+            self.one_pass()
+            e1.record()
+        torch.cuda.synchronize()
+        step_ms = [e0.elapsed_time(e1) for e0, e1 in ev]
+        if world > 1:
+            dist.barrier()
+        clk = clocks.stop() if clocks is not None else None
+        rc, kms, klaunch = B.gleam_cache_profile_read(cache.handle, 2)
+        B.gleam_cache_profile(cache.handle, False)
+        # each timed step starts from the snapshot's counters: the difference is
+        # the last timed step's
+        spec_chunks = cache.stats()["spec_chunks"] - st0["spec_chunks"]
+        # algorithmic bytes of the fingerprint/probe/verify kernel: the payload
+        # once and the cached copy of every cache hit (in-call duplicates
+        # counted as whole chunks: exact for every workload here, none of which
+        # repeats a short last chunk within a call), plus the two writes of
+        # every chunk written ahead (write-through of likely misses)
+        hit_cache_bytes = self.total - miss_bytes - hit_intra * C
+        kernel0_bytes = self.total + hit_cache_bytes + 2 * spec_chunks * C
+        # the pipeline's minimal traffic: payload read once, the cached copy of
+        # every cache hit read, the miss bytes written once (an in-call
+        # duplicate needs neither: its first occurrence is part of the payload)
+        pipeline_bytes = self.total + hit_cache_bytes + miss_bytes
+        return {"step_ms": step_ms, "ms": sum(step_ms), "kms": kms, "klaunch": klaunch,
+                "n_miss": n_miss, "miss_bytes": miss_bytes, "hit_intra": hit_intra,
+                "evictions": st1["evictions"] - st0["evictions"], "spec_chunks": spec_chunks,
+                "kernel0_bytes": kernel0_bytes, "pipeline_bytes": pipeline_bytes, "clocks": clk}
+
+    def per_call(self, steps, sync_calls=0, flags=0):
+        """The same pass as one gleam_dedup_copy_async call per payload (and,
+        if sync_calls, that many synchronous gleam_dedup_copy calls), on the
+        cache made with the extra creation flags `flags` if given."""
+        import torch
+        from paper_2607_23115_gb300 import binding as B
+        cache, snap, nt = self.cache, self.snap, self.nt
+        if flags:
+            cache, snap = self.extra[flags], self.extra_snap[flags]
         cache.restore(snap)
         for k in range(nt):
-            cache.dedup_async(bufs[k], outs[k], results[k], stream=None)
+            cache.dedup_async(self.bufs[k], self.outs[k], self.results[k], stream=None)
         torch.cuda.synchronize()
         c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         th = time.perf_counter()
         c0.record()
-        for _ in range(calls_steps):
+        for _ in range(steps):
             cache.restore(snap)
             for k in range(nt):
-                cache.dedup_async(bufs[k], outs[k], results[k], stream=None)
+                cache.dedup_async(self.bufs[k], self.outs[k], self.results[k], stream=None)
         c1.record()
         torch.cuda.synchronize()
-        wall = (time.perf_counter() - th) / calls_steps
-        calls_ms = c0.elapsed_time(c1) / calls_steps
-        rcall = results.cpu().numpy()
-        assert (rcall[:, 0] == 0).all() and int(rcall[:, 1].sum()) == n_miss
-        per_call = {"ms_per_step": round(calls_ms, 3),
-                    "value": round(total / (calls_ms * 1e-3) / 1e9, 2),
-                    "us_per_call": round(calls_ms * 1e3 / nt, 3),
-                    "host_wall_us_per_call": round(wall * 1e6 / nt, 3),
-                    "calls_per_s": round(nt / (calls_ms * 1e-3)),
-                    "insert_gbs": round(miss_bytes / (calls_ms * 1e-3) / 1e9, 2),
-                    "how": "same step as %d gleam_dedup_copy_async calls (one per payload) "
-                           "instead of one gleam_dedup_copy_batch call" % nt}
-        if nt > 1000:  # synchronous calls, like cudaMemcpy, on the first 2000 payloads
-            from paper_2607_23115_gb300 import binding as BB
+        wall = (time.perf_counter() - th) / steps
+        calls_ms = c0.elapsed_time(c1) / steps
+        rcall = self.results.cpu().numpy()
+        assert (rcall[:, 0] == 0).all()
+        if self.wl.expect_misses is not None:
+            assert int(rcall[:, 1].sum()) == self.wl.expect_misses
+        miss_bytes = int(rcall[:, 5].sum())
+        out = {"ms_per_step": round(calls_ms, 3),
+               "value": round(self.total / (calls_ms * 1e-3) / 1e9, 2),
+               "us_per_call": round(calls_ms * 1e3 / nt, 3),
+               "host_wall_us_per_call": round(wall * 1e6 / nt, 3),
+               "calls_per_s": round(nt / (calls_ms * 1e-3)),
+               "insert_gbs": round(miss_bytes / (calls_ms * 1e-3) / 1e9, 2),
+               "how": "same step as %d gleam_dedup_copy_async calls (one per payload) "
+                      "instead of one gleam_dedup_copy_batch call" % nt}
+        if sync_calls:  # synchronous calls, like cudaMemcpy
             cache.restore(snap)
             torch.cuda.synchronize()
             th = time.perf_counter()
-            for k in range(2000):
-                rcs = BB.gleam_dedup_copy(cache.handle, bufs[k], up.sizes[k], outs[k].hit_mask,
-                                          outs[k].miss_idx, outs[k].miss_bytes)
+            for k in range(sync_calls):
+                rcs = B.gleam_dedup_copy(cache.handle, self.bufs[k], self.wl.up.sizes[k],
+                                         self.outs[k].hit_mask, self.outs[k].miss_idx,
+                                         self.outs[k].miss_bytes)
                 assert rcs >= 0, rcs
-            per_call["sync_us_per_call"] = round((time.perf_counter() - th) * 1e6 / 2000, 3)
-    ms, value = replica_timing(ms, total, args.steps, world, dev)
+            out["sync_us_per_call"] = round((time.perf_counter() - th) * 1e6 / sync_calls, 3)
+            out["sync_calls"] = sync_calls
+        return out
+
+    def close(self):
+        import torch
+        self.cache.close()
+        for c in self.extra.values():
+            c.close()
+        self.__dict__.clear()
+        torch.cuda.empty_cache()
+
+
+def summarize(raw, total, steps, hbm):
+    """Per-step rates of one timed workload: payload GB/s, the pipeline's
+    minimal-traffic fraction, the hash kernel's algorithmic fraction."""
+    ms_per_step = raw["ms"] / steps
+    k0_ms = raw["kms"][0] / max(1, raw["klaunch"][0])
+    k0_gbs = raw["kernel0_bytes"] / (k0_ms * 1e-3) / 1e9 if k0_ms else 0.0
+    pipe_gbs = raw["pipeline_bytes"] / (ms_per_step * 1e-3) / 1e9
+    return {"gbs": round(total / (ms_per_step * 1e-3) / 1e9, 2),
+            "ms_per_step": round(ms_per_step, 4),
+            "pipeline_frac": round(pipe_gbs / hbm, 4),
+            "hash_frac": round(k0_gbs / hbm, 4),
+            "hash_ms": round(k0_ms, 4),
+            "dedup_pack_ms": round(raw["kms"][1] / max(1, raw["klaunch"][1]), 4),
+            "misses": raw["n_miss"]}
+
+
+# The rows of the `configs` object: every configuration of the target besides
+# the headline one (the Llama-3-8B upload), at full size.
+CONFIG_ROWS = ["fp16-64m", "gpt2-small-pass1", "gpt2-small", "small-calls"] + \
+    ["adversarial-%dk%s" % (c, m) for c in (1, 4, 16, 64) for m in ("", "-key16")]
+
+
+def run_configs(args, dev, hbm):
+    """Each configuration of CONFIG_ROWS timed like the headline (warm-up,
+    per-step CUDA events, snapshot restore between steps), one after the other
+    on this GPU; clocks sampled over all of their timed regions."""
+    import torch
+    rows = {}
+    clocks = ClockSampler(dev.index or 0)
+    clocks.start()
+    for name in CONFIG_ROWS:
+        from paper_2607_23115_gb300 import binding as B
+        wl = build_workload(name, dev, 0)
+        per_call = name == "small-calls"
+        run = Run(wl, dev, (B.GLEAM_OVERLAP_CALLS,) if per_call else ())
+        raw = run.timed(args.steps, args.warmup)
+        row = {"workload": wl.name, "chunks_per_step": run.nchunks,
+               "payload_bytes_per_step": run.total}
+        row.update(summarize(raw, run.total, args.steps, hbm))
+        if per_call:  # per-call overhead: async calls and synchronous ones
+            pc = run.per_call(1, sync_calls=2000)
+            row["async_us_per_call"] = pc["us_per_call"]
+            row["async_gbs"] = pc["value"]
+            row["sync_us_per_call"] = pc["sync_us_per_call"]
+            pc = run.per_call(1, flags=B.GLEAM_OVERLAP_CALLS)
+            row["async_overlap_us_per_call"] = pc["us_per_call"]
+            row["async_overlap_gbs"] = pc["value"]
+        run.close()
+        del wl, run
+        torch.cuda.empty_cache()
+        rows[name] = row
+    return {"rows": rows, "clocks": clocks.stop(),
+            "how": "each configuration at full size, %d warm-up and %d timed steps (one "
+                   "gleam_dedup_copy_batch call per step over all of its payloads); gbs = "
+                   "payload GB/s, pipeline_frac = (payload + cached copies of cache hits + "
+                   "miss bytes) / step time / measured copy peak, hash_frac = the hash "
+                   "kernel's algorithmic bytes / its CUDA-event time / that peak; "
+                   "small-call stream: also 100,000 async calls (on a plain cache and on one created with "
+                   "GLEAM_OVERLAP_CALLS) and 2,000 synchronous calls"
+                   % (args.warmup, args.steps)}
+
+
+def run_gleam(args, rank, world, local_rank):
+    import torch
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    do_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline and not args.profile_launches
+    from paper_2607_23115_gb300 import binding as B
+    wl = build_workload(args.workload, dev, args.cpu_sample_bytes if do_cpu else 0)
+    # a second cache made with GLEAM_OVERLAP_CALLS, for the per-call pass whose
+    # calls may overlap (not with eviction, where calls never overlap)
+    overlap = not args.profile_launches and not (wl.flags & B.GLEAM_EVICT_LRU)
+    run = Run(wl, dev, (B.GLEAM_OVERLAP_CALLS,) if overlap else ())
+    C, up, nt, total = wl.C, wl.up, run.nt, run.total
+    hbm, hbm_src = measured_peaks()
+
+    clocks = None if args.profile_launches else ClockSampler(local_rank)
+    raw = run.timed(args.steps, args.warmup, world, clocks)
+    ms, value = replica_timing(raw["ms"], total, args.steps, world, dev)
     ms_per_step = ms / args.steps
 
-    hbm, hbm_src = measured_peaks()
+    # the same pass as one call per payload (secondary figures)
+    per_call = per_call_ov = None
+    if not args.profile_launches:
+        pc_steps = 1 if nt > 1000 else max(1, min(args.steps, 5))
+        per_call = run.per_call(pc_steps, sync_calls=2000 if nt > 1000 else 0)
+        if overlap:
+            per_call_ov = run.per_call(pc_steps, flags=B.GLEAM_OVERLAP_CALLS)
+            per_call_ov["how"] += ", on a cache created with GLEAM_OVERLAP_CALLS (each call " \
+                                  "fingerprints while the calls before it still run)"
+
+    kms, klaunch = raw["kms"], raw["klaunch"]
     k0_ms = kms[0] / max(1, klaunch[0])
-    k0_bytes = kernel0_bytes  # one launch covers the whole step
+    k0_bytes = raw["kernel0_bytes"]  # one launch covers the whole step
     k0_gbs = k0_bytes / (k0_ms * 1e-3) / 1e9
     traffic = committed_traffic(wl.name)
     roofline = {"bound": "hbm", "kernel": "k_hash_probe_staged (fingerprint + probe + verify)",
@@ -570,8 +707,9 @@ def run_gleam(args, rank, world, local_rank):
                 "unit": "GB/s", "frac": round(k0_gbs / hbm, 4),
                 "traffic": traffic, "algorithmic_bytes_per_launch": round(k0_bytes),
                 "avg_launch_ms": round(k0_ms, 5),
-                "kernel_share_of_step": round((kms[0]) / ms if ms else 0, 4),
+                "kernel_share_of_step": round((kms[0]) / raw["ms"] if raw["ms"] else 0, 4),
                 "k_dedup_k_pack_avg_ms": round(kms[1] / max(1, klaunch[1]), 5)}
+    pipeline_bytes, miss_bytes = raw["pipeline_bytes"], raw["miss_bytes"]
     pipe_gbs = pipeline_bytes / (ms_per_step * 1e-3) / 1e9
     pipeline = {"min_bytes_per_step": pipeline_bytes,
                 "achieved_gbs": round(pipe_gbs, 1),
@@ -580,6 +718,7 @@ def run_gleam(args, rank, world, local_rank):
                 "with_arena_write_bytes": pipeline_bytes + miss_bytes,
                 "with_arena_write_frac_of_measured": round(
                     (pipeline_bytes + miss_bytes) / (ms_per_step * 1e-3) / 1e9 / hbm, 4)}
+    step_ms = raw["step_ms"]
 
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
@@ -588,33 +727,32 @@ def run_gleam(args, rank, world, local_rank):
                     "min": round(min(step_ms), 4), "max": round(max(step_ms), 4)},
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
         "data": "synthetic",
-        "config": {"workload": wl.name, "description": wl.desc,
-                   "payload_bytes_per_step": total, "payloads_per_step": nt, "calls_per_step": 1,
-                   "api": "gleam_dedup_copy_batch (one call = %d payloads)" % nt,
-                   "chunk_bytes": C, "chunks_per_step": nchunks, "misses_per_step": n_miss,
-                   "evictions_per_step": evictions,
-                   "written_ahead_chunks_per_step": spec_chunks,
-                   "cache_capacity_bytes": wl.capacity, "key16": bool(wl.flags & 1),
-                   "l2": ("inputs (%.2f GB) fit in the 129 MB L2's reach: a 256 MiB buffer is "
-                          "written between timed steps, after the cache snapshot is restored, "
-                          "both outside each step's events" % (total / 1e9))
-                         if flush is not None else
-                         ("inputs (%.1f GB per step) far larger than the 129 MB L2; no flush"
-                          % (total / 1e9)),
-                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "config": workload_config(wl),
+        "run": {"calls_per_step": 1,
+                "api": "gleam_dedup_copy_batch (one call = %d payloads)" % nt,
+                "misses_per_step": raw["n_miss"], "evictions_per_step": raw["evictions"],
+                "written_ahead_chunks_per_step": raw["spec_chunks"],
+                "l2": ("inputs (%.2f GB) fit in the 129 MB L2's reach: a 256 MiB buffer is "
+                       "written between timed steps, after the cache snapshot is restored, "
+                       "both outside each step's events" % (total / 1e9))
+                      if run.flush is not None else
+                      ("inputs (%.1f GB per step) far larger than the 129 MB L2; no flush"
+                       % (total / 1e9)),
+                "parallelism": "replicas" if world > 1 else "single GPU"},
         "pipeline_roofline": pipeline,
         "roofline": roofline,
         "per_call_async": per_call,
+        "per_call_async_overlap": per_call_ov,
         # the library's kernels in the timed region, counted by its profile
         # events: one hash launch and one k_dedup + k_pack pair per call
         "gpu_launches": int(klaunch[0]) + 2 * int(klaunch[1]),
-        "clocks": clk,
+        "clocks": raw["clocks"],
     }
 
     if not args.profile_launches:
-        step()  # the per-call runs above changed the cache; redo the batch pass
+        run.step()  # the per-call runs above changed the cache; redo the batch pass
         torch.cuda.synchronize()
-        line["block_check"] = run_block_check(up, cache, chunk_slots, C, hbm)
+        line["block_check"] = run_block_check(up, run.cache, run.chunk_slots, C, hbm)
 
     if do_cpu:
         nbytes, dt, text = oracle_time(wl, args.cpu_sample_bytes)
@@ -625,11 +763,16 @@ def run_gleam(args, rank, world, local_rank):
     if not args.no_e2e and not args.profile_launches and nt <= 1000:
         host = torch.empty(up.buf.numel(), dtype=torch.uint8, pin_memory=True)
         host.copy_(up.buf)
-        line["e2e"] = run_e2e_host(args, up, host, cache, snap, outs, results, miss_bytes)
-        line["e2e_copy_then_dedup"] = run_e2e(args, up, host, cache, snap, outs, results,
-                                              miss_bytes)
+        line["e2e"] = run_e2e_host(args, up, host, run.cache, run.snap, run.outs, run.results,
+                                   miss_bytes)
+        line["e2e_copy_then_dedup"] = run_e2e(args, up, host, run.cache, run.snap, run.outs,
+                                              run.results, miss_bytes)
+        del host
 
-    cache.close()
+    run.close()
+    del wl, run
+    if not args.no_configs and not args.profile_launches and world == 1:
+        line["configs"] = run_configs(args, dev, hbm)
     return line
 
 
@@ -852,7 +995,9 @@ def run_reference(args, rank, world):
         "ms_per_step": round(t / args.steps * 1e3, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "u8", "data": "synthetic",
         "impl": "reference",
-        "config": {"workload": wl.name, "description": wl.desc, "chunk_bytes": wl.C},
+        "config": workload_config(wl),
+        "run": {"api": "the oracle's dedup, one call per payload", "parallelism":
+                "one host core"},
         "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
                          "sample": "per step: " + text, "host_cpus": os.cpu_count(),
                          "host_cpu_model": cpu_model()},

@@ -85,6 +85,25 @@ enum gleam_status {
                                    instead of failing with GLEAM_ERR_CAPACITY.
                                    A batch is one call for this.  Costs 9 bytes
                                    of device memory per slot. */
+#define GLEAM_OVERLAP_CALLS 0x10u /* consecutive calls of the cache on one
+                                   stream may overlap on the GPU: a call of up
+                                   to 8192 chunks fingerprints its payload
+                                   while the calls before it are still running
+                                   and waits for them (on the GPU, by
+                                   programmatic dependent launch) only before
+                                   it reads the cache's index; outputs and
+                                   cache state are those of calls run one after
+                                   another.  The caller promises that each
+                                   payload is complete when its call is
+                                   enqueued, or is written by work that the
+                                   call already waits for without it: a copy,
+                                   memset or event wait on the stream between
+                                   the writer and the call, or a kernel that
+                                   does not trigger its dependents early.  Not
+                                   applied to GLEAM_EVICT_LRU caches (an
+                                   eviction rewrites slots) nor with
+                                   GLEAM_PAPER_IDS (the key is known after one
+                                   stage); both stay correct. */
 
 /* Cumulative counters of one cache (successful calls only). */
 typedef struct gleam_stats {
@@ -141,8 +160,8 @@ typedef struct gleam_payload {
  * slots of chunk_bytes each and an empty index (paper Sec. 4.1.3: the
  * server-side shareable pool; Sec. 4.1.2: the set of resident identifiers).
  * chunk_bytes: multiple of 32, 32..16 MiB.  The slot count must be 1..2^32-2.
- * flags: 0 or a combination of GLEAM_KEY16, GLEAM_DEBUG_CHECKS, GLEAM_PAPER_IDS
- * and GLEAM_EVICT_LRU.
+ * flags: 0 or a combination of GLEAM_KEY16, GLEAM_DEBUG_CHECKS, GLEAM_PAPER_IDS,
+ * GLEAM_EVICT_LRU and GLEAM_OVERLAP_CALLS.
  * On success *out owns about capacity_bytes + 32 B * slots of device memory.
  * Returns GLEAM_OK, GLEAM_ERR_INVALID_ARG, GLEAM_ERR_NOMEM or GLEAM_ERR_CUDA. */
 int gleam_cache_create(size_t capacity_bytes, size_t chunk_bytes, gleam_cache_t** out);

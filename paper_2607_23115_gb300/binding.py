@@ -26,6 +26,7 @@ GLEAM_KEY16 = 0x1
 GLEAM_DEBUG_CHECKS = 0x2
 GLEAM_PAPER_IDS = 0x4
 GLEAM_EVICT_LRU = 0x8
+GLEAM_OVERLAP_CALLS = 0x10
 GLEAM_DEBUG_WAIT_LIMIT_NS = 1
 GLEAM_DEBUG_SKIP_ARRIVE = 2
 GLEAM_DEBUG_CLOCK = 3

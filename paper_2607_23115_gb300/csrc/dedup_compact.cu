@@ -1213,11 +1213,15 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
 }
 
 __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
+  pdl_trigger();
+  pdl_wait();
   resolve_rank(a, gridDim.x, blockIdx.x);
 }
 
 __global__ void GLEAM_PACK_BOUNDS k_pack(DedupArgs a) {
   extern __shared__ __align__(128) uint8_t pack_smem[];
+  pdl_trigger();
+  pdl_wait();
   pack_publish(a, gridDim.x, blockIdx.x, pack_smem);
 }
 
@@ -1236,6 +1240,8 @@ __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
 template <bool kAhead>
 __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a) {
   extern __shared__ __align__(128) uint8_t small_smem[];
+  pdl_trigger();
+  if (!h.wait_late) pdl_wait();  // else in staged_range, before the first probe
   // Device-resident payloads (16-byte aligned here) are prefetched into L2 at
   // once, lane p taking payload p in 16 KiB pieces, so that the hash stages
   // wait for L2 rather than HBM.
@@ -1377,31 +1383,33 @@ int dedup_blocks_per_sm() {
   return nb < GLEAM_DEDUP_BLOCKS_PER_SM ? nb : GLEAM_DEDUP_BLOCKS_PER_SM;
 }
 
-cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s) {
-  DedupArgs copy = a;
-  void* args[] = {&copy};
-  cudaError_t e =
-      cudaLaunchCooperativeKernel((void*)k_dedup, dim3(grid), dim3(kThreads), args, 0, s);
+cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s, bool pdl) {
+  cudaError_t e;
+  if (pdl) {
+    e = launch_kernel(k_dedup, dim3(grid), dim3(kThreads), 0, s, true, a);
+  } else {
+    DedupArgs copy = a;
+    void* args[] = {&copy};
+    e = cudaLaunchCooperativeKernel((void*)k_dedup, dim3(grid), dim3(kThreads), args, 0, s);
+  }
   if (e != cudaSuccess) return e;
   if (kPackSmem > 48 * 1024)
     cudaFuncSetAttribute((const void*)k_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          kPackSmem);
-  k_pack<<<pack_grid, kThreads, kPackSmem, s>>>(a);
-  return cudaGetLastError();
+  return launch_kernel(k_pack, dim3(pack_grid), dim3(kThreads), kPackSmem, s, pdl, a);
 }
 
 uint32_t small_call_groups() { return kSmallGroups; }
 
 template <bool kAhead>
-cudaError_t launch_small(const HashArgs& h, const DedupArgs& a, cudaStream_t s) {
+cudaError_t launch_small(const HashArgs& h, const DedupArgs& a, cudaStream_t s, bool pdl) {
   cudaFuncSetAttribute((const void*)k_small_call<kAhead>,
                        cudaFuncAttributeMaxDynamicSharedMemorySize, kSmallSmem);
-  k_small_call<kAhead><<<1, kThreads, kSmallSmem, s>>>(h, a);
-  return cudaGetLastError();
+  return launch_kernel(k_small_call<kAhead>, dim3(1), dim3(kThreads), kSmallSmem, s, pdl, h, a);
 }
 
-cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_t s) {
-  return h.spec_mode ? launch_small<true>(h, a, s) : launch_small<false>(h, a, s);
+cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_t s, bool pdl) {
+  return h.spec_mode ? launch_small<true>(h, a, s, pdl) : launch_small<false>(h, a, s, pdl);
 }
 
 cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s) {

@@ -77,6 +77,10 @@ struct gleam_cache {
   unsigned long long wait_ns = 4000000000ULL;
   int skip_block = -1;
 
+  // id (cudaStreamGetId) of the stream `done` was last recorded on: a call on
+  // that same stream is ordered after it without an event wait
+  unsigned long long done_stream = ~0ull;
+
   // device address of the allocation-free call's scratch array on this GPU,
   // looked up when the cache is created
   uint8_t* na_scratch = nullptr;
@@ -463,6 +467,64 @@ void note_call(gleam_cache* c, uint64_t Ntot) {
   c->slots_bound = std::min<uint64_t>(c->nslots, c->slots_bound + Ntot);
 }
 
+// Chained calls.  A call that leaves most of the GPU idle (at most
+// kChainMaxChunks chunks and kChainMaxBytes bytes) launches its kernels with
+// programmatic stream serialization: each kernel lets the next one on the
+// stream be launched as soon as all of its blocks have started, so that a
+// kernel's blocks are waiting on the GPU when the one before finishes instead
+// of being launched then.  The resolve kernel is then a regular launch (a
+// cooperative one is never launched early) on at most kChainDedupBlocks
+// blocks, and the pack kernel runs on at most kChainPackBlocks: every waiting
+// block holds its SM resources.  With GLEAM_OVERLAP_CALLS the hash kernel also
+// fingerprints before it waits (HashArgs::wait_late).  Evicting caches and the
+// test hook that makes a block skip a barrier keep the plain launches.
+#ifndef GLEAM_CHAIN_MAX_CHUNKS
+#define GLEAM_CHAIN_MAX_CHUNKS 8192
+#endif
+#ifndef GLEAM_CHAIN_DEDUP_BLOCKS
+#define GLEAM_CHAIN_DEDUP_BLOCKS 32
+#endif
+#ifndef GLEAM_CHAIN_PACK_BLOCKS
+#define GLEAM_CHAIN_PACK_BLOCKS 76
+#endif
+constexpr uint64_t kChainMaxChunks = GLEAM_CHAIN_MAX_CHUNKS;
+constexpr uint64_t kChainMaxBytes = 1ull << 30;
+constexpr int kChainDedupBlocks = GLEAM_CHAIN_DEDUP_BLOCKS;
+constexpr int kChainPackBlocks = GLEAM_CHAIN_PACK_BLOCKS;
+
+bool chain_call(const gleam_cache* c, uint64_t Ntot, uint64_t nbytes, int skip_block) {
+  return Ntot <= kChainMaxChunks && nbytes <= kChainMaxBytes && skip_block < 0 &&
+         !(c->flags & GLEAM_EVICT_LRU);
+}
+
+// Orders a call on stream s after the cache's previous work: an event wait,
+// unless that work ended on s itself (stream order already holds, and a wait
+// between two kernels would keep the second from being launched early).
+int order_after_done(gleam_cache* c, cudaStream_t s, unsigned long long* sid) {
+  if (cudaStreamGetId(s, sid) != cudaSuccess) {
+    cudaGetLastError();
+    *sid = ~0ull;
+  }
+  if (*sid != ~0ull && *sid == c->done_stream) return GLEAM_OK;
+  return cuda_err(cudaStreamWaitEvent(s, c->done, 0));
+}
+
+// Records the end of the cache's latest work on stream s.
+int record_done(gleam_cache* c, cudaStream_t s, unsigned long long sid) {
+  const int rc = cuda_err(cudaEventRecord(c->done, s));
+  c->done_stream = rc == GLEAM_OK ? sid : ~0ull;
+  return rc;
+}
+
+unsigned long long stream_id(cudaStream_t s) {
+  unsigned long long id = ~0ull;
+  if (cudaStreamGetId(s, &id) != cudaSuccess) {
+    cudaGetLastError();
+    id = ~0ull;
+  }
+  return id;
+}
+
 // The write-through fields of a call's kernel arguments.  It needs the staged
 // hash (16-byte-aligned payloads, C a multiple of 32), 16-byte-aligned packed
 // buffers (device or page-locked host memory), and 64-bit or KEY16 keys.  In the automatic
@@ -539,7 +601,8 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   }
   if ((rc = ensure_ws(c, std::max<uint64_t>(Ntot, 1))) != GLEAM_OK) return rc;
 
-  if ((rc = cuda_err(cudaStreamWaitEvent(s, c->done, 0))) != GLEAM_OK) return rc;
+  unsigned long long sid = ~0ull;
+  if ((rc = order_after_done(c, s, &sid)) != GLEAM_OK) return rc;
   if (count > 1) {
     if ((rc = cuda_err(cudaMemcpyAsync(c->d_table, c->h_table, count * sizeof(PayloadDesc),
                                        cudaMemcpyHostToDevice, s))) != GLEAM_OK)
@@ -604,9 +667,14 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     if (d.skip_block >= grid) d.skip_block = grid - 1;
   }
   const bool fused = small_call(c, aligned, Ntot, nbytes, d.skip_block);
+  const bool chain = chain_call(c, Ntot, nbytes, d.skip_block);
+  // overlapping calls: the staged hash kernels fingerprint before they wait
+  // (others ignore the field and wait first); the write-through stays off, as
+  // it writes arena slots counted from a slot count that may still change
+  h.wait_late = chain && (c->flags & GLEAM_OVERLAP_CALLS) && !(c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   // host payloads too: a chunk written ahead then spares the pack a second
   // read over the CPU-GPU link (managed memory stays out)
-  set_spec(c, &h, &d, aligned && packed_aligned && !chk.saw_managed());
+  set_spec(c, &h, &d, aligned && packed_aligned && !chk.saw_managed() && !h.wait_late);
 
   cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
   if (c->profile) {
@@ -620,12 +688,17 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     cudaEventRecord(ev[0], s);
   }
   if (fused) {  // one kernel: all of its time is phase 0
-    if ((rc = cuda_err(launch_small_call(h, d, s))) != GLEAM_OK) return rc;
+    if ((rc = cuda_err(launch_small_call(h, d, s, chain))) != GLEAM_OK) return rc;
     if (ev[1]) cudaEventRecord(ev[1], s);
   } else {
-    if ((rc = cuda_err(launch_hash(h, aligned, s))) != GLEAM_OK) return rc;
+    if ((rc = cuda_err(launch_hash(h, aligned, s, chain))) != GLEAM_OK) return rc;
     if (ev[1]) cudaEventRecord(ev[1], s);
-    if ((rc = cuda_err(launch_dedup(d, grid, pack_grid(c, Ntot, nbytes), s))) != GLEAM_OK) {
+    int pgrid = pack_grid(c, Ntot, nbytes);
+    if (chain) {
+      grid = std::min(grid, kChainDedupBlocks);
+      pgrid = std::min(pgrid, kChainPackBlocks);
+    }
+    if ((rc = cuda_err(launch_dedup(d, grid, pgrid, s, chain))) != GLEAM_OK) {
       cudaMemsetAsync(c->ctl, 0, sizeof(DevCtl), s);  // the hash kernel may have flagged it
       return rc;
     }
@@ -633,7 +706,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   if (ev[2]) cudaEventRecord(ev[2], s);
   note_call(c, Ntot);
   if ((rc = enqueue_index_check(c, d, s)) != GLEAM_OK) return rc;
-  return cuda_err(cudaEventRecord(c->done, s));
+  return record_done(c, s, sid);
 }
 
 gleam_payload_t make_payload(const void* d_buf, size_t n, uint32_t* d_hit_mask,
@@ -677,7 +750,8 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   *out = nullptr;
   if (chunk_bytes < kMinChunk || chunk_bytes > kMaxChunk || chunk_bytes % 32 != 0)
     return GLEAM_ERR_INVALID_ARG;
-  if ((flags & ~(GLEAM_KEY16 | GLEAM_DEBUG_CHECKS | GLEAM_PAPER_IDS | GLEAM_EVICT_LRU)) != 0)
+  if ((flags & ~(GLEAM_KEY16 | GLEAM_DEBUG_CHECKS | GLEAM_PAPER_IDS | GLEAM_EVICT_LRU |
+                 GLEAM_OVERLAP_CALLS)) != 0)
     return GLEAM_ERR_INVALID_ARG;
   const uint64_t nslots = capacity_bytes / chunk_bytes;
   if (nslots == 0 || nslots > 0xFFFFFFFEull) return GLEAM_ERR_INVALID_ARG;
@@ -987,7 +1061,7 @@ int gleam_cache_debug_insert(gleam_cache_t* c, uint64_t key, const void* d_bytes
                                       (uint32_t)used, (uint32_t)len, c->ctl, c->last_use,
                                       c->last_use ? ++c->epoch : 0u, nullptr));
   if (rc == GLEAM_OK) rc = cuda_err(cudaDeviceSynchronize());
-  if (rc == GLEAM_OK) rc = cuda_err(cudaEventRecord(c->done, nullptr));
+  if (rc == GLEAM_OK) rc = record_done(c, nullptr, stream_id(nullptr));
   if (rc == GLEAM_OK) note_call(c, 1);
   return rc;
 }
@@ -1139,7 +1213,7 @@ int gleam_cache_restore(gleam_cache_t* c, const gleam_snapshot_t* s) {
   }
   if (rc == GLEAM_OK) {
     c->slots_bound = s->slots_bound;
-    rc = cuda_err(cudaEventRecord(c->done, nullptr));
+    rc = record_done(c, nullptr, stream_id(nullptr));
   }
   return rc;
 }
@@ -1259,7 +1333,8 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   const uint64_t tcap = std::min<uint64_t>(kNaTable, next_pow2(std::max<uint64_t>(64, 2 * N)));
 
   // the array keeps the previous call's contents: clear what must start at zero
-  if ((rc = cuda_err(cudaStreamWaitEvent(s, c->done, 0))) != GLEAM_OK) return rc;
+  unsigned long long sid = ~0ull;
+  if ((rc = order_after_done(c, s, &sid)) != GLEAM_OK) return rc;
   if ((rc = cuda_err(cudaMemsetAsync(ctl, 0, sizeof(DevCtl), s))) != GLEAM_OK) return rc;
   if ((rc = cuda_err(cudaMemsetAsync(tbl, 0, tcap * sizeof(CallEntry), s))) != GLEAM_OK) return rc;
 
@@ -1320,5 +1395,5 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   }
   note_call(c, N);
   if ((rc = enqueue_index_check(c, d, s)) != GLEAM_OK) return rc;
-  return cuda_err(cudaEventRecord(c->done, s));
+  return record_done(c, s, sid);
 }

@@ -165,6 +165,12 @@ struct HashArgs {
   uint8_t* arena_w;                // the arena, for those writes
   uint32_t cache_empty;            // the host knows the cache holds no chunk yet
   unsigned long long nslots;
+  // Calls that overlap (GLEAM_OVERLAP_CALLS): the kernel was launched while the
+  // cache's previous call may still be running, and waits for it only before
+  // it probes the index.  Until then it reads the payload and, for the
+  // speculative verify, the hint table and arena bytes of the slots counted as
+  // used when it started, which no later call changes (no eviction).
+  uint32_t wait_late;
 };
 
 struct DedupArgs {
@@ -214,18 +220,26 @@ constexpr uint32_t kLruBins = 65536;
 // Paper-identifier mode (App. B.1): chunks shorter than this get no entry.
 constexpr uint32_t kPaperMinCached = 1024;
 
-cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s);
+// pdl: launched with programmatic stream serialization (the kernel waits on the
+// GPU for the one before it; see pdl_trigger/pdl_wait).
+cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s, bool pdl = false);
 // Loads the hash kernels' device code on the current GPU (cache creation does
 // it, so that no later call loads code, which allocates device memory).
 cudaError_t load_hash_kernels();
 // The cooperative resolve/rank kernel on `grid` blocks, then the pack kernel
-// (masks, indices, copies, inserts, publish) on `pack_grid` blocks.
-cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s);
+// (masks, indices, copies, inserts, publish) on `pack_grid` blocks.  pdl: both
+// launched with programmatic stream serialization, the resolve kernel then as
+// a regular launch (a cooperative one is never launched early); its grid must
+// fit the GPU at once, and every block of it is resident before anything
+// later on the stream can start, so its grid barriers still complete.
+cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s,
+                         bool pdl = false);
 // A whole call (hash, resolve and rank, pack) as one single-block kernel, for
 // calls with few chunks whose payloads suit the staged hash (16-byte aligned)
 // outside GLEAM_PAPER_IDS mode; the block hashes small_call_groups() chunks at
 // a time.
-cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_t s);
+cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_t s,
+                              bool pdl = false);
 uint32_t small_call_groups();
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
                                 unsigned long long* dstats, unsigned long long key,
@@ -291,6 +305,23 @@ __device__ __forceinline__ unsigned int ld_acquire_u32(const unsigned int* p) {
 __device__ __forceinline__ int ld_volatile_s32(const int* p) {
   return *reinterpret_cast<const volatile int*>(p);
 }
+
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Programmatic dependent launch.  Every hot kernel lets the next kernel of its
+// stream be launched as soon as all of its blocks have started (the next
+// kernel's blocks then wait on the GPU instead of behind a launch), and waits
+// for the kernel before it to finish, with its memory visible, before it
+// touches anything that kernel may write.  Both are no-ops for a kernel
+// launched without the attribute (or one whose predecessor is not a kernel).
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 // Grid-wide barrier for a cooperative launch.  Every wait is bounded by
 // `wait_ns`: a block that gives up records GLEAM_ERR_TIMEOUT and every block
@@ -398,6 +429,28 @@ __device__ __forceinline__ uint32_t block_find_payload(const PayloadDesc* table,
   if (lo == 31 && p0 + 32 < count && __ldg(&table[p0 + 32].chunk_base) <= g)
     return find_payload_in(table, p0 + 32, count, g);
   return p0 + lo;
+}
+
+// Launches kern<<<grid, block, smem, s>>>(args...), with programmatic stream
+// serialization when pdl is set.
+template <typename... Params, typename... Args>
+cudaError_t launch_kernel(void (*kern)(Params...), dim3 grid, dim3 block, size_t smem,
+                          cudaStream_t s, bool pdl, Args&&... args) {
+  if (!pdl) {
+    kern<<<grid, block, smem, s>>>(static_cast<Args&&>(args)...);
+    return cudaGetLastError();
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
 }
 
 #endif  // __CUDACC__

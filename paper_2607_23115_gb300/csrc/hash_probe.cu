@@ -122,6 +122,8 @@ __device__ __forceinline__ unsigned long long lane_stripes_cmp(
 
 template <bool kAligned, bool kProbe>
 __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
+  pdl_trigger();
+  pdl_wait();  // this variant reads nothing before the previous call is complete
   const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
   __shared__ unsigned long long s_scratch[33];
   const uint32_t pid_b =
@@ -261,6 +263,8 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
 template <bool kProbe, bool kAhead, bool kVerify>
 __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
+  pdl_trigger();
+  if (!a.wait_late) pdl_wait();  // else in staged_range, before the probe
   const unsigned long long nvb = (a.Ntot * 4 + kStagedThreads - 1) / kStagedThreads;
   for (unsigned long long vb = blockIdx.x; vb < nvb; vb += gridDim.x) {
     __syncthreads();  // the previous range's groups are done with the shared memory
@@ -269,15 +273,15 @@ __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a
 }
 
 template <bool kProbe, bool kAhead, bool kVerify>
-cudaError_t launch_staged(const HashArgs& a, cudaStream_t s) {
+cudaError_t launch_staged(const HashArgs& a, cudaStream_t s, bool pdl) {
   constexpr int smem = (kStagedThreads / 4) * group_bytes(kVerify);
   // per device and cheap: set on every launch
   cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kAhead, kVerify>,
                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   const unsigned long long threads = a.Ntot * 4;
   const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
-  k_hash_probe_staged<kProbe, kAhead, kVerify><<<sg, kStagedThreads, smem, s>>>(a);
-  return cudaGetLastError();
+  return launch_kernel(k_hash_probe_staged<kProbe, kAhead, kVerify>, dim3(sg),
+                       dim3(kStagedThreads), smem, s, pdl, a);
 }
 
 // ---------------------------------------------------------------------------
@@ -352,6 +356,8 @@ __device__ unsigned long long md5_prefix_key(const uint8_t* p, uint32_t m, const
 
 template <bool kAligned>
 __global__ void __launch_bounds__(kHashThreads) k_probe_paper(HashArgs a, Md5Table tab) {
+  pdl_trigger();
+  pdl_wait();
   const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
   __shared__ unsigned long long s_scratch[33];
   const uint32_t pid_b =
@@ -428,6 +434,8 @@ __global__ void __launch_bounds__(kHashThreads) k_probe_paper(HashArgs a, Md5Tab
 // stage; further candidates after a mismatch are compared by re-reading.
 __global__ void __launch_bounds__(kStagedThreads) k_probe_paper_staged(HashArgs a, Md5Table tab) {
   extern __shared__ __align__(16) uint8_t smem[];
+  pdl_trigger();
+  pdl_wait();  // the key is known after the first stage: nothing to overlap
   const unsigned long long g = ((unsigned long long)blockIdx.x * blockDim.x + threadIdx.x) >> 2;
   const uint32_t pid_b =
       a.count > 1 ? block_find_payload(a.table, a.count,
@@ -590,7 +598,7 @@ cudaError_t load_hash_kernels() {
   return cudaFuncGetAttributes(&fa, k_hash_probe_staged<true, false, true>);
 }
 
-cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
+cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s, bool pdl) {
   if (a.Ntot == 0) return cudaSuccess;
   const unsigned long long threads = a.Ntot * 4;
   const unsigned grid = (unsigned)((threads + kHashThreads - 1) / kHashThreads);
@@ -600,31 +608,32 @@ cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s) {
 #if GLEAM_STAGED_HASH
     if (aligned && a.C % 32 == 0) {
       const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
-      k_probe_paper_staged<<<sg, kStagedThreads, kStagedSmem, s>>>(a, tab);
-      return cudaGetLastError();
+      return launch_kernel(k_probe_paper_staged, dim3(sg), dim3(kStagedThreads), kStagedSmem, s,
+                           pdl, a, tab);
     }
 #endif
-    if (aligned) k_probe_paper<true><<<grid, kHashThreads, 0, s>>>(a, tab);
-    else k_probe_paper<false><<<grid, kHashThreads, 0, s>>>(a, tab);
-    return cudaGetLastError();
+    return aligned ? launch_kernel(k_probe_paper<true>, dim3(grid), dim3(kHashThreads), 0, s,
+                                   pdl, a, tab)
+                   : launch_kernel(k_probe_paper<false>, dim3(grid), dim3(kHashThreads), 0, s,
+                                   pdl, a, tab);
   }
 #if GLEAM_STAGED_HASH
   if (aligned && (a.C % 32 == 0 || a.Ntot == 1)) {
     // no cached copy can be streamed when only fingerprints are wanted or the
     // cache is known to be empty: the variant without those buffers
-    if (!probe) return launch_staged<false, false, false>(a, s);
+    if (!probe) return launch_staged<false, false, false>(a, s, pdl);
     if (a.cache_empty)
-      return a.spec_mode ? launch_staged<true, true, false>(a, s)
-                         : launch_staged<true, false, false>(a, s);
-    return a.spec_mode ? launch_staged<true, true, true>(a, s)
-                       : launch_staged<true, false, true>(a, s);
+      return a.spec_mode ? launch_staged<true, true, false>(a, s, pdl)
+                         : launch_staged<true, false, false>(a, s, pdl);
+    return a.spec_mode ? launch_staged<true, true, true>(a, s, pdl)
+                       : launch_staged<true, false, true>(a, s, pdl);
   }
 #endif
-  if (aligned && probe) k_hash_probe<true, true><<<grid, kHashThreads, 0, s>>>(a);
-  else if (aligned) k_hash_probe<true, false><<<grid, kHashThreads, 0, s>>>(a);
-  else if (probe) k_hash_probe<false, true><<<grid, kHashThreads, 0, s>>>(a);
-  else k_hash_probe<false, false><<<grid, kHashThreads, 0, s>>>(a);
-  return cudaGetLastError();
+  const dim3 g3(grid), b3(kHashThreads);
+  if (aligned && probe) return launch_kernel(k_hash_probe<true, true>, g3, b3, 0, s, pdl, a);
+  if (aligned) return launch_kernel(k_hash_probe<true, false>, g3, b3, 0, s, pdl, a);
+  if (probe) return launch_kernel(k_hash_probe<false, true>, g3, b3, 0, s, pdl, a);
+  return launch_kernel(k_hash_probe<false, false>, g3, b3, 0, s, pdl, a);
 }
 
 }  // namespace gleam

