@@ -234,15 +234,20 @@ def build_workload(name, dev, sample_budget):
         return wl
 
     if name.startswith("adversarial-"):
+        # adversarial-<C>k[-key16][-<M>m]: the 1 GiB payload, or M MiB of the
+        # same make (the small cases for ncu captures)
         parts = name.split("-")
         C = int(parts[1].rstrip("k")) * KiB
-        key16 = len(parts) > 2 and parts[2] == "key16"
+        key16 = "key16" in parts[2:]
+        size = next((int(p[:-1]) * MiB for p in parts[2:] if p.endswith("m")), GiB)
         from paper_2607_23115_gb300 import binding as B
-        wl = Workload("adversarial-1gib-c%dk%s" % (C // KiB, "-key16" if key16 else ""),
-                      "1 GiB: 25%% zero chunks, 25%% copies of 16 patterns, 50%% random, C = %d "
-                      "KiB%s" % (C // KiB, "; KEY16 test mode with 64 crafted colliding entries"
-                                 if key16 else ""), C, 2 * GiB, B.GLEAM_KEY16 if key16 else 0)
-        adv = W.adversarial_payload(1 * GiB, C, device=dev)
+        tag = "1gib" if size == GiB else "%dmib" % (size // MiB)
+        wl = Workload("adversarial-%s-c%dk%s" % (tag, C // KiB, "-key16" if key16 else ""),
+                      "%s: 25%% zero chunks, 25%% copies of 16 patterns, 50%% random, C = %d "
+                      "KiB%s" % ("1 GiB" if size == GiB else "%d MiB" % (size // MiB), C // KiB,
+                                 "; KEY16 test mode with 64 crafted colliding entries"
+                                 if key16 else ""), C, 2 * size, B.GLEAM_KEY16 if key16 else 0)
+        adv = W.adversarial_payload(size, C, device=dev)
         wl.up = Upload(adv.buf, [0], [adv.buf.numel()])
         npat = len(set(adv.pattern_id[adv.kind == 1].tolist()))
         wl.expect_misses = 1 + npat + int((adv.kind == 2).sum())
@@ -269,7 +274,8 @@ WORKLOADS = ["llama3-8b", "llama3-8b-paper-ids", "llama3-8b-lru", "llama3-8b-lay
              "llama3-8b-4layers",
              "gpt2-small",
              "gpt2-small-pass1", "fp16-64m", "small-calls", "small-calls-10k"] + \
-    ["adversarial-%dk%s" % (c, m) for c in (1, 4, 16, 64) for m in ("", "-key16")]
+    ["adversarial-%dk%s" % (c, m) for c in (1, 4, 16, 64) for m in ("", "-key16")] + \
+    ["adversarial-<C>k[-key16]-<M>m (M MiB of the adversarial make)"]
 
 
 # ---------------------------------------------------------------------------

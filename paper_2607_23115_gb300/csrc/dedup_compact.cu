@@ -303,17 +303,24 @@ __device__ bool index_insert(IndexEntry* index, uint64_t mask, unsigned long lon
   return false;
 }
 
-// Finds or claims the per-call group entry of (key, len) for chunk g.
+// Finds or claims the per-call group entry of (key, len) for chunk g;
+// *claimed tells whether g claimed it (else another chunk of the group did).
 __device__ uint32_t group_entry(const DedupArgs& a, uint32_t g, unsigned long long k,
-                                uint32_t len) {
+                                uint32_t len, bool* claimed = nullptr) {
   uint64_t pos = mix64(k ^ ((unsigned long long)len << 40)) & a.tbl_mask;
   for (uint64_t probe = 0; probe <= a.tbl_mask; ++probe) {
     uint32_t o = ldcg_u32(&a.tbl[pos].owner);
     if (o == 0) {
       o = atomicCAS(&a.tbl[pos].owner, 0u, g + 1);
-      if (o == 0) return (uint32_t)pos;
+      if (o == 0) {
+        if (claimed) *claimed = true;
+        return (uint32_t)pos;
+      }
     }
-    if (a.ch.key[o - 1] == k && a.ch.len[o - 1] == len) return (uint32_t)pos;
+    if (a.ch.key[o - 1] == k && a.ch.len[o - 1] == len) {
+      if (claimed) *claimed = false;
+      return (uint32_t)pos;
+    }
     pos = (pos + 1) & a.tbl_mask;
   }
   return 0xFFFFFFFFu;  // cannot happen: the table has >= 2 Ntot entries
@@ -575,8 +582,11 @@ __device__ __forceinline__ void post_minimum(const DedupArgs& a, uint32_t e, uin
 }
 
 // The first-occurrence resolution and miss ranks of a call, run by block
-// `bid` of a grid of G co-resident blocks.
-__device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uint32_t bid) {
+// `bid` of a grid of G co-resident blocks.  claimed: the caller has done
+// phase A (claims and minima posted, outputs cleared) and passed a grid
+// barrier since, with outcome `ok0`.
+__device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uint32_t bid,
+                                             bool claimed = false, bool ok0 = true) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ uint32_t warp_cnt[kWarps];
   __shared__ uint32_t warp_off[kWarps];
@@ -598,7 +608,7 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
       threadIdx.x == 0 ? *(volatile const unsigned long long*)&a.dstats[ST_SLOTS_USED] : 0ull;
 
   // ---- A: clear outputs, round-1 claims; LRU: stamp the slots hit ----------
-  {
+  if (!claimed) {
     unsigned long long distinct = 0;
     for (uint32_t p = tid; p < a.count; p += nth) {
       gleam_result_t* r = desc(a, p).result;
@@ -649,7 +659,7 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
       if (threadIdx.x == 0 && distinct) atomicAdd(&a.ctl->acc_distinct, distinct);
     }
   }
-  bool ok = grid_barrier(a.ctl, G, a.wait_ns, skip);
+  bool ok = claimed ? ok0 : grid_barrier(a.ctl, G, a.wait_ns, skip);
 
   // ---- B/C: rounds until every chunk is a hit, duplicate or leader ---------
   uint32_t round = 1;
@@ -849,6 +859,124 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
   }
 }
 
+// The end of a call, run by every block: the last block to get here
+// publishes the counters and results and leaves the per-call state (group
+// table, control block) as the next call expects it.  total/stored/evict/
+// vbytes: the call's misses, stored misses, evicted slots and their bytes;
+// s_sum: a grid of one block's sums (hits, intra hits, rejects, miss bytes,
+// stored bytes, chunks written ahead, of them used), else the control block's.
+__device__ __forceinline__ void finish_call(const DedupArgs& a, uint32_t G,
+                                            unsigned long long slots0,
+                                            unsigned long long total,
+                                            unsigned long long s_stored,
+                                            unsigned long long evict,
+                                            unsigned long long s_vbytes,
+                                            const unsigned long long* s_sum) {
+  const uint32_t N = (uint32_t)a.Ntot;
+  __shared__ int s_last;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (G == 1) {  // the block barrier already orders the block's own writes
+      s_last = 1;
+    } else {
+      __threadfence();
+      s_last = atomicAdd(&a.ctl->done, 1u) == G - 1;
+    }
+  }
+  __syncthreads();
+  if (!s_last) return;
+  if (G > 1) __threadfence();
+  const int err = ld_volatile_s32(&a.ctl->err);
+  if (threadIdx.x == 0) {
+    const bool one = G == 1;
+    const unsigned long long misses = total;
+    const unsigned long long hc = one ? s_sum[0] : __ldcg(&a.ctl->acc_hits_cache);
+    const unsigned long long hi2 = one ? s_sum[1] : __ldcg(&a.ctl->acc_hits_intra);
+    const unsigned long long rej = one ? s_sum[2] : __ldcg(&a.ctl->acc_rejects);
+    const unsigned long long mbytes = one ? s_sum[3] : __ldcg(&a.ctl->acc_miss_bytes);
+    const unsigned long long sbytes = one ? s_sum[4] : __ldcg(&a.ctl->acc_stored_bytes);
+    const unsigned long long stored = s_stored;
+    const unsigned long long vbytes = s_vbytes;
+    const unsigned long long spec = one ? s_sum[5] : __ldcg(&a.ctl->spec_tried);
+    const unsigned long long spec_used = one ? s_sum[6] : __ldcg(&a.ctl->spec_used);
+    if (err == 0 && a.spec_state) {
+      // automatic write-through: stays on while at least half of the chunks
+      // written ahead were used; once off, tried again after 256 calls
+      uint32_t* st = a.spec_state;
+      if (spec) {
+        st[0] = 2 * spec_used >= spec ? 1u : 0u;
+        st[1] = 0;
+      } else if (st[0] == 0 && ++st[1] >= 256) {
+        st[0] = 1;
+        st[1] = 0;
+      }
+      *a.spec_mirror = st[0];
+    }
+    if (err == 0) {  // no reads: the counters change by atomic adds
+      atomicAdd(&a.dstats[ST_CALLS], a.ncalls);
+      atomicAdd(&a.dstats[ST_CHUNKS], (unsigned long long)N);
+      atomicAdd(&a.dstats[ST_HITS_CACHE], hc);
+      atomicAdd(&a.dstats[ST_HITS_INTRA], hi2);
+      atomicAdd(&a.dstats[ST_MISSES], misses);
+      atomicAdd(&a.dstats[ST_INSERTS], stored);
+      atomicAdd(&a.dstats[ST_REJECTS], rej);
+      a.dstats[ST_SLOTS_USED] = slots0 + stored - evict;
+      atomicAdd(&a.dstats[ST_BYTES_USED], sbytes - vbytes);
+      atomicAdd(&a.dstats[ST_EVICTIONS], evict);
+      if (spec) atomicAdd(&a.dstats[ST_SPEC_CHUNKS], spec);
+    }
+    gleam_result_t* t = a.total;
+    t->status = err;
+    t->n_miss = err ? 0 : misses;
+    t->n_hit_cache = err ? 0 : hc;
+    t->n_hit_intra = err ? 0 : hi2;
+    t->verify_rejects = err ? 0 : rej;
+    t->miss_bytes = err ? 0 : mbytes;
+  }
+  for (uint32_t p = threadIdx.x; p < a.count; p += kThreads) {
+    gleam_result_t* r = desc(a, p).result;
+    if (!r) continue;
+    r->status = err;
+    if (err) {
+      r->n_miss = 0;
+      r->n_hit_cache = 0;
+      r->n_hit_intra = 0;
+      r->verify_rejects = 0;
+      r->miss_bytes = 0;
+    }
+  }
+  // Leave the per-call state as the next call expects it: the group table
+  // (cleared entry by entry by the leaders, or here in full after an error
+  // that may have stopped them) and the control block.
+  if (err) {
+    for (unsigned long long e = threadIdx.x; e <= a.tbl_mask; e += kThreads) {
+      a.tbl[e].owner = 0u;
+      a.tbl[e].minv = 0u;
+    }
+    if (a.lru) {  // an eviction that stopped half-way may have left these set
+      for (uint32_t j = threadIdx.x; j < kLruBins; j += kThreads) a.bins[j] = 0u;
+      for (unsigned long long j = threadIdx.x; j < a.nslots; j += kThreads) a.vflag[j] = 0;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    DevCtl* c = a.ctl;
+    c->bar_count = 0;
+    c->err = 0;
+    c->unres[0] = c->unres[1] = c->unres[2] = 0;
+    c->shared_groups = 0;
+    c->acc_hits_cache = c->acc_hits_intra = c->acc_rejects = 0;
+    c->acc_misses = c->acc_miss_bytes = 0;
+    c->acc_stored = c->acc_stored_bytes = 0;
+    c->acc_distinct = c->evict_k = c->lru_below = c->lru_ties = c->acc_victim_bytes = 0;
+    c->lru_hi = c->lru_cut = 0;
+    c->spec_tried = c->spec_used = 0;
+    c->done = 0;
+  }
+  __threadfence();
+}
+
+
 // Second kernel of the call (a regular launch sized for the copies): hit
 // masks, miss indices, chunk slots, per-payload counters, then every miss by
 // rank copied by whole warps to the packed output and its arena slot and
@@ -1001,59 +1129,69 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
       }
     }
     flush();
-    // Every miss, by rank.  Warp gw owns the contiguous ranks [lo, hi): its
-    // lanes fetch the metadata of 32 ranks at once, the whole warp copies the
-    // 32 chunks one after the other to the packed output and their arena
-    // slots (all but those the hash kernel already wrote there), then each
-    // lane inserts its own chunk (32 independent probes).
+    // Every miss's bytes, in pieces of kPackPiece bytes: piece k of the miss
+    // of rank r is number r * ppc + k (ppc = pieces of a whole chunk; a
+    // shorter miss has fewer), and warp gw owns the contiguous numbers
+    // [plo, phi), so that a call with few misses still spreads its copies over
+    // every warp (one 64 KiB miss is 32 pieces) and a call with many streams
+    // whole runs of chunks per warp.  The lanes fetch the metadata of 32
+    // pieces at once (mostly one chunk's: the same addresses), then the pieces
+    // go to the packed output and the miss's arena slot, all but those of
+    // misses the hash kernel already wrote there.
     const unsigned long long nw = (unsigned long long)G * kWarps;
     const unsigned long long gw = (unsigned long long)bid * kWarps + w;
-    const unsigned long long lo = total * gw / nw, hi = total * (gw + 1) / nw;
-    for (unsigned long long base = lo; base < hi; base += 32) {
-      const unsigned long long r = base + lane;
-      const bool have = r < hi;
-      uint32_t gg = 0, ln = 0;
-      bool cached = false, copy = false;
-      unsigned long long slot = 0, src = 0, d1 = 0, d2 = 0;
-      if (have) {
-        gg = ch.order[r];
-        const uint32_t pp = ch.pidx[gg];
-        const PayloadDesc& P = desc(a, pp);
-        ln = ch.len[gg];
-        src = ch.src[gg];
-        d1 = (unsigned long long)(P.packed + (r - a.pstart[pp]) * a.C);
-        cached = !(ch.res[gg] & kResNoSlot);  // else sent, never cached
-        uint32_t sr = 0xFFFFFFFFu;
-        if (cached) {
-          sr = ch.srank[gg];
-          slot = slot_of(sr);
-          d2 = (unsigned long long)(a.arena + slot * a.C);
+    const unsigned long long ppc = (a.C + kPackPiece - 1) / kPackPiece;
+    const unsigned long long npieces = total * ppc;
+    const unsigned long long plo = npieces * gw / nw, phi = npieces * (gw + 1) / nw;
+    // written ahead by the hash kernel exactly where it belongs: with no
+    // eviction, stored rank g means every earlier chunk of the call is a
+    // stored miss, so the chunk's packed offset is i*C and its slot
+    // slots_used + g, the places it was written to
+    auto written_ahead = [&](uint32_t gg, uint32_t sr) {
+      return a.spec_active && evict == 0 && sr == gg && ch.spec[gg];
+    };
+    for (unsigned long long base = plo; base < phi; base += 32) {
+      const unsigned long long pc = base + lane;
+      uint32_t bytes = 0;
+      bool copy = false;
+      unsigned long long src = 0, d1 = 0, d2 = 0;
+      if (pc < phi) {
+        const unsigned long long r = pc / ppc;
+        const uint32_t off = (uint32_t)(pc - r * ppc) * kPackPiece;
+        const uint32_t gg = ch.order[r];
+        const uint32_t ln = ch.len[gg];
+        if (off < ln) {
+          const uint32_t pp = ch.pidx[gg];
+          const PayloadDesc& P = desc(a, pp);
+          bytes = min(kPackPiece, ln - off);
+          src = ch.src[gg] + off;
+          d1 = (unsigned long long)(P.packed + (r - a.pstart[pp]) * a.C + off);
+          uint32_t sr = 0xFFFFFFFFu;
+          if (!(ch.res[gg] & kResNoSlot)) {  // else sent, never cached
+            sr = ch.srank[gg];
+            d2 = (unsigned long long)(a.arena + slot_of(sr) * a.C + off);
+          }
+          copy = !written_ahead(gg, sr);
         }
-        // written ahead by the hash kernel exactly where it belongs: with no
-        // eviction, stored rank g means every earlier chunk of the call is a
-        // stored miss, so the chunk's packed offset is i*C and its slot
-        // slots_used + g, the places it was written to
-        copy = !(a.spec_active && evict == 0 && sr == gg && ch.spec[gg]);
-        n_spec_used += !copy;
       }
-      const unsigned cmask = __ballot_sync(0xffffffffu, copy);  // lanes whose chunk is copied
+      const unsigned cmask = __ballot_sync(0xffffffffu, copy);  // lanes whose piece is copied
       const uint32_t m = __popc(cmask);
 #if GLEAM_PACK_BULK
       const bool bulk =
           !a.plain_copy && __all_sync(0xffffffffu, !copy || ((src | d1 | d2) & 15) == 0);
       if (bulk) {
-        if (copy) meta[__popc(cmask & ((1u << lane) - 1u))] = PackMeta{src, d1, d2, ln, 0u};
+        if (copy) meta[__popc(cmask & ((1u << lane) - 1u))] = PackMeta{src, d1, d2, bytes, 0u};
         __syncwarp();
         if (lane == 0 && m && !bulk_failed &&
             !bulk_copy_batch(meta, m, bufs, bars, ring, a.wait_ns)) {
           bulk_failed = true;
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_TIMEOUT);
         }
-        if (copy) {  // the last len % 16 bytes
+        if (copy) {  // the piece's last bytes % 16 (only a miss's last piece has any)
           const uint8_t* sp = reinterpret_cast<const uint8_t*>(src);
           uint8_t* x = reinterpret_cast<uint8_t*>(d1);
           uint8_t* y = reinterpret_cast<uint8_t*>(d2);
-          for (uint32_t k = ln & ~15u; k < ln; ++k) {
+          for (uint32_t k = bytes & ~15u; k < bytes; ++k) {
             x[k] = sp[k];
             if (y) y[k] = sp[k];
           }
@@ -1066,19 +1204,31 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
         const unsigned long long sj = __shfl_sync(0xffffffffu, src, j);
         const unsigned long long xj = __shfl_sync(0xffffffffu, d1, j);
         const unsigned long long yj = __shfl_sync(0xffffffffu, d2, j);
-        const uint32_t lj = __shfl_sync(0xffffffffu, ln, j);
+        const uint32_t lj = __shfl_sync(0xffffffffu, bytes, j);
         warp_copy2(reinterpret_cast<uint8_t*>(xj), reinterpret_cast<uint8_t*>(yj),
                    reinterpret_cast<const uint8_t*>(sj), lj, ((sj | xj | yj) & 15) == 0);
       }
-      if (have && cached) {
-        a.slot_len[slot] = ln;
-        if (a.lru) a.last_use[slot] = a.epoch;
-        if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
-          atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-        if (!a.paper && ln >= kPrefixBytes &&
-            !index_insert(a.hints, a.index_mask, ch.hint[gg], (uint32_t)slot, ln))
-          atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-      }
+    }
+    // Every miss's index and hint-table entries, by rank: warp gw owns the
+    // contiguous ranks [lo, hi), each lane inserting its own chunk (32
+    // independent probes at a time).
+    const unsigned long long lo = total * gw / nw, hi = total * (gw + 1) / nw;
+    for (unsigned long long base = lo; base < hi; base += 32) {
+      const unsigned long long r = base + lane;
+      if (r >= hi) continue;
+      const uint32_t gg = ch.order[r];
+      if (ch.res[gg] & kResNoSlot) continue;  // sent, never cached
+      const uint32_t ln = ch.len[gg];
+      const uint32_t sr = ch.srank[gg];
+      const unsigned long long slot = slot_of(sr);
+      n_spec_used += written_ahead(gg, sr);
+      a.slot_len[slot] = ln;
+      if (a.lru) a.last_use[slot] = a.epoch;
+      if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
+        atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+      if (!a.paper && ln >= kPrefixBytes &&
+          !index_insert(a.hints, a.index_mask, ch.hint[gg], (uint32_t)slot, ln))
+        atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
     }
 #if GLEAM_PACK_BULK
     if (lane == 0) bulk_wait_all<0>();  // every piece written before the block ends
@@ -1109,107 +1259,306 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
     }
   }
 
-  // ---- epilogue: the last block publishes ----------------------------------
-  __shared__ int s_last;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    if (G == 1) {  // the block barrier already orders the block's own writes
-      s_last = 1;
+  finish_call(a, G, slots0, total, s_stored, evict, s_vbytes, s_sum);
+}
+
+// ---- one-launch resolve + pack of a one-payload call --------------------------
+//
+// A call of one payload that is launched chained (few enough chunks to leave
+// most of the GPU idle) runs its resolution, ranks, packing and publishing in
+// one launch.  Block b owns the contiguous chunks [b * per, (b + 1) * per),
+// at most one per thread.  Phase 1 classifies them and claims their (key,
+// length) groups without posting minima.  If no chunk of the call found its
+// group claimed by another (no in-call duplicate and no key collision: the
+// common case), every chunk that is not a cache hit is a miss of round one
+// (its own group's first chunk), so after one grid barrier each block knows
+// its misses' ranks from the blocks' counts and copies and inserts its own
+// misses.  Otherwise the general algorithm takes over: the minima are posted
+// and resolve_rank and pack_publish run on the same grid.
+struct LeadCopy {  // a block's miss, by its rank in the block
+  unsigned long long src, d1, d2;
+  uint32_t len, copy;
+};
+constexpr uint32_t kLeadBytes = kThreads * (uint32_t)sizeof(LeadCopy);
+constexpr uint32_t kResolvePackSmem = kPackSmem + kLeadBytes;
+
+__device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G, uint32_t bid,
+                                                  uint8_t* smem) {
+  __shared__ unsigned long long red64[kWarps];
+  __shared__ uint32_t wcnt[kWarps], swcnt[kWarps];
+  __shared__ unsigned long long s_slots0, s_sum[7], s_tot[4];
+  __shared__ int s_shared, s_err;
+  const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const ChunkArrays& ch = a.ch;
+  const PayloadDesc& P = a.one;
+  const uint32_t N = (uint32_t)a.Ntot;
+  const uint32_t per = (N + G - 1) / G;  // <= kThreads (the host sizes the grid)
+  const uint32_t g = bid * per + threadIdx.x;
+  const bool valid = threadIdx.x < per && g < N;
+  if (per > kThreads && threadIdx.x == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+  const unsigned long long my_slots0 =
+      threadIdx.x == 0 ? *(volatile const unsigned long long*)&a.dstats[ST_SLOTS_USED] : 0ull;
+  if (threadIdx.x == 0) s_shared = 0;
+
+  // ---- 1: classify, clear the outputs, claim the groups ----------------------
+  if (bid == 0 && threadIdx.x == 0 && P.result) {
+    gleam_result_t* r = P.result;
+    r->n_miss = r->n_hit_cache = r->n_hit_intra = r->verify_rejects = r->miss_bytes = 0;
+  }
+  uint8_t st = kMissNoCand;
+  uint32_t len = 0, e = 0xFFFFFFFFu;
+  unsigned long long key = 0;
+  bool lead = false, stored = false, shared = false;
+  if (valid) {
+    st = ch.status[g];
+    if ((g & 31) == 0) P.mask[g >> 5] = 0;
+    if (st == kHit0) {
+      ch.res[g] = kResHit0;
+    } else if (st == kUncached) {  // never cached: a miss of its own, in no group
+      ch.ent[g] = 0xFFFFFFFFu;
+      ch.res[g] = kResLeader | kResNoSlot | 1u;
+      lead = true;
+      len = ch.len[g];
     } else {
-      __threadfence();
-      s_last = atomicAdd(&a.ctl->done, 1u) == G - 1;
-    }
-  }
-  __syncthreads();
-  if (!s_last) return;
-  if (G > 1) __threadfence();
-  const int err = ld_volatile_s32(&a.ctl->err);
-  if (threadIdx.x == 0) {
-    const bool one = G == 1;
-    const unsigned long long misses = total;
-    const unsigned long long hc = one ? s_sum[0] : __ldcg(&a.ctl->acc_hits_cache);
-    const unsigned long long hi2 = one ? s_sum[1] : __ldcg(&a.ctl->acc_hits_intra);
-    const unsigned long long rej = one ? s_sum[2] : __ldcg(&a.ctl->acc_rejects);
-    const unsigned long long mbytes = one ? s_sum[3] : __ldcg(&a.ctl->acc_miss_bytes);
-    const unsigned long long sbytes = one ? s_sum[4] : __ldcg(&a.ctl->acc_stored_bytes);
-    const unsigned long long stored = s_stored;
-    const unsigned long long vbytes = s_vbytes;
-    const unsigned long long spec = one ? s_sum[5] : __ldcg(&a.ctl->spec_tried);
-    const unsigned long long spec_used = one ? s_sum[6] : __ldcg(&a.ctl->spec_used);
-    if (err == 0 && a.spec_state) {
-      // automatic write-through: stays on while at least half of the chunks
-      // written ahead were used; once off, tried again after 256 calls
-      uint32_t* st = a.spec_state;
-      if (spec) {
-        st[0] = 2 * spec_used >= spec ? 1u : 0u;
-        st[1] = 0;
-      } else if (st[0] == 0 && ++st[1] >= 256) {
-        st[0] = 1;
-        st[1] = 0;
+      key = ch.key[g];
+      len = ch.len[g];
+      bool claimed = true;
+      e = group_entry(a, g, key, len, &claimed);
+      if (e == 0xFFFFFFFFu) {
+        atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+        ch.res[g] = kResLeader | 1u;
+      } else {
+        ch.res[g] = kResUnresolved;
       }
-      *a.spec_mirror = st[0];
-    }
-    if (err == 0) {  // no reads: the counters change by atomic adds
-      atomicAdd(&a.dstats[ST_CALLS], a.ncalls);
-      atomicAdd(&a.dstats[ST_CHUNKS], (unsigned long long)N);
-      atomicAdd(&a.dstats[ST_HITS_CACHE], hc);
-      atomicAdd(&a.dstats[ST_HITS_INTRA], hi2);
-      atomicAdd(&a.dstats[ST_MISSES], misses);
-      atomicAdd(&a.dstats[ST_INSERTS], stored);
-      atomicAdd(&a.dstats[ST_REJECTS], rej);
-      a.dstats[ST_SLOTS_USED] = slots0 + stored - evict;
-      atomicAdd(&a.dstats[ST_BYTES_USED], sbytes - vbytes);
-      atomicAdd(&a.dstats[ST_EVICTIONS], evict);
-      if (spec) atomicAdd(&a.dstats[ST_SPEC_CHUNKS], spec);
-    }
-    gleam_result_t* t = a.total;
-    t->status = err;
-    t->n_miss = err ? 0 : misses;
-    t->n_hit_cache = err ? 0 : hc;
-    t->n_hit_intra = err ? 0 : hi2;
-    t->verify_rejects = err ? 0 : rej;
-    t->miss_bytes = err ? 0 : mbytes;
-  }
-  for (uint32_t p = threadIdx.x; p < a.count; p += kThreads) {
-    gleam_result_t* r = desc(a, p).result;
-    if (!r) continue;
-    r->status = err;
-    if (err) {
-      r->n_miss = 0;
-      r->n_hit_cache = 0;
-      r->n_hit_intra = 0;
-      r->verify_rejects = 0;
-      r->miss_bytes = 0;
+      ch.ent[g] = e;
+      shared = !claimed;
+      lead = stored = true;
     }
   }
-  // Leave the per-call state as the next call expects it: the group table
-  // (cleared entry by entry by the leaders, or here in full after an error
-  // that may have stopped them) and the control block.
-  if (err) {
-    for (unsigned long long e = threadIdx.x; e <= a.tbl_mask; e += kThreads) {
-      a.tbl[e].owner = 0u;
-      a.tbl[e].minv = 0u;
-    }
-    if (a.lru) {  // an eviction that stopped half-way may have left these set
-      for (uint32_t j = threadIdx.x; j < kLruBins; j += kThreads) a.bins[j] = 0u;
-      for (unsigned long long j = threadIdx.x; j < a.nslots; j += kThreads) a.vflag[j] = 0;
-    }
+  const uint32_t c_b = __syncthreads_count(lead);
+  const uint32_t s_b = __syncthreads_count(stored);
+  if (__syncthreads_or(shared) && threadIdx.x == 0) {
+    s_shared = 1;
+    if (G > 1) atomicOr(&a.ctl->shared_groups, 1u);
+  }
+  if (G > 1 && threadIdx.x == 0) {
+    a.bcount[bid] = c_b;
+    a.bcount[G + bid] = s_b;
+  }
+  bool ok = grid_barrier(a.ctl, G, a.wait_ns, false);
+  if (threadIdx.x == 0) {
+    if (G > 1) s_shared = (int)ldcg_u32(&a.ctl->shared_groups);
+    s_slots0 = my_slots0;
+    s_err = G == 1 ? ld_volatile_s32(&a.ctl->err) : 0;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    DevCtl* c = a.ctl;
-    c->bar_count = 0;
-    c->err = 0;
-    c->unres[0] = c->unres[1] = c->unres[2] = 0;
-    c->acc_hits_cache = c->acc_hits_intra = c->acc_rejects = 0;
-    c->acc_misses = c->acc_miss_bytes = 0;
-    c->acc_stored = c->acc_stored_bytes = 0;
-    c->acc_distinct = c->evict_k = c->lru_below = c->lru_ties = c->acc_victim_bytes = 0;
-    c->lru_hi = c->lru_cut = 0;
-    c->spec_tried = c->spec_used = 0;
-    c->done = 0;
+  if (G == 1) ok = s_err == 0;  // a grid of one did not read the error word
+
+  if (s_shared) {
+    // the general algorithm: post the group minima, then the rounds, ranks
+    // and copies of k_dedup and k_pack on this grid
+    if (ok) {  // every lane of the block takes part (one chunk per thread at most)
+      const bool post = valid && e != 0xFFFFFFFFu && st != kHit0 && st != kUncached;
+      post_minimum(a, post ? e : 0xFFFFFFFFu, g);
+    }
+    ok = grid_barrier(a.ctl, G, a.wait_ns, false);
+    resolve_rank(a, G, bid, true, ok);
+    grid_barrier(a.ctl, G, a.wait_ns, false);
+    pack_publish(a, G, bid, smem);
+    return;
   }
-  __threadfence();
+
+  // ---- 2: the fast path: ranks, outputs, copies, inserts ---------------------
+  const unsigned long long slots0 = s_slots0;
+  unsigned long long before = 0, total = c_b, sbefore = 0, stotal = s_b;
+  if (G > 1) {
+    unsigned long long b0 = 0, t0 = 0, sb0 = 0, st0 = 0;
+    for (uint32_t j = threadIdx.x; j < G; j += kThreads) {
+      const uint32_t v = ldcg_u32(&a.bcount[j]), sv = ldcg_u32(&a.bcount[G + j]);
+      t0 += v;
+      st0 += sv;
+      if (j < bid) {
+        b0 += v;
+        sb0 += sv;
+      }
+    }
+    before = block_sum<unsigned long long>(b0, red64);
+    total = block_sum<unsigned long long>(t0, red64);
+    sbefore = block_sum<unsigned long long>(sb0, red64);
+    stotal = block_sum<unsigned long long>(st0, red64);
+  }
+  if (ok && stotal > a.nslots - slots0) {  // every block decides the same
+    if (threadIdx.x == 0) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_CAPACITY);
+    ok = false;
+  }
+  unsigned long long n_hc = 0, n_rej = 0, n_bytes = 0, n_sbytes = 0;
+  uint32_t n_spec = 0, n_spec_used = 0;
+  LeadCopy* leads = reinterpret_cast<LeadCopy*>(smem + kPackSmem);
+  if (ok) {
+    // ranks within the block, in chunk order
+    const uint32_t mb = __ballot_sync(0xffffffffu, lead);
+    const uint32_t sb = __ballot_sync(0xffffffffu, stored);
+    if (lane == 0) {
+      wcnt[w] = __popc(mb);
+      swcnt[w] = __popc(sb);
+    }
+    __syncthreads();
+    uint32_t woff = 0, swoff = 0;
+    for (uint32_t k2 = 0; k2 < w; ++k2) {
+      woff += wcnt[k2];
+      swoff += swcnt[k2];
+    }
+    const uint32_t below = (1u << lane) - 1u;
+    const uint32_t lr = woff + __popc(mb & below);
+    const unsigned long long r = before + lr;
+    const unsigned long long sr = sbefore + swoff + __popc(sb & below);
+    const unsigned long long slot = slots0 + sr;
+    const bool spec = a.spec_active && valid && ch.spec[g];
+    // written ahead by the hash kernel where it belongs: stored rank g means
+    // every earlier chunk is a stored miss (no eviction here)
+    const bool ahead = spec && stored && sr == g;
+    n_spec += spec;
+    n_spec_used += ahead;
+    if (lead) {
+      P.miss_idx[r] = g;
+      n_rej += st == kMissCand;
+      n_bytes += len;
+      if (stored) n_sbytes += len;
+      leads[lr] = LeadCopy{(unsigned long long)(P.buf + (unsigned long long)g * a.C),
+                           (unsigned long long)(P.packed + r * a.C),
+                           stored ? (unsigned long long)(a.arena + slot * a.C) : 0ull, len,
+                           ahead ? 0u : 1u};
+    }
+    // hit-mask words: one atomic per group of lanes that share a word
+    const bool hit = valid && st == kHit0;
+    n_hc += hit;
+    const unsigned long long mw = hit ? (unsigned long long)(P.mask + (g >> 5)) : 0ull;
+    const unsigned mpeers = __match_any_sync(0xffffffffu, mw);
+    const uint32_t bits = __reduce_or_sync(mpeers, hit ? 1u << (g & 31) : 0u);
+    if (mw && lane == (uint32_t)(__ffs(mpeers) - 1)) atomicOr((uint32_t*)mw, bits);
+    if (P.chunk_slot && valid)
+      P.chunk_slot[g] = hit ? ch.ent[g] : stored ? (uint32_t)slot : kEmptySlot;
+    __syncthreads();  // the block's miss table is written
+
+    // the block's misses, in pieces of kPackPiece bytes spread over its warps
+    const unsigned long long ppc = (a.C + kPackPiece - 1) / kPackPiece;
+    const unsigned long long npieces = (unsigned long long)c_b * ppc;
+    const unsigned long long plo = npieces * w / kWarps, phi = npieces * (w + 1) / kWarps;
+#if GLEAM_PACK_BULK
+    const uint32_t wbase = (uint32_t)__cvta_generic_to_shared(smem) + w * kPackWarpBytes;
+    const uint32_t bufs = wbase, bars = wbase + kPackBufs * kPackPiece;
+    PackMeta* meta = reinterpret_cast<PackMeta*>(smem + w * kPackWarpBytes + kPackBufs * kPackPiece + 64);
+    PackRing ring{0u, 0u, 0u};
+    bool bulk_failed = false;
+    if (lane == 0) {
+      for (uint32_t b = 0; b < kPackBufs; ++b) mbar_init(bars + 8 * b);
+      mbar_fence_init();
+    }
+    __syncwarp();
+#endif
+    for (unsigned long long base = plo; base < phi; base += 32) {
+      const unsigned long long pc = base + lane;
+      uint32_t bytes = 0;
+      bool copy = false;
+      unsigned long long src = 0, d1 = 0, d2 = 0;
+      if (pc < phi) {
+        const LeadCopy& L = leads[pc / ppc];
+        const uint32_t off = (uint32_t)(pc % ppc) * kPackPiece;
+        if (off < L.len && L.copy) {
+          bytes = min(kPackPiece, L.len - off);
+          src = L.src + off;
+          d1 = L.d1 + off;
+          d2 = L.d2 ? L.d2 + off : 0ull;
+          copy = true;
+        }
+      }
+      const unsigned cmask = __ballot_sync(0xffffffffu, copy);
+#if GLEAM_PACK_BULK
+      const bool bulk =
+          !a.plain_copy && __all_sync(0xffffffffu, !copy || ((src | d1 | d2) & 15) == 0);
+      if (bulk) {
+        if (copy) meta[__popc(cmask & ((1u << lane) - 1u))] = PackMeta{src, d1, d2, bytes, 0u};
+        __syncwarp();
+        if (lane == 0 && cmask && !bulk_failed &&
+            !bulk_copy_batch(meta, __popc(cmask), bufs, bars, ring, a.wait_ns)) {
+          bulk_failed = true;
+          atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_TIMEOUT);
+        }
+        if (copy) {  // the piece's last bytes % 16
+          const uint8_t* sp = reinterpret_cast<const uint8_t*>(src);
+          uint8_t* x = reinterpret_cast<uint8_t*>(d1);
+          uint8_t* y = reinterpret_cast<uint8_t*>(d2);
+          for (uint32_t k2 = bytes & ~15u; k2 < bytes; ++k2) {
+            x[k2] = sp[k2];
+            if (y) y[k2] = sp[k2];
+          }
+        }
+        __syncwarp();
+      } else
+#endif
+      for (unsigned todo = cmask; todo; todo &= todo - 1) {
+        const int j = __ffs(todo) - 1;
+        const unsigned long long sj = __shfl_sync(0xffffffffu, src, j);
+        const unsigned long long xj = __shfl_sync(0xffffffffu, d1, j);
+        const unsigned long long yj = __shfl_sync(0xffffffffu, d2, j);
+        const uint32_t lj = __shfl_sync(0xffffffffu, bytes, j);
+        warp_copy2(reinterpret_cast<uint8_t*>(xj), reinterpret_cast<uint8_t*>(yj),
+                   reinterpret_cast<const uint8_t*>(sj), lj, ((sj | xj | yj) & 15) == 0);
+      }
+    }
+    // each stored miss inserts itself and frees the group entry it claimed
+    if (stored) {
+      a.slot_len[slot] = len;
+      if (!index_insert(a.index, a.index_mask, key, (uint32_t)slot, len))
+        atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+      if (!a.paper && len >= kPrefixBytes &&
+          !index_insert(a.hints, a.index_mask, ch.hint[g], (uint32_t)slot, len))
+        atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+      if (e != 0xFFFFFFFFu) a.tbl[e].owner = 0u;
+    }
+#if GLEAM_PACK_BULK
+    if (lane == 0) bulk_wait_all<0>();  // every piece written before the block ends
+#endif
+  }
+  n_hc = block_sum<unsigned long long>(n_hc, red64);
+  n_rej = block_sum<unsigned long long>(n_rej, red64);
+  n_bytes = block_sum<unsigned long long>(n_bytes, red64);
+  n_sbytes = block_sum<unsigned long long>(n_sbytes, red64);
+  const unsigned long long b_spec = block_sum<unsigned long long>(n_spec, red64);
+  const unsigned long long b_spec_used = block_sum<unsigned long long>(n_spec_used, red64);
+  if (threadIdx.x == 0 && P.result) {  // the payload's own counters (cleared in phase 1)
+    gleam_result_t* res = P.result;
+    if (n_hc) atomicAdd((unsigned long long*)&res->n_hit_cache, n_hc);
+    if (c_b) atomicAdd((unsigned long long*)&res->n_miss, (unsigned long long)c_b);
+    if (n_rej) atomicAdd((unsigned long long*)&res->verify_rejects, n_rej);
+    if (n_bytes) atomicAdd((unsigned long long*)&res->miss_bytes, n_bytes);
+  }
+  if (threadIdx.x == 0) {
+    if (G == 1) {
+      s_sum[0] = n_hc;
+      s_sum[1] = 0;  // no in-call duplicate on this path
+      s_sum[2] = n_rej;
+      s_sum[3] = n_bytes;
+      s_sum[4] = n_sbytes;
+      s_sum[5] = b_spec;
+      s_sum[6] = b_spec_used;
+    } else {
+      if (n_hc) atomicAdd(&a.ctl->acc_hits_cache, n_hc);
+      if (n_rej) atomicAdd(&a.ctl->acc_rejects, n_rej);
+      if (n_bytes) atomicAdd(&a.ctl->acc_miss_bytes, n_bytes);
+      if (n_sbytes) atomicAdd(&a.ctl->acc_stored_bytes, n_sbytes);
+      if (b_spec) atomicAdd(&a.ctl->spec_tried, b_spec);
+      if (b_spec_used) atomicAdd(&a.ctl->spec_used, b_spec_used);
+    }
+  }
+  finish_call(a, G, slots0, total, stotal, 0ull, 0ull, s_sum);
+}
+
+__global__ void __launch_bounds__(kThreads) k_resolve_pack(DedupArgs a) {
+  extern __shared__ __align__(128) uint8_t rp_smem[];
+  pdl_trigger();
+  pdl_wait();
+  resolve_pack_fast(a, gridDim.x, blockIdx.x, rp_smem);
 }
 
 __global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
@@ -1397,6 +1746,12 @@ cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream
     cudaFuncSetAttribute((const void*)k_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          kPackSmem);
   return launch_kernel(k_pack, dim3(pack_grid), dim3(kThreads), kPackSmem, s, pdl, a);
+}
+
+cudaError_t launch_resolve_pack(const DedupArgs& a, int grid, cudaStream_t s) {
+  cudaFuncSetAttribute((const void*)k_resolve_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       kResolvePackSmem);
+  return launch_kernel(k_resolve_pack, dim3(grid), dim3(kThreads), kResolvePackSmem, s, true, a);
 }
 
 uint32_t small_call_groups() { return kSmallGroups; }

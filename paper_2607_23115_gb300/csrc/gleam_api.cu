@@ -472,12 +472,15 @@ void note_call(gleam_cache* c, uint64_t Ntot) {
 // programmatic stream serialization: each kernel lets the next one on the
 // stream be launched as soon as all of its blocks have started, so that a
 // kernel's blocks are waiting on the GPU when the one before finishes instead
-// of being launched then.  The resolve kernel is then a regular launch (a
-// cooperative one is never launched early) on at most kChainDedupBlocks
-// blocks, and the pack kernel runs on at most kChainPackBlocks: every waiting
-// block holds its SM resources.  With GLEAM_OVERLAP_CALLS the hash kernel also
-// fingerprints before it waits (HashArgs::wait_late).  Evicting caches and the
-// test hook that makes a block skip a barrier keep the plain launches.
+// of being launched then.  After the hash kernel, a call of one payload runs
+// resolve, ranks, pack and publish as one launch (k_resolve_pack, one block
+// per 256 chunks or kChainBytesPerBlock of payload, at most kChainPackBlocks);
+// a batch runs the resolve kernel as a regular launch (a cooperative one is
+// never launched early) on at most kChainDedupBlocks blocks and the pack
+// kernel on at most kChainPackBlocks: every waiting block holds its SM
+// resources.  With GLEAM_OVERLAP_CALLS the hash kernel also fingerprints
+// before it waits (HashArgs::wait_late).  Evicting caches and the test hook
+// that makes a block skip a barrier keep the plain launches.
 #ifndef GLEAM_CHAIN_MAX_CHUNKS
 #define GLEAM_CHAIN_MAX_CHUNKS 8192
 #endif
@@ -491,6 +494,9 @@ constexpr uint64_t kChainMaxChunks = GLEAM_CHAIN_MAX_CHUNKS;
 constexpr uint64_t kChainMaxBytes = 1ull << 30;
 constexpr int kChainDedupBlocks = GLEAM_CHAIN_DEDUP_BLOCKS;
 constexpr int kChainPackBlocks = GLEAM_CHAIN_PACK_BLOCKS;
+constexpr uint64_t kChainBytesPerBlock = 2ull << 20;
+// the one-launch resolve kernel holds at most one chunk per thread
+static_assert(kChainMaxChunks <= (uint64_t)kChainPackBlocks * 256, "chain limit");
 
 bool chain_call(const gleam_cache* c, uint64_t Ntot, uint64_t nbytes, int skip_block) {
   return Ntot <= kChainMaxChunks && nbytes <= kChainMaxBytes && skip_block < 0 &&
@@ -695,10 +701,23 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
     if (ev[1]) cudaEventRecord(ev[1], s);
     int pgrid = pack_grid(c, Ntot, nbytes);
     if (chain) {
-      grid = std::min(grid, kChainDedupBlocks);
+      // one chunk per thread of the resolve kernel: a call of at most 256
+      // chunks resolves in one block, without any grid-wide barrier
+      grid = (int)std::min<uint64_t>(kChainDedupBlocks, (Ntot + 255) / 256);
       pgrid = std::min(pgrid, kChainPackBlocks);
     }
-    if ((rc = cuda_err(launch_dedup(d, grid, pgrid, s, chain))) != GLEAM_OK) {
+    if (chain && count == 1) {
+      // one launch: at most one chunk per thread, and one block per
+      // kChainBytesPerBlock of payload so that the misses' copies spread
+      const uint64_t want = std::max<uint64_t>((Ntot + dedup_threads() - 1) / dedup_threads(),
+                                               (nbytes + kChainBytesPerBlock - 1) /
+                                                   kChainBytesPerBlock);
+      rc = cuda_err(launch_resolve_pack(
+          d, (int)std::min<uint64_t>(std::max<uint64_t>(1, want), kChainPackBlocks), s));
+    } else {
+      rc = cuda_err(launch_dedup(d, grid, pgrid, s, chain));
+    }
+    if (rc != GLEAM_OK) {
       cudaMemsetAsync(c->ctl, 0, sizeof(DevCtl), s);  // the hash kernel may have flagged it
       return rc;
     }

@@ -60,7 +60,7 @@ struct DevCtl {
   int err;
   unsigned int done;
   unsigned int unres[3];
-  unsigned int pad0;
+  unsigned int shared_groups;  // a chunk found its (key, length) group claimed by another
   unsigned long long acc_hits_cache;
   unsigned long long acc_hits_intra;
   unsigned long long acc_rejects;
@@ -234,6 +234,9 @@ cudaError_t load_hash_kernels();
 // later on the stream can start, so its grid barriers still complete.
 cudaError_t launch_dedup(const DedupArgs& a, int grid, int pack_grid, cudaStream_t s,
                          bool pdl = false);
+// Resolve, rank, pack and publish of a one-payload call in one launch on
+// `grid` blocks (see k_resolve_pack), with programmatic stream serialization.
+cudaError_t launch_resolve_pack(const DedupArgs& a, int grid, cudaStream_t s);
 // A whole call (hash, resolve and rank, pack) as one single-block kernel, for
 // calls with few chunks whose payloads suit the staged hash (16-byte aligned)
 // outside GLEAM_PAPER_IDS mode; the block hashes small_call_groups() chunks at
