@@ -57,6 +57,9 @@ constexpr int kWarps = kThreads / 32;
 #ifndef GLEAM_DEDUP_CHUNKS_PER_BLOCK
 #define GLEAM_DEDUP_CHUNKS_PER_BLOCK 1024
 #endif
+#ifndef GLEAM_CHAIN_PREFETCH
+#define GLEAM_CHAIN_PREFETCH 1
+#endif
 #ifndef GLEAM_PACK_MINBLOCKS
 #define GLEAM_PACK_MINBLOCKS 3
 #endif
@@ -285,6 +288,10 @@ __device__ bool bulk_copy_batch(const PackMeta* meta, uint32_t m, uint32_t bufs,
     }
   }
   return true;
+}
+
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
 // Claims a free index entry for (key, slot, len); false if the table is full.
@@ -1272,15 +1279,13 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
 // group claimed by another (no in-call duplicate and no key collision: the
 // common case), every chunk that is not a cache hit is a miss of round one
 // (its own group's first chunk), so after one grid barrier each block knows
-// its misses' ranks from the blocks' counts and copies and inserts its own
-// misses.  Otherwise the general algorithm takes over: the minima are posted
-// and resolve_rank and pack_publish run on the same grid.
-struct LeadCopy {  // a block's miss, by its rank in the block
-  unsigned long long src, d1, d2;
-  uint32_t len, copy;
-};
-constexpr uint32_t kLeadBytes = kThreads * (uint32_t)sizeof(LeadCopy);
-constexpr uint32_t kResolvePackSmem = kPackSmem + kLeadBytes;
+// its misses' ranks from the blocks' counts, writes the outputs and inserts
+// its misses; after a second barrier every warp of the grid copies its share
+// of all misses' bytes (a block's own misses would leave the blocks that hold
+// the most of them as the call's tail).  Otherwise the general algorithm
+// takes over: the minima are posted and resolve_rank and pack_publish run on
+// the same grid.
+constexpr uint32_t kResolvePackSmem = kPackSmem;
 
 __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G, uint32_t bid,
                                                   uint8_t* smem) {
@@ -1368,7 +1373,7 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
     return;
   }
 
-  // ---- 2: the fast path: ranks, outputs, copies, inserts ---------------------
+  // ---- 2: the fast path: ranks, outputs, inserts; then copies ----------------
   const unsigned long long slots0 = s_slots0;
   unsigned long long before = 0, total = c_b, sbefore = 0, stotal = s_b;
   if (G > 1) {
@@ -1393,7 +1398,7 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
   }
   unsigned long long n_hc = 0, n_rej = 0, n_bytes = 0, n_sbytes = 0;
   uint32_t n_spec = 0, n_spec_used = 0;
-  LeadCopy* leads = reinterpret_cast<LeadCopy*>(smem + kPackSmem);
+  unsigned long long ins_slot = ~0ull;  // the slot this thread's stored miss takes
   if (ok) {
     // ranks within the block, in chunk order
     const uint32_t mb = __ballot_sync(0xffffffffu, lead);
@@ -1409,25 +1414,19 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
       swoff += swcnt[k2];
     }
     const uint32_t below = (1u << lane) - 1u;
-    const uint32_t lr = woff + __popc(mb & below);
-    const unsigned long long r = before + lr;
+    const unsigned long long r = before + woff + __popc(mb & below);
     const unsigned long long sr = sbefore + swoff + __popc(sb & below);
     const unsigned long long slot = slots0 + sr;
     const bool spec = a.spec_active && valid && ch.spec[g];
-    // written ahead by the hash kernel where it belongs: stored rank g means
-    // every earlier chunk is a stored miss (no eviction here)
-    const bool ahead = spec && stored && sr == g;
     n_spec += spec;
-    n_spec_used += ahead;
+    n_spec_used += spec && stored && sr == g;
     if (lead) {
       P.miss_idx[r] = g;
+      ch.order[r] = g;  // for the copies, spread over the grid below
+      ch.srank[g] = stored ? (uint32_t)sr : kEmptySlot;
       n_rej += st == kMissCand;
       n_bytes += len;
       if (stored) n_sbytes += len;
-      leads[lr] = LeadCopy{(unsigned long long)(P.buf + (unsigned long long)g * a.C),
-                           (unsigned long long)(P.packed + r * a.C),
-                           stored ? (unsigned long long)(a.arena + slot * a.C) : 0ull, len,
-                           ahead ? 0u : 1u};
     }
     // hit-mask words: one atomic per group of lanes that share a word
     const bool hit = valid && st == kHit0;
@@ -1438,12 +1437,20 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
     if (mw && lane == (uint32_t)(__ffs(mpeers) - 1)) atomicOr((uint32_t*)mw, bits);
     if (P.chunk_slot && valid)
       P.chunk_slot[g] = hit ? ch.ent[g] : stored ? (uint32_t)slot : kEmptySlot;
-    __syncthreads();  // the block's miss table is written
-
-    // the block's misses, in pieces of kPackPiece bytes spread over its warps
+    ins_slot = stored ? slot : ~0ull;
+  }
+  ok = grid_barrier(a.ctl, G, a.wait_ns, false) && ok;
+  if (ok) {
+    // every miss's bytes, in pieces of kPackPiece bytes spread over all the
+    // grid's warps (piece k of the miss of rank r is number r * ppc + k), all
+    // but those of misses the hash kernel already wrote where they belong
+    // (stored rank g means every earlier chunk is a stored miss: no eviction
+    // here)
+    const unsigned long long nw = (unsigned long long)G * kWarps;
+    const unsigned long long gw = (unsigned long long)bid * kWarps + w;
     const unsigned long long ppc = (a.C + kPackPiece - 1) / kPackPiece;
-    const unsigned long long npieces = (unsigned long long)c_b * ppc;
-    const unsigned long long plo = npieces * w / kWarps, phi = npieces * (w + 1) / kWarps;
+    const unsigned long long npieces = total * ppc;
+    const unsigned long long plo = npieces * gw / nw, phi = npieces * (gw + 1) / nw;
 #if GLEAM_PACK_BULK
     const uint32_t wbase = (uint32_t)__cvta_generic_to_shared(smem) + w * kPackWarpBytes;
     const uint32_t bufs = wbase, bars = wbase + kPackBufs * kPackPiece;
@@ -1456,20 +1463,42 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
     }
     __syncwarp();
 #endif
+#if GLEAM_CHAIN_PREFETCH
+    // the warp's source pieces start their way into L2 at once (up to 32),
+    // so that the copies below wait for L2 rather than HBM
+    if (plo + lane < phi && !a.plain_copy) {
+      const unsigned long long pc = plo + lane, rr = pc / ppc;
+      const uint32_t off = (uint32_t)(pc - rr * ppc) * kPackPiece;
+      const uint32_t gg = __ldcg(&ch.order[rr]);
+      const uint32_t ln = (uint32_t)min(a.C, P.n - (unsigned long long)gg * a.C);
+      const uint8_t* src = P.buf + (unsigned long long)gg * a.C + off;
+      if (off < ln && ((uintptr_t)src & 15) == 0) {  // the prefetch wants 16-byte alignment
+        const uint32_t pb = min(kPackPiece, ln - off) & ~15u;
+        if (pb) prefetch_l2(src, pb);
+      }
+    }
+#endif
     for (unsigned long long base = plo; base < phi; base += 32) {
       const unsigned long long pc = base + lane;
       uint32_t bytes = 0;
       bool copy = false;
       unsigned long long src = 0, d1 = 0, d2 = 0;
       if (pc < phi) {
-        const LeadCopy& L = leads[pc / ppc];
-        const uint32_t off = (uint32_t)(pc % ppc) * kPackPiece;
-        if (off < L.len && L.copy) {
-          bytes = min(kPackPiece, L.len - off);
-          src = L.src + off;
-          d1 = L.d1 + off;
-          d2 = L.d2 ? L.d2 + off : 0ull;
-          copy = true;
+        const unsigned long long rr = pc / ppc;
+        const uint32_t off = (uint32_t)(pc - rr * ppc) * kPackPiece;
+        const uint32_t gg = __ldcg(&ch.order[rr]);
+        const uint32_t ln = (uint32_t)min(a.C, P.n - (unsigned long long)gg * a.C);
+        if (off < ln) {
+          const uint32_t srr = __ldcg(&ch.srank[gg]);
+          const bool ahead = a.spec_active && srr == gg && ch.spec[gg];
+          if (!ahead) {
+            bytes = min(kPackPiece, ln - off);
+            src = (unsigned long long)(P.buf + (unsigned long long)gg * a.C + off);
+            d1 = (unsigned long long)(P.packed + rr * a.C + off);
+            d2 = srr != kEmptySlot ? (unsigned long long)(a.arena + (slots0 + srr) * a.C + off)
+                                   : 0ull;
+            copy = true;
+          }
         }
       }
       const unsigned cmask = __ballot_sync(0xffffffffu, copy);
@@ -1506,13 +1535,14 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
                    reinterpret_cast<const uint8_t*>(sj), lj, ((sj | xj | yj) & 15) == 0);
       }
     }
-    // each stored miss inserts itself and frees the group entry it claimed
-    if (stored) {
-      a.slot_len[slot] = len;
-      if (!index_insert(a.index, a.index_mask, key, (uint32_t)slot, len))
+    // each stored miss inserts itself and frees the group entry it claimed,
+    // while the last pieces' stores are still in flight
+    if (ins_slot != ~0ull) {
+      a.slot_len[ins_slot] = len;
+      if (!index_insert(a.index, a.index_mask, key, (uint32_t)ins_slot, len))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       if (!a.paper && len >= kPrefixBytes &&
-          !index_insert(a.hints, a.index_mask, ch.hint[g], (uint32_t)slot, len))
+          !index_insert(a.hints, a.index_mask, ch.hint[g], (uint32_t)ins_slot, len))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       if (e != 0xFFFFFFFFu) a.tbl[e].owner = 0u;
     }
@@ -1582,9 +1612,6 @@ constexpr uint32_t kSmallGroups = kThreads / 4;
 constexpr uint32_t kSmallHashSmem = kSmallGroups * (uint32_t)kGroupBytes;
 constexpr uint32_t kSmallSmem = kSmallHashSmem > kPackSmem ? kSmallHashSmem : kPackSmem;
 
-__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
-}
 
 template <bool kAhead>
 __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a) {
@@ -1607,9 +1634,16 @@ __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a
     staged_range<true, kAhead>(h, vb, small_smem);
   }
   __syncthreads();  // every chunk's probe outcome written (and its stage copies landed)
-  resolve_rank(a, 1, 0);
-  __syncthreads();
-  pack_publish(a, 1, 0, small_smem);
+  if (a.count == 1 && !a.lru && a.Ntot <= (unsigned long long)kThreads) {
+    // one payload of at most one chunk per thread: the one-launch path's
+    // steps, which for a call without duplicates rank the misses by a block
+    // scan (no LRU: they stamp no last use)
+    resolve_pack_fast(a, 1, 0, small_smem);
+  } else {
+    resolve_rank(a, 1, 0);
+    __syncthreads();
+    pack_publish(a, 1, 0, small_smem);
+  }
 }
 
 // One warp per record: does the block still hold the recorded chunk's bytes?

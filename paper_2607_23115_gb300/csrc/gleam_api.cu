@@ -494,7 +494,10 @@ constexpr uint64_t kChainMaxChunks = GLEAM_CHAIN_MAX_CHUNKS;
 constexpr uint64_t kChainMaxBytes = 1ull << 30;
 constexpr int kChainDedupBlocks = GLEAM_CHAIN_DEDUP_BLOCKS;
 constexpr int kChainPackBlocks = GLEAM_CHAIN_PACK_BLOCKS;
-constexpr uint64_t kChainBytesPerBlock = 2ull << 20;
+#ifndef GLEAM_CHAIN_BYTES_PER_BLOCK
+#define GLEAM_CHAIN_BYTES_PER_BLOCK (2ull << 20)
+#endif
+constexpr uint64_t kChainBytesPerBlock = GLEAM_CHAIN_BYTES_PER_BLOCK;
 // the one-launch resolve kernel holds at most one chunk per thread
 static_assert(kChainMaxChunks <= (uint64_t)kChainPackBlocks * 256, "chain limit");
 
