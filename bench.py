@@ -109,10 +109,10 @@ def build_workload(name, dev, sample_budget):
     from paper_2607_23115_gb300 import workloads as W
     from paper_2607_23115_gb300.workloads import Upload
 
-    if name == "llama3-8b-paper-ids":
+    if name.startswith("llama3-8b") and name.endswith("-paper-ids"):
         from paper_2607_23115_gb300 import binding as B
-        wl = build_workload("llama3-8b", dev, sample_budget)
-        wl.name = "llama3-8b-bf16-per-tensor-paper-ids"
+        wl = build_workload(name[: -len("-paper-ids")], dev, sample_budget)
+        wl.name = wl.name + "-paper-ids"
         wl.desc = wl.desc + "; the paper's identifier (MD5 of each chunk's first 1024 bits) " \
                             "instead of XXH64, byte verify kept"
         wl.flags = B.GLEAM_PAPER_IDS
@@ -271,7 +271,7 @@ def build_workload(name, dev, sample_budget):
 
 
 WORKLOADS = ["llama3-8b", "llama3-8b-paper-ids", "llama3-8b-lru", "llama3-8b-layer",
-             "llama3-8b-4layers",
+             "llama3-8b-4layers", "llama3-8b-layer-paper-ids", "llama3-8b-4layers-paper-ids",
              "gpt2-small",
              "gpt2-small-pass1", "fp16-64m", "small-calls", "small-calls-10k"] + \
     ["adversarial-%dk%s" % (c, m) for c in (1, 4, 16, 64) for m in ("", "-key16")] + \

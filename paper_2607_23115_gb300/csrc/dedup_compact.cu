@@ -333,6 +333,29 @@ __device__ uint32_t group_entry(const DedupArgs& a, uint32_t g, unsigned long lo
   return 0xFFFFFFFFu;  // cannot happen: the table has >= 2 Ntot entries
 }
 
+// KEY16 with XXH64 keys: finds or claims chunk g's entry in the per-call table
+// of (16-bit index key, length) classes.
+__device__ uint32_t class_entry(const DedupArgs& a, uint32_t g, unsigned long long k16,
+                                uint32_t len) {
+  uint64_t pos = mix64(k16 ^ ((unsigned long long)len << 40)) & a.tbl_mask;
+  for (uint64_t probe = 0; probe <= a.tbl_mask; ++probe) {
+    uint32_t o = ldcg_u32(&a.cls_tbl[pos].owner);
+    if (o == 0) {
+      o = atomicCAS(&a.cls_tbl[pos].owner, 0u, g + 1);
+      if (o == 0) return (uint32_t)pos;
+    }
+    if ((a.ch.key[o - 1] & 0xFFFFull) == k16 && a.ch.len[o - 1] == len) return (uint32_t)pos;
+    pos = (pos + 1) & a.tbl_mask;
+  }
+  return 0xFFFFFFFFu;  // cannot happen: the table has >= 2 Ntot entries
+}
+
+// The index key of a group key (KEY16 mode: its low 16 bits).
+__device__ __forceinline__ unsigned long long index_key(const DedupArgs& a,
+                                                        unsigned long long k) {
+  return a.key16 ? (k & 0xFFFFull) : k;
+}
+
 __device__ __forceinline__ const PayloadDesc& desc(const DedupArgs& a, uint32_t p) {
   return a.count > 1 ? a.table[p] : a.one;
 }
@@ -578,14 +601,17 @@ __device__ bool lru_evict(const DedupArgs& a, uint32_t G, uint32_t bid,
 
 // Posts ~g as a candidate minimum of group entry `e` (0xFFFFFFFF: none), one
 // atomic per group of lanes that share the entry.  Called by the whole warp.
-__device__ __forceinline__ void post_minimum(const DedupArgs& a, uint32_t e, uint32_t g) {
+__device__ __forceinline__ void post_minimum(CallEntry* tbl, uint32_t e, uint32_t g) {
   const unsigned peers = __match_any_sync(0xffffffffu, e);
   const uint32_t m = __reduce_max_sync(peers, e != 0xFFFFFFFFu ? ~g : 0u);
   // a group of many chunks (all-zero chunks, say) would queue its atomics on
   // one address: skip the atomic when a smaller number is already posted
   if (e != 0xFFFFFFFFu && (threadIdx.x & 31) == (uint32_t)(__ffs(peers) - 1) &&
-      ldcg_u32(&a.tbl[e].minv) < m)
-    atomicMax(&a.tbl[e].minv, m);
+      ldcg_u32(&tbl[e].minv) < m)
+    atomicMax(&tbl[e].minv, m);
+}
+__device__ __forceinline__ void post_minimum(const DedupArgs& a, uint32_t e, uint32_t g) {
+  post_minimum(a.tbl, e, g);
 }
 
 // The first-occurrence resolution and miss ranks of a call, run by block
@@ -631,7 +657,8 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
     // minimum with one atomic (all-zero chunks, say, share a group)
     for (uint32_t base = tid - lane; base < N; base += nth) {
       const uint32_t g = base + lane;
-      uint32_t post = 0xFFFFFFFFu;  // group entry that gets this chunk's number
+      uint32_t post = 0xFFFFFFFFu;   // group entry that gets this chunk's number
+      uint32_t cpost = 0xFFFFFFFFu;  // class entry that gets it (KEY16)
       if (g < N) {
         const PayloadDesc& P = desc(a, ch.pidx[g]);
         const unsigned long long i = g - P.chunk_base;
@@ -657,9 +684,15 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
             ch.res[g] = kResUnresolved;
             post = e;
           }
+          if (a.classes) {
+            cpost = class_entry(a, g, ch.key[g] & 0xFFFFull, ch.len[g]);
+            if (cpost == 0xFFFFFFFFu) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+            ch.cls[g] = cpost;
+          }
         }
       }
       post_minimum(a, post, g);
+      if (a.classes) post_minimum(a.cls_tbl, cpost, g);
     }
     if (a.lru) {
       distinct = block_sum<unsigned long long>(distinct, red64);
@@ -758,6 +791,14 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
       if (r & kResLeader) {
         ++cnt;
         if (!(r & kResNoSlot)) ++scnt;
+        // a verify reject: the cache had a key+length candidate, or an
+        // earlier miss of the call has this key and length (another leader
+        // of a later round; with classes, any earlier chunk of the class)
+        const bool rej =
+            !(r & kResNoSlot) &&
+            (ch.status[g] == kMissCand ||
+             (a.classes ? ~ldcg_u32(&a.cls_tbl[ch.cls[g]].minv) < g : (r & kResRoundMask) > 1));
+        if (rej) ch.res[g] = r | kResReject;
         // leave the group table zeroed for the next call: every claimed entry
         // belongs to a group with at least one leader
         const uint32_t e = ch.ent[g];
@@ -839,6 +880,11 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
       __syncthreads();
       const uint32_t below = (1u << lane) - 1u;
       if (valid) {
+        // every read of the class table happened before the last barrier
+        if (a.classes && !(rv & (kResHit0 | kResNoSlot)) && ch.cls[g] != 0xFFFFFFFFu) {
+          a.cls_tbl[ch.cls[g]].owner = 0u;
+          a.cls_tbl[ch.cls[g]].minv = 0u;
+        }
         const uint32_t r = (uint32_t)(running + warp_off[w] + __popc(mb & below));
         ch.rank[g] = r;
         if (miss) ch.order[r] = g;
@@ -959,6 +1005,10 @@ __device__ __forceinline__ void finish_call(const DedupArgs& a, uint32_t G,
     for (unsigned long long e = threadIdx.x; e <= a.tbl_mask; e += kThreads) {
       a.tbl[e].owner = 0u;
       a.tbl[e].minv = 0u;
+      if (a.classes) {
+        a.cls_tbl[e].owner = 0u;
+        a.cls_tbl[e].minv = 0u;
+      }
     }
     if (a.lru) {  // an eviction that stopped half-way may have left these set
       for (uint32_t j = threadIdx.x; j < kLruBins; j += kThreads) a.bins[j] = 0u;
@@ -1101,7 +1151,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
         if (miss) {
           len = ch.len[g];
           P.miss_idx[ch.rank[g] - __ldcg(&a.pstart[p])] = (uint32_t)i;
-          rej = (r & kResRoundMask) > 1 || ch.status[g] == kMissCand;
+          rej = (r & kResReject) != 0;
         }
       }
       n_spec += a.spec_active && valid && ch.spec[g];
@@ -1231,7 +1281,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
       n_spec_used += written_ahead(gg, sr);
       a.slot_len[slot] = ln;
       if (a.lru) a.last_use[slot] = a.epoch;
-      if (!index_insert(a.index, a.index_mask, ch.key[gg], (uint32_t)slot, ln))
+      if (!index_insert(a.index, a.index_mask, index_key(a, ch.key[gg]), (uint32_t)slot, ln))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       if (!a.paper && ln >= kPrefixBytes &&
           !index_insert(a.hints, a.index_mask, ch.hint[gg], (uint32_t)slot, ln))
@@ -1539,7 +1589,7 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
     // while the last pieces' stores are still in flight
     if (ins_slot != ~0ull) {
       a.slot_len[ins_slot] = len;
-      if (!index_insert(a.index, a.index_mask, key, (uint32_t)ins_slot, len))
+      if (!index_insert(a.index, a.index_mask, index_key(a, key), (uint32_t)ins_slot, len))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       if (!a.paper && len >= kPrefixBytes &&
           !index_insert(a.hints, a.index_mask, ch.hint[g], (uint32_t)ins_slot, len))
@@ -1634,7 +1684,7 @@ __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a
     staged_range<true, kAhead>(h, vb, small_smem);
   }
   __syncthreads();  // every chunk's probe outcome written (and its stage copies landed)
-  if (a.count == 1 && !a.lru && a.Ntot <= (unsigned long long)kThreads) {
+  if (a.count == 1 && !a.lru && !a.classes && a.Ntot <= (unsigned long long)kThreads) {
     // one payload of at most one chunk per thread: the one-launch path's
     // steps, which for a call without duplicates rank the misses by a block
     // scan (no LRU: they stamp no last use)

@@ -45,6 +45,7 @@ struct gleam_cache {
   void* ws = nullptr;
   ChunkArrays ch{};
   CallEntry* tbl = nullptr;
+  CallEntry* cls_tbl = nullptr;  // KEY16: (16-bit key, length) classes, tbl_cap entries
   uint64_t tbl_cap = 0;
 
   // payload tables of multi-payload calls
@@ -247,6 +248,7 @@ void free_ws(gleam_cache* c) {
   c->tbl_cap = 0;
   c->ch = ChunkArrays{};
   c->tbl = nullptr;
+  c->cls_tbl = nullptr;
 }
 
 // Grows the per-chunk workspace to hold `nchunks` chunks.  Waits for the
@@ -257,11 +259,12 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   cap = std::min<uint64_t>(cap, kMaxChunks);
   if (cap < nchunks) cap = nchunks;
   const uint64_t tcap = next_pow2(2 * cap);
-  const uint64_t sz[14] = {align256(cap),     align256(cap * 8), align256(cap * 4),
+  const uint64_t sz[16] = {align256(cap),     align256(cap * 8), align256(cap * 4),
                            align256(cap * 8), align256(cap * 4), align256(cap * 4),
                            align256(cap * 4), align256(cap * 4), align256(cap * 8),
                            align256(cap * 4), align256(cap * 4), align256(cap * 4),
-                           align256(cap),     align256(tcap * sizeof(CallEntry))};
+                           align256(cap),     align256(tcap * sizeof(CallEntry)),
+                           align256(cap * 4), align256(tcap * sizeof(CallEntry))};
   uint64_t total = 0;
   for (uint64_t x : sz) total += x;
   int rc = cuda_err(cudaEventSynchronize(c->done));
@@ -302,6 +305,10 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   c->ch.spec = b;
   b += sz[12];
   c->tbl = reinterpret_cast<CallEntry*>(b);
+  b += sz[13];
+  c->ch.cls = reinterpret_cast<uint32_t*>(b);
+  b += sz[14];
+  c->cls_tbl = reinterpret_cast<CallEntry*>(b);
   c->tbl_cap = tcap;
   c->ws_chunks = cap;
   return GLEAM_OK;
@@ -657,6 +664,9 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   d.ch = c->ch;
   d.pstart = count > 1 ? c->d_pstart : c->bcount + 2 * c->coop_max_blocks;
   d.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
+  d.key16 = (c->flags & GLEAM_KEY16) ? 1u : 0u;
+  d.classes = d.key16 && !d.paper ? 1u : 0u;
+  d.cls_tbl = c->cls_tbl;
   d.plain_copy = (host_payloads || chk.saw_managed()) ? 1u : 0u;
   d.tbl = c->tbl;
   d.tbl_mask = tcap - 1;
@@ -709,7 +719,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
       grid = (int)std::min<uint64_t>(kChainDedupBlocks, (Ntot + 255) / 256);
       pgrid = std::min(pgrid, kChainPackBlocks);
     }
-    if (chain && count == 1) {
+    if (chain && count == 1 && !d.classes) {
       // one launch: at most one chunk per thread, and one block per
       // kChainBytesPerBlock of payload so that the misses' copies spread
       const uint64_t want = std::max<uint64_t>((Ntot + dedup_threads() - 1) / dedup_threads(),
@@ -1287,10 +1297,12 @@ constexpr uint64_t kNaOffSrank = kNaOffOrder + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffOld = kNaOffSrank + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffSpec = kNaOffOld + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffTbl = kNaOffSpec + na_align(kNaChunks);
-constexpr uint64_t kNaOffCtl = kNaOffTbl + na_align(kNaTable * sizeof(CallEntry));
+constexpr uint64_t kNaOffCls = kNaOffTbl + na_align(kNaTable * sizeof(CallEntry));
+constexpr uint64_t kNaOffClsTbl = kNaOffCls + na_align(kNaChunks * 4);
+constexpr uint64_t kNaOffCtl = kNaOffClsTbl + na_align(kNaTable * sizeof(CallEntry));
 constexpr uint64_t kNaOffBcount = kNaOffCtl + na_align(sizeof(DevCtl));
 constexpr uint64_t kNaOffResult = kNaOffBcount + na_align((2 * kNaBlocks + 1) * 4);
-constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~4.6 MiB
+constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~5.9 MiB
 
 }  // namespace
 
@@ -1348,7 +1360,9 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   ch.srank = reinterpret_cast<uint32_t*>(base + kNaOffSrank);
   ch.old = reinterpret_cast<uint32_t*>(base + kNaOffOld);
   ch.spec = base + kNaOffSpec;
+  ch.cls = reinterpret_cast<uint32_t*>(base + kNaOffCls);
   CallEntry* tbl = reinterpret_cast<CallEntry*>(base + kNaOffTbl);
+  CallEntry* cls_tbl = reinterpret_cast<CallEntry*>(base + kNaOffClsTbl);
   DevCtl* ctl = reinterpret_cast<DevCtl*>(base + kNaOffCtl);
   uint32_t* bcount = reinterpret_cast<uint32_t*>(base + kNaOffBcount);
   gleam_result_t* total = reinterpret_cast<gleam_result_t*>(base + kNaOffResult);
@@ -1359,6 +1373,10 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   if ((rc = order_after_done(c, s, &sid)) != GLEAM_OK) return rc;
   if ((rc = cuda_err(cudaMemsetAsync(ctl, 0, sizeof(DevCtl), s))) != GLEAM_OK) return rc;
   if ((rc = cuda_err(cudaMemsetAsync(tbl, 0, tcap * sizeof(CallEntry), s))) != GLEAM_OK) return rc;
+  const bool classes = (c->flags & GLEAM_KEY16) && !(c->flags & GLEAM_PAPER_IDS);
+  if (classes &&
+      (rc = cuda_err(cudaMemsetAsync(cls_tbl, 0, tcap * sizeof(CallEntry), s))) != GLEAM_OK)
+    return rc;
 
   HashArgs h{};
   h.one = one;
@@ -1391,6 +1409,9 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.ch = ch;
   d.pstart = bcount + 2 * kNaBlocks;
   d.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
+  d.key16 = (c->flags & GLEAM_KEY16) ? 1u : 0u;
+  d.classes = classes ? 1u : 0u;
+  d.cls_tbl = cls_tbl;
   d.tbl = tbl;
   d.tbl_mask = tcap - 1;
   d.bcount = bcount;

@@ -44,7 +44,8 @@ constexpr uint32_t kResHit0 = 0x20000000u;     // byte-equal to a cached chunk
 constexpr uint32_t kResDup = 0x40000000u;      // byte-equal to an earlier miss
 constexpr uint32_t kResLeader = 0x80000000u;   // | round in which it was resolved
 constexpr uint32_t kResNoSlot = 0x10000000u;   // a miss that is never cached
-constexpr uint32_t kResRoundMask = 0x0FFFFFFFu;
+constexpr uint32_t kResReject = 0x08000000u;   // a miss that had a key+length candidate
+constexpr uint32_t kResRoundMask = 0x07FFFFFFu;
 
 // Device counters of one cache, in gleam_stats_t order (the fields that
 // change; capacity, slot count and chunk size are host constants).
@@ -114,7 +115,8 @@ struct __align__(16) PayloadDesc {
 // Per-chunk workspace, indexed by global chunk number.
 struct ChunkArrays {
   uint8_t* status;           // kHit0 / kMissCand / kMissNoCand
-  unsigned long long* key;   // index key (XXH64, or its low 16 bits)
+  unsigned long long* key;   // group key: the whole XXH64 (also in KEY16 mode, whose
+                             // index key is its low 16 bits), or the paper's key
   uint32_t* len;             // true length
   unsigned long long* src;   // device address of the chunk's first byte
   uint32_t* pidx;            // payload number
@@ -128,6 +130,7 @@ struct ChunkArrays {
   uint32_t* old;             // LRU: last use of a hit's slot before this call stamped it
   uint8_t* spec;             // 1: the hash kernel wrote the chunk to packed offset
                              // i*C of its payload and to arena slot slots_used + g
+  uint32_t* cls;             // KEY16: the chunk's entry in the per-call class table
 };
 
 // Speculative verify.  After the first kPrefixBytes of a chunk the four XXH64
@@ -197,6 +200,13 @@ struct DedupArgs {
   unsigned long long wait_ns;
   int skip_block;
   uint32_t paper;            // no prefix hints are kept in GLEAM_PAPER_IDS mode
+  uint32_t key16;            // GLEAM_KEY16: index key = low 16 bits of the group key
+  // KEY16 with XXH64 keys: chunks are grouped by their whole fingerprint, so a
+  // miss's verify rejects inside the call (an earlier chunk with the same
+  // 16-bit key and length) come from this second per-call table of (16-bit
+  // key, length) classes, each holding its smallest chunk number
+  uint32_t classes;
+  CallEntry* cls_tbl;        // same size as tbl
   uint32_t plain_copy;       // copy misses with loads and stores, not bulk copies
                              // (payloads or outputs in host or managed memory)
   // LRU eviction (GLEAM_EVICT_LRU; lru == 0: the other fields are unused)

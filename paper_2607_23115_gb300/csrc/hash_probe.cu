@@ -250,7 +250,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
   }
   if (lane == 0) {
     a.ch.status[g] = hit ? kHit0 : (cand ? kMissCand : kMissNoCand);
-    a.ch.key[g] = key;
+    a.ch.key[g] = h;  // the group key: the whole fingerprint
     a.ch.len[g] = len;
     a.ch.src[g] = (unsigned long long)p;
     a.ch.pidx[g] = pid;

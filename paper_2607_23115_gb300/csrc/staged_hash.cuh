@@ -452,7 +452,7 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   }
   if (lane == 0) {
     a.ch.status[g] = hit ? kHit0 : (cand ? kMissCand : kMissNoCand);
-    a.ch.key[g] = key;
+    a.ch.key[g] = h;  // the group key: the whole fingerprint
     a.ch.len[g] = len;
     a.ch.src[g] = (unsigned long long)p;
     a.ch.pidx[g] = pid;
