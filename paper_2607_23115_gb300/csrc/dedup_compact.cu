@@ -1280,6 +1280,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
       const unsigned long long slot = slot_of(sr);
       n_spec_used += written_ahead(gg, sr);
       a.slot_len[slot] = ln;
+      a.slot_key[slot] = ch.key[gg];
       if (a.lru) a.last_use[slot] = a.epoch;
       if (!index_insert(a.index, a.index_mask, index_key(a, ch.key[gg]), (uint32_t)slot, ln))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
@@ -1589,6 +1590,7 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
     // while the last pieces' stores are still in flight
     if (ins_slot != ~0ull) {
       a.slot_len[ins_slot] = len;
+      a.slot_key[ins_slot] = key;
       if (!index_insert(a.index, a.index_mask, index_key(a, key), (uint32_t)ins_slot, len))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       if (!a.paper && len >= kPrefixBytes &&
@@ -1725,14 +1727,16 @@ __global__ void __launch_bounds__(kThreads) k_block_check(BlockCheckArgs a) {
 }
 
 __global__ void k_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
-                               unsigned long long* dstats, unsigned long long key, uint32_t slot,
-                               uint32_t len, DevCtl* ctl, uint32_t* last_use, uint32_t epoch) {
+                               unsigned long long* slot_key, unsigned long long* dstats,
+                               unsigned long long key, uint32_t slot, uint32_t len, DevCtl* ctl,
+                               uint32_t* last_use, uint32_t epoch) {
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   if (!index_insert(index, index_mask, key, slot, len)) {
     ctl->err = GLEAM_ERR_INTERNAL;
     return;
   }
   slot_len[slot] = len;
+  slot_key[slot] = key;
   if (last_use) last_use[slot] = epoch;
   dstats[ST_SLOTS_USED] = (unsigned long long)slot + 1;
   dstats[ST_INSERTS] += 1;
@@ -1860,11 +1864,11 @@ cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
-                                unsigned long long* dstats, unsigned long long key,
-                                uint32_t slot, uint32_t len, DevCtl* ctl, uint32_t* last_use,
-                                uint32_t epoch, cudaStream_t s) {
-  k_debug_insert<<<1, 32, 0, s>>>(index, index_mask, slot_len, dstats, key, slot, len, ctl,
-                                  last_use, epoch);
+                                unsigned long long* slot_key, unsigned long long* dstats,
+                                unsigned long long key, uint32_t slot, uint32_t len, DevCtl* ctl,
+                                uint32_t* last_use, uint32_t epoch, cudaStream_t s) {
+  k_debug_insert<<<1, 32, 0, s>>>(index, index_mask, slot_len, slot_key, dstats, key, slot, len,
+                                  ctl, last_use, epoch);
   return cudaGetLastError();
 }
 

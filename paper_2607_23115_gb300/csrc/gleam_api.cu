@@ -27,6 +27,7 @@ struct gleam_cache {
   IndexEntry* hints = nullptr;  // prefix-hint table, index_cap entries
   uint64_t index_cap = 0;  // power of two >= 2 * nslots
   uint32_t* slot_len = nullptr;
+  unsigned long long* slot_key = nullptr;  // per slot: the stored chunk's group key
   unsigned long long* dstats = nullptr;
 
   // LRU eviction (GLEAM_EVICT_LRU)
@@ -101,7 +102,8 @@ struct gleam_snapshot {
   IndexEntry* hints = nullptr;
   uint64_t index_cap = 0;
   unsigned long long* dstats = nullptr;
-  uint32_t* slot_len = nullptr;  // LRU caches: slot lengths and last uses too
+  uint32_t* slot_len = nullptr;  // LRU caches: slot lengths, keys and last uses too
+  unsigned long long* slot_key = nullptr;
   uint32_t* last_use = nullptr;
   uint64_t nslots = 0;
   uint64_t slots_bound = 0;  // the cache's host-side bound of its used slots
@@ -344,6 +346,7 @@ void destroy_cache(gleam_cache* c) {
     if (c->index) cudaFree(c->index);
     if (c->hints) cudaFree(c->hints);
     if (c->slot_len) cudaFree(c->slot_len);
+    if (c->slot_key) cudaFree(c->slot_key);
     if (c->dstats) cudaFree(c->dstats);
     if (c->last_use) cudaFree(c->last_use);
     if (c->vflag) cudaFree(c->vflag);
@@ -646,6 +649,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   h.index_mask = c->index_cap - 1;
   h.hints = c->hints;
   h.arena = c->arena;
+  h.slot_key = c->slot_key;
   h.dstats = c->dstats;
   h.key16 = (c->flags & GLEAM_KEY16) ? 1u : 0u;
   h.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
@@ -665,6 +669,7 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   d.hints = c->hints;
   d.nslots = c->nslots;
   d.slot_len = c->slot_len;
+  d.slot_key = c->slot_key;
   d.dstats = c->dstats;
   d.ch = c->ch;
   d.pstart = count > 1 ? c->d_pstart : c->bcount + 2 * c->coop_max_blocks;
@@ -817,6 +822,7 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
   step(cudaMalloc(&c->index, c->index_cap * sizeof(IndexEntry)));
   step(cudaMalloc(&c->hints, c->index_cap * sizeof(IndexEntry)));
   step(cudaMalloc(&c->slot_len, nslots * sizeof(uint32_t)));
+  step(cudaMalloc(&c->slot_key, nslots * sizeof(unsigned long long)));
   step(cudaMalloc(&c->dstats, ST_COUNT * sizeof(unsigned long long)));
   if (flags & GLEAM_DEBUG_CHECKS) {
     step(cudaMalloc(&c->dbg_count, nslots * sizeof(uint32_t)));
@@ -1097,7 +1103,8 @@ int gleam_cache_debug_insert(gleam_cache_t* c, uint64_t key, const void* d_bytes
   const unsigned long long k = (c->flags & GLEAM_KEY16) ? (key & 0xFFFFull) : key;
   rc = cuda_err(cudaMemcpy(c->arena + used * c->C, d_bytes, len, cudaMemcpyDeviceToDevice));
   if (rc == GLEAM_OK)
-    rc = cuda_err(launch_debug_insert(c->index, c->index_cap - 1, c->slot_len, c->dstats, k,
+    rc = cuda_err(launch_debug_insert(c->index, c->index_cap - 1, c->slot_len, c->slot_key,
+                                      c->dstats, k,
                                       (uint32_t)used, (uint32_t)len, c->ctl, c->last_use,
                                       c->last_use ? ++c->epoch : 0u, nullptr));
   if (rc == GLEAM_OK) rc = cuda_err(cudaDeviceSynchronize());
@@ -1212,7 +1219,12 @@ int gleam_cache_snapshot(gleam_cache_t* c, gleam_snapshot_t** out) {
   if (rc == GLEAM_OK && c->last_use) {
     s->nslots = c->nslots;
     rc = cuda_err(cudaMalloc(&s->slot_len, c->nslots * sizeof(uint32_t)));
+    if (rc == GLEAM_OK)
+      rc = cuda_err(cudaMalloc(&s->slot_key, c->nslots * sizeof(unsigned long long)));
     if (rc == GLEAM_OK) rc = cuda_err(cudaMalloc(&s->last_use, c->nslots * sizeof(uint32_t)));
+    if (rc == GLEAM_OK)
+      rc = cuda_err(cudaMemcpy(s->slot_key, c->slot_key, c->nslots * sizeof(unsigned long long),
+                               cudaMemcpyDeviceToDevice));
     if (rc == GLEAM_OK)
       rc = cuda_err(cudaMemcpy(s->slot_len, c->slot_len, c->nslots * sizeof(uint32_t),
                                cudaMemcpyDeviceToDevice));
@@ -1248,6 +1260,10 @@ int gleam_cache_restore(gleam_cache_t* c, const gleam_snapshot_t* s) {
     rc = cuda_err(cudaMemcpyAsync(c->slot_len, s->slot_len, s->nslots * sizeof(uint32_t),
                                   cudaMemcpyDeviceToDevice, nullptr));
     if (rc == GLEAM_OK)
+      rc = cuda_err(cudaMemcpyAsync(c->slot_key, s->slot_key,
+                                    s->nslots * sizeof(unsigned long long),
+                                    cudaMemcpyDeviceToDevice, nullptr));
+    if (rc == GLEAM_OK)
       rc = cuda_err(cudaMemcpyAsync(c->last_use, s->last_use, s->nslots * sizeof(uint32_t),
                                     cudaMemcpyDeviceToDevice, nullptr));
   }
@@ -1266,6 +1282,7 @@ void gleam_snapshot_destroy(gleam_snapshot_t* s) {
   if (s->hints) cudaFree(s->hints);
   if (s->dstats) cudaFree(s->dstats);
   if (s->slot_len) cudaFree(s->slot_len);
+  if (s->slot_key) cudaFree(s->slot_key);
   if (s->last_use) cudaFree(s->last_use);
   cudaGetLastError();
   delete s;
@@ -1395,6 +1412,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   h.index_mask = c->index_cap - 1;
   h.hints = c->hints;
   h.arena = c->arena;
+  h.slot_key = c->slot_key;
   h.dstats = c->dstats;
   h.key16 = (c->flags & GLEAM_KEY16) ? 1u : 0u;
   h.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
@@ -1413,6 +1431,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   d.hints = c->hints;
   d.nslots = c->nslots;
   d.slot_len = c->slot_len;
+  d.slot_key = c->slot_key;
   d.dstats = c->dstats;
   d.ch = ch;
   d.pstart = bcount + 2 * kNaBlocks;

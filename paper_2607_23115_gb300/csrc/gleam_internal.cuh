@@ -155,6 +155,7 @@ struct HashArgs {
   unsigned long long index_mask;
   const IndexEntry* hints;   // prefix-hint table (same size as the index)
   const uint8_t* arena;
+  const unsigned long long* slot_key;  // per slot: the stored chunk's whole fingerprint
   const unsigned long long* dstats;
   uint32_t key16;
   uint32_t paper;            // GLEAM_PAPER_IDS: MD5-prefix keys, small chunks uncached
@@ -188,6 +189,7 @@ struct DedupArgs {
   IndexEntry* hints;
   unsigned long long nslots;
   uint32_t* slot_len;
+  unsigned long long* slot_key;  // per slot: the group key of the stored chunk
   unsigned long long* dstats;
   ChunkArrays ch;
   uint32_t* pstart;          // per payload: misses before its first chunk
@@ -255,9 +257,9 @@ cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_
                               bool pdl = false);
 uint32_t small_call_groups();
 cudaError_t launch_debug_insert(IndexEntry* index, uint64_t index_mask, uint32_t* slot_len,
-                                unsigned long long* dstats, unsigned long long key,
-                                uint32_t slot, uint32_t len, DevCtl* ctl, uint32_t* last_use,
-                                uint32_t epoch, cudaStream_t s);
+                                unsigned long long* slot_key, unsigned long long* dstats,
+                                unsigned long long key, uint32_t slot, uint32_t len, DevCtl* ctl,
+                                uint32_t* last_use, uint32_t epoch, cudaStream_t s);
 struct BlockCheckArgs {
   const uint8_t* block;
   unsigned long long block_bytes;

@@ -238,6 +238,7 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
               : a.wait_late ? ld_acquire_u64(&a.dstats[ST_SLOTS_USED]) : a.dstats[ST_SLOTS_USED];
   unsigned long long hint = 0, diff = 0;
   uint32_t hint_slot = kEmptySlot;
+  unsigned long long hint_key = 0;  // the whole fingerprint stored for hint_slot
   const uint8_t* q = nullptr;
   bool cmp = false;
   // write-through of a likely miss, decided once the prefix hint is known
@@ -320,6 +321,8 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
       }
       if (cmp) {
         q = a.arena + (unsigned long long)hint_slot * a.C;
+        // loaded now, used once the chunk is hashed: no lookup waits then
+        hint_key = a.slot_key[hint_slot];
         // the prefix, still in stage buffer 0, against the cached copy's prefix
 #pragma unroll 4
         for (uint32_t s = 0; s < (uint32_t)kStage / 32; ++s)
@@ -402,7 +405,15 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
     const unsigned wmask = present_lanes(vb, a.Ntot);
     const uint32_t wl = threadIdx.x & 31, nl = __popc(wmask);
     unsigned long long pos = mix64(key) & a.index_mask, probe = 0;
+    // the hinted slot holds these very bytes and this fingerprint: the index
+    // lists it under this key and length (both are written for every stored
+    // chunk), so it is the hit and the probe can be skipped
     bool done = false;
+    if (spec_equal && hint_key == h) {
+      hit = true;
+      hit_slot = hint_slot;
+      done = true;
+    }
     for (;;) {
       uint32_t want = kEmptySlot;  // a candidate for the warp to compare
       while (!done) {
