@@ -208,20 +208,23 @@ def build_workload(name, dev, sample_budget):
                                              "prefilled with the same half (untimed)")
         return wl
 
-    if name in ("small-calls", "small-calls-10k"):
+    if name == "small-calls" or (name.startswith("small-calls-") and name.endswith("k")):
+        # small-calls: the 100,000-payload stream; small-calls-<N>k: N thousand
+        # payloads of the same make, prefill and cache scaled (profiling sizes)
         C = 4 * KiB
-        count = 100000 if name == "small-calls" else 10000
+        count = 100000 if name == "small-calls" else int(name[len("small-calls-"):-1]) * 1000
         if count == 100000:
             wl = Workload("small-call-stream-100k", "100,000 payloads of uniform random bytes, "
                           "sizes log-uniform in 4 KiB-1 MiB (18.8 GB); cache prefilled with 2 GB "
                           "of unrelated chunks; 32 GiB cache", C, 32 * GiB)
         else:
-            wl = Workload("small-call-stream-10k", "10,000 payloads of uniform random bytes, "
-                          "sizes log-uniform in 4 KiB-1 MiB (1.9 GB); cache prefilled with 0.2 GB "
-                          "of unrelated chunks; 4 GiB cache (a profiling-size case)", C, 4 * GiB)
+            wl = Workload("small-call-stream-%dk" % (count // 1000),
+                          "%d payloads of uniform random bytes, sizes log-uniform in 4 KiB-1 MiB; "
+                          "cache prefilled with unrelated chunks (2 GB per 100,000 payloads); a "
+                          "profiling-size case" % count, C, max(1, count * 32 // 100000) * GiB)
         up = W.small_call_upload(count, device=dev)
         wl.up = up
-        pre_bytes = 2 * 10**9 if count == 100000 else 2 * 10**8
+        pre_bytes = 2 * 10**9 * count // 100000
         wl.prefill = [[W.random_bytes(pre_bytes // C * C, seed=W.SEED_PREFILL, device=dev)]]
         wl.expect_misses = sum((s + C - 1) // C for s in up.sizes)
 
@@ -273,7 +276,7 @@ def build_workload(name, dev, sample_budget):
 WORKLOADS = ["llama3-8b", "llama3-8b-paper-ids", "llama3-8b-lru", "llama3-8b-layer",
              "llama3-8b-4layers", "llama3-8b-layer-paper-ids", "llama3-8b-4layers-paper-ids",
              "gpt2-small",
-             "gpt2-small-pass1", "fp16-64m", "small-calls", "small-calls-10k"] + \
+             "gpt2-small-pass1", "fp16-64m", "small-calls", "small-calls-10k", "small-calls-<N>k"] + \
     ["adversarial-%dk%s" % (c, m) for c in (1, 4, 16, 64) for m in ("", "-key16")] + \
     ["adversarial-<C>k[-key16]-<M>m (M MiB of the adversarial make)"]
 
