@@ -501,7 +501,11 @@ void note_call(gleam_cache* c, uint64_t Ntot) {
 #define GLEAM_CHAIN_PACK_BLOCKS 76
 #endif
 constexpr uint64_t kChainMaxChunks = GLEAM_CHAIN_MAX_CHUNKS;
-constexpr uint64_t kChainMaxBytes = 1ull << 30;
+// A large payload keeps the full grids of the unchained path: its in-call
+// duplicates (a 1 GiB payload of 64 KiB chunks, a quarter of them copies) are
+// compared by every warp the resolve kernel has (0.47 ms with 456 blocks,
+// 1.15 ms with 32).
+constexpr uint64_t kChainMaxBytes = 256ull << 20;
 constexpr int kChainDedupBlocks = GLEAM_CHAIN_DEDUP_BLOCKS;
 constexpr int kChainPackBlocks = GLEAM_CHAIN_PACK_BLOCKS;
 #ifndef GLEAM_CHAIN_BYTES_PER_BLOCK
