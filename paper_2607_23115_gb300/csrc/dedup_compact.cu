@@ -69,6 +69,12 @@ constexpr int kWarps = kThreads / 32;
 #define GLEAM_PACK_BOUNDS __launch_bounds__(kThreads)
 #endif
 constexpr int kCopyVec = GLEAM_COPY_VEC;  // 16-byte vectors per lane in flight while copying
+// In-call duplicates of at most this many bytes are compared kSmallCmpWays at a time.
+#ifndef GLEAM_SMALL_CMP_WAYS
+#define GLEAM_SMALL_CMP_WAYS 2
+#endif
+constexpr uint32_t kSmallCmpBytes = 1024;
+constexpr uint32_t kSmallCmpWays = GLEAM_SMALL_CMP_WAYS;
 
 __device__ __forceinline__ uint32_t ldcg_u32(const uint32_t* p) { return __ldcg(p); }
 
@@ -660,21 +666,25 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
       uint32_t post = 0xFFFFFFFFu;   // group entry that gets this chunk's number
       uint32_t cpost = 0xFFFFFFFFu;  // class entry that gets it (KEY16)
       if (g < N) {
+        // every operand at once: the claim below then waits for none of them
+        const uint8_t st = ch.status[g];
+        const unsigned long long key = ch.key[g];
+        const uint32_t len = ch.len[g];
         const PayloadDesc& P = desc(a, ch.pidx[g]);
         const unsigned long long i = g - P.chunk_base;
         if ((i & 31) == 0) P.mask[i >> 5] = 0;
-        if (ch.status[g] == kHit0) {
+        if (st == kHit0) {
           ch.res[g] = kResHit0;
           if (a.lru) {  // the first chunk to stamp a slot keeps its old value
             const uint32_t old = atomicExch(&a.last_use[ch.ent[g]], a.epoch);
             ch.old[g] = old;
             distinct += old != a.epoch;
           }
-        } else if (ch.status[g] == kUncached) {  // never cached: a miss of its own, in no group
+        } else if (st == kUncached) {  // never cached: a miss of its own, in no group
           ch.ent[g] = 0xFFFFFFFFu;
           ch.res[g] = kResLeader | kResNoSlot | 1u;
         } else {
-          const uint32_t e = group_entry(a, g, ch.key[g], ch.len[g]);
+          const uint32_t e = group_entry(a, g, key, len);
           if (e == 0xFFFFFFFFu) {
             atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
             ch.ent[g] = 0xFFFFFFFFu;
@@ -685,7 +695,7 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
             post = e;
           }
           if (a.classes) {
-            cpost = class_entry(a, g, ch.key[g] & 0xFFFFull, ch.len[g]);
+            cpost = class_entry(a, g, key & 0xFFFFull, len);
             if (cpost == 0xFFFFFFFFu) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
             ch.cls[g] = cpost;
           }
@@ -741,14 +751,13 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
         ys = ch.src[m];
         ln = ch.len[g];
       }
-      while (todo) {
-        const int j = __ffs(todo) - 1;
-        todo &= todo - 1;
-        const uint8_t* x = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, xs, j));
-        const uint8_t* y = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, ys, j));
-        const uint32_t len = __shfl_sync(0xffffffffu, ln, j);
-        const bool vec = (((uintptr_t)x | (uintptr_t)y) & 15) == 0;
-        const bool eq = warp_equal(x, y, len, vec);
+      // duplicates of at most kSmallCmpBytes (whole 16-byte pieces, aligned
+      // operands) are compared up to kSmallCmpWays at a time, every lane loading
+      // its pieces of all of them before any result is needed; the others one
+      // by one
+      unsigned small = __ballot_sync(0xffffffffu, need && ln <= kSmallCmpBytes && (ln & 15) == 0 &&
+                                                      ((xs | ys) & 15) == 0);
+      auto settle = [&](int j, bool eq) {
         if (lane == (uint32_t)j) {
           if (eq) {
             ch.ent[g] = m;  // the leader, for the hit's classification
@@ -758,6 +767,50 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
             stay = true;
           }
         }
+      };
+      while (kSmallCmpWays > 1 && __popc(small) >= 2) {
+        int js[kSmallCmpWays];
+        uint32_t cnt = 0;
+        while (cnt < kSmallCmpWays && small) {
+          js[cnt++] = __ffs(small) - 1;
+          small &= small - 1;
+        }
+        uint4 u[kSmallCmpWays][kSmallCmpBytes / 512], v[kSmallCmpWays][kSmallCmpBytes / 512];
+#pragma unroll
+        for (uint32_t c = 0; c < kSmallCmpWays; ++c) {
+          if (c < cnt) {
+            const uint4* x = reinterpret_cast<const uint4*>(__shfl_sync(0xffffffffu, xs, js[c]));
+            const uint4* y = reinterpret_cast<const uint4*>(__shfl_sync(0xffffffffu, ys, js[c]));
+            const uint32_t np = __shfl_sync(0xffffffffu, ln, js[c]) >> 4;
+#pragma unroll
+            for (uint32_t r = 0; r < kSmallCmpBytes / 512; ++r) {
+              const uint32_t k = r * 32 + lane;
+              u[c][r] = k < np ? __ldcs(x + k) : make_uint4(0, 0, 0, 0);
+              v[c][r] = k < np ? __ldcs(y + k) : make_uint4(0, 0, 0, 0);
+            }
+          }
+        }
+#pragma unroll
+        for (uint32_t c = 0; c < kSmallCmpWays; ++c) {
+          if (c < cnt) {
+            bool diff = false;
+#pragma unroll
+            for (uint32_t r = 0; r < kSmallCmpBytes / 512; ++r)
+              diff |= (u[c][r].x != v[c][r].x) | (u[c][r].y != v[c][r].y) |
+                      (u[c][r].z != v[c][r].z) | (u[c][r].w != v[c][r].w);
+            settle(js[c], !__any_sync(0xffffffffu, diff));
+            todo &= ~(1u << js[c]);
+          }
+        }
+      }
+      while (todo) {
+        const int j = __ffs(todo) - 1;
+        todo &= todo - 1;
+        const uint8_t* x = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, xs, j));
+        const uint8_t* y = reinterpret_cast<const uint8_t*>(__shfl_sync(0xffffffffu, ys, j));
+        const uint32_t len = __shfl_sync(0xffffffffu, ln, j);
+        const bool vec = (((uintptr_t)x | (uintptr_t)y) & 15) == 0;
+        settle(j, warp_equal(x, y, len, vec));
       }
     }
     if (G == 1) {  // the block's own count, without the round trip to the counter
@@ -1643,7 +1696,12 @@ __global__ void __launch_bounds__(kThreads) k_resolve_pack(DedupArgs a) {
   resolve_pack_fast(a, gridDim.x, blockIdx.x, rp_smem);
 }
 
-__global__ void __launch_bounds__(kThreads) k_dedup(DedupArgs a) {
+#ifndef GLEAM_DEDUP_MINBLOCKS
+#define GLEAM_DEDUP_MINBLOCKS 3
+#endif
+// three co-resident blocks per SM (at most 85 registers): the resolve kernel's
+// phases are chains of round trips that want every thread of the grid
+__global__ void __launch_bounds__(kThreads, GLEAM_DEDUP_MINBLOCKS) k_dedup(DedupArgs a) {
   pdl_trigger();
   pdl_wait();
   resolve_rank(a, gridDim.x, blockIdx.x);
