@@ -316,13 +316,45 @@ __device__ bool index_insert(IndexEntry* index, uint64_t mask, unsigned long lon
   return false;
 }
 
+// index_insert in two halves: the first claim attempt at the key's home
+// position (issued early; its result is not waited for until it is needed),
+// then, given that attempt's result, the entry's fields or the rest of the
+// probe.  Together they do what index_insert does.
+struct PendingInsert {
+  uint64_t pos;
+  uint32_t old;
+};
+__device__ __forceinline__ PendingInsert index_insert_begin(IndexEntry* index, uint64_t mask,
+                                                            unsigned long long key, uint32_t slot) {
+  const uint64_t pos = mix64(key) & mask;
+  return PendingInsert{pos, atomicCAS(&index[pos].slot, kEmptySlot, slot)};
+}
+__device__ bool index_insert_end(IndexEntry* index, uint64_t mask, unsigned long long key,
+                                 uint32_t slot, uint32_t len, PendingInsert p) {
+  uint64_t pos = p.pos;
+  uint32_t old = p.old;
+  for (uint64_t probe = 0;;) {
+    if (old == kEmptySlot) {
+      index[pos].key = key;
+      index[pos].len = len;
+      return true;
+    }
+    if (++probe > mask) return false;
+    pos = (pos + 1) & mask;
+    old = atomicCAS(&index[pos].slot, kEmptySlot, slot);
+  }
+}
+
 // Finds or claims the per-call group entry of (key, len) for chunk g;
 // *claimed tells whether g claimed it (else another chunk of the group did).
+// cas_first: claim without reading the entry first (one round trip fewer
+// where entries are mostly free; the read spares a contended entry the
+// atomics of every chunk of a large group).
 __device__ uint32_t group_entry(const DedupArgs& a, uint32_t g, unsigned long long k,
-                                uint32_t len, bool* claimed = nullptr) {
+                                uint32_t len, bool* claimed = nullptr, bool cas_first = false) {
   uint64_t pos = mix64(k ^ ((unsigned long long)len << 40)) & a.tbl_mask;
   for (uint64_t probe = 0; probe <= a.tbl_mask; ++probe) {
-    uint32_t o = ldcg_u32(&a.tbl[pos].owner);
+    uint32_t o = cas_first && probe == 0 ? 0u : ldcg_u32(&a.tbl[pos].owner);
     if (o == 0) {
       o = atomicCAS(&a.tbl[pos].owner, 0u, g + 1);
       if (o == 0) {
@@ -1416,10 +1448,14 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
   }
   uint8_t st = kMissNoCand;
   uint32_t len = 0, e = 0xFFFFFFFFu;
-  unsigned long long key = 0;
+  unsigned long long key = 0, hint = 0;
   bool lead = false, stored = false, shared = false;
   if (valid) {
+    // the chunk's record at once (one round trip, whatever its status)
     st = ch.status[g];
+    const unsigned long long key0 = ch.key[g];
+    const uint32_t len0 = ch.len[g];
+    hint = a.paper ? 0ull : ch.hint[g];
     if ((g & 31) == 0) P.mask[g >> 5] = 0;
     if (st == kHit0) {
       ch.res[g] = kResHit0;
@@ -1427,12 +1463,12 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
       ch.ent[g] = 0xFFFFFFFFu;
       ch.res[g] = kResLeader | kResNoSlot | 1u;
       lead = true;
-      len = ch.len[g];
+      len = len0;
     } else {
-      key = ch.key[g];
-      len = ch.len[g];
+      key = key0;
+      len = len0;
       bool claimed = true;
-      e = group_entry(a, g, key, len, &claimed);
+      e = group_entry(a, g, key, len, &claimed, true);
       if (e == 0xFFFFFFFFu) {
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
         ch.res[g] = kResLeader | 1u;
@@ -1545,6 +1581,17 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
   }
   ok = grid_barrier(a.ctl, G, a.wait_ns, false) && ok;
   if (ok) {
+    // each stored miss records its slot and starts its index inserts (the
+    // first claim attempts), which complete after the copies below
+    const bool ins = ins_slot != ~0ull;
+    const bool ins_hint = ins && !a.paper && len >= kPrefixBytes;
+    PendingInsert pi{0ull, 0u}, ph{0ull, 0u};
+    if (ins) {
+      a.slot_len[ins_slot] = len;
+      a.slot_key[ins_slot] = key;
+      pi = index_insert_begin(a.index, a.index_mask, index_key(a, key), (uint32_t)ins_slot);
+      if (ins_hint) ph = index_insert_begin(a.hints, a.index_mask, hint, (uint32_t)ins_slot);
+    }
     // every miss's bytes, in pieces of kPackPiece bytes spread over all the
     // grid's warps (piece k of the miss of rank r is number r * ppc + k), all
     // but those of misses the hash kernel already wrote where they belong
@@ -1639,15 +1686,13 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
                    reinterpret_cast<const uint8_t*>(sj), lj, ((sj | xj | yj) & 15) == 0);
       }
     }
-    // each stored miss inserts itself and frees the group entry it claimed,
-    // while the last pieces' stores are still in flight
-    if (ins_slot != ~0ull) {
-      a.slot_len[ins_slot] = len;
-      a.slot_key[ins_slot] = key;
-      if (!index_insert(a.index, a.index_mask, index_key(a, key), (uint32_t)ins_slot, len))
+    // each stored miss completes its inserts and frees the group entry it
+    // claimed, while the last pieces' stores are still in flight
+    if (ins) {
+      if (!index_insert_end(a.index, a.index_mask, index_key(a, key), (uint32_t)ins_slot, len, pi))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-      if (!a.paper && len >= kPrefixBytes &&
-          !index_insert(a.hints, a.index_mask, ch.hint[g], (uint32_t)ins_slot, len))
+      if (ins_hint &&
+          !index_insert_end(a.hints, a.index_mask, hint, (uint32_t)ins_slot, len, ph))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       if (e != 0xFFFFFFFFu) a.tbl[e].owner = 0u;
     }
@@ -1723,7 +1768,7 @@ constexpr uint32_t kSmallHashSmem = kSmallGroups * (uint32_t)kGroupBytes;
 constexpr uint32_t kSmallSmem = kSmallHashSmem > kPackSmem ? kSmallHashSmem : kPackSmem;
 
 
-template <bool kAhead>
+template <bool kAhead, bool kPrefixAsync>
 __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a) {
   extern __shared__ __align__(128) uint8_t small_smem[];
   pdl_trigger();
@@ -1741,7 +1786,7 @@ __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a
   const unsigned long long nvb = (h.Ntot * 4 + kThreads - 1) / kThreads;
   for (unsigned long long vb = 0; vb < nvb; ++vb) {
     __syncthreads();  // the previous range's groups are done with the shared memory
-    staged_range<true, kAhead>(h, vb, small_smem);
+    staged_range<true, kAhead, true, kPrefixAsync>(h, vb, small_smem);
   }
   __syncthreads();  // every chunk's probe outcome written (and its stage copies landed)
   if (a.count == 1 && !a.lru && !a.classes && a.Ntot <= (unsigned long long)kThreads) {
@@ -1870,6 +1915,19 @@ int pack_blocks_per_sm() {
   return nb;
 }
 
+// Co-resident blocks per SM of the one-launch resolve + pack kernel (its grid
+// barriers need every block of the grid resident at once).
+int resolve_pack_blocks_per_sm() {
+  int nb = 0;
+  if (cudaFuncSetAttribute((const void*)k_resolve_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kResolvePackSmem) != cudaSuccess)
+    return 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k_resolve_pack, kThreads,
+                                                    kResolvePackSmem) != cudaSuccess)
+    return 0;
+  return nb;
+}
+
 // Co-resident blocks per SM for the cooperative launch (capped).
 int dedup_blocks_per_sm() {
   int nb = 0;
@@ -1902,15 +1960,20 @@ cudaError_t launch_resolve_pack(const DedupArgs& a, int grid, cudaStream_t s) {
 
 uint32_t small_call_groups() { return kSmallGroups; }
 
-template <bool kAhead>
+template <bool kAhead, bool kPrefixAsync>
 cudaError_t launch_small(const HashArgs& h, const DedupArgs& a, cudaStream_t s, bool pdl) {
-  cudaFuncSetAttribute((const void*)k_small_call<kAhead>,
+  cudaFuncSetAttribute((const void*)k_small_call<kAhead, kPrefixAsync>,
                        cudaFuncAttributeMaxDynamicSharedMemorySize, kSmallSmem);
-  return launch_kernel(k_small_call<kAhead>, dim3(1), dim3(kThreads), kSmallSmem, s, pdl, h, a);
+  return launch_kernel(k_small_call<kAhead, kPrefixAsync>, dim3(1), dim3(kThreads), kSmallSmem, s,
+                       pdl, h, a);
 }
 
 cudaError_t launch_small_call(const HashArgs& h, const DedupArgs& a, cudaStream_t s, bool pdl) {
-  return h.spec_mode ? launch_small<true>(h, a, s, pdl) : launch_small<false>(h, a, s, pdl);
+  if (h.C <= kPrefixAsyncMaxChunk)
+    return h.spec_mode ? launch_small<true, true>(h, a, s, pdl)
+                       : launch_small<false, true>(h, a, s, pdl);
+  return h.spec_mode ? launch_small<true, false>(h, a, s, pdl)
+                     : launch_small<false, false>(h, a, s, pdl);
 }
 
 cudaError_t launch_block_check(const BlockCheckArgs& a, cudaStream_t s) {

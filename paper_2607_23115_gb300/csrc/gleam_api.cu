@@ -63,6 +63,7 @@ struct gleam_cache {
   gleam_result_t* h_result_dev = nullptr;  // its device address
   int coop_max_blocks = 0;
   int pack_max_blocks = 0;  // pack kernel: all co-resident blocks
+  int rp_max_blocks = 0;    // one-launch resolve + pack: all co-resident blocks
   cudaEvent_t done = nullptr;
 
   // single-block calls: the largest call (in chunks) that runs as one kernel,
@@ -516,7 +517,13 @@ constexpr uint64_t kChainBytesPerBlock = GLEAM_CHAIN_BYTES_PER_BLOCK;
 // its one-launch resolve kernel may take a block per 512 KiB, up to one per SM
 // (a 64 MiB call of 16,384 chunks: 0.101 -> 0.092 ms); with it, blocks that
 // wait for an earlier call hold resources that the calls in flight want.
-constexpr uint64_t kSoloBytesPerBlock = 512ull << 10;
+#ifndef GLEAM_SOLO_KIB_PER_BLOCK
+#define GLEAM_SOLO_KIB_PER_BLOCK 512
+#endif
+#ifndef GLEAM_SOLO_CAP_DIV
+#define GLEAM_SOLO_CAP_DIV 3
+#endif
+constexpr uint64_t kSoloBytesPerBlock = (uint64_t)GLEAM_SOLO_KIB_PER_BLOCK << 10;
 // the one-launch resolve kernel holds at most one chunk per thread
 static_assert(kChainMaxChunks <= (uint64_t)kChainPackBlocks * 256, "chain limit");
 
@@ -738,8 +745,10 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
       // kChainBytesPerBlock of payload so that the misses' copies spread
       const bool solo = !(c->flags & GLEAM_OVERLAP_CALLS);
       const uint64_t per_block = solo ? kSoloBytesPerBlock : kChainBytesPerBlock;
-      const uint64_t cap = solo ? (uint64_t)std::max(kChainPackBlocks, c->coop_max_blocks / 3)
-                                : (uint64_t)kChainPackBlocks;
+      const uint64_t cap =
+          solo ? (uint64_t)std::min(c->rp_max_blocks,
+                                    std::max(kChainPackBlocks, c->coop_max_blocks / GLEAM_SOLO_CAP_DIV))
+               : (uint64_t)kChainPackBlocks;
       const uint64_t want = std::max<uint64_t>((Ntot + dedup_threads() - 1) / dedup_threads(),
                                                (nbytes + per_block - 1) / per_block);
       rc = cuda_err(launch_resolve_pack(
@@ -852,8 +861,10 @@ int gleam_cache_create_ex(size_t capacity_bytes, size_t chunk_bytes, uint32_t fl
     const int per_sm = dedup_blocks_per_sm();
     c->coop_max_blocks = sms * per_sm;
     c->pack_max_blocks = sms * pack_blocks_per_sm();
+    c->rp_max_blocks = sms * resolve_pack_blocks_per_sm();
     c->small_max_chunks = small_call_groups();
-    if (c->coop_max_blocks <= 0 || c->pack_max_blocks <= 0) rc = GLEAM_ERR_CUDA;
+    if (c->coop_max_blocks <= 0 || c->pack_max_blocks <= 0 || c->rp_max_blocks < kChainPackBlocks)
+      rc = GLEAM_ERR_CUDA;
   }
   // per-block miss and stored-miss counts, then one word used as the single
   // payload's start rank

@@ -298,6 +298,7 @@ int dedup_threads();
 int dedup_chunks_per_block();
 int dedup_blocks_per_sm();
 int pack_blocks_per_sm();
+int resolve_pack_blocks_per_sm();
 
 // ---------------------------------------------------------------------------
 // Device helpers

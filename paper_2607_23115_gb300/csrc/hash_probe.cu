@@ -260,7 +260,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
 }
 
 
-template <bool kProbe, bool kAhead, bool kVerify>
+template <bool kProbe, bool kAhead, bool kVerify, bool kPrefixAsync = false>
 __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   pdl_trigger();
@@ -268,19 +268,23 @@ __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a
   const unsigned long long nvb = (a.Ntot * 4 + kStagedThreads - 1) / kStagedThreads;
   for (unsigned long long vb = blockIdx.x; vb < nvb; vb += gridDim.x) {
     __syncthreads();  // the previous range's groups are done with the shared memory
-    staged_range<kProbe, kAhead, kVerify>(a, vb, smem);
+    staged_range<kProbe, kAhead, kVerify, kPrefixAsync>(a, vb, smem);
   }
 }
 
-template <bool kProbe, bool kAhead, bool kVerify>
+template <bool kProbe, bool kAhead, bool kVerify, bool kPrefixAsync = false>
 cudaError_t launch_staged(const HashArgs& a, cudaStream_t s, bool pdl) {
+  if constexpr (kVerify && !kPrefixAsync) {
+    if (a.C <= kPrefixAsyncMaxChunk)
+      return launch_staged<kProbe, kAhead, kVerify, true>(a, s, pdl);
+  }
   constexpr int smem = (kStagedThreads / 4) * group_bytes(kVerify);
   // per device and cheap: set on every launch
-  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kAhead, kVerify>,
+  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kAhead, kVerify, kPrefixAsync>,
                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   const unsigned long long threads = a.Ntot * 4;
   const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
-  return launch_kernel(k_hash_probe_staged<kProbe, kAhead, kVerify>, dim3(sg),
+  return launch_kernel(k_hash_probe_staged<kProbe, kAhead, kVerify, kPrefixAsync>, dim3(sg),
                        dim3(kStagedThreads), smem, s, pdl, a);
 }
 

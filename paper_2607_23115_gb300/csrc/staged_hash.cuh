@@ -132,6 +132,12 @@ __device__ __forceinline__ unsigned present_lanes(unsigned long long vb, unsigne
 #ifndef GLEAM_STAGE_DEPTH
 #define GLEAM_STAGE_DEPTH 2
 #endif
+// Chunks of at most this many bytes fetch a hinted chunk's cached prefix by
+// cp.async into stage buffer 0, in the same round trip as the cached copy's
+// next stages (GPT-2 pass 2, 4 KiB chunks: hash kernel -3%); larger chunks
+// compare it with direct loads first (64 KiB chunks: 3% faster that way, their
+// one prefix per 128 stages costs little and the simpler loop streams better).
+constexpr uint32_t kPrefixAsyncMaxChunk = 16u << 10;
 #ifndef GLEAM_STAGED_THREADS
 #define GLEAM_STAGED_THREADS 32
 #endif
@@ -187,7 +193,7 @@ __device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uin
 // kVerify = false: no speculative verify and no buffers for a cached copy
 // (an empty cache has none to stream), so twice as many groups fit an SM; a
 // key+length candidate, if any, is still compared with direct loads.
-template <bool kProbe, bool kAhead = false, bool kVerify = true>
+template <bool kProbe, bool kAhead = false, bool kVerify = true, bool kPrefixAsync = false>
 __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long long vb,
                                              uint8_t* smem) {
   const unsigned long long g = (vb * blockDim.x + threadIdx.x) >> 2;
@@ -323,17 +329,33 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
         q = a.arena + (unsigned long long)hint_slot * a.C;
         // loaded now, used once the chunk is hashed: no lookup waits then
         hint_key = a.slot_key[hint_slot];
-        // the prefix, still in stage buffer 0, against the cached copy's prefix
+        if constexpr (kPrefixAsync) {
+          // the cached copy's prefix into the free half of stage buffer 0, in
+          // a group of its own, and its next stages behind it: one round trip
+          // for both
+          stage_copy(pay_s(0) + kStage, q, (uint32_t)kStage, lane);
+          cp_commit();
+        } else {
+          // the prefix, still in stage buffer 0, against the cached copy's prefix
 #pragma unroll 4
-        for (uint32_t s = 0; s < (uint32_t)kStage / 32; ++s)
-          d |= *reinterpret_cast<const unsigned long long*>(sp + s * 32 + lane * 8) ^
-               load_arena_word(q + s * 32 + lane * 8);
+          for (uint32_t s = 0; s < (uint32_t)kStage / 32; ++s)
+            d |= *reinterpret_cast<const unsigned long long*>(sp + s * 32 + lane * 8) ^
+                 load_arena_word(q + s * 32 + lane * 8);
+        }
         // the cached copy of the stages already in flight
         for (uint32_t tt = 1; tt < (uint32_t)kDepth && tt < nst; ++tt)
           stage_copy(pay_s(tt) + kStage, q + (unsigned long long)tt * kStage, sbytes(tt), lane);
       }
     }
     if (t == 0) cp_commit();  // the late group (empty without a hint)
+    if (kPrefixAsync && t == 0 && cmp) {
+      // the prefix's group is complete once at most the late group pends
+      cp_wait<1>();
+      __syncwarp(gmask);
+#pragma unroll
+      for (uint32_t s = 0; s < (uint32_t)kStage / 32; ++s)
+        d |= word(sp, s) ^ word(sp + kStage, s);
+    }
     if (cmp) {
       // a lane that found a difference stops streaming its share of the
       // cached copy; the others may then compare stale words, which can only
