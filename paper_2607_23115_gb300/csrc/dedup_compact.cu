@@ -1104,6 +1104,7 @@ __device__ __forceinline__ void finish_call(const DedupArgs& a, uint32_t G,
   if (threadIdx.x == 0) {
     DevCtl* c = a.ctl;
     c->bar_count = 0;
+    c->copy_next = 0;
     c->err = 0;
     c->unres[0] = c->unres[1] = c->unres[2] = 0;
     c->shared_groups = 0;
@@ -1422,6 +1423,46 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
 // takes over: the minima are posted and resolve_rank and pack_publish run on
 // the same grid.
 constexpr uint32_t kResolvePackSmem = kPackSmem;
+// The one-launch kernel's copies: pieces handed out by a shared counter,
+// GLEAM_RP_STEAL at a time (0: an equal share of consecutive pieces per warp).
+#ifndef GLEAM_RP_STEAL
+#define GLEAM_RP_STEAL 0
+#endif
+constexpr uint32_t kRpGrab = GLEAM_RP_STEAL;
+static_assert(kRpGrab <= 32, "a grab is at most one batch of 32 pieces");
+
+// Bit k of the result: byte k of w (k < 4) is not kHit0.
+__device__ __forceinline__ uint32_t not_hit_bits(uint32_t w) {
+  const uint32_t x = w ^ (0x01010101u * kHit0);
+  const uint32_t t = (((x & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | x) & 0x80808080u;  // bit 8k+7: byte k != 0
+  return ((t >> 7) & 1u) | ((t >> 14) & 2u) | ((t >> 21) & 4u) | ((t >> 28) & 8u);
+}
+
+// This thread's share of the call's chunks that are not cache hits: among
+// chunks [0, lim) (*below) and among all N (*all); the block's threads
+// together cover every chunk once.
+__device__ __forceinline__ void count_not_hit(const uint8_t* status, uint32_t N, uint32_t lim,
+                                              uint32_t* below, uint32_t* all) {
+  uint32_t b = 0, t = 0;
+  const bool vec = ((uintptr_t)status & 15) == 0;
+  for (uint32_t v = threadIdx.x; v * 16 < N; v += blockDim.x) {
+    const uint32_t b0 = v * 16;
+    uint32_t m = 0;
+    if (vec && b0 + 16 <= N) {
+      const uint4 q = __ldcg(reinterpret_cast<const uint4*>(status) + v);
+      m = not_hit_bits(q.x) | not_hit_bits(q.y) << 4 | not_hit_bits(q.z) << 8 |
+          not_hit_bits(q.w) << 12;
+    } else {
+      for (uint32_t k = 0; k < 16 && b0 + k < N; ++k)
+        m |= (uint32_t)(__ldcg(status + b0 + k) != kHit0) << k;
+    }
+    t += __popc(m);
+    const uint32_t nb = lim <= b0 ? 0u : min(lim - b0, 16u);
+    b += __popc(m & ((1u << nb) - 1u));
+  }
+  *below = b;
+  *all = t;
+}
 
 __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G, uint32_t bid,
                                                   uint8_t* smem) {
@@ -1450,11 +1491,15 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
   uint32_t len = 0, e = 0xFFFFFFFFu;
   unsigned long long key = 0, hint = 0;
   bool lead = false, stored = false, shared = false;
+  // the hash kernel claimed the groups: every miss is stored (the staged
+  // kernel marks no chunk uncached) and was given its entry there
+  const bool pre = a.pre_claimed != 0;
   if (valid) {
     // the chunk's record at once (one round trip, whatever its status)
     st = ch.status[g];
     const unsigned long long key0 = ch.key[g];
     const uint32_t len0 = ch.len[g];
+    const uint32_t ent0 = pre ? ch.ent[g] : 0u;
     hint = a.paper ? 0ull : ch.hint[g];
     if ((g & 31) == 0) P.mask[g >> 5] = 0;
     if (st == kHit0) {
@@ -1468,14 +1513,14 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
       key = key0;
       len = len0;
       bool claimed = true;
-      e = group_entry(a, g, key, len, &claimed, true);
+      e = pre ? ent0 : group_entry(a, g, key, len, &claimed, true);
       if (e == 0xFFFFFFFFu) {
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
         ch.res[g] = kResLeader | 1u;
-      } else {
+      } else if (!pre) {
         ch.res[g] = kResUnresolved;
       }
-      ch.ent[g] = e;
+      if (!pre) ch.ent[g] = e;
       shared = !claimed;
       lead = stored = true;
     }
@@ -1486,20 +1531,55 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
     s_shared = 1;
     if (G > 1) atomicOr(&a.ctl->shared_groups, 1u);
   }
-  if (G > 1 && threadIdx.x == 0) {
-    a.bcount[bid] = c_b;
-    a.bcount[G + bid] = s_b;
+  bool ok = true;
+  unsigned long long pre_before = 0, pre_total = 0;
+  if (pre) {
+    // no barrier: every block counts the misses before its chunks, and in
+    // all, from the statuses the hash kernel wrote (at most 16 KiB of them)
+    uint32_t mb = 0, mt = 0;
+    count_not_hit(ch.status, N, bid * per, &mb, &mt);
+    pre_before = block_sum<unsigned long long>(mb, red64);
+    pre_total = block_sum<unsigned long long>(mt, red64);
+    if (threadIdx.x == 0) {
+      s_shared = (int)ldcg_u32(&a.ctl->shared_groups);
+      s_slots0 = my_slots0;
+      s_err = ld_volatile_s32(&a.ctl->err);
+    }
+    __syncthreads();
+    ok = s_err == 0;
+  } else {
+    if (G > 1 && threadIdx.x == 0) {
+      a.bcount[bid] = c_b;
+      a.bcount[G + bid] = s_b;
+    }
+    ok = grid_barrier(a.ctl, G, a.wait_ns, false);
+    if (threadIdx.x == 0) {
+      if (G > 1) s_shared = (int)ldcg_u32(&a.ctl->shared_groups);
+      s_slots0 = my_slots0;
+      s_err = G == 1 ? ld_volatile_s32(&a.ctl->err) : 0;
+    }
+    __syncthreads();
+    if (G == 1) ok = s_err == 0;  // a grid of one did not read the error word
   }
-  bool ok = grid_barrier(a.ctl, G, a.wait_ns, false);
-  if (threadIdx.x == 0) {
-    if (G > 1) s_shared = (int)ldcg_u32(&a.ctl->shared_groups);
-    s_slots0 = my_slots0;
-    s_err = G == 1 ? ld_volatile_s32(&a.ctl->err) : 0;
-  }
-  __syncthreads();
-  if (G == 1) ok = s_err == 0;  // a grid of one did not read the error word
 
   if (s_shared) {
+    if (pre) {
+      // a chunk found an entry with its tag: the groups are claimed again,
+      // by the whole group key and length, in the cleared table
+      const bool mine = valid && st != kHit0 && st != kUncached;
+      if (mine && e != 0xFFFFFFFFu)
+        *reinterpret_cast<volatile unsigned long long*>(&a.tbl[e]) = 0ull;
+      ok = grid_barrier(a.ctl, G, a.wait_ns, false) && ok;
+      if (ok && mine) {
+        bool claimed = true;
+        e = group_entry(a, g, key, len, &claimed, true);
+        if (e == 0xFFFFFFFFu) {
+          atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+          ch.res[g] = kResLeader | 1u;
+        }
+        ch.ent[g] = e;
+      }
+    }
     // the general algorithm: post the group minima, then the rounds, ranks
     // and copies of k_dedup and k_pack on this grid
     if (ok) {  // every lane of the block takes part (one chunk per thread at most)
@@ -1516,7 +1596,10 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
   // ---- 2: the fast path: ranks, outputs, inserts; then copies ----------------
   const unsigned long long slots0 = s_slots0;
   unsigned long long before = 0, total = c_b, sbefore = 0, stotal = s_b;
-  if (G > 1) {
+  if (pre) {
+    before = sbefore = pre_before;
+    total = stotal = pre_total;
+  } else if (G > 1) {
     unsigned long long b0 = 0, t0 = 0, sb0 = 0, st0 = 0;
     for (uint32_t j = threadIdx.x; j < G; j += kThreads) {
       const uint32_t v = ldcg_u32(&a.bcount[j]), sv = ldcg_u32(&a.bcount[G + j]);
@@ -1614,6 +1697,80 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
     }
     __syncwarp();
 #endif
+    // pieces [lo, hi) of the call, 32 at a time
+    auto copy_range = [&](unsigned long long lo, unsigned long long hi) {
+      for (unsigned long long base = lo; base < hi; base += 32) {
+        const unsigned long long pc = base + lane;
+        uint32_t bytes = 0;
+        bool copy = false;
+        unsigned long long src = 0, d1 = 0, d2 = 0;
+        if (pc < hi) {
+          const unsigned long long rr = pc / ppc;
+          const uint32_t off = (uint32_t)(pc - rr * ppc) * kPackPiece;
+          const uint32_t gg = __ldcg(&ch.order[rr]);
+          const uint32_t ln = (uint32_t)min(a.C, P.n - (unsigned long long)gg * a.C);
+          if (off < ln) {
+            const uint32_t srr = __ldcg(&ch.srank[gg]);
+            const bool ahead = a.spec_active && srr == gg && ch.spec[gg];
+            if (!ahead) {
+              bytes = min(kPackPiece, ln - off);
+              src = (unsigned long long)(P.buf + (unsigned long long)gg * a.C + off);
+              d1 = (unsigned long long)(P.packed + rr * a.C + off);
+              d2 = srr != kEmptySlot ? (unsigned long long)(a.arena + (slots0 + srr) * a.C + off)
+                                     : 0ull;
+              copy = true;
+            }
+          }
+        }
+        const unsigned cmask = __ballot_sync(0xffffffffu, copy);
+#if GLEAM_PACK_BULK
+        const bool bulk =
+            !a.plain_copy && __all_sync(0xffffffffu, !copy || ((src | d1 | d2) & 15) == 0);
+        if (bulk) {
+          if (copy) meta[__popc(cmask & ((1u << lane) - 1u))] = PackMeta{src, d1, d2, bytes, 0u};
+          __syncwarp();
+          if (lane == 0 && cmask && !bulk_failed &&
+              !bulk_copy_batch(meta, __popc(cmask), bufs, bars, ring, a.wait_ns)) {
+            bulk_failed = true;
+            atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_TIMEOUT);
+          }
+          if (copy) {  // the piece's last bytes % 16
+            const uint8_t* sp = reinterpret_cast<const uint8_t*>(src);
+            uint8_t* x = reinterpret_cast<uint8_t*>(d1);
+            uint8_t* y = reinterpret_cast<uint8_t*>(d2);
+            for (uint32_t k2 = bytes & ~15u; k2 < bytes; ++k2) {
+              x[k2] = sp[k2];
+              if (y) y[k2] = sp[k2];
+            }
+          }
+          __syncwarp();
+        } else
+#endif
+        for (unsigned todo = cmask; todo; todo &= todo - 1) {
+          const int j = __ffs(todo) - 1;
+          const unsigned long long sj = __shfl_sync(0xffffffffu, src, j);
+          const unsigned long long xj = __shfl_sync(0xffffffffu, d1, j);
+          const unsigned long long yj = __shfl_sync(0xffffffffu, d2, j);
+          const uint32_t lj = __shfl_sync(0xffffffffu, bytes, j);
+          warp_copy2(reinterpret_cast<uint8_t*>(xj), reinterpret_cast<uint8_t*>(yj),
+                     reinterpret_cast<const uint8_t*>(sj), lj, ((sj | xj | yj) & 15) == 0);
+        }
+      }
+    };
+#if GLEAM_RP_STEAL
+    // the pieces taken kRpGrab at a time from a counter of the call, the
+    // warp's next grab requested before its current one is copied: warps on
+    // SMs that copy faster take more
+    uint32_t nxt = 0;
+    if (lane == 0) nxt = atomicAdd(&a.ctl->copy_next, kRpGrab);
+    nxt = __shfl_sync(0xffffffffu, nxt, 0);
+    while (nxt < npieces) {
+      uint32_t nn = 0;
+      if (lane == 0) nn = atomicAdd(&a.ctl->copy_next, kRpGrab);
+      copy_range(nxt, min(npieces, (unsigned long long)nxt + kRpGrab));
+      nxt = __shfl_sync(0xffffffffu, nn, 0);
+    }
+#else
 #if GLEAM_CHAIN_PREFETCH
     // the warp's source pieces start their way into L2 at once (up to 32),
     // so that the copies below wait for L2 rather than HBM
@@ -1629,63 +1786,8 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
       }
     }
 #endif
-    for (unsigned long long base = plo; base < phi; base += 32) {
-      const unsigned long long pc = base + lane;
-      uint32_t bytes = 0;
-      bool copy = false;
-      unsigned long long src = 0, d1 = 0, d2 = 0;
-      if (pc < phi) {
-        const unsigned long long rr = pc / ppc;
-        const uint32_t off = (uint32_t)(pc - rr * ppc) * kPackPiece;
-        const uint32_t gg = __ldcg(&ch.order[rr]);
-        const uint32_t ln = (uint32_t)min(a.C, P.n - (unsigned long long)gg * a.C);
-        if (off < ln) {
-          const uint32_t srr = __ldcg(&ch.srank[gg]);
-          const bool ahead = a.spec_active && srr == gg && ch.spec[gg];
-          if (!ahead) {
-            bytes = min(kPackPiece, ln - off);
-            src = (unsigned long long)(P.buf + (unsigned long long)gg * a.C + off);
-            d1 = (unsigned long long)(P.packed + rr * a.C + off);
-            d2 = srr != kEmptySlot ? (unsigned long long)(a.arena + (slots0 + srr) * a.C + off)
-                                   : 0ull;
-            copy = true;
-          }
-        }
-      }
-      const unsigned cmask = __ballot_sync(0xffffffffu, copy);
-#if GLEAM_PACK_BULK
-      const bool bulk =
-          !a.plain_copy && __all_sync(0xffffffffu, !copy || ((src | d1 | d2) & 15) == 0);
-      if (bulk) {
-        if (copy) meta[__popc(cmask & ((1u << lane) - 1u))] = PackMeta{src, d1, d2, bytes, 0u};
-        __syncwarp();
-        if (lane == 0 && cmask && !bulk_failed &&
-            !bulk_copy_batch(meta, __popc(cmask), bufs, bars, ring, a.wait_ns)) {
-          bulk_failed = true;
-          atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_TIMEOUT);
-        }
-        if (copy) {  // the piece's last bytes % 16
-          const uint8_t* sp = reinterpret_cast<const uint8_t*>(src);
-          uint8_t* x = reinterpret_cast<uint8_t*>(d1);
-          uint8_t* y = reinterpret_cast<uint8_t*>(d2);
-          for (uint32_t k2 = bytes & ~15u; k2 < bytes; ++k2) {
-            x[k2] = sp[k2];
-            if (y) y[k2] = sp[k2];
-          }
-        }
-        __syncwarp();
-      } else
+    copy_range(plo, phi);
 #endif
-      for (unsigned todo = cmask; todo; todo &= todo - 1) {
-        const int j = __ffs(todo) - 1;
-        const unsigned long long sj = __shfl_sync(0xffffffffu, src, j);
-        const unsigned long long xj = __shfl_sync(0xffffffffu, d1, j);
-        const unsigned long long yj = __shfl_sync(0xffffffffu, d2, j);
-        const uint32_t lj = __shfl_sync(0xffffffffu, bytes, j);
-        warp_copy2(reinterpret_cast<uint8_t*>(xj), reinterpret_cast<uint8_t*>(yj),
-                   reinterpret_cast<const uint8_t*>(sj), lj, ((sj | xj | yj) & 15) == 0);
-      }
-    }
     // each stored miss completes its inserts and frees the group entry it
     // claimed, while the last pieces' stores are still in flight
     if (ins) {
@@ -1694,7 +1796,7 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
       if (ins_hint &&
           !index_insert_end(a.hints, a.index_mask, hint, (uint32_t)ins_slot, len, ph))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-      if (e != 0xFFFFFFFFu) a.tbl[e].owner = 0u;
+      if (e != 0xFFFFFFFFu) a.tbl[e] = CallEntry{0u, 0u};  // owner and the claim's tag
     }
 #if GLEAM_PACK_BULK
     if (lane == 0) bulk_wait_all<0>();  // every piece written before the block ends

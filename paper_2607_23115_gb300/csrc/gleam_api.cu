@@ -715,6 +715,29 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   // host payloads too: a chunk written ahead then spares the pack a second
   // read over the CPU-GPU link (managed memory stays out)
   set_spec(c, &h, &d, aligned && packed_aligned && !chk.saw_managed() && !h.wait_late);
+  // a payload resolved by the one-launch kernel: its staged hash kernel
+  // claims the misses' groups as it records them
+  const bool one_launch = !fused && chain && count == 1 && !d.classes;
+  int rp_grid = 1;
+  if (one_launch) {
+    // at most one chunk per thread, and one block per kChainBytesPerBlock of
+    // payload so that the misses' copies spread
+    const bool solo = !(c->flags & GLEAM_OVERLAP_CALLS);
+    const uint64_t per_block = solo ? kSoloBytesPerBlock : kChainBytesPerBlock;
+    const uint64_t cap =
+        solo ? (uint64_t)std::min(c->rp_max_blocks,
+                                  std::max(kChainPackBlocks, c->coop_max_blocks / GLEAM_SOLO_CAP_DIV))
+             : (uint64_t)kChainPackBlocks;
+    const uint64_t want = std::max<uint64_t>((Ntot + dedup_threads() - 1) / dedup_threads(),
+                                             (nbytes + per_block - 1) / per_block);
+    rp_grid = (int)std::min<uint64_t>(std::max<uint64_t>(1, want), cap);
+  }
+  // (a grid of one block needs no barrier before its ranks anyway)
+  if (one_launch && rp_grid > 1 && hash_is_staged(h, aligned)) {
+    h.claim_tbl = d.tbl;
+    h.claim_mask = d.tbl_mask;
+    d.pre_claimed = 1u;
+  }
 
   cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
   if (c->profile) {
@@ -740,24 +763,15 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
       grid = (int)std::min<uint64_t>(kChainDedupBlocks, (Ntot + 255) / 256);
       pgrid = std::min(pgrid, kChainPackBlocks);
     }
-    if (chain && count == 1 && !d.classes) {
-      // one launch: at most one chunk per thread, and one block per
-      // kChainBytesPerBlock of payload so that the misses' copies spread
-      const bool solo = !(c->flags & GLEAM_OVERLAP_CALLS);
-      const uint64_t per_block = solo ? kSoloBytesPerBlock : kChainBytesPerBlock;
-      const uint64_t cap =
-          solo ? (uint64_t)std::min(c->rp_max_blocks,
-                                    std::max(kChainPackBlocks, c->coop_max_blocks / GLEAM_SOLO_CAP_DIV))
-               : (uint64_t)kChainPackBlocks;
-      const uint64_t want = std::max<uint64_t>((Ntot + dedup_threads() - 1) / dedup_threads(),
-                                               (nbytes + per_block - 1) / per_block);
-      rc = cuda_err(launch_resolve_pack(
-          d, (int)std::min<uint64_t>(std::max<uint64_t>(1, want), cap), s));
+    if (one_launch) {
+      rc = cuda_err(launch_resolve_pack(d, rp_grid, s));
     } else {
       rc = cuda_err(launch_dedup(d, grid, pgrid, s, chain));
     }
     if (rc != GLEAM_OK) {
       cudaMemsetAsync(c->ctl, 0, sizeof(DevCtl), s);  // the hash kernel may have flagged it
+      if (d.pre_claimed)  // and claimed group entries
+        cudaMemsetAsync(d.tbl, 0, (d.tbl_mask + 1) * sizeof(CallEntry), s);
       return rc;
     }
   }

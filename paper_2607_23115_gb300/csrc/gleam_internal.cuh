@@ -57,7 +57,7 @@ enum StatIdx {
 // Per-call control block; starts zeroed and every dedup kernel leaves it zeroed.
 struct DevCtl {
   unsigned int bar_count;  // grid-barrier arrivals of the call (nblocks per barrier)
-  unsigned int pad1;
+  unsigned int copy_next;  // next piece to hand out (one-launch resolve + pack copies)
   int err;
   unsigned int done;
   unsigned int unres[3];
@@ -175,6 +175,15 @@ struct HashArgs {
   // speculative verify, the hint table and arena bytes of the slots counted as
   // used when it started, which no later call changes (no eviction).
   uint32_t wait_late;
+  // Calls resolved by the one-launch kernel on more than one block (one
+  // payload): the staged hash kernel claims each miss's entry in the per-call
+  // group table as it records the chunk (ent and res as the resolve kernel
+  // would set them; the entry's minv holds a tag of the chunk's (group key,
+  // length) until the resolve kernel frees it; shared_groups if an entry with
+  // the same tag was found), so that the resolve kernel needs no claims and
+  // no barrier before its ranks.  Null: no claims here.
+  CallEntry* claim_tbl;
+  unsigned long long claim_mask;
 };
 
 struct DedupArgs {
@@ -225,6 +234,8 @@ struct DedupArgs {
   uint32_t spec_active;
   uint32_t* spec_state;
   uint32_t* spec_mirror;
+  // the hash kernel claimed the misses' groups (HashArgs::claim_tbl)
+  uint32_t pre_claimed;
 };
 
 constexpr uint32_t kLruBins = 65536;
@@ -235,6 +246,9 @@ constexpr uint32_t kPaperMinCached = 1024;
 // pdl: launched with programmatic stream serialization (the kernel waits on the
 // GPU for the one before it; see pdl_trigger/pdl_wait).
 cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s, bool pdl = false);
+// Whether launch_hash runs the staged XXH64 kernel for these arguments (the
+// one that can claim groups, HashArgs::claim_tbl).
+bool hash_is_staged(const HashArgs& a, bool aligned);
 // Loads the hash kernels' device code on the current GPU (cache creation does
 // it, so that no later call loads code, which allocates device memory).
 cudaError_t load_hash_kernels();

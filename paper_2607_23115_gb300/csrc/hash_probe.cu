@@ -602,6 +602,14 @@ cudaError_t load_hash_kernels() {
   return cudaFuncGetAttributes(&fa, k_hash_probe_staged<true, false, true>);
 }
 
+bool hash_is_staged(const HashArgs& a, bool aligned) {
+#if GLEAM_STAGED_HASH
+  return a.Ntot > 0 && !(a.index != nullptr && a.paper) && aligned && (a.C % 32 == 0 || a.Ntot == 1);
+#else
+  return false;
+#endif
+}
+
 cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s, bool pdl) {
   if (a.Ntot == 0) return cudaSuccess;
   const unsigned long long threads = a.Ntot * 4;

@@ -491,7 +491,37 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
     a.ch.pidx[g] = pid;
     a.ch.hint[g] = hint;
     if (kAhead) a.ch.spec[g] = ahead ? 1 : 0;
-    if (hit) a.ch.ent[g] = hit_slot;
+    if (hit) {
+      a.ch.ent[g] = hit_slot;
+    } else if (kProbe && a.claim_tbl != nullptr) {
+      // the miss's (group key, length) entry of the per-call table, claimed
+      // with one 64-bit CAS that also stores a 32-bit tag of the pair (where
+      // the resolve kernel keeps a minimum): an entry found holding the same
+      // tag may be the chunk's group, which sends the call down the general
+      // path (shared_groups), where the groups are claimed again by the whole
+      // key; a different tag is another group's entry
+      const unsigned long long mixed = mix64(h ^ ((unsigned long long)len << 40));
+      const unsigned long long tag = mixed >> 32;
+      unsigned long long pos = mixed & a.claim_mask;
+      uint32_t e = 0xFFFFFFFFu;
+      for (unsigned long long probe = 0; probe <= a.claim_mask; ++probe) {
+        const unsigned long long old =
+            atomicCAS(reinterpret_cast<unsigned long long*>(&a.claim_tbl[pos]), 0ull,
+                      (tag << 32) | ((unsigned long long)g + 1ull));
+        if (old == 0) {
+          e = (uint32_t)pos;
+          break;
+        }
+        if ((old >> 32) == tag) {
+          e = (uint32_t)pos;
+          atomicOr(&a.ctl->shared_groups, 1u);
+          break;
+        }
+        pos = (pos + 1) & a.claim_mask;
+      }
+      a.ch.ent[g] = e;
+      a.ch.res[g] = kResUnresolved;
+    }
   }
 }
 
