@@ -1423,13 +1423,7 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
 // takes over: the minima are posted and resolve_rank and pack_publish run on
 // the same grid.
 constexpr uint32_t kResolvePackSmem = kPackSmem;
-// The one-launch kernel's copies: pieces handed out by a shared counter,
-// GLEAM_RP_STEAL at a time (0: an equal share of consecutive pieces per warp).
-#ifndef GLEAM_RP_STEAL
-#define GLEAM_RP_STEAL 0
-#endif
-constexpr uint32_t kRpGrab = GLEAM_RP_STEAL;
-static_assert(kRpGrab <= 32, "a grab is at most one batch of 32 pieces");
+
 
 // Bit k of the result: byte k of w (k < 4) is not kHit0.
 __device__ __forceinline__ uint32_t not_hit_bits(uint32_t w) {
@@ -1757,37 +1751,38 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
         }
       }
     };
-#if GLEAM_RP_STEAL
-    // the pieces taken kRpGrab at a time from a counter of the call, the
-    // warp's next grab requested before its current one is copied: warps on
-    // SMs that copy faster take more
-    uint32_t nxt = 0;
-    if (lane == 0) nxt = atomicAdd(&a.ctl->copy_next, kRpGrab);
-    nxt = __shfl_sync(0xffffffffu, nxt, 0);
-    while (nxt < npieces) {
-      uint32_t nn = 0;
-      if (lane == 0) nn = atomicAdd(&a.ctl->copy_next, kRpGrab);
-      copy_range(nxt, min(npieces, (unsigned long long)nxt + kRpGrab));
-      nxt = __shfl_sync(0xffffffffu, nn, 0);
-    }
-#else
-#if GLEAM_CHAIN_PREFETCH
-    // the warp's source pieces start their way into L2 at once (up to 32),
-    // so that the copies below wait for L2 rather than HBM
-    if (plo + lane < phi && !a.plain_copy) {
-      const unsigned long long pc = plo + lane, rr = pc / ppc;
-      const uint32_t off = (uint32_t)(pc - rr * ppc) * kPackPiece;
-      const uint32_t gg = __ldcg(&ch.order[rr]);
-      const uint32_t ln = (uint32_t)min(a.C, P.n - (unsigned long long)gg * a.C);
-      const uint8_t* src = P.buf + (unsigned long long)gg * a.C + off;
-      if (off < ln && ((uintptr_t)src & 15) == 0) {  // the prefetch wants 16-byte alignment
-        const uint32_t pb = min(kPackPiece, ln - off) & ~15u;
-        if (pb) prefetch_l2(src, pb);
+    if (a.copy_grab) {
+      // the pieces taken copy_grab at a time from a counter of the call, the
+      // warp's next grab requested before its current one is copied: warps
+      // on SMs that copy faster take more
+      const uint32_t grab = a.copy_grab;
+      uint32_t nxt = 0;
+      if (lane == 0) nxt = atomicAdd(&a.ctl->copy_next, grab);
+      nxt = __shfl_sync(0xffffffffu, nxt, 0);
+      while (nxt < npieces) {
+        uint32_t nn = 0;
+        if (lane == 0) nn = atomicAdd(&a.ctl->copy_next, grab);
+        copy_range(nxt, min(npieces, (unsigned long long)nxt + grab));
+        nxt = __shfl_sync(0xffffffffu, nn, 0);
       }
+    } else {
+#if GLEAM_CHAIN_PREFETCH
+      // the warp's source pieces start their way into L2 at once (up to 32),
+      // so that the copies below wait for L2 rather than HBM
+      if (plo + lane < phi && !a.plain_copy) {
+        const unsigned long long pc = plo + lane, rr = pc / ppc;
+        const uint32_t off = (uint32_t)(pc - rr * ppc) * kPackPiece;
+        const uint32_t gg = __ldcg(&ch.order[rr]);
+        const uint32_t ln = (uint32_t)min(a.C, P.n - (unsigned long long)gg * a.C);
+        const uint8_t* src = P.buf + (unsigned long long)gg * a.C + off;
+        if (off < ln && ((uintptr_t)src & 15) == 0) {  // the prefetch wants 16-byte alignment
+          const uint32_t pb = min(kPackPiece, ln - off) & ~15u;
+          if (pb) prefetch_l2(src, pb);
+        }
+      }
+#endif
+      copy_range(plo, phi);
     }
-#endif
-    copy_range(plo, phi);
-#endif
     // each stored miss completes its inserts and frees the group entry it
     // claimed, while the last pieces' stores are still in flight
     if (ins) {

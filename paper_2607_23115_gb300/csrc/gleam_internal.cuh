@@ -236,6 +236,9 @@ struct DedupArgs {
   uint32_t* spec_mirror;
   // the hash kernel claimed the misses' groups (HashArgs::claim_tbl)
   uint32_t pre_claimed;
+  // one-launch resolve + pack: pieces of misses a warp takes at a time from a
+  // counter of the call (1..32), or 0 for an equal share per warp
+  uint32_t copy_grab;
 };
 
 constexpr uint32_t kLruBins = 65536;
