@@ -432,8 +432,11 @@ __device__ __forceinline__ uint32_t block_find_payload(const PayloadDesc* table,
   unsigned long long* s_p0 = scratch + 32;
   if (threadIdx.x < 32) {
     const uint32_t lane = threadIdx.x;
-    uint32_t lo = 0, hi = count;  // table[lo].chunk_base <= g0; hi == count or its base > g0
-    while (hi - lo > 1) {
+    // table[lo].chunk_base <= g0; hi == count or its base > g0.  Narrowed
+    // until the 32-entry window at lo holds g0's payload (one round for up
+    // to 1,024 payloads), not to one entry: the window load settles the rest.
+    uint32_t lo = 0, hi = count;
+    while (hi - lo > 32) {
       const uint32_t span = hi - lo;
       const uint32_t q = lo + 1 + (uint32_t)(((unsigned long long)(span - 1) * lane) >> 5);
       const unsigned m = __ballot_sync(0xffffffffu, __ldg(&table[q].chunk_base) <= g0);
