@@ -509,13 +509,13 @@ constexpr uint64_t kChainMaxChunks = GLEAM_CHAIN_MAX_CHUNKS;
 constexpr uint64_t kChainMaxBytes = 256ull << 20;
 constexpr int kChainDedupBlocks = GLEAM_CHAIN_DEDUP_BLOCKS;
 constexpr int kChainPackBlocks = GLEAM_CHAIN_PACK_BLOCKS;
-// Overlapping calls: a block of the one-launch kernel per 1 MiB of payload
-// (Llama-3-8B one call per tensor: 1,315 GB/s with 2 MiB, 1,342 with 1 MiB,
-// 1,304 with 512 KiB), or per 512 KiB for calls under 4 MiB, whose copies
-// would otherwise fall to one block (the 10,000-call stream's calls of
-// 256 KiB-1 MiB: 38.8 -> 34.2 us each).
+// Overlapping calls: a block of the one-launch kernel per 2 MiB of payload
+// (Llama-3-8B, one call per tensor: 1,558-1,571 GB/s, against 1,480-1,495
+// with 1 MiB), or per 512 KiB for calls under 4 MiB, whose copies would
+// otherwise fall to one block (the 10,000-call stream's calls of 256 KiB-
+// 1 MiB: 38.8 -> 34.2 us each).
 #ifndef GLEAM_CHAIN_BYTES_PER_BLOCK
-#define GLEAM_CHAIN_BYTES_PER_BLOCK (1ull << 20)
+#define GLEAM_CHAIN_BYTES_PER_BLOCK (2ull << 20)
 #endif
 constexpr uint64_t kChainSmallCall = 4ull << 20;
 constexpr uint64_t kChainBytesPerBlock = GLEAM_CHAIN_BYTES_PER_BLOCK;
@@ -746,8 +746,8 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   // (a grid of one block needs no barrier before its ranks anyway)
   // overlapping calls give the one-launch kernel few blocks (a block per
   // kChainBytesPerBlock): its warps then share the copies out as they go
-  // (Llama-3-8B, one call per tensor: +4.5%), where an equal share per warp
-  // suits the one-block-per-SM grid of a call on its own
+  // (Llama-3-8B, one call per tensor: +1%, four layers of it: +3%), where an
+  // equal share per warp suits the one-block-per-SM grid of a call on its own
   if (one_launch && rp_grid > 1 && (c->flags & GLEAM_OVERLAP_CALLS)) d.copy_grab = kOverlapCopyGrab;
   if (one_launch && rp_grid > 1 && hash_is_staged(h, aligned)) {
     h.claim_tbl = d.tbl;
