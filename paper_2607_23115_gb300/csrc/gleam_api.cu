@@ -676,7 +676,10 @@ int enqueue(gleam_cache* c, const gleam_payload_t* payloads, uint64_t count,
   h.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   h.ch = c->ch;
   h.ctl = c->ctl;
-  h.cache_empty = c->slots_bound == 0 ? 1u : 0u;  // an upper bound of the used slots
+  // slots_bound: an upper bound of the used slots
+  h.no_hints = c->slots_bound == 0 ||
+                       (c->C <= kHintedMaxChunk && c->slots_bound * kHintedMinRatio < Ntot)
+                   ? 1u : 0u;
 
   DedupArgs d{};
   d.table = c->d_table;
@@ -1463,7 +1466,9 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   h.paper = (c->flags & GLEAM_PAPER_IDS) ? 1u : 0u;
   h.ch = ch;
   h.ctl = ctl;
-  h.cache_empty = c->slots_bound == 0 ? 1u : 0u;
+  h.no_hints = c->slots_bound == 0 ||
+                       (c->C <= kHintedMaxChunk && c->slots_bound * kHintedMinRatio < N)
+                   ? 1u : 0u;
 
   DedupArgs d{};
   d.one = one;

@@ -167,7 +167,15 @@ struct HashArgs {
   // to arena slot slots_used + g as it streams by
   uint32_t spec_mode;
   uint8_t* arena_w;                // the arena, for those writes
-  uint32_t cache_empty;            // the host knows the cache holds no chunk yet
+  // the host knows the cache holds no chunk, or (chunks of at most
+  // kHintedMaxChunk) so few against the call's chunks (fewer than one per
+  // kHintedMinRatio) that the prefix-hinted verify would rarely find a copy to
+  // stream: the kernel variant without it (and without its stage buffers, so
+  // twice the groups per SM) runs, and every key+length candidate is compared
+  // after the probe, which costs a larger chunk two more reads of its bytes
+  // (KEY16 adversarial payloads with 64 cached entries: 1 KiB chunks +13%,
+  // 64 KiB chunks -7% when they too took this variant)
+  uint32_t no_hints;
   unsigned long long nslots;
   // Calls that overlap (GLEAM_OVERLAP_CALLS): the kernel was launched while the
   // cache's previous call may still be running, and waits for it only before
@@ -248,6 +256,8 @@ constexpr uint32_t kPaperMinCached = 1024;
 
 // pdl: launched with programmatic stream serialization (the kernel waits on the
 // GPU for the one before it; see pdl_trigger/pdl_wait).
+constexpr unsigned long long kHintedMinRatio = 16;
+constexpr unsigned long long kHintedMaxChunk = 4096;
 cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s, bool pdl = false);
 // Whether launch_hash runs the staged XXH64 kernel for these arguments (the
 // one that can claim groups, HashArgs::claim_tbl).

@@ -631,10 +631,11 @@ cudaError_t launch_hash(const HashArgs& a, bool aligned, cudaStream_t s, bool pd
   }
 #if GLEAM_STAGED_HASH
   if (aligned && (a.C % 32 == 0 || a.Ntot == 1)) {
-    // no cached copy can be streamed when only fingerprints are wanted or the
-    // cache is known to be empty: the variant without those buffers
+    // no cached copy is streamed when only fingerprints are wanted or the
+    // cache holds no chunk (or too few to be worth the hint lookups): the
+    // variant without those buffers
     if (!probe) return launch_staged<false, false, false>(a, s, pdl);
-    if (a.cache_empty)
+    if (a.no_hints)
       return a.spec_mode ? launch_staged<true, true, false>(a, s, pdl)
                          : launch_staged<true, false, false>(a, s, pdl);
     return a.spec_mode ? launch_staged<true, true, true>(a, s, pdl)

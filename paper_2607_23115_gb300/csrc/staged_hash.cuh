@@ -191,8 +191,9 @@ __device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uin
 // shared memory holds one region of group_bytes(kVerify) per group.  kAhead:
 // with the write-through of likely misses (written ahead of the pack step).
 // kVerify = false: no speculative verify and no buffers for a cached copy
-// (an empty cache has none to stream), so twice as many groups fit an SM; a
-// key+length candidate, if any, is still compared with direct loads.
+// (for a cache that holds no chunk, or too few to be worth the lookups), so
+// twice as many groups fit an SM; a key+length candidate, if any, is still
+// compared with direct loads.
 template <bool kProbe, bool kAhead = false, bool kVerify = true, bool kPrefixAsync = false>
 __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long long vb,
                                              uint8_t* smem) {
