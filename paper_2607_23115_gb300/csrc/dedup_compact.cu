@@ -936,6 +936,14 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
       }
     }
   }
+  if (ok && a.classes) {
+    // every read of the class table happened before the last barrier: the
+    // grid clears the call's whole table with plain 16-byte stores (a
+    // clear per chunk would first load the chunk's class entry)
+    uint4* t4 = reinterpret_cast<uint4*>(a.cls_tbl);
+    const unsigned long long n4 = (a.tbl_mask + 1) / 2;
+    for (unsigned long long e = tid; e < n4; e += nth) t4[e] = make_uint4(0u, 0u, 0u, 0u);
+  }
   if (ok) {
     unsigned long long running = before, srunning = sbefore;
     for (uint32_t t = lo; t < hi; t += kThreads) {
@@ -965,11 +973,6 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
       __syncthreads();
       const uint32_t below = (1u << lane) - 1u;
       if (valid) {
-        // every read of the class table happened before the last barrier
-        if (a.classes && !(rv & (kResHit0 | kResNoSlot)) && ch.cls[g] != 0xFFFFFFFFu) {
-          a.cls_tbl[ch.cls[g]].owner = 0u;
-          a.cls_tbl[ch.cls[g]].minv = 0u;
-        }
         const uint32_t r = (uint32_t)(running + warp_off[w] + __popc(mb & below));
         ch.rank[g] = r;
         if (miss) ch.order[r] = g;
