@@ -260,7 +260,7 @@ __global__ void __launch_bounds__(kHashThreads) k_hash_probe(HashArgs a) {
 }
 
 
-template <bool kProbe, bool kAhead, bool kVerify, bool kPrefixAsync = false>
+template <bool kProbe, bool kAhead, bool kVerify, bool kPrefixAsync = false, int kS = kStage>
 __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   pdl_trigger();
@@ -268,23 +268,54 @@ __global__ void __launch_bounds__(kStagedThreads) k_hash_probe_staged(HashArgs a
   const unsigned long long nvb = (a.Ntot * 4 + kStagedThreads - 1) / kStagedThreads;
   for (unsigned long long vb = blockIdx.x; vb < nvb; vb += gridDim.x) {
     __syncthreads();  // the previous range's groups are done with the shared memory
-    staged_range<kProbe, kAhead, kVerify, kPrefixAsync>(a, vb, smem);
+    staged_range<kProbe, kAhead, kVerify, kPrefixAsync, kS>(a, vb, smem);
   }
 }
 
-template <bool kProbe, bool kAhead, bool kVerify, bool kPrefixAsync = false>
+// Blocks of the kS-stage variant resident at once on the whole GPU (0 if
+// unknown); cached per instantiation (the machine's GPUs are all alike).
+template <bool kProbe, bool kAhead, bool kVerify, int kS>
+int staged_wave_blocks() {
+  static int wave = -1;
+  if (wave < 0) {
+    constexpr int smem = (kStagedThreads / 4) * group_bytes(kVerify, kS);
+    int dev = 0, nsm = 0, occ = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kAhead, kVerify, false, kS>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+            &occ, k_hash_probe_staged<kProbe, kAhead, kVerify, false, kS>, kStagedThreads, smem) !=
+            cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    wave = nsm * occ;
+  }
+  return wave;
+}
+
+template <bool kProbe, bool kAhead, bool kVerify, bool kPrefixAsync = false, int kS = kStage>
 cudaError_t launch_staged(const HashArgs& a, cudaStream_t s, bool pdl) {
-  if constexpr (kVerify && !kPrefixAsync) {
+  const unsigned long long threads = a.Ntot * 4;
+  const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
+  if constexpr (kS == kStage && kProbe && !kPrefixAsync) {
+    // a call whose large chunks all fit one wave of the large-stage variant,
+    // unless calls overlap (then the calls in flight share the SMs, and the
+    // variant's larger blocks would crowd them out)
+    if (a.C >= kBigStageMinChunk && !a.wait_late &&
+        (unsigned long long)sg <= (unsigned long long)staged_wave_blocks<kProbe, kAhead, kVerify, kBigStage>())
+      return launch_staged<kProbe, kAhead, kVerify, false, kBigStage>(a, s, pdl);
+  }
+  if constexpr (kVerify && !kPrefixAsync && kS == kStage) {
     if (a.C <= kPrefixAsyncMaxChunk)
       return launch_staged<kProbe, kAhead, kVerify, true>(a, s, pdl);
   }
-  constexpr int smem = (kStagedThreads / 4) * group_bytes(kVerify);
+  constexpr int smem = (kStagedThreads / 4) * group_bytes(kVerify, kS);
   // per device and cheap: set on every launch
-  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kAhead, kVerify, kPrefixAsync>,
+  cudaFuncSetAttribute((const void*)k_hash_probe_staged<kProbe, kAhead, kVerify, kPrefixAsync, kS>,
                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  const unsigned long long threads = a.Ntot * 4;
-  const unsigned sg = (unsigned)((threads + kStagedThreads - 1) / kStagedThreads);
-  return launch_kernel(k_hash_probe_staged<kProbe, kAhead, kVerify, kPrefixAsync>, dim3(sg),
+  return launch_kernel(k_hash_probe_staged<kProbe, kAhead, kVerify, kPrefixAsync, kS>, dim3(sg),
                        dim3(kStagedThreads), smem, s, pdl, a);
 }
 

@@ -146,9 +146,16 @@ constexpr int kDepth = GLEAM_STAGE_DEPTH;                   // stages in flight
 // A group's stage buffers: kDepth stages of its chunk and, when it may
 // compare against a cached copy (verify), kDepth stages of that copy too
 // (+32: bank skew).
-__host__ __device__ constexpr int group_bytes(bool verify) {
-  return kDepth * (verify ? 2 : 1) * kStage + 32;
+__host__ __device__ constexpr int group_bytes(bool verify, int stage = kStage) {
+  return kDepth * (verify ? 2 : 1) * stage + 32;
 }
+// Stage size of the variant for calls that leave most of the GPU idle (fewer
+// chunks than one wave of it holds, chunks of at least kBigStageMinChunk):
+// each stage's bookkeeping (its copies, waits and branches) then serves 64
+// XXH64 rounds of a lane instead of 16, which is what a chunk's dependent
+// chain waits on when nothing else shares the SM.
+constexpr int kBigStage = 2048;
+constexpr unsigned long long kBigStageMinChunk = 32768;
 constexpr int kGroupBytes = group_bytes(true);
 constexpr int kStagedThreads = GLEAM_STAGED_THREADS;
 constexpr int kStagedSmem = (kStagedThreads / 4) * kGroupBytes;
@@ -176,12 +183,13 @@ __device__ __forceinline__ void cp_wait_upto(uint32_t n) {
   }
 }
 
-// This lane's share (4 lanes x 8 x 16 bytes) of one stage of `src` into `dst`;
-// `bytes` (multiple of 32, <= kStage) of the stage exist.
+// This lane's share (4 lanes x kS / 64 x 16 bytes) of one stage of kS bytes
+// of `src` into `dst`; `bytes` (multiple of 32, <= kS) of the stage exist.
+template <int kS = kStage>
 __device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uint32_t bytes,
                                            uint32_t lane) {
 #pragma unroll
-  for (int j = 0; j < kStage / 64; ++j) {
+  for (int j = 0; j < kS / 64; ++j) {
     const uint32_t off = (uint32_t)j * 64 + lane * 16;
     if (off < bytes) cp_async16(dst + off, src + off);
   }
@@ -194,9 +202,11 @@ __device__ __forceinline__ void stage_copy(uint32_t dst, const uint8_t* src, uin
 // (for a cache that holds no chunk, or too few to be worth the lookups), so
 // twice as many groups fit an SM; a key+length candidate, if any, is still
 // compared with direct loads.
-template <bool kProbe, bool kAhead = false, bool kVerify = true, bool kPrefixAsync = false>
+template <bool kProbe, bool kAhead = false, bool kVerify = true, bool kPrefixAsync = false,
+          int kS = kStage>
 __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long long vb,
                                              uint8_t* smem) {
+  static_assert(kS % kPrefixBytes == 0 && kS % 256 == 0, "stages hold whole prefixes and batches");
   const unsigned long long g = (vb * blockDim.x + threadIdx.x) >> 2;
   // the payload search borrows the start of the stage buffers (no static
   // shared memory: any would cost this kernel a fifth of its bandwidth)
@@ -208,10 +218,10 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   const uint32_t lane = threadIdx.x & 3;
   const int gbase = threadIdx.x & 28;
   const unsigned gmask = 0xFu << gbase;
-  uint8_t* region = smem + (threadIdx.x >> 2) * group_bytes(kVerify);
+  uint8_t* region = smem + (threadIdx.x >> 2) * group_bytes(kVerify, kS);
   const uint32_t sbase = (uint32_t)__cvta_generic_to_shared(region);
-  // stage buffer t % kDepth: payload at [0, kStage), cached copy at [kStage, 2 kStage)
-  constexpr uint32_t kBuf = (kVerify ? 2 : 1) * kStage;  // one stage's buffers
+  // stage buffer t % kDepth: payload at [0, kS), cached copy at [kS, 2 kS)
+  constexpr uint32_t kBuf = (kVerify ? 2 : 1) * kS;  // one stage's buffers
   auto pay_s = [&](uint32_t t) { return sbase + (t % kDepth) * kBuf; };
   auto pay_p = [&](uint32_t t) { return region + (t % kDepth) * kBuf; };
 
@@ -233,8 +243,8 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   const uint8_t* p = buf + start;
   const uint32_t ns = len >> 5;
   const uint32_t full = ns * 32;                       // bytes in whole stripes
-  const uint32_t nst = (full + kStage - 1) / kStage;   // stages
-  auto sbytes = [&](uint32_t t) { return min((uint32_t)kStage, full - t * kStage); };
+  const uint32_t nst = (full + kS - 1) / kS;   // stages
+  auto sbytes = [&](uint32_t t) { return min((uint32_t)kS, full - t * kS); };
 
   const bool speculate = kProbe && len >= kPrefixBytes;
   // slots in use as the hint lookups see them; with a late wait (calls that
@@ -255,18 +265,20 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
   uint8_t* ahead_ar = nullptr;  // arena slot slots_used + g
 
   unsigned long long acc = xlane_start(lane);
+  // the accumulator after the prefix (stage 0 may hold more than the prefix)
+  unsigned long long acc_pre = 0;
   // prologue: payload stages 0 .. kDepth-2
 #pragma unroll
   for (int t = 0; t < kDepth - 1; ++t) {
-    if ((uint32_t)t < nst) stage_copy(pay_s(t), p + t * kStage, sbytes(t), lane);
+    if ((uint32_t)t < nst) stage_copy<kS>(pay_s(t), p + t * kS, sbytes(t), lane);
     cp_commit();
   }
   for (uint32_t t = 0; t < nst; ++t) {
     // issue stage t + kDepth - 1 into the buffer consumed at t - 1
     const uint32_t tn = t + kDepth - 1;
     if (tn < nst) {
-      stage_copy(pay_s(tn), p + (unsigned long long)tn * kStage, sbytes(tn), lane);
-      if (cmp) stage_copy(pay_s(tn) + kStage, q + (unsigned long long)tn * kStage, sbytes(tn), lane);
+      stage_copy<kS>(pay_s(tn), p + (unsigned long long)tn * kS, sbytes(tn), lane);
+      if (cmp) stage_copy<kS>(pay_s(tn) + kS, q + (unsigned long long)tn * kS, sbytes(tn), lane);
     }
     cp_commit();
     // groups committed so far, oldest first: prologue stages, then one per
@@ -282,23 +294,24 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
     auto word = [&](const uint8_t* b, uint32_t s) {
       return *reinterpret_cast<const unsigned long long*>(b + s * 32 + lane * 8);
     };
-    if (sst == (uint32_t)kStage / 32) {
+    if (sst == (uint32_t)kS / 32) {
       // a whole stage, eight stripes at a time: the loads and the compare
       // overlap the XXH64 chain instead of waiting in it
 #pragma unroll
-      for (uint32_t h = 0; h < (uint32_t)kStage / 32; h += 8) {
+      for (uint32_t h = 0; h < (uint32_t)kS / 32; h += 8) {
         unsigned long long w[8];
 #pragma unroll
         for (uint32_t u = 0; u < 8; ++u) w[u] = word(sp, h + u);
         if (cmp && t > 0) {
 #pragma unroll
-          for (uint32_t u = 0; u < 8; ++u) d |= w[u] ^ word(sp + kStage, h + u);
+          for (uint32_t u = 0; u < 8; ++u) d |= w[u] ^ word(sp + kS, h + u);
         }
 #pragma unroll
         for (uint32_t u = 0; u < 8; ++u) acc = xstep(acc, w[u]);
+        if (kS > (int)kPrefixBytes && h + 8 == kPrefixBytes / 32) acc_pre = acc;
       }
     } else if (cmp && t > 0) {
-      const uint8_t* sq = sp + kStage;
+      const uint8_t* sq = sp + kS;
 #pragma unroll 4
       for (uint32_t s = 0; s < sst; ++s) {
         const unsigned long long w = *reinterpret_cast<const unsigned long long*>(sp + s * 32 + lane * 8);
@@ -308,14 +321,17 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
       }
     } else {
 #pragma unroll 4
-      for (uint32_t s = 0; s < sst; ++s)
+      for (uint32_t s = 0; s < sst; ++s) {
         acc = xstep(acc, *reinterpret_cast<const unsigned long long*>(sp + s * 32 + lane * 8));
+        if (kS > (int)kPrefixBytes && s + 1 == kPrefixBytes / 32) acc_pre = acc;
+      }
     }
+    if (kS == (int)kPrefixBytes) acc_pre = acc;
     if (t == 0 && speculate) {
-      const unsigned long long b0 = group_shfl(acc, gmask, gbase + 0);
-      const unsigned long long b1 = group_shfl(acc, gmask, gbase + 1);
-      const unsigned long long b2 = group_shfl(acc, gmask, gbase + 2);
-      const unsigned long long b3 = group_shfl(acc, gmask, gbase + 3);
+      const unsigned long long b0 = group_shfl(acc_pre, gmask, gbase + 0);
+      const unsigned long long b1 = group_shfl(acc_pre, gmask, gbase + 1);
+      const unsigned long long b2 = group_shfl(acc_pre, gmask, gbase + 2);
+      const unsigned long long b3 = group_shfl(acc_pre, gmask, gbase + 3);
       hint = b0 ^ xrotl(b1, 16) ^ xrotl(b2, 32) ^ xrotl(b3, 48);
       // an empty cache has no hints to look up
       hint_slot = kVerify && slots_used ? hint_lookup(a.hints, a.index_mask, hint, len, slots_used)
@@ -334,18 +350,19 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
           // the cached copy's prefix into the free half of stage buffer 0, in
           // a group of its own, and its next stages behind it: one round trip
           // for both
-          stage_copy(pay_s(0) + kStage, q, (uint32_t)kStage, lane);
+          stage_copy<kS>(pay_s(0) + kS, q, kS == (int)kPrefixBytes ? (uint32_t)kS : sbytes(0), lane);
           cp_commit();
         } else {
-          // the prefix, still in stage buffer 0, against the cached copy's prefix
+          // stage 0 (the prefix, and more in a larger stage), still in its
+          // buffer, against the cached copy's
 #pragma unroll 4
-          for (uint32_t s = 0; s < (uint32_t)kStage / 32; ++s)
+          for (uint32_t s = 0; s < (kS == (int)kPrefixBytes ? (uint32_t)kS / 32 : sst); ++s)
             d |= *reinterpret_cast<const unsigned long long*>(sp + s * 32 + lane * 8) ^
                  load_arena_word(q + s * 32 + lane * 8);
         }
         // the cached copy of the stages already in flight
         for (uint32_t tt = 1; tt < (uint32_t)kDepth && tt < nst; ++tt)
-          stage_copy(pay_s(tt) + kStage, q + (unsigned long long)tt * kStage, sbytes(tt), lane);
+          stage_copy<kS>(pay_s(tt) + kS, q + (unsigned long long)tt * kS, sbytes(tt), lane);
       }
     }
     if (t == 0) cp_commit();  // the late group (empty without a hint)
@@ -353,9 +370,13 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
       // the prefix's group is complete once at most the late group pends
       cp_wait<1>();
       __syncwarp(gmask);
+      if constexpr (kS == (int)kPrefixBytes) {
 #pragma unroll
-      for (uint32_t s = 0; s < (uint32_t)kStage / 32; ++s)
-        d |= word(sp, s) ^ word(sp + kStage, s);
+        for (uint32_t s = 0; s < (uint32_t)kS / 32; ++s) d |= word(sp, s) ^ word(sp + kS, s);
+      } else {
+#pragma unroll 4
+        for (uint32_t s = 0; s < sst; ++s) d |= word(sp, s) ^ word(sp + kS, s);
+      }
     }
     if (cmp) {
       // a lane that found a difference stops streaming its share of the
@@ -367,11 +388,11 @@ __device__ __forceinline__ void staged_range(const HashArgs& a, unsigned long lo
     if (ahead) {  // this lane's own pieces of stage t, to both destinations
       const uint32_t sb = sbytes(t);
 #pragma unroll
-      for (int j = 0; j < kStage / 64; ++j) {
+      for (int j = 0; j < kS / 64; ++j) {
         const uint32_t off = (uint32_t)j * 64 + lane * 16;
         if (off < sb) {
           const uint4 v = *reinterpret_cast<const uint4*>(sp + off);
-          const unsigned long long o = (unsigned long long)t * kStage + off;
+          const unsigned long long o = (unsigned long long)t * kS + off;
           __stcs(reinterpret_cast<uint4*>(ahead_pk + o), v);
           __stcs(reinterpret_cast<uint4*>(ahead_ar + o), v);
         }
