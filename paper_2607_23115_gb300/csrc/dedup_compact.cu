@@ -1461,6 +1461,22 @@ __device__ __forceinline__ void count_not_hit(const uint8_t* status, uint32_t N,
   *all = t;
 }
 
+// The general algorithm on the one-launch kernel's grid, for a call with a
+// shared group: post the group minima, then the rounds, ranks and copies of
+// k_dedup and k_pack.  Out of line, so that the common path's code stays
+// compact (the kernel runs once per call, on SMs whose instruction caches are
+// cold).  Every thread of every block calls it; post_e: the entry to post
+// this thread's chunk number to, or 0xFFFFFFFF.
+__device__ __noinline__ void resolve_pack_general(const DedupArgs& a, uint32_t G, uint32_t bid,
+                                                  uint8_t* smem, bool ok, uint32_t post_e,
+                                                  uint32_t g) {
+  if (ok) post_minimum(a, post_e, g);  // one chunk per thread at most
+  ok = grid_barrier(a.ctl, G, a.wait_ns, false);
+  resolve_rank(a, G, bid, true, ok);
+  grid_barrier(a.ctl, G, a.wait_ns, false);
+  pack_publish(a, G, bid, smem);
+}
+
 __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G, uint32_t bid,
                                                   uint8_t* smem) {
   __shared__ unsigned long long red64[kWarps];
@@ -1577,16 +1593,8 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
         ch.ent[g] = e;
       }
     }
-    // the general algorithm: post the group minima, then the rounds, ranks
-    // and copies of k_dedup and k_pack on this grid
-    if (ok) {  // every lane of the block takes part (one chunk per thread at most)
-      const bool post = valid && e != 0xFFFFFFFFu && st != kHit0 && st != kUncached;
-      post_minimum(a, post ? e : 0xFFFFFFFFu, g);
-    }
-    ok = grid_barrier(a.ctl, G, a.wait_ns, false);
-    resolve_rank(a, G, bid, true, ok);
-    grid_barrier(a.ctl, G, a.wait_ns, false);
-    pack_publish(a, G, bid, smem);
+    const bool post = valid && e != 0xFFFFFFFFu && st != kHit0 && st != kUncached;
+    resolve_pack_general(a, G, bid, smem, ok, post ? e : 0xFFFFFFFFu, g);
     return;
   }
 
