@@ -1876,6 +1876,15 @@ constexpr uint32_t kSmallHashSmem = kSmallGroups * (uint32_t)kGroupBytes;
 constexpr uint32_t kSmallSmem = kSmallHashSmem > kPackSmem ? kSmallHashSmem : kPackSmem;
 
 
+// k_dedup's and k_pack's steps on a grid of one block (several payloads, LRU,
+// a class table, or more chunks than threads): out of line, so that the small
+// kernel's common path stays compact.
+__device__ __noinline__ void small_call_general(const DedupArgs& a, uint8_t* smem) {
+  resolve_rank(a, 1, 0);
+  __syncthreads();
+  pack_publish(a, 1, 0, smem);
+}
+
 template <bool kAhead, bool kPrefixAsync>
 __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a) {
   extern __shared__ __align__(128) uint8_t small_smem[];
@@ -1903,9 +1912,7 @@ __global__ void __launch_bounds__(kThreads) k_small_call(HashArgs h, DedupArgs a
     // scan (no LRU: they stamp no last use)
     resolve_pack_fast(a, 1, 0, small_smem);
   } else {
-    resolve_rank(a, 1, 0);
-    __syncthreads();
-    pack_publish(a, 1, 0, small_smem);
+    small_call_general(a, small_smem);
   }
 }
 
