@@ -1006,6 +1006,25 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
 // vbytes: the call's misses, stored misses, evicted slots and their bytes;
 // s_sum: a grid of one block's sums (hits, intra hits, rejects, miss bytes,
 // stored bytes, chunks written ahead, of them used), else the control block's.
+// After an error that may have stopped the leaders before they cleared their
+// entries: the whole group table (and class table), and an eviction's
+// histogram and flags.  Out of line: rare, and kept out of the code that
+// every call runs.
+__device__ __noinline__ void clear_after_error(const DedupArgs& a) {
+  for (unsigned long long e = threadIdx.x; e <= a.tbl_mask; e += kThreads) {
+    a.tbl[e].owner = 0u;
+    a.tbl[e].minv = 0u;
+    if (a.classes) {
+      a.cls_tbl[e].owner = 0u;
+      a.cls_tbl[e].minv = 0u;
+    }
+  }
+  if (a.lru) {  // an eviction that stopped half-way may have left these set
+    for (uint32_t j = threadIdx.x; j < kLruBins; j += kThreads) a.bins[j] = 0u;
+    for (unsigned long long j = threadIdx.x; j < a.nslots; j += kThreads) a.vflag[j] = 0;
+  }
+}
+
 __device__ __forceinline__ void finish_call(const DedupArgs& a, uint32_t G,
                                             unsigned long long slots0,
                                             unsigned long long total,
@@ -1089,20 +1108,7 @@ __device__ __forceinline__ void finish_call(const DedupArgs& a, uint32_t G,
   // Leave the per-call state as the next call expects it: the group table
   // (cleared entry by entry by the leaders, or here in full after an error
   // that may have stopped them) and the control block.
-  if (err) {
-    for (unsigned long long e = threadIdx.x; e <= a.tbl_mask; e += kThreads) {
-      a.tbl[e].owner = 0u;
-      a.tbl[e].minv = 0u;
-      if (a.classes) {
-        a.cls_tbl[e].owner = 0u;
-        a.cls_tbl[e].minv = 0u;
-      }
-    }
-    if (a.lru) {  // an eviction that stopped half-way may have left these set
-      for (uint32_t j = threadIdx.x; j < kLruBins; j += kThreads) a.bins[j] = 0u;
-      for (unsigned long long j = threadIdx.x; j < a.nslots; j += kThreads) a.vflag[j] = 0;
-    }
-  }
+  if (err) clear_after_error(a);
   __syncthreads();
   if (threadIdx.x == 0) {
     DevCtl* c = a.ctl;
@@ -1462,15 +1468,32 @@ __device__ __forceinline__ void count_not_hit(const uint8_t* status, uint32_t N,
 }
 
 // The general algorithm on the one-launch kernel's grid, for a call with a
-// shared group: post the group minima, then the rounds, ranks and copies of
-// k_dedup and k_pack.  Out of line, so that the common path's code stays
-// compact (the kernel runs once per call, on SMs whose instruction caches are
-// cold).  Every thread of every block calls it; post_e: the entry to post
-// this thread's chunk number to, or 0xFFFFFFFF.
+// shared group: if the hash kernel claimed the groups (pre), their entries are
+// cleared and claimed again by the whole group key and length (a shared tag
+// may be two different pairs'); then the group minima are posted, and the
+// rounds, ranks and copies of k_dedup and k_pack run.  Out of line, so that
+// the common path's code stays compact (the kernel runs once per call, on SMs
+// whose instruction caches are cold).  Every thread of every block calls it;
+// mine: this thread holds a chunk of a group (entry e, group key and length).
 __device__ __noinline__ void resolve_pack_general(const DedupArgs& a, uint32_t G, uint32_t bid,
-                                                  uint8_t* smem, bool ok, uint32_t post_e,
-                                                  uint32_t g) {
-  if (ok) post_minimum(a, post_e, g);  // one chunk per thread at most
+                                                  uint8_t* smem, bool ok, bool pre, bool mine,
+                                                  uint32_t e, unsigned long long key,
+                                                  uint32_t len, uint32_t g) {
+  if (pre) {
+    if (mine && e != 0xFFFFFFFFu)
+      *reinterpret_cast<volatile unsigned long long*>(&a.tbl[e]) = 0ull;
+    ok = grid_barrier(a.ctl, G, a.wait_ns, false) && ok;
+    if (ok && mine) {
+      bool claimed = true;
+      e = group_entry(a, g, key, len, &claimed, true);
+      if (e == 0xFFFFFFFFu) {
+        atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+        a.ch.res[g] = kResLeader | 1u;
+      }
+      a.ch.ent[g] = e;
+    }
+  }
+  if (ok) post_minimum(a, mine && e != 0xFFFFFFFFu ? e : 0xFFFFFFFFu, g);  // one chunk per thread
   ok = grid_barrier(a.ctl, G, a.wait_ns, false);
   resolve_rank(a, G, bid, true, ok);
   grid_barrier(a.ctl, G, a.wait_ns, false);
@@ -1576,25 +1599,8 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
   }
 
   if (s_shared) {
-    if (pre) {
-      // a chunk found an entry with its tag: the groups are claimed again,
-      // by the whole group key and length, in the cleared table
-      const bool mine = valid && st != kHit0 && st != kUncached;
-      if (mine && e != 0xFFFFFFFFu)
-        *reinterpret_cast<volatile unsigned long long*>(&a.tbl[e]) = 0ull;
-      ok = grid_barrier(a.ctl, G, a.wait_ns, false) && ok;
-      if (ok && mine) {
-        bool claimed = true;
-        e = group_entry(a, g, key, len, &claimed, true);
-        if (e == 0xFFFFFFFFu) {
-          atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-          ch.res[g] = kResLeader | 1u;
-        }
-        ch.ent[g] = e;
-      }
-    }
-    const bool post = valid && e != 0xFFFFFFFFu && st != kHit0 && st != kUncached;
-    resolve_pack_general(a, G, bid, smem, ok, post ? e : 0xFFFFFFFFu, g);
+    resolve_pack_general(a, G, bid, smem, ok, pre, valid && st != kHit0 && st != kUncached, e,
+                         key, len, g);
     return;
   }
 
