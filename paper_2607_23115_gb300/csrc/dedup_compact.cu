@@ -112,8 +112,10 @@ __device__ bool warp_equal(const uint8_t* x, const uint8_t* y, uint32_t len, boo
 }
 
 // Whole-warp copy of one chunk to the packed output and to its arena slot
-// (d2 == nullptr: to the packed output only).
-__device__ void warp_copy2(uint8_t* d1, uint8_t* d2, const uint8_t* s, uint32_t len, bool vec) {
+// (d2 == nullptr: to the packed output only).  The path of copies that cannot
+// be bulk copies (host or managed memory, unaligned addresses): out of line,
+// away from the code that every call runs.
+__device__ __noinline__ void warp_copy2(uint8_t* d1, uint8_t* d2, const uint8_t* s, uint32_t len, bool vec) {
   const uint32_t lane = threadIdx.x & 31;
   uint32_t done = 0;
   if (vec) {
