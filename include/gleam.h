@@ -264,7 +264,7 @@ int gleam_dedup_copy_host_batch(gleam_cache_t* cache, const gleam_payload_t* pay
  * memory map it keeps for the application.
  *
  * Same operation, outputs and cache update as gleam_dedup_copy_async, but the
- * per-call workspace is one fixed array of about 5.9 MiB in the library's
+ * per-call workspace is one fixed array of about 7.2 MiB in the library's
  * device image instead of memory allocated by the cache; the call itself only
  * enqueues memsets and kernels and allocates nothing.  Every GPU that loads
  * the library holds that array until the process exits.

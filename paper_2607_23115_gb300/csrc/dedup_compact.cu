@@ -302,10 +302,57 @@ __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
+// The rest of an insert's linear probe in KEY16 mode, from `pos` (the probe's
+// `probe`-th position): all chunks of one 16-bit key share a home position,
+// so an insert walks the cluster of the key's earlier entries.  The slot words
+// of the next kScanEntries entries are read at once and the first that was
+// free is claimed: one round trip per kScanEntries entries instead of one per
+// entry.  While a call inserts, entries only go from free to used (evictions
+// finish before), so an entry read as used stays used and is passed over
+// safely; a claim that loses the race moves on to the next entry.  (With full
+// 64-bit keys the entry after a used home is mostly free, and claiming it
+// directly is one round trip fewer.)  False if the table is full.
+constexpr uint32_t kScanEntries = 8;
+__device__ __noinline__ bool index_insert_scan(IndexEntry* index, uint64_t mask,
+                                               unsigned long long key, uint32_t slot,
+                                               uint32_t len, uint64_t pos, uint64_t probe) {
+  while (probe <= mask) {
+    uint32_t free_bits = 0;
+#pragma unroll
+    for (uint32_t k = 0; k < kScanEntries; ++k)
+      free_bits |= (ldcg_u32(&index[(pos + k) & mask].slot) == kEmptySlot ? 1u : 0u) << k;
+    if (free_bits == 0) {
+      pos = (pos + kScanEntries) & mask;
+      probe += kScanEntries;
+      continue;
+    }
+    const uint32_t k = __ffs(free_bits) - 1;
+    probe += k;
+    if (probe > mask) break;
+    pos = (pos + k) & mask;
+    if (atomicCAS(&index[pos].slot, kEmptySlot, slot) == kEmptySlot) {
+      index[pos].key = key;
+      index[pos].len = len;
+      return true;
+    }
+    pos = (pos + 1) & mask;
+    ++probe;
+  }
+  return false;
+}
+
 // Claims a free index entry for (key, slot, len); false if the table is full.
+// scan: the rest of the probe by index_insert_scan (KEY16 index keys).
+// place: the probe starts that many entries after the key's home position.
+// With KEY16 classes the misses of a call that share an index key (and
+// length) have the places 0 .. n-1, so each starts at its own entry instead
+// of walking past the others; an entry stays reachable from the home
+// position: a free entry left between the home position and a miss's entry
+// (at place q) would have been taken by the miss whose place is q.
 __device__ bool index_insert(IndexEntry* index, uint64_t mask, unsigned long long key,
-                             uint32_t slot, uint32_t len) {
-  uint64_t pos = mix64(key) & mask;
+                             uint32_t slot, uint32_t len, bool scan = false,
+                             uint32_t place = 0) {
+  uint64_t pos = (mix64(key) + place) & mask;
   for (uint64_t probe = 0; probe <= mask; ++probe) {
     const uint32_t old = atomicCAS(&index[pos].slot, kEmptySlot, slot);
     if (old == kEmptySlot) {
@@ -314,6 +361,7 @@ __device__ bool index_insert(IndexEntry* index, uint64_t mask, unsigned long lon
       return true;
     }
     pos = (pos + 1) & mask;
+    if (scan) return index_insert_scan(index, mask, key, slot, len, pos, probe + 1);
   }
   return false;
 }
@@ -332,7 +380,7 @@ __device__ __forceinline__ PendingInsert index_insert_begin(IndexEntry* index, u
   return PendingInsert{pos, atomicCAS(&index[pos].slot, kEmptySlot, slot)};
 }
 __device__ bool index_insert_end(IndexEntry* index, uint64_t mask, unsigned long long key,
-                                 uint32_t slot, uint32_t len, PendingInsert p) {
+                                 uint32_t slot, uint32_t len, PendingInsert p, bool scan = false) {
   uint64_t pos = p.pos;
   uint32_t old = p.old;
   for (uint64_t probe = 0;;) {
@@ -343,6 +391,7 @@ __device__ bool index_insert_end(IndexEntry* index, uint64_t mask, unsigned long
     }
     if (++probe > mask) return false;
     pos = (pos + 1) & mask;
+    if (scan) return index_insert_scan(index, mask, key, slot, len, pos, probe);
     old = atomicCAS(&index[pos].slot, kEmptySlot, slot);
   }
 }
@@ -641,14 +690,33 @@ __device__ bool lru_evict(const DedupArgs& a, uint32_t G, uint32_t bid,
 
 // Posts ~g as a candidate minimum of group entry `e` (0xFFFFFFFF: none), one
 // atomic per group of lanes that share the entry.  Called by the whole warp.
-__device__ __forceinline__ void post_minimum(CallEntry* tbl, uint32_t e, uint32_t g) {
-  const unsigned peers = __match_any_sync(0xffffffffu, e);
+template <typename Entry>
+__device__ __forceinline__ void post_minimum(Entry* tbl, uint32_t e, uint32_t g,
+                                             unsigned peers) {
   const uint32_t m = __reduce_max_sync(peers, e != 0xFFFFFFFFu ? ~g : 0u);
   // a group of many chunks (all-zero chunks, say) would queue its atomics on
   // one address: skip the atomic when a smaller number is already posted
   if (e != 0xFFFFFFFFu && (threadIdx.x & 31) == (uint32_t)(__ffs(peers) - 1) &&
       ldcg_u32(&tbl[e].minv) < m)
     atomicMax(&tbl[e].minv, m);
+}
+__device__ __forceinline__ void post_minimum(CallEntry* tbl, uint32_t e, uint32_t g) {
+  post_minimum(tbl, e, g, __match_any_sync(0xffffffffu, e));
+}
+
+// KEY16 classes: posts ~g as a candidate minimum of class entry `e`
+// (0xFFFFFFFF: none) and returns the lane's place among the misses of the
+// class (counted in the entry), one atomic of each kind per group of lanes
+// that share the entry.  Called by the whole warp.
+__device__ __forceinline__ uint32_t post_class(ClassEntry* tbl, uint32_t e, uint32_t g) {
+  const uint32_t lane = threadIdx.x & 31;
+  const unsigned peers = __match_any_sync(0xffffffffu, e);
+  post_minimum(tbl, e, g, peers);
+  const int first = __ffs(peers) - 1;
+  uint32_t base = 0;
+  if (e != 0xFFFFFFFFu && lane == (uint32_t)first)
+    base = atomicAdd(&tbl[e].count, (uint32_t)__popc(peers));
+  return __shfl_sync(0xffffffffu, base, first) + __popc(peers & ((1u << lane) - 1u));
 }
 __device__ __forceinline__ void post_minimum(const DedupArgs& a, uint32_t e, uint32_t g) {
   post_minimum(a.tbl, e, g);
@@ -697,8 +765,7 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
     // minimum with one atomic (all-zero chunks, say, share a group)
     for (uint32_t base = tid - lane; base < N; base += nth) {
       const uint32_t g = base + lane;
-      uint32_t post = 0xFFFFFFFFu;   // group entry that gets this chunk's number
-      uint32_t cpost = 0xFFFFFFFFu;  // class entry that gets it (KEY16)
+      uint32_t post = 0xFFFFFFFFu;  // group entry that gets this chunk's number
       if (g < N) {
         // every operand at once: the claim below then waits for none of them
         const uint8_t st = ch.status[g];
@@ -728,15 +795,9 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
             ch.res[g] = kResUnresolved;
             post = e;
           }
-          if (a.classes) {
-            cpost = class_entry(a, g, key & 0xFFFFull, len);
-            if (cpost == 0xFFFFFFFFu) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
-            ch.cls[g] = cpost;
-          }
         }
       }
       post_minimum(a, post, g);
-      if (a.classes) post_minimum(a.cls_tbl, cpost, g);
     }
     if (a.lru) {
       distinct = block_sum<unsigned long long>(distinct, red64);
@@ -757,15 +818,17 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
     while (W > 1 && (unsigned long long)N < (unsigned long long)nwarps * W) W >>= 1;
     for (uint32_t base = (tid / 32) * W; base < N; base += nwarps * W) {
       const uint32_t g = base + lane;
-      bool need = false;
+      bool need = false, lead = false;
       uint32_t m = 0;
       if (lane < W && g < N && ldcg_u32(&ch.res[g]) == kResUnresolved) {
         m = ~ldcg_u32(&a.tbl[ch.ent[g]].minv);
         if (m == g) {
           ch.res[g] = kResLeader | round;
+          lead = true;
         } else if (m > g) {  // the group minimum can only be below g: table damaged
           atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
           ch.res[g] = kResLeader | round;
+          lead = true;
         } else if (ch.hint[g] != ch.hint[m]) {
           // different first 512 bytes (the prefix hints differ), so different
           // chunks: no byte compare, the chunk waits for a later round
@@ -774,6 +837,22 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
         } else {
           need = true;
         }
+      }
+      if (a.classes) {
+        // KEY16: a new leader (a miss) claims the class of its 16-bit index
+        // key and length, posts its number there and takes its place among
+        // the class's misses (where its index insert starts); after the last
+        // round a class minimum below a leader's number is an earlier miss of
+        // its index key and length (a reject).  Groups are whole fingerprints, so
+        // nearly all leaders are found in round 1, while the other warps
+        // compare their duplicates.
+        uint32_t cpost = 0xFFFFFFFFu;
+        if (lead) {
+          cpost = class_entry(a, g, ch.key[g] & 0xFFFFull, ch.len[g]);
+          if (cpost == 0xFFFFFFFFu) atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
+        }
+        const uint32_t place = post_class(a.cls_tbl, cpost, g);
+        if (lead) ch.cls[g] = cpost | ((unsigned long long)place << 32);
       }
       uint32_t todo = __ballot_sync(0xffffffffu, need);
       // every lane fetches its own chunk's operands at once, so that each
@@ -880,11 +959,15 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
         if (!(r & kResNoSlot)) ++scnt;
         // a verify reject: the cache had a key+length candidate, or an
         // earlier miss of the call has this key and length (another leader
-        // of a later round; with classes, any earlier chunk of the class)
-        const bool rej =
-            !(r & kResNoSlot) &&
-            (ch.status[g] == kMissCand ||
-             (a.classes ? ~ldcg_u32(&a.cls_tbl[ch.cls[g]].minv) < g : (r & kResRoundMask) > 1));
+        // of a later round; with classes, an earlier leader of the class)
+        bool earlier;
+        if (a.classes) {
+          const uint32_t cl = (uint32_t)ch.cls[g];  // in range unless the call failed
+          earlier = cl <= a.tbl_mask && ~ldcg_u32(&a.cls_tbl[cl].minv) < g;
+        } else {
+          earlier = (r & kResRoundMask) > 1;
+        }
+        const bool rej = !(r & kResNoSlot) && (ch.status[g] == kMissCand || earlier);
         if (rej) ch.res[g] = r | kResReject;
         // leave the group table zeroed for the next call: every claimed entry
         // belongs to a group with at least one leader
@@ -943,7 +1026,7 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
     // grid clears the call's whole table with plain 16-byte stores (a
     // clear per chunk would first load the chunk's class entry)
     uint4* t4 = reinterpret_cast<uint4*>(a.cls_tbl);
-    const unsigned long long n4 = (a.tbl_mask + 1) / 2;
+    const unsigned long long n4 = a.tbl_mask + 1;  // one 16-byte store per entry
     for (unsigned long long e = tid; e < n4; e += nth) t4[e] = make_uint4(0u, 0u, 0u, 0u);
   }
   if (ok) {
@@ -1016,10 +1099,7 @@ __device__ __noinline__ void clear_after_error(const DedupArgs& a) {
   for (unsigned long long e = threadIdx.x; e <= a.tbl_mask; e += kThreads) {
     a.tbl[e].owner = 0u;
     a.tbl[e].minv = 0u;
-    if (a.classes) {
-      a.cls_tbl[e].owner = 0u;
-      a.cls_tbl[e].minv = 0u;
-    }
+    if (a.classes) a.cls_tbl[e] = ClassEntry{0u, 0u, 0u, 0u};
   }
   if (a.lru) {  // an eviction that stopped half-way may have left these set
     for (uint32_t j = threadIdx.x; j < kLruBins; j += kThreads) a.bins[j] = 0u;
@@ -1379,7 +1459,8 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
       a.slot_len[slot] = ln;
       a.slot_key[slot] = ch.key[gg];
       if (a.lru) a.last_use[slot] = a.epoch;
-      if (!index_insert(a.index, a.index_mask, index_key(a, ch.key[gg]), (uint32_t)slot, ln))
+      if (!index_insert(a.index, a.index_mask, index_key(a, ch.key[gg]), (uint32_t)slot, ln,
+                        a.key16, a.classes ? (uint32_t)(ch.cls[gg] >> 32) : 0u))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       if (!a.paper && ln >= kPrefixBytes &&
           !index_insert(a.hints, a.index_mask, ch.hint[gg], (uint32_t)slot, ln))
@@ -1805,7 +1886,8 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
     // each stored miss completes its inserts and frees the group entry it
     // claimed, while the last pieces' stores are still in flight
     if (ins) {
-      if (!index_insert_end(a.index, a.index_mask, index_key(a, key), (uint32_t)ins_slot, len, pi))
+      if (!index_insert_end(a.index, a.index_mask, index_key(a, key), (uint32_t)ins_slot, len, pi,
+                            a.key16))
         atomicCAS(&a.ctl->err, 0, (int)GLEAM_ERR_INTERNAL);
       if (ins_hint &&
           !index_insert_end(a.hints, a.index_mask, hint, (uint32_t)ins_slot, len, ph))

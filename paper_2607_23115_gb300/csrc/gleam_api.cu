@@ -46,7 +46,7 @@ struct gleam_cache {
   void* ws = nullptr;
   ChunkArrays ch{};
   CallEntry* tbl = nullptr;
-  CallEntry* cls_tbl = nullptr;  // KEY16: (16-bit key, length) classes, tbl_cap entries
+  ClassEntry* cls_tbl = nullptr;  // KEY16: (16-bit key, length) classes, tbl_cap entries
   uint64_t tbl_cap = 0;
 
   // payload tables of multi-payload calls
@@ -267,7 +267,7 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
                            align256(cap * 4), align256(cap * 4), align256(cap * 8),
                            align256(cap * 4), align256(cap * 4), align256(cap * 4),
                            align256(cap),     align256(tcap * sizeof(CallEntry)),
-                           align256(cap * 4), align256(tcap * sizeof(CallEntry))};
+                           align256(cap * 8), align256(tcap * sizeof(ClassEntry))};
   uint64_t total = 0;
   for (uint64_t x : sz) total += x;
   int rc = cuda_err(cudaEventSynchronize(c->done));
@@ -309,9 +309,9 @@ int ensure_ws(gleam_cache* c, uint64_t nchunks) {
   b += sz[12];
   c->tbl = reinterpret_cast<CallEntry*>(b);
   b += sz[13];
-  c->ch.cls = reinterpret_cast<uint32_t*>(b);
+  c->ch.cls = reinterpret_cast<unsigned long long*>(b);
   b += sz[14];
-  c->cls_tbl = reinterpret_cast<CallEntry*>(b);
+  c->cls_tbl = reinterpret_cast<ClassEntry*>(b);
   c->tbl_cap = tcap;
   c->ws_chunks = cap;
   return GLEAM_OK;
@@ -1371,11 +1371,11 @@ constexpr uint64_t kNaOffOld = kNaOffSrank + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffSpec = kNaOffOld + na_align(kNaChunks * 4);
 constexpr uint64_t kNaOffTbl = kNaOffSpec + na_align(kNaChunks);
 constexpr uint64_t kNaOffCls = kNaOffTbl + na_align(kNaTable * sizeof(CallEntry));
-constexpr uint64_t kNaOffClsTbl = kNaOffCls + na_align(kNaChunks * 4);
-constexpr uint64_t kNaOffCtl = kNaOffClsTbl + na_align(kNaTable * sizeof(CallEntry));
+constexpr uint64_t kNaOffClsTbl = kNaOffCls + na_align(kNaChunks * 8);
+constexpr uint64_t kNaOffCtl = kNaOffClsTbl + na_align(kNaTable * sizeof(ClassEntry));
 constexpr uint64_t kNaOffBcount = kNaOffCtl + na_align(sizeof(DevCtl));
 constexpr uint64_t kNaOffResult = kNaOffBcount + na_align((2 * kNaBlocks + 1) * 4);
-constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~5.9 MiB
+constexpr uint64_t kNaBytes = kNaOffResult + na_align(sizeof(gleam_result_t));  // ~7.2 MiB
 
 }  // namespace
 
@@ -1433,9 +1433,9 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   ch.srank = reinterpret_cast<uint32_t*>(base + kNaOffSrank);
   ch.old = reinterpret_cast<uint32_t*>(base + kNaOffOld);
   ch.spec = base + kNaOffSpec;
-  ch.cls = reinterpret_cast<uint32_t*>(base + kNaOffCls);
+  ch.cls = reinterpret_cast<unsigned long long*>(base + kNaOffCls);
   CallEntry* tbl = reinterpret_cast<CallEntry*>(base + kNaOffTbl);
-  CallEntry* cls_tbl = reinterpret_cast<CallEntry*>(base + kNaOffClsTbl);
+  ClassEntry* cls_tbl = reinterpret_cast<ClassEntry*>(base + kNaOffClsTbl);
   DevCtl* ctl = reinterpret_cast<DevCtl*>(base + kNaOffCtl);
   uint32_t* bcount = reinterpret_cast<uint32_t*>(base + kNaOffBcount);
   gleam_result_t* total = reinterpret_cast<gleam_result_t*>(base + kNaOffResult);
@@ -1448,7 +1448,7 @@ extern "C" int gleam_dedup_copy_noalloc(gleam_cache_t* c, const void* d_buf, siz
   if ((rc = cuda_err(cudaMemsetAsync(tbl, 0, tcap * sizeof(CallEntry), s))) != GLEAM_OK) return rc;
   const bool classes = (c->flags & GLEAM_KEY16) && !(c->flags & GLEAM_PAPER_IDS);
   if (classes &&
-      (rc = cuda_err(cudaMemsetAsync(cls_tbl, 0, tcap * sizeof(CallEntry), s))) != GLEAM_OK)
+      (rc = cuda_err(cudaMemsetAsync(cls_tbl, 0, tcap * sizeof(ClassEntry), s))) != GLEAM_OK)
     return rc;
 
   HashArgs h{};

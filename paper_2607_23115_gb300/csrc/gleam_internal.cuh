@@ -35,6 +35,18 @@ struct __align__(8) CallEntry {
   uint32_t minv;
 };
 
+// One entry of the per-call table of (16-bit index key, length) classes
+// (KEY16 with XXH64 keys), over the call's misses: owner and minv as in
+// CallEntry; count = misses of the class so far, so that each miss gets its
+// own place (0, 1, ...) in the run of index entries that the class's misses
+// occupy from the key's home position on.
+struct __align__(16) ClassEntry {
+  uint32_t owner;
+  uint32_t minv;
+  uint32_t count;
+  uint32_t pad;
+};
+
 // Per-chunk outcome of the probe/verify kernel.
 enum : uint8_t { kMissNoCand = 0, kMissCand = 1, kHit0 = 2, kUncached = 3 };
 
@@ -130,7 +142,8 @@ struct ChunkArrays {
   uint32_t* old;             // LRU: last use of a hit's slot before this call stamped it
   uint8_t* spec;             // 1: the hash kernel wrote the chunk to packed offset
                              // i*C of its payload and to arena slot slots_used + g
-  uint32_t* cls;             // KEY16: the chunk's entry in the per-call class table
+  unsigned long long* cls;   // KEY16, a miss: its entry in the per-call class table (low
+                             // 32 bits) and its place among the class's misses (high 32)
 };
 
 // Speculative verify.  After the first kPrefixBytes of a chunk the four XXH64
@@ -221,11 +234,11 @@ struct DedupArgs {
   uint32_t paper;            // no prefix hints are kept in GLEAM_PAPER_IDS mode
   uint32_t key16;            // GLEAM_KEY16: index key = low 16 bits of the group key
   // KEY16 with XXH64 keys: chunks are grouped by their whole fingerprint, so a
-  // miss's verify rejects inside the call (an earlier chunk with the same
+  // miss's verify rejects inside the call (an earlier miss with the same
   // 16-bit key and length) come from this second per-call table of (16-bit
-  // key, length) classes, each holding its smallest chunk number
+  // key, length) classes, each holding its smallest miss and its miss count
   uint32_t classes;
-  CallEntry* cls_tbl;        // same size as tbl
+  ClassEntry* cls_tbl;       // KEY16 classes: as many entries as tbl
   uint32_t plain_copy;       // copy misses with loads and stores, not bulk copies
                              // (payloads or outputs in host or managed memory)
   // LRU eviction (GLEAM_EVICT_LRU; lru == 0: the other fields are unused)
