@@ -844,7 +844,7 @@ __device__ __forceinline__ void resolve_rank(const DedupArgs& a, uint32_t G, uin
         // the class's misses (where its index insert starts); after the last
         // round a class minimum below a leader's number is an earlier miss of
         // its index key and length (a reject).  Groups are whole fingerprints, so
-        // nearly all leaders are found in round 1, while the other warps
+        // nearly all leaders are found in the first round, while the other warps
         // compare their duplicates.
         uint32_t cpost = 0xFFFFFFFFu;
         if (lead) {
