@@ -161,6 +161,9 @@ __device__ __noinline__ void warp_copy2(uint8_t* d1, uint8_t* d2, const uint8_t*
 // copies write it to the packed output and the arena slot.  Up to kPackBufs
 // pieces are in flight per warp across chunk boundaries.  Needs 16-byte
 // aligned addresses; a chunk's last len % 16 bytes are copied by its lane.
+#ifndef GLEAM_PACK_GRAB
+#define GLEAM_PACK_GRAB 1
+#endif
 #ifndef GLEAM_PACK_BULK
 #define GLEAM_PACK_BULK 1
 #endif
@@ -1384,12 +1387,33 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
     auto written_ahead = [&](uint32_t gg, uint32_t sr) {
       return a.spec_active && evict == 0 && sr == gg && ch.spec[gg];
     };
-    for (unsigned long long base = plo; base < phi; base += 32) {
-      const unsigned long long pc = base + lane;
+#if GLEAM_PACK_GRAB
+    // With GLEAM_PACK_GRAB the warps take their steps of 32 pieces from a
+    // counter of the call instead (each asks for its next step before it
+    // copies the current one), so that warps on SMs that copy faster take
+    // more.  The static ranges remain where the hash kernel wrote likely
+    // misses ahead (the steps then copy little, and the counter's round trip
+    // would be most of a step) and for counts the 32-bit counter cannot hold.
+    const bool grab = !a.spec_active && npieces < (1ull << 31);
+#else
+    const bool grab = false;
+#endif
+    unsigned long long step = plo, step_end = phi;
+    if (grab) {
+      uint32_t b0 = 0;
+      if (lane == 0) b0 = atomicAdd(&a.ctl->copy_next, 32u);
+      step = __shfl_sync(0xffffffffu, b0, 0);
+      step_end = npieces;
+    }
+    while (step < step_end) {
+      uint32_t next = 0;
+      if (grab && lane == 0) next = atomicAdd(&a.ctl->copy_next, 32u);
+      const unsigned long long shi = min(step_end, step + 32);
+      const unsigned long long pc = step + lane;
       uint32_t bytes = 0;
       bool copy = false;
       unsigned long long src = 0, d1 = 0, d2 = 0;
-      if (pc < phi) {
+      if (pc < shi) {
         const unsigned long long r = pc / ppc;
         const uint32_t off = (uint32_t)(pc - r * ppc) * kPackPiece;
         const uint32_t gg = ch.order[r];
@@ -1442,6 +1466,8 @@ __device__ __forceinline__ void pack_publish(const DedupArgs& a, uint32_t G, uin
         warp_copy2(reinterpret_cast<uint8_t*>(xj), reinterpret_cast<uint8_t*>(yj),
                    reinterpret_cast<const uint8_t*>(sj), lj, ((sj | xj | yj) & 15) == 0);
       }
+      if (grab) step = __shfl_sync(0xffffffffu, next, 0);
+      else step += 32;
     }
     // Every miss's index and hint-table entries, by rank: warp gw owns the
     // contiguous ranks [lo, hi), each lane inserting its own chunk (32
