@@ -1613,7 +1613,7 @@ __device__ __forceinline__ void resolve_pack_fast(const DedupArgs& a, uint32_t G
                                                   uint8_t* smem) {
   __shared__ unsigned long long red64[kWarps];
   __shared__ uint32_t wcnt[kWarps], swcnt[kWarps];
-  __shared__ unsigned long long s_slots0, s_sum[7], s_tot[4];
+  __shared__ unsigned long long s_slots0, s_sum[7];
   __shared__ int s_shared, s_err;
   const uint32_t lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const ChunkArrays& ch = a.ch;
